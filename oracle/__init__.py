@@ -1,0 +1,155 @@
+"""ctypes binding of the CPU oracle (``smetric_oracle.c``).
+
+TEST INFRASTRUCTURE ONLY: the test suite, the package smoke check and the
+benchmark's CPU-baseline leg may import this module; the product path never
+does. The oracle shares no code with the CUDA path. ``build()`` compiles it
+with gcc into ``oracle/_build/liboracle.so``.
+"""
+
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "smetric_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB = os.path.join(_BUILD, "liboracle.so")
+_lib = None
+
+u64p = np.ctypeslib.ndpointer(dtype=np.uint64, flags="C_CONTIGUOUS")
+i64p = np.ctypeslib.ndpointer(dtype=np.int64, flags="C_CONTIGUOUS")
+i32p = np.ctypeslib.ndpointer(dtype=np.int32, flags="C_CONTIGUOUS")
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (plain C11, OpenMP for the optional
+    request-parallel loop)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", "-O2", "-std=c11", "-Wall", "-Wextra", "-fopenmp",
+                               "-shared", "-fPIC", _SRC, "-o", tmp])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def load_library(path: str):
+    """Load an oracle build from `path` and declare its prototypes."""
+    L = C.CDLL(path)
+    L.oracle_mix64.restype = C.c_uint64
+    L.oracle_mix64.argtypes = [C.c_uint64]
+    L.oracle_block_hashes.restype = C.c_int64
+    L.oracle_block_hashes.argtypes = [i32p, C.c_int64, C.c_int32, C.c_uint64, u64p]
+    L.oracle_index_create.restype = C.c_void_p
+    L.oracle_index_create.argtypes = [C.c_int32]
+    L.oracle_index_destroy.restype = None
+    L.oracle_index_destroy.argtypes = [C.c_void_p]
+    for f in (L.oracle_index_insert, L.oracle_index_evict):
+        f.restype = C.c_int
+        f.argtypes = [C.c_void_p, u64p, i32p, C.c_int64]
+    L.oracle_index_contains.restype = C.c_int
+    L.oracle_index_contains.argtypes = [C.c_void_p, C.c_uint64, C.c_int32]
+    L.oracle_prefix_hits.restype = None
+    L.oracle_prefix_hits.argtypes = [C.c_void_p, u64p, C.c_int64, i64p, i64p]
+    L.oracle_route_batch.restype = C.c_int
+    L.oracle_route_batch.argtypes = [
+        C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p,
+        C.c_int64, C.c_int64, C.c_int64, i32p, i32p, i32p, u64p, C.c_void_p, C.c_int32]
+    return L
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        _lib = load_library(build())
+    return _lib
+
+
+def mix64(z: int, L=None) -> int:
+    return int((L or lib()).oracle_mix64(C.c_uint64(z & 0xFFFFFFFFFFFFFFFF)))
+
+
+def block_hashes(tokens: np.ndarray, block_size: int, seed: int = 0, L=None) -> np.ndarray:
+    t = np.ascontiguousarray(tokens, dtype=np.int32)
+    out = np.zeros(max(len(t) // block_size, 1), dtype=np.uint64)
+    n = (L or lib()).oracle_block_hashes(t if len(t) else np.zeros(1, np.int32), len(t), block_size,
+                                  seed & 0xFFFFFFFFFFFFFFFF, out)
+    if n < 0:
+        raise ValueError("invalid block size")
+    return out[:n]
+
+
+class OracleIndex:
+    """Two-tier KV$ index: local tier per instance plus one global tier (-1)."""
+
+    def __init__(self, num_instances: int, L=None):
+        self.N = num_instances
+        self._L = L or lib()
+        self._h = self._L.oracle_index_create(num_instances)
+        if not self._h:
+            raise ValueError("oracle_index_create failed")
+
+    def close(self):
+        if getattr(self, "_h", None):
+            self._L.oracle_index_destroy(self._h)
+            self._h = None
+
+    __del__ = close
+
+    def insert(self, keys, tiers):
+        k = np.ascontiguousarray(keys, dtype=np.uint64)
+        t = np.ascontiguousarray(np.broadcast_to(tiers, k.shape), dtype=np.int32)
+        if len(k) == 0:
+            return
+        rc = self._L.oracle_index_insert(self._h, k, t, len(k))
+        if rc != 0:
+            raise ValueError(f"oracle_index_insert: {rc}")
+
+    def evict(self, keys, tiers):
+        k = np.ascontiguousarray(keys, dtype=np.uint64)
+        t = np.ascontiguousarray(np.broadcast_to(tiers, k.shape), dtype=np.int32)
+        if len(k) == 0:
+            return
+        rc = self._L.oracle_index_evict(self._h, k, t, len(k))
+        if rc != 0:
+            raise ValueError(f"oracle_index_evict: {rc}")
+
+    def contains(self, key: int, tier: int) -> bool:
+        return bool(self._L.oracle_index_contains(self._h, C.c_uint64(int(key)), tier))
+
+    def prefix_hits(self, hashes: np.ndarray):
+        h = np.ascontiguousarray(hashes, dtype=np.uint64)
+        c = np.zeros(self.N, dtype=np.int64)
+        g = np.zeros(1, dtype=np.int64)
+        self._L.oracle_prefix_hits(self._h, h if len(h) else np.zeros(1, np.uint64), len(h), c, g)
+        return c, int(g[0])
+
+    def route_batch(self, block_size: int, session_blocks: int, seed: int, tokens, offsets,
+                    load, w_load: int, w_miss: int, w_glob: int, want_hashes: bool = False,
+                    n_threads: int = 1):
+        """Returns dict(instance, local_hit, global_hit, session_key[, block_hashes])."""
+        t = np.ascontiguousarray(tokens, dtype=np.int32)
+        o = np.ascontiguousarray(offsets, dtype=np.int64)
+        ld = np.ascontiguousarray(load, dtype=np.int64)
+        if len(ld) != self.N:
+            raise ValueError("load must have one entry per instance")
+        n = len(o) - 1
+        inst = np.zeros(max(n, 1), np.int32)
+        lh = np.zeros(max(n, 1), np.int32)
+        gh = np.zeros(max(n, 1), np.int32)
+        sk = np.zeros(max(n, 1), np.uint64)
+        nblk = int((np.diff(o) // block_size).sum()) if n > 0 else 0
+        hb = np.zeros(max(nblk, 1), np.uint64) if want_hashes else None
+        rc = self._L.oracle_route_batch(
+            self._h, block_size, session_blocks, seed & 0xFFFFFFFFFFFFFFFF,
+            t if len(t) else np.zeros(1, np.int32), o, n, ld, w_load, w_miss, w_glob,
+            inst, lh, gh, sk, hb.ctypes.data if hb is not None else None, n_threads)
+        if rc != 0:
+            raise ValueError(f"oracle_route_batch: {rc}")
+        out = dict(instance=inst[:n], local_hit=lh[:n], global_hit=gh[:n], session_key=sk[:n])
+        if want_hashes:
+            out["block_hashes"] = hb[:nblk]
+        return out

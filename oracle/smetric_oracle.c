@@ -1,0 +1,297 @@
+/*
+ * CPU oracle for the batched routing decision of balanced session-centric
+ * scheduling (SMetric, arXiv 2607.08565).
+ *
+ * TEST INFRASTRUCTURE ONLY. Only the test suite, the package smoke check and
+ * the benchmark's CPU-baseline leg may load this library. It shares no code,
+ * header, table or constant generator with the CUDA path; it is written from
+ * the definitions below so that a reader can check it against them by eye.
+ * It is deliberately plain: scalar loops, a chained hash map, a block-by-block
+ * prefix walk per tier and an exhaustive argmin.
+ *
+ * What it computes (per request r of a batch):
+ *
+ *  Block chain hash (Section 3.1: reuse is measured at KV$ block granularity;
+ *  Appendix A: a follow-up request's block-hash sequence starts with its
+ *  parent's, so the hash of block b must identify the whole prefix up to b).
+ *  The paper fixes no hash function; the definition here is SplitMix64-style:
+ *    mix64(z): the SplitMix64 output function (Steele, Lea & Flood, OOPSLA
+ *              2014, with Stafford's "Mix13" multipliers).
+ *    word k of block b: the little-endian u64 made of tokens bB+2k (low half)
+ *              and bB+2k+1 (high half), each as u32.
+ *    digest:   d_b = fold over k = 0..B/2-1 of x <- mix64(x ^ w_k), starting
+ *              from x = mix64(seed ^ B).
+ *    chain:    h_{-1} = mix64(seed + GAMMA);
+ *              h_b = mix64((h_{b-1} + GAMMA) ^ d_b), then h_b |= 2 when
+ *              h_b < 2 (0 and 1 are reserved), and the remapped value chains.
+ *    Only full blocks are hashed: n_r = floor(L_r / B); a partial tail block
+ *    is never a hit (Section 3.1 counts reuse in whole hit blocks).
+ *
+ *  Session key (Section 4.2, "Basic solution": sessions are identified from
+ *  the request itself, without per-session state): sk_r = h_{min(n_r,S)-1},
+ *  or 0 when n_r = 0.
+ *
+ *  Two-tier longest prefix match (Figure 6 / Figure 10: c = kvc.hit_len(req),
+ *  the per-instance local KV$ prefix hit; Section 2 and Section 4.2: a local
+ *  miss can be fetched from the global tier):
+ *    c_i = largest k <= n_r with h_0..h_{k-1} all in instance i's local tier,
+ *    g   = largest k <= n_r with h_0..h_{k-1} all in the global tier,
+ *    g_i = max(c_i, g).
+ *
+ *  Integer cost and argmin (Figure 6, instances.argmin(f(c, l)); Figure 10(c):
+ *  load = queued prefill plus the request's own new tokens):
+ *    miss_i  = L_r - B*g_i            (tokens instance i must prefill)
+ *    fetch_i = B*(g_i - c_i)          (tokens fetched from the global tier)
+ *    cost_i  = w_load*load_i + w_miss*miss_i + w_glob*fetch_i   (int64)
+ *    i*      = smallest i attaining the minimum cost.
+ *  Outputs: instance = i*, local_hit = B*c_{i*}, global_hit = fetch_{i*},
+ *  session_key = sk_r.
+ *
+ * Every request of a batch sees the same index and load (snapshot semantics).
+ */
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORACLE_GAMMA 0x9E3779B97F4A7C15ULL
+
+enum {
+  ORACLE_OK = 0,
+  ORACLE_ERR_INVALID_ARG = -1,
+  ORACLE_ERR_OOM = -2,
+};
+
+/* ------------------------------------------------------------------------ */
+/* Hashing                                                                  */
+/* ------------------------------------------------------------------------ */
+
+uint64_t oracle_mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+  return z ^ (z >> 31);
+}
+
+static uint64_t oracle_word(const int32_t* t, int64_t i) {
+  uint64_t lo = (uint64_t)(uint32_t)t[i];
+  uint64_t hi = (uint64_t)(uint32_t)t[i + 1];
+  return lo | (hi << 32);
+}
+
+/* Full-block chain hashes of one request. Writes floor(L/B) values to out and
+ * returns that count, or a negative error for an invalid block size. */
+int64_t oracle_block_hashes(const int32_t* tokens, int64_t L, int32_t B, uint64_t seed,
+                            uint64_t* out) {
+  if (B < 2 || (B % 2) != 0 || L < 0) return ORACLE_ERR_INVALID_ARG;
+  int64_t n = L / B;
+  uint64_t h = oracle_mix64(seed + ORACLE_GAMMA);
+  for (int64_t b = 0; b < n; ++b) {
+    uint64_t d = oracle_mix64(seed ^ (uint64_t)B);
+    for (int32_t k = 0; k < B / 2; ++k) d = oracle_mix64(d ^ oracle_word(tokens, b * B + 2 * k));
+    h = oracle_mix64((h + ORACLE_GAMMA) ^ d);
+    if (h < 2) h |= 2;
+    out[b] = h;
+  }
+  return n;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Index: key -> set of tiers (bit i < N: local tier of instance i; bit N:   */
+/* global tier). A chained hash map; nodes are never removed, a key whose    */
+/* tier set becomes empty is simply a member of no tier.                      */
+/* ------------------------------------------------------------------------ */
+
+typedef struct oracle_node {
+  uint64_t key;
+  struct oracle_node* next;
+  uint8_t tiers[]; /* (N + 1) bits */
+} oracle_node;
+
+typedef struct oracle_index {
+  int32_t N;
+  size_t tier_bytes;
+  uint64_t nbuckets;
+  uint64_t count;
+  oracle_node** buckets;
+} oracle_index;
+
+oracle_index* oracle_index_create(int32_t N) {
+  if (N < 1) return NULL;
+  oracle_index* x = (oracle_index*)calloc(1, sizeof(oracle_index));
+  if (!x) return NULL;
+  x->N = N;
+  x->tier_bytes = (size_t)(N + 1 + 7) / 8;
+  x->nbuckets = 1024;
+  x->buckets = (oracle_node**)calloc(x->nbuckets, sizeof(oracle_node*));
+  if (!x->buckets) { free(x); return NULL; }
+  return x;
+}
+
+void oracle_index_destroy(oracle_index* x) {
+  if (!x) return;
+  for (uint64_t i = 0; i < x->nbuckets; ++i) {
+    oracle_node* p = x->buckets[i];
+    while (p) { oracle_node* q = p->next; free(p); p = q; }
+  }
+  free(x->buckets);
+  free(x);
+}
+
+static oracle_node* oracle_find(const oracle_index* x, uint64_t key) {
+  for (oracle_node* p = x->buckets[key % x->nbuckets]; p; p = p->next)
+    if (p->key == key) return p;
+  return NULL;
+}
+
+static int oracle_grow(oracle_index* x) {
+  uint64_t nb = x->nbuckets * 2;
+  oracle_node** nbk = (oracle_node**)calloc(nb, sizeof(oracle_node*));
+  if (!nbk) return ORACLE_ERR_OOM;
+  for (uint64_t i = 0; i < x->nbuckets; ++i) {
+    oracle_node* p = x->buckets[i];
+    while (p) {
+      oracle_node* q = p->next;
+      p->next = nbk[p->key % nb];
+      nbk[p->key % nb] = p;
+      p = q;
+    }
+  }
+  free(x->buckets);
+  x->buckets = nbk;
+  x->nbuckets = nb;
+  return ORACLE_OK;
+}
+
+static int oracle_tier_bit(const oracle_index* x, int32_t tier) {
+  if (tier == -1) return x->N;
+  if (tier >= 0 && tier < x->N) return tier;
+  return -1;
+}
+
+/* Insert each (keys[j], tiers[j]) pair; tier -1 is the global tier. */
+int oracle_index_insert(oracle_index* x, const uint64_t* keys, const int32_t* tiers, int64_t n) {
+  if (!x || n < 0) return ORACLE_ERR_INVALID_ARG;
+  for (int64_t j = 0; j < n; ++j) {
+    int bit = oracle_tier_bit(x, tiers[j]);
+    if (bit < 0 || keys[j] < 2) return ORACLE_ERR_INVALID_ARG;
+    oracle_node* p = oracle_find(x, keys[j]);
+    if (!p) {
+      if (x->count >= x->nbuckets && oracle_grow(x) != ORACLE_OK) return ORACLE_ERR_OOM;
+      p = (oracle_node*)calloc(1, sizeof(oracle_node) + x->tier_bytes);
+      if (!p) return ORACLE_ERR_OOM;
+      p->key = keys[j];
+      p->next = x->buckets[keys[j] % x->nbuckets];
+      x->buckets[keys[j] % x->nbuckets] = p;
+      x->count++;
+    }
+    p->tiers[bit / 8] |= (uint8_t)(1u << (bit % 8));
+  }
+  return ORACLE_OK;
+}
+
+/* Remove each (keys[j], tiers[j]) membership; absent pairs are ignored. */
+int oracle_index_evict(oracle_index* x, const uint64_t* keys, const int32_t* tiers, int64_t n) {
+  if (!x || n < 0) return ORACLE_ERR_INVALID_ARG;
+  for (int64_t j = 0; j < n; ++j) {
+    int bit = oracle_tier_bit(x, tiers[j]);
+    if (bit < 0) return ORACLE_ERR_INVALID_ARG;
+    oracle_node* p = oracle_find(x, keys[j]);
+    if (p) p->tiers[bit / 8] &= (uint8_t)~(1u << (bit % 8));
+  }
+  return ORACLE_OK;
+}
+
+/* 1 if key is in the given tier (-1 = global), else 0. */
+int oracle_index_contains(const oracle_index* x, uint64_t key, int32_t tier) {
+  int bit = oracle_tier_bit(x, tier);
+  if (bit < 0) return 0;
+  const oracle_node* p = oracle_find(x, key);
+  return p && ((p->tiers[bit / 8] >> (bit % 8)) & 1u);
+}
+
+/* ------------------------------------------------------------------------ */
+/* Routing                                                                  */
+/* ------------------------------------------------------------------------ */
+
+/* Prefix hits of one hashed request: c[i] for each instance i and g for the
+ * global tier. Each tier's run starts at block 0 and stops at the first block
+ * that the tier does not hold; block k's tier set is looked up once and
+ * checked against every tier whose run is still going. */
+void oracle_prefix_hits(const oracle_index* x, const uint64_t* h, int64_t n, int64_t* c,
+                        int64_t* g) {
+  const int32_t N = x->N;
+  int32_t running = N + 1; /* tiers whose run has not stopped yet */
+  for (int32_t i = 0; i < N; ++i) c[i] = -1;
+  *g = -1;
+  for (int64_t k = 0; k < n && running > 0; ++k) {
+    const oracle_node* p = oracle_find(x, h[k]);
+    for (int32_t i = 0; i < N; ++i) {
+      if (c[i] >= 0) continue;
+      int held = p && ((p->tiers[i / 8] >> (i % 8)) & 1u);
+      if (!held) { c[i] = k; running--; }
+    }
+    if (*g < 0) {
+      int held = p && ((p->tiers[N / 8] >> (N % 8)) & 1u);
+      if (!held) { *g = k; running--; }
+    }
+  }
+  for (int32_t i = 0; i < N; ++i) if (c[i] < 0) c[i] = n; /* held every block */
+  if (*g < 0) *g = n;
+}
+
+/* Route one batch. offsets has n_requests + 1 entries; tokens holds
+ * offsets[n_requests] entries. block_hashes (may be NULL) receives every
+ * request's full-block hashes, request after request. n_threads > 1 routes
+ * requests in parallel (they are independent under snapshot semantics). */
+int oracle_route_batch(const oracle_index* x, int32_t B, int32_t S, uint64_t seed,
+                       const int32_t* tokens, const int64_t* offsets, int32_t n_requests,
+                       const int64_t* load, int64_t w_load, int64_t w_miss, int64_t w_glob,
+                       int32_t* instance, int32_t* local_hit, int32_t* global_hit,
+                       uint64_t* session_key, uint64_t* block_hashes, int32_t n_threads) {
+  if (!x || B < 2 || (B % 2) != 0 || S < 1 || n_requests < 0) return ORACLE_ERR_INVALID_ARG;
+  for (int32_t r = 0; r < n_requests; ++r)
+    if (offsets[r + 1] < offsets[r] || offsets[r] < 0) return ORACLE_ERR_INVALID_ARG;
+  const int32_t N = x->N;
+  int failed = 0;
+  /* first block index of each request in block_hashes */
+  int64_t* before = (int64_t*)malloc((size_t)(n_requests + 1) * sizeof(int64_t));
+  if (!before) return ORACLE_ERR_OOM;
+  before[0] = 0;
+  for (int32_t r = 0; r < n_requests; ++r) before[r + 1] = before[r] + (offsets[r + 1] - offsets[r]) / B;
+  (void)n_threads;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(n_threads > 0 ? n_threads : 1)
+  for (int32_t r = 0; r < n_requests; ++r) {
+    int64_t L = offsets[r + 1] - offsets[r];
+    int64_t n = L / B;
+    uint64_t* h = (uint64_t*)malloc((size_t)(n > 0 ? n : 1) * sizeof(uint64_t));
+    int64_t* c = (int64_t*)malloc((size_t)N * sizeof(int64_t));
+    if (!h || !c) {
+      free(h); free(c);
+#pragma omp atomic write
+      failed = 1;
+      continue;
+    }
+    oracle_block_hashes(tokens + offsets[r], L, B, seed, h);
+    if (block_hashes) memcpy(block_hashes + before[r], h, (size_t)n * sizeof(uint64_t));
+    int64_t g;
+    oracle_prefix_hits(x, h, n, c, &g);
+    int32_t best = -1;
+    int64_t best_cost = 0;
+    for (int32_t i = 0; i < N; ++i) {
+      int64_t gi = c[i] > g ? c[i] : g;
+      int64_t miss = L - (int64_t)B * gi;
+      int64_t fetch = (int64_t)B * (gi - c[i]);
+      int64_t cost = w_load * load[i] + w_miss * miss + w_glob * fetch;
+      if (best < 0 || cost < best_cost) { best = i; best_cost = cost; }
+    }
+    int64_t gb = c[best] > g ? c[best] : g;
+    instance[r] = best;
+    local_hit[r] = (int32_t)((int64_t)B * c[best]);
+    global_hit[r] = (int32_t)((int64_t)B * (gb - c[best]));
+    if (n == 0) session_key[r] = 0;
+    else session_key[r] = h[(n < S ? n : S) - 1];
+    free(h);
+    free(c);
+  }
+  free(before);
+  return failed ? ORACLE_ERR_OOM : ORACLE_OK;
+}

@@ -1,0 +1,400 @@
+"""Pins for the CPU oracle: checks against what the paper and mathematics fix.
+
+Each check takes an oracle library handle so the same checks can be run
+against deliberately broken oracle builds (test_oracle_mutants.py) to show
+that a plausible mistake anywhere in the oracle fails at least one of them.
+"""
+
+from __future__ import annotations
+
+import json
+import os
+from fractions import Fraction
+
+import numpy as np
+
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+M64 = (1 << 64) - 1
+GAMMA = 0x9E3779B97F4A7C15
+
+
+def _golden_hex(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return [int(x, 16) for x in f.read().split("\n") if x and not x.startswith("#")]
+
+
+def _golden_json(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+# ---------------------------------------------------------------------------
+# mix64
+# ---------------------------------------------------------------------------
+
+def check_published_vector(L):
+    """The SplitMix64 generator's published first outputs for seed 0."""
+    want = _golden_hex("splitmix64_seed0.txt")
+    state = 0
+    for w in want:
+        state = (state + GAMMA) & M64
+        assert oracle.mix64(state, L) == w, hex(w)
+
+
+def _py_mix64(z):
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & M64
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & M64
+    return z ^ (z >> 31)
+
+
+def _unxorshift(z, s):
+    x = z
+    for _ in range(64 // s + 1):
+        x = z ^ (x >> s)
+    return x
+
+
+def py_mix64_inverse(z):
+    """Inverse of the SplitMix64 output function (each step is a bijection:
+    xor-shift right by s >= 1, and multiplication by an odd constant)."""
+    z = _unxorshift(z, 31)
+    z = (z * pow(0x94D049BB133111EB, -1, 1 << 64)) & M64
+    z = _unxorshift(z, 27)
+    z = (z * pow(0xBF58476D1CE4E5B9, -1, 1 << 64)) & M64
+    return _unxorshift(z, 30)
+
+
+def check_bijection(L):
+    rng = np.random.default_rng(7)
+    for z in rng.integers(0, 2**63, size=64).tolist() + [0, 1, M64]:
+        assert py_mix64_inverse(oracle.mix64(z, L)) == z
+
+
+# ---------------------------------------------------------------------------
+# chain hash
+# ---------------------------------------------------------------------------
+
+def check_prefix_locality(L):
+    """h_b depends on exactly tokens [0, (b+1)B): flipping token p leaves
+    every h_b with b < p // B unchanged and changes every later one."""
+    rng = np.random.default_rng(1)
+    for B in (2, 4, 16):
+        t = rng.integers(0, 151936, size=B * 9 + B // 2, dtype=np.int32)
+        h = oracle.block_hashes(t, B, 0, L)
+        assert len(h) == 9
+        for p in rng.choice(len(t), size=12, replace=False):
+            u = t.copy()
+            u[p] ^= 0x55
+            hu = oracle.block_hashes(u, B, 0, L)
+            j = p // B
+            assert np.array_equal(h[:min(j, 9)], hu[:min(j, 9)])
+            assert np.all(h[j:] != hu[j:])
+        # every block position matters, not only its content: repeating one
+        # block's tokens must not repeat its hash
+        rep = np.tile(t[:B], 6)
+        hr = oracle.block_hashes(rep, B, 0, L)
+        assert len(set(hr.tolist())) == 6
+
+
+def check_tail_and_empty(L):
+    rng = np.random.default_rng(2)
+    B = 8
+    t = rng.integers(0, 151936, size=5 * B, dtype=np.int32)
+    base = oracle.block_hashes(t, B, 0, L)
+    for extra in range(B):
+        u = np.concatenate([t, rng.integers(0, 151936, size=extra, dtype=np.int32)])
+        assert np.array_equal(oracle.block_hashes(u, B, 0, L), base)
+    assert len(oracle.block_hashes(t[:B - 1], B, 0, L)) == 0
+    assert len(oracle.block_hashes(t[:0], B, 0, L)) == 0
+
+
+def check_seed_and_block_size(L):
+    rng = np.random.default_rng(3)
+    t = rng.integers(0, 151936, size=64, dtype=np.int32)
+    a = oracle.block_hashes(t, 16, 0, L)
+    b = oracle.block_hashes(t, 16, 12345, L)
+    assert np.all(a != b)
+    c = oracle.block_hashes(t, 32, 0, L)
+    assert c[0] != a[1] and c[0] != a[0]
+
+
+def sentinel_tokens(target_pre_remap: int, seed: int = 0):
+    """Two tokens (B = 2) whose block-0 chain value before the remap equals
+    `target_pre_remap`, constructed by inverting the definition."""
+    h_init = _py_mix64((seed + GAMMA) & M64)
+    # h_0 = mix64((h_init + GAMMA) ^ d_0); want h_0 == target
+    d0 = py_mix64_inverse(target_pre_remap) ^ ((h_init + GAMMA) & M64)
+    # d_0 = mix64(mix64(seed ^ B) ^ w_0), B = 2
+    w0 = py_mix64_inverse(d0) ^ _py_mix64(seed ^ 2)
+    lo, hi = w0 & 0xFFFFFFFF, w0 >> 32
+    return np.array([lo, hi], dtype=np.uint32).view(np.int32)
+
+
+def check_sentinel_remap(L):
+    """0 and 1 are reserved: a chain value of 0 becomes 2, 1 becomes 3, and the
+    remapped value is what the next block chains from."""
+    rng = np.random.default_rng(4)
+    for target, want in ((0, 2), (1, 3)):
+        for seed in (0, 99):
+            t = sentinel_tokens(target, seed)
+            h = oracle.block_hashes(t, 2, seed, L)
+            assert len(h) == 1 and int(h[0]) == want
+            more = np.concatenate([t, rng.integers(0, 151936, size=2, dtype=np.int32)])
+            h2 = oracle.block_hashes(more, 2, seed, L)
+            w1 = int(more[2].astype(np.uint32)) | (int(more[3].astype(np.uint32)) << 32)
+            d1 = _py_mix64(_py_mix64(seed ^ 2) ^ w1)
+            assert int(h2[1]) == _py_mix64(((want + GAMMA) & M64) ^ d1)
+
+
+# ---------------------------------------------------------------------------
+# routing
+# ---------------------------------------------------------------------------
+
+def _route(ix, B, S, tokens_list, load, w=(1, 4, 2), seed=0):
+    from synth.traces import pack
+    tokens, offsets = pack(tokens_list)
+    return ix.route_batch(B, S, seed, tokens, offsets, np.asarray(load, np.int64), *w,
+                          want_hashes=True)
+
+
+def check_session_key(L):
+    rng = np.random.default_rng(5)
+    B = 4
+    for S in (1, 3, 7):
+        ix = oracle.OracleIndex(2, L)
+        shared = rng.integers(0, 151936, size=S * B, dtype=np.int32)
+        reqs = [np.concatenate([shared, rng.integers(0, 151936, size=k, dtype=np.int32)])
+                for k in (0, 3, 9, 40)]
+        reqs += [shared[:B * (S - 1)] if S > 1 else shared[:0], shared[:2]]
+        out = _route(ix, B, S, reqs, [0, 0])
+        sk = out["session_key"]
+        assert len(set(sk[:4].tolist())) == 1 and sk[0] != 0
+        for r, t in enumerate(reqs):
+            h = oracle.block_hashes(t, B, 0, L)
+            want = 0 if len(h) == 0 else h[min(len(h), S) - 1]
+            assert sk[r] == want
+        assert sk[-1] == 0  # fewer than B tokens: no full block
+        other = np.concatenate([shared[:B * (S - 1)], shared[B * (S - 1):] ^ 1])
+        assert _route(ix, B, S, [other], [0, 0])["session_key"][0] != sk[0]
+
+
+def brute_hit(req, stored, B):
+    """Longest k such that every request prefix of 1..k blocks equals a
+    block-aligned prefix of some stored prompt, by token comparison."""
+    prefixes = set()
+    for p in stored:
+        for j in range(1, len(p) // B + 1):
+            prefixes.add(tuple(p[:j * B].tolist()))
+    k = 0
+    while k < len(req) // B and tuple(req[:(k + 1) * B].tolist()) in prefixes:
+        k += 1
+    return k
+
+
+def _mutate(rng, base, n_tokens):
+    """A prompt sharing a random-length prefix with base (alphabet {0,1,2})."""
+    keep = int(rng.integers(0, min(len(base), n_tokens) + 1))
+    return np.concatenate([base[:keep], rng.integers(0, 3, size=n_tokens - keep, dtype=np.int32)])
+
+
+def check_brute_force_prefix(L):
+    rng = np.random.default_rng(6)
+    for trial in range(60):
+        B = int(rng.choice([2, 4]))
+        N = int(rng.integers(1, 6))
+        base = rng.integers(0, 3, size=8 * B, dtype=np.int32)
+        stored = {t: [_mutate(rng, base, int(rng.integers(0, 9 * B)))
+                      for _ in range(int(rng.integers(0, 4)))] for t in range(-1, N)}
+        ix = oracle.OracleIndex(N, L)
+        for t, prompts in stored.items():
+            for p in prompts:
+                ix.insert(oracle.block_hashes(p, B, 0, L), t)
+        for _ in range(6):
+            req = _mutate(rng, base, int(rng.integers(0, 9 * B)))
+            h = oracle.block_hashes(req, B, 0, L)
+            c, g = ix.prefix_hits(h)
+            assert g == brute_hit(req, stored[-1], B)
+            for i in range(N):
+                assert c[i] == brute_hit(req, stored[i], B), (trial, i)
+            # the routing outputs agree with these hits
+            load = rng.integers(0, 50, size=N)
+            out = _route(ix, B, 2, [req], load)
+            i = int(out["instance"][0])
+            gi = max(c[i], g)
+            assert out["local_hit"][0] == B * c[i]
+            assert out["global_hit"][0] == B * (gi - c[i])
+            cost = [1 * load[j] + 4 * (len(req) - B * max(c[j], g)) + 2 * B * (max(c[j], g) - c[j])
+                    for j in range(N)]
+            assert i == int(np.argmin(cost))
+
+
+def check_non_prefix_closed(L):
+    """A tier that holds a deep block but not an earlier one stops at the gap."""
+    rng = np.random.default_rng(8)
+    B = 4
+    t = rng.integers(0, 151936, size=10 * B, dtype=np.int32)
+    h = oracle.block_hashes(t, B, 0, L)
+    ix = oracle.OracleIndex(2, L)
+    ix.insert(h[[0, 1, 2, 4, 5]], 0)
+    ix.insert(h[[1, 2, 3]], 1)
+    ix.insert(h[:7], -1)
+    c, g = ix.prefix_hits(h)
+    assert list(c) == [3, 0] and g == 7
+
+
+def check_jsq_when_index_empty(L):
+    """Empty index: cost_i = w_load*load_i + w_miss*L, so routing is
+    join-the-shortest-queue (Section 4.1, 'Load-balance-only'), ties to the
+    lowest id."""
+    rng = np.random.default_rng(9)
+    for N in (1, 3, 8, 33):
+        ix = oracle.OracleIndex(N, L)
+        reqs = [rng.integers(0, 151936, size=int(rng.integers(0, 200)), dtype=np.int32)
+                for _ in range(20)]
+        for _ in range(5):
+            load = rng.integers(0, 4, size=N)  # many ties
+            out = _route(ix, 8, 3, reqs, load)
+            assert np.all(out["instance"] == int(np.argmin(load)))
+            assert np.all(out["local_hit"] == 0) and np.all(out["global_hit"] == 0)
+
+
+def check_argmax_hit_when_load_ignored(L):
+    """w_load = 0 and an empty global tier: cost_i = w_miss*(L - B*c_i), so
+    routing picks the instance with the longest local hit (the paper's
+    prev = argmax(c), Figure 10), ties to the lowest id."""
+    rng = np.random.default_rng(10)
+    B = 2
+    for trial in range(30):
+        N = int(rng.integers(1, 7))
+        base = rng.integers(0, 3, size=10 * B, dtype=np.int32)
+        stored = {i: [_mutate(rng, base, int(rng.integers(0, 11 * B)))
+                      for _ in range(int(rng.integers(0, 3)))] for i in range(N)}
+        ix = oracle.OracleIndex(N, L)
+        for i, ps in stored.items():
+            for p in ps:
+                ix.insert(oracle.block_hashes(p, B, 0, L), i)
+        req = _mutate(rng, base, int(rng.integers(0, 11 * B)))
+        c = [brute_hit(req, stored[i], B) for i in range(N)]
+        out = _route(ix, B, 1, [req], rng.integers(0, 1000, size=N), w=(0, 3, 5))
+        assert int(out["instance"][0]) == int(np.argmax(c))
+
+
+def check_equal_costs_pick_zero(L):
+    ix = oracle.OracleIndex(5, L)
+    rng = np.random.default_rng(11)
+    reqs = [rng.integers(0, 151936, size=50, dtype=np.int32) for _ in range(4)]
+    out = _route(ix, 4, 1, reqs, [7] * 5)
+    assert np.all(out["instance"] == 0)
+
+
+def check_paper_examples(L):
+    ex = _golden_json("paper_examples.json")
+    rng = np.random.default_rng(12)
+    a = ex["three_token_two_hits"]
+    B = a["block_size"]
+    t = rng.integers(0, 151936, size=a["prompt_len"], dtype=np.int32)
+    ix = oracle.OracleIndex(1, L)
+    ix.insert(oracle.block_hashes(t, B, 0, L)[:a["cached_blocks"]], 0)
+    out = _route(ix, B, 1, [t], [0])
+    assert out["local_hit"][0] == a["expect_local_hit"]
+    assert a["prompt_len"] - out["local_hit"][0] - out["global_hit"][0] == a["expect_tokens_to_compute"]
+
+    b = ex["reuse_70_to_80"]
+    B = b["block_size"]
+    t = rng.integers(0, 151936, size=b["prompt_len"], dtype=np.int32)
+    h = oracle.block_hashes(t, B, 0, L)
+    comp = []
+    for k in (b["cached_blocks_low"], b["cached_blocks_high"]):
+        ix = oracle.OracleIndex(1, L)
+        ix.insert(h[:k], 0)
+        out = _route(ix, B, 1, [t], [0])
+        comp.append(b["prompt_len"] - int(out["local_hit"][0]))
+    assert comp == [b["expect_compute_low"], b["expect_compute_high"]]
+    assert Fraction(comp[0] - comp[1], comp[0]) == Fraction(b["expect_cut_num"], b["expect_cut_den"])
+
+
+def check_hand_costs(L):
+    ex = _golden_json("hand_costs.json")
+    B, Lp, N = ex["block_size"], ex["prompt_len"], ex["num_instances"]
+    rng = np.random.default_rng(13)
+    t = rng.integers(0, 151936, size=Lp, dtype=np.int32)
+    h = oracle.block_hashes(t, B, 0, L)
+    ix = oracle.OracleIndex(N, L)
+    ix.insert(h[:ex["global_blocks"]], -1)
+    for i, k in enumerate(ex["local_blocks"]):
+        ix.insert(h[:k], i)
+    for case in ex["cases"]:
+        out = _route(ix, B, 1, [t], case["load"], w=tuple(ex["weights"]))
+        assert int(out["instance"][0]) == case["instance"], case
+        assert int(out["local_hit"][0]) == case["local_hit"], case
+        assert int(out["global_hit"][0]) == case["global_hit"], case
+
+
+def check_batch_invariants(L):
+    """Invariants on a synthetic multi-turn batch: hits never exceed the full
+    blocks, and a session's key is the same on every turn."""
+    from synth import agent_trace, ReplayDriver
+    tr = agent_trace("c1_tiny", scale=0.25, seed=3)
+    p = tr.params
+    ix = oracle.OracleIndex(p.num_instances, L)
+    drv = ReplayDriver(p.num_instances, p.block_size)
+    keys_by_session = {}
+    for bt in tr.batches():
+        out = ix.route_batch(p.block_size, p.session_blocks, 0, bt.tokens, bt.offsets, drv.load,
+                             p.w_load, p.w_miss, p.w_glob, want_hashes=True)
+        lens = bt.lengths()
+        nfull = (lens // p.block_size) * p.block_size
+        assert np.all(out["local_hit"] + out["global_hit"] <= nfull)
+        assert np.all(out["local_hit"] >= 0) and np.all(out["global_hit"] >= 0)
+        for s, k in zip(bt.sessions.tolist(), out["session_key"].tolist()):
+            assert keys_by_session.setdefault(s, k) == k
+        ins_k, ins_t, ev_k, ev_t = drv.after_batch(bt.offsets, out["instance"], out["local_hit"],
+                                                   out["block_hashes"])
+        ix.insert(ins_k, ins_t)
+        ix.evict(ev_k, ev_t)
+    assert len(keys_by_session) == tr.n_sessions
+
+
+def check_index_set_semantics(L):
+    """Insert/evict behave as set operations per tier (against Python sets)."""
+    rng = np.random.default_rng(14)
+    N = 5
+    ix = oracle.OracleIndex(N, L)
+    ref = {t: set() for t in range(-1, N)}
+    universe = rng.integers(2, 2**62, size=300).astype(np.uint64)
+    for step in range(40):
+        k = rng.choice(universe, size=int(rng.integers(0, 60)))
+        t = rng.integers(-1, N, size=len(k)).astype(np.int32)
+        if rng.random() < 0.6:
+            ix.insert(k, t)
+            for a, b in zip(k.tolist(), t.tolist()):
+                ref[b].add(a)
+        else:
+            ix.evict(k, t)
+            for a, b in zip(k.tolist(), t.tolist()):
+                ref[b].discard(a)
+        for key in rng.choice(universe, size=30).tolist():
+            for tier in range(-1, N):
+                assert ix.contains(key, tier) == (key in ref[tier])
+
+
+ALL_CHECKS = [
+    check_published_vector,
+    check_bijection,
+    check_prefix_locality,
+    check_tail_and_empty,
+    check_seed_and_block_size,
+    check_sentinel_remap,
+    check_session_key,
+    check_brute_force_prefix,
+    check_non_prefix_closed,
+    check_jsq_when_index_empty,
+    check_argmax_hit_when_load_ignored,
+    check_equal_costs_pick_zero,
+    check_paper_examples,
+    check_hand_costs,
+    check_batch_invariants,
+    check_index_set_semantics,
+]

@@ -1,0 +1,96 @@
+"""The pins catch plausible oracle mistakes.
+
+Each mutant below is the oracle source with one plausible slip (a dropped
+term, a wrong sign or index, a transposed operand, a flipped tie-break). Each
+is compiled on the CPU and must fail at least one pin in pins.ALL_CHECKS.
+"""
+
+import os
+import subprocess
+import sys
+
+import pytest
+
+import oracle
+from pins import ALL_CHECKS
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "smetric_oracle.c")
+
+MUTANTS = {
+    "mix64_shift": ("z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;",
+                    "z = (z ^ (z >> 31)) * 0xBF58476D1CE4E5B9ULL;"),
+    "word_halves_swapped": ("return lo | (hi << 32);", "return hi | (lo << 32);"),
+    "digest_start_drops_block_size": ("uint64_t d = oracle_mix64(seed ^ (uint64_t)B);",
+                                      "uint64_t d = oracle_mix64(seed);"),
+    "chain_drops_previous": ("h = oracle_mix64((h + ORACLE_GAMMA) ^ d);",
+                             "h = oracle_mix64(ORACLE_GAMMA ^ d);"),
+    "chain_xor_for_add": ("h = oracle_mix64((h + ORACLE_GAMMA) ^ d);",
+                          "h = oracle_mix64((h ^ ORACLE_GAMMA) ^ d);"),
+    "no_sentinel_remap": ("if (h < 2) h |= 2;", ""),
+    "word_index_off_by_one": ("oracle_word(tokens, b * B + 2 * k)",
+                              "oracle_word(tokens, b * B + k)"),
+    "session_key_index": ("session_key[r] = h[(n < S ? n : S) - 1];",
+                          "session_key[r] = h[(n - 1 < S ? n - 1 : S)];"),
+    "walk_counts_missing_block": ("if (!held) { c[i] = k; running--; }",
+                                  "if (!held) { c[i] = k + 1; running--; }"),
+    "global_walk_ignored": ("if (!held) { *g = k; running--; }",
+                            "if (!held || 1) { *g = k; running--; }"),
+    "miss_uses_local_hit": ("int64_t miss = L - (int64_t)B * gi;",
+                            "int64_t miss = L - (int64_t)B * c[i];"),
+    "fetch_sign": ("int64_t fetch = (int64_t)B * (gi - c[i]);",
+                   "int64_t fetch = (int64_t)B * (c[i] - gi);"),
+    "global_weight_dropped": ("+ w_glob * fetch;", ";"),
+    "tie_to_highest": ("if (best < 0 || cost < best_cost)", "if (best < 0 || cost <= best_cost)"),
+    "global_hit_reports_g": ("global_hit[r] = (int32_t)((int64_t)B * (gb - c[best]));",
+                             "global_hit[r] = (int32_t)((int64_t)B * gb);"),
+    "tail_block_hashed": ("int64_t n = L / B;\n  uint64_t h = oracle_mix64",
+                          "int64_t n = (L + B - 1) / B;\n  uint64_t h = oracle_mix64"),
+}
+
+
+def _build_mutant(name, tmp_path):
+    src = open(SRC).read()
+    old, new = MUTANTS[name]
+    assert src.count(old) >= 1, name
+    path_c = tmp_path / f"{name}.c"
+    path_so = tmp_path / f"{name}.so"
+    path_c.write_text(src.replace(old, new, 1))
+    subprocess.check_call(["gcc", "-O1", "-std=c11", "-w", "-fopenmp", "-shared", "-fPIC",
+                           str(path_c), "-o", str(path_so)])
+    return oracle.load_library(str(path_so))
+
+
+_RUNNER = """
+import sys
+sys.path[:0] = [{root!r}, {tests!r}]
+import oracle
+from pins import ALL_CHECKS
+L = oracle.load_library({so!r})
+failed = []
+for check in ALL_CHECKS:
+    try:
+        check(L)
+    except Exception as e:
+        failed.append(check.__name__)
+print("FAILED_CHECKS", ",".join(failed))
+"""
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name, tmp_path):
+    src = open(SRC).read()
+    old, new = MUTANTS[name]
+    assert src.count(old) >= 1, name
+    path_c = tmp_path / f"{name}.c"
+    path_so = tmp_path / f"{name}.so"
+    path_c.write_text(src.replace(old, new, 1))
+    subprocess.check_call(["gcc", "-O1", "-std=c11", "-w", "-fopenmp", "-shared", "-fPIC",
+                           str(path_c), "-o", str(path_so)])
+    here = os.path.dirname(os.path.abspath(__file__))
+    code = _RUNNER.format(root=os.path.dirname(here), tests=here, so=str(path_so))
+    p = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, timeout=300)
+    if p.returncode != 0:
+        return  # the mutant crashed (e.g. read past its buffer): caught
+    line = [x for x in p.stdout.splitlines() if x.startswith("FAILED_CHECKS")][-1]
+    failed = line.split(" ", 1)[1].strip() if " " in line else ""
+    assert failed, f"mutant {name} passed every pin"
