@@ -1,0 +1,471 @@
+#!/usr/bin/env python3
+"""Benchmark of the batched routing path on the config-4 burst workload.
+
+One step = one smetric_route_batch call over one batch of 8,192 requests
+(block hash, session key, two-tier prefix match, cost, argmin). Inputs are
+resident in HBM when the timed region starts; four distinct batches of
+~820 MB each rotate, so every step reads inputs larger than L2.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 the script runs under torchrun, one rank per GPU: every rank holds
+a replica of the (static) index and routes its own batches; there is no
+collective on the data path (weak scaling). Rank 0 prints one JSON line.
+--impl reference times the CPU oracle on the host cores instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "routed requests/sec and prompt tokens hashed+matched/sec on 1 GB300; % HBM roofline"
+UNIT = "requests/s"
+WORKLOAD = ("c4_burst: 65536 concurrent sessions, Zipf(1.1) popularity, 64 instances, block 32, "
+            "prompts U[8k,40k] tokens with a 95% cached prefix, index pre-populated at load "
+            "factor 0.7, batches of 8192 requests")
+N_DISTINCT_BATCHES = 4
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--e2e-steps", type=int, default=8)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist  # noqa: F811
+        backend = "nccl" if args.impl == "ours" else "gloo"
+        if backend == "nccl":
+            import torch
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return rank, world, local, dist
+
+
+# ---------------------------------------------------------------------------
+# clocks
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock, power and throttle reasons."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu: str):
+        self.gpu = gpu
+        self.proc = None
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.t0 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.gpu)], stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        self.t0 = time.time()
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        self.f.flush()
+        self.f.seek(0)
+        rows = [r.split(", ") for r in self.f.read().strip().splitlines() if r.strip()]
+        os.unlink(self.f.name)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+                for n, v in zip(names, r[5:9]):
+                    if v.strip().lower() == "active":
+                        reasons.add(n)
+            except (IndexError, ValueError):
+                continue
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm),
+                "window": "warm-up and timed steps"}
+
+
+def peak_hbm():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def ncu_traffic(kernel: str):
+    """Per-launch DRAM bytes of `kernel` from the committed ncu summary, if
+    that summary was taken on the current kernel source; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)[kernel]
+    except (OSError, KeyError, ValueError):
+        return None
+    src = os.path.join(ROOT, "paper_2607_08565_gb300", "csrc", rec["source"])
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    return rec["bytes_per_launch"] if sha == rec["source_sha"] else None
+
+
+# ---------------------------------------------------------------------------
+# workload
+# ---------------------------------------------------------------------------
+
+def c4_trace():
+    from synth import burst_trace
+    return burst_trace()
+
+
+def populate_index(ix, tr, device, chunk=4096):
+    import torch
+    B = tr.params.block_size
+    buf = np.empty(int(tr.prefix_len.max()) * chunk, np.int32)
+    for ids, tok, off in tr.prepopulation(chunk=chunk, out=buf):
+        hb, _ = ix.block_hashes(torch.from_numpy(tok).to(device), torch.from_numpy(off).to(device))
+        nb = torch.from_numpy(tr.prefix_len[ids] // B).to(device)
+        hb = hb[:int(nb.sum())]
+        owner = torch.repeat_interleave(torch.arange(len(ids), device=device), nb)
+        sess = torch.from_numpy(ids).to(device)[owner]
+        ix.insert(hb, -1)
+        for tier_of, member in ((tr.home, tr.in_home), (tr.second, tr.in_second)):
+            m = torch.from_numpy(member).to(device)[sess]
+            t = torch.from_numpy(tier_of).to(device)[sess]
+            ix.insert(hb[m].contiguous(), t[m].contiguous())
+    ix.check()
+
+
+def algorithmic_bytes(lens, local_hit, global_hit, B, W):
+    """Per-kernel algorithmic bytes of one route call: digest reads 4 B per
+    hashed token; walk reads one index entry (key + W
+    mask words) per probed block, P_r = min(n_r, reach_r + 1), plus offsets
+    and outputs; prep reads offsets and loads."""
+    nb = lens // B
+    reach = (local_hit.astype(np.int64) + global_hit) // B
+    probes = np.minimum(nb, reach + 1)
+    n = len(lens)
+    return {
+        "k_digest": int(4 * B * nb.sum()),
+        "k_walk": int(probes.sum() * (8 + 8 * W) + 16 * n + 20 * n),
+        "k_prep": int(16 * n),
+        "path": int(4 * lens.sum() + probes.sum() * (8 + 8 * W) + 8 * (n + 1) + 20 * n),
+    }
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing
+# ---------------------------------------------------------------------------
+
+def oracle_index_for(tr, batches):
+    """Oracle index holding every session prefix the given batches use."""
+    import oracle
+    p = tr.params
+    ox = oracle.OracleIndex(p.num_instances)
+    sessions = np.unique(np.concatenate([b.sessions for b in batches]))
+    for s in sessions.tolist():
+        h = oracle.block_hashes(tr.session_prefix(s), p.block_size, p.hash_seed)
+        for t in tr.session_tiers(s):
+            ox.insert(h, t)
+    return ox
+
+
+def oracle_route(tr, ox, bt, m, threads):
+    """Seconds the oracle takes to route the first m requests of bt."""
+    p = tr.params
+    off = bt.offsets[:m + 1]
+    t0 = time.perf_counter()
+    ox.route_batch(p.block_size, p.session_blocks, p.hash_seed, bt.tokens[:off[-1]], off,
+                   bt.load, p.w_load, p.w_miss, p.w_glob, n_threads=threads)
+    return time.perf_counter() - t0
+
+
+def oracle_calibrate(tr, ox, bt, seconds, threads):
+    """Largest prefix m of the batch (doubling from 64) routed in about
+    `seconds`; returns (m, seconds taken)."""
+    m = min(64, bt.n_requests)
+    while True:
+        dt = oracle_route(tr, ox, bt, m, threads)
+        if dt >= seconds / 2 or m == bt.n_requests:
+            return m, dt
+        m = min(bt.n_requests, max(m * 2, int(m * seconds / max(dt, 1e-3))))
+
+
+def run_reference(args, rank, world, dist):
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    tr = c4_trace()
+    threads = os.cpu_count() or 1
+    batches = [tr.batch(k) for k in range(N_DISTINCT_BATCHES)]
+    ox = oracle_index_for(tr, batches)
+    per_step = min(2.0, 150.0 / max(1, args.warmup + args.steps))
+    m, _ = oracle_calibrate(tr, ox, batches[0], per_step, threads)
+    for i in range(args.warmup):
+        oracle_route(tr, ox, batches[i % len(batches)], m, threads)
+    times, toks = [], 0
+    for i in range(args.steps):
+        bt = batches[i % len(batches)]
+        times.append(oracle_route(tr, ox, bt, m, threads))
+        toks += int(bt.offsets[m])
+    total = sum(times)
+    rps = args.steps * m / total
+    sample = (f"first {m} of the 8192 requests of a config-4 batch per step (4 batches rotated), "
+              f"oracle index holding those batches' sessions, {threads} threads")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": rps, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u64",
+        "data": "synthetic", "tokens_per_s": toks / total,
+        "config": {"workload": WORKLOAD, "l2": "host run"},
+        "cpu_baseline": {"value": rps, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": rps, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args, rank, world, local, dist):
+    import torch
+    import paper_2607_08565_gb300 as pkg
+    from paper_2607_08565_gb300 import build_lib
+
+    if rank == 0 or not build_lib.up_to_date():
+        build_lib.build()
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    tr = c4_trace()
+    p = tr.params
+    N, B = p.num_instances, p.block_size
+
+    # this rank's batches: ids rank, rank + world, ... (distinct across ranks)
+    ids = [rank + world * i for i in range(N_DISTINCT_BATCHES)]
+    host = [tr.batch(k) for k in ids]
+    max_tok = max(b.n_tokens for b in host)
+    nkeys = tr.n_prefix_blocks()
+    ix = pkg.SMetricIndex(N, B, p.session_blocks, capacity_slots=int(nkeys / 0.7) + 1,
+                          max_batch_requests=tr.batch_size, max_batch_tokens=max_tok,
+                          hash_seed=p.hash_seed, host_staging=True)
+    populate_index(ix, tr, device)
+    dev_b = []
+    for b in host:
+        dev_b.append(dict(tok=torch.from_numpy(b.tokens).to(device),
+                          off=torch.from_numpy(b.offsets).to(device),
+                          load=torch.from_numpy(b.load).to(device), n=b.n_requests,
+                          n_tokens=b.n_tokens))
+    n = tr.batch_size
+    outs = dict(instance=torch.empty(n, dtype=torch.int32, device=device),
+                local_hit=torch.empty(n, dtype=torch.int32, device=device),
+                global_hit=torch.empty(n, dtype=torch.int32, device=device),
+                session_key=torch.empty(n, dtype=torch.uint64, device=device))
+    w = (p.w_load, p.w_miss, p.w_glob)
+    stream = torch.cuda.current_stream(device)
+
+    def step(i):
+        b = dev_b[i % len(dev_b)]
+        pkg.smetric_route_batch(ix.handle, b["tok"], b["n_tokens"], b["off"], b["n"], b["load"], w,
+                                outs["instance"], outs["local_hit"], outs["global_hit"],
+                                outs["session_key"], None, 0, stream)
+
+    # per-batch outputs (for the algorithmic-byte count)
+    per_batch = []
+    for i in range(len(dev_b)):
+        step(i)
+        ix.check()
+        per_batch.append({k: v.cpu().numpy().copy() for k, v in outs.items()})
+
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(local).uuid)
+    except Exception:
+        gpu_id = str(local)
+    clocks = ClockSampler(gpu_id)
+    clocks.start()
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    launches0 = pkg.smetric_launch_count(ix.handle)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1)
+    launches = pkg.smetric_launch_count(ix.handle) - launches0
+    clk = clocks.stop()
+    rc = ix.status()
+    if rc != pkg.SMETRIC_OK:
+        raise pkg.SmetricError(rc, "bench")
+    if dist is not None:
+        t = torch.tensor([ms], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        if dist is not None:
+            dist.barrier()
+
+    reqs_per_step = np.mean([b.n_requests for b in host])
+    toks_per_step = np.mean([b.n_tokens for b in host])
+    value = world * args.steps * reqs_per_step / (ms / 1e3)
+    tokens_per_s = world * args.steps * toks_per_step / (ms / 1e3)
+
+    # per-kernel durations, measured live with CUDA events on the launch stream
+    pkg.smetric_profile_enable(ix.handle, True)
+    kprof_steps = max(20, min(args.steps, 200))
+    for i in range(kprof_steps):
+        step(i)
+    prof = pkg.smetric_profile_read(ix.handle)
+    pkg.smetric_profile_enable(ix.handle, False)
+    algo = [algorithmic_bytes(b.lengths(), pb["local_hit"], pb["global_hit"], B, ix.W)
+            for b, pb in zip(host, per_batch)]
+    algo_mean = {k: float(np.mean([a[k] for a in algo])) for k in algo[0]}
+    peak, peak_kind = peak_hbm()
+    dom = max(prof, key=lambda k: prof[k][0])
+    dom_ms = prof[dom][0] / max(prof[dom][1], 1)
+    achieved = algo_mean[dom] / (dom_ms / 1e3) / 1e9
+    path_ms = ms / args.steps
+    path_gbs = algo_mean["path"] / (path_ms / 1e3) / 1e9
+    traffic = ncu_traffic(dom)
+
+    # end to end through the host-buffer entry point: H2D of the batch, route,
+    # D2H of the outputs, every step
+    pinned = []
+    for b in host[:2]:
+        t = torch.empty(b.n_tokens, dtype=torch.int32, pin_memory=True)
+        t.numpy()[:] = b.tokens
+        pinned.append(dict(tok=t, off=torch.from_numpy(b.offsets).pin_memory(),
+                           load=torch.from_numpy(b.load).pin_memory(), n=b.n_requests,
+                           n_tokens=b.n_tokens))
+    hout = dict(instance=torch.empty(n, dtype=torch.int32, pin_memory=True),
+                local_hit=torch.empty(n, dtype=torch.int32, pin_memory=True),
+                global_hit=torch.empty(n, dtype=torch.int32, pin_memory=True),
+                session_key=torch.empty(n, dtype=torch.uint64, pin_memory=True))
+
+    def e2e_step(i):
+        b = pinned[i % len(pinned)]
+        rc = pkg.smetric_route_batch_host(ix.handle, b["tok"], b["n_tokens"], b["off"], b["n"],
+                                          b["load"], w, hout["instance"], hout["local_hit"],
+                                          hout["global_hit"], hout["session_key"], stream)
+        if rc != pkg.SMETRIC_OK:
+            raise pkg.SmetricError(rc, "e2e")
+
+    for i in range(2):
+        e2e_step(i)
+    if dist is not None:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for i in range(args.e2e_steps):
+        e2e_step(i)
+    e2e_s = time.perf_counter() - t0
+    if dist is not None:
+        t = torch.tensor([e2e_s], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e_reqs = np.mean([b["n"] for b in pinned])
+    e2e_value = world * args.e2e_steps * e2e_reqs / e2e_s
+    h2d = float(np.mean([4 * b["n_tokens"] + 8 * (b["n"] + 1) + 8 * N for b in pinned]))
+    d2h = float(20 * e2e_reqs)
+    # the host-buffer path must agree with the device path
+    last = per_batch[(args.e2e_steps - 1) % len(pinned)]
+    for k in hout:
+        if not np.array_equal(hout[k].numpy(), last[k]):
+            raise RuntimeError(f"host-buffer route differs from the device route in {k}")
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        threads = os.cpu_count() or 1
+        ox = oracle_index_for(tr, host[:1])
+        m, dt = oracle_calibrate(tr, ox, host[0], args.cpu_seconds, threads)
+        cpu = {"value": m / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+               "sample": f"first {m} of the 8192 requests of config-4 batch {ids[0]} "
+                         f"({dt:.1f} s on {threads} threads), oracle index holding that batch's "
+                         f"sessions", "tokens_per_s": float(host[0].offsets[m]) / dt}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": path_ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+            "tokens_per_s": tokens_per_s,
+            "config": {"workload": WORKLOAD, "batch": int(reqs_per_step),
+                       "num_instances": N, "block_size": B, "index_keys": nkeys,
+                       "l2": f"inputs larger than L2: {N_DISTINCT_BATCHES} distinct batches of "
+                             f"{toks_per_step * 4 / 1e6:.0f} MB rotated"},
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
+                         "unit": "GB/s", "frac": achieved / peak, "peak_kind": f"{peak_kind} copy",
+                         "traffic": traffic, "algorithmic_bytes_per_launch": algo_mean[dom],
+                         "ms_per_launch": dom_ms},
+            "roofline_path": {"achieved": path_gbs, "frac": path_gbs / peak,
+                              "algorithmic_bytes_per_step": algo_mean["path"]},
+            "kernels_ms_per_launch": {k: v[0] / max(v[1], 1) for k, v in prof.items()},
+            "clocks": clk,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "steps": args.e2e_steps},
+            "gpu_launches": int(launches),
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    ix.close()
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    rank, world, local, dist = dist_setup(args)
+    if args.impl == "reference":
+        run_reference(args, rank, world, dist)
+        if dist is not None:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
+    run_ours(args, rank, world, local, dist)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,204 @@
+/*
+ * smetric.h - C ABI of the batched routing path of balanced session-centric
+ * scheduling (SMetric, arXiv 2607.08565), for one NVIDIA GB300 (sm_103a).
+ *
+ * For a batch of agent requests the library
+ *   (a) chain-hashes each prompt's int32 tokens in blocks of B tokens,
+ *   (b) derives a stateless session key from the leading S blocks,
+ *   (c) longest-prefix-matches the block-hash chain against a two-tier KV$
+ *       index (one local tier per serving instance plus one global tier),
+ *   (d) scores every instance with an integer cost and takes the argmin.
+ * The paper's router scores instances per request (Section 4.1, Figure 6:
+ * "route to argmin over instances of f(c_i, l_i)", with c_i the prefix hit of
+ * the prompt in instance i's local KV$ and l_i its load) and keeps only
+ * per-instance state (Section 4.2, Challenge 1); the two-tier store is the
+ * local GPU tier plus the cluster-wide global tier (Section 2, Figure 2).
+ *
+ * Definitions (exact; every output is bit-reproducible):
+ *   mix64(z)  SplitMix64 output function: z ^= z>>30; z *= 0xBF58476D1CE4E5B9;
+ *             z ^= z>>27; z *= 0x94D049BB133111EB; z ^= z>>31 (mod 2^64).
+ *   GAMMA     0x9E3779B97F4A7C15.
+ *   w_{b,k}   (uint32)t[bB+2k] | (uint32)t[bB+2k+1] << 32, k < B/2.
+ *   d_b       x = mix64(seed ^ B); for k: x = mix64(x ^ w_{b,k}); d_b = x.
+ *   h_b       h_{-1} = mix64(seed + GAMMA); h_b = mix64((h_{b-1}+GAMMA) ^ d_b),
+ *             then h_b |= 2 if h_b < 2. Only the n_r = floor(L_r/B) full
+ *             blocks are hashed.
+ *   sk_r      h_{min(n_r,S)-1}, or 0 if n_r = 0.
+ *   c_i       largest k <= n_r with h_0..h_{k-1} all in instance i's local tier.
+ *   g         largest k <= n_r with h_0..h_{k-1} all in the global tier.
+ *   cost_i    w_load*load_i + w_miss*(L_r - B*max(c_i,g))
+ *             + w_glob*B*(max(c_i,g) - c_i), in int64.
+ *   i*        smallest i with minimal cost_i.
+ * Every request of one batch sees the same index and load (snapshot).
+ *
+ * Conventions
+ *   - "d_" pointers are device memory of the device that was current at
+ *     smetric_index_create; "h_" pointers are host memory (pinned memory
+ *     gives the fastest copies). The caller owns every buffer it passes.
+ *   - Calls are stream-ordered: inserts, evictions and routes enqueued on one
+ *     stream see each other's effects in enqueue order. Calls on one index
+ *     share that index's scratch, so they must not run concurrently on
+ *     different streams.
+ *   - Host-detectable errors return immediately with nothing enqueued.
+ *     Device-detectable errors (bad offsets, out-of-range tiers or loads, a
+ *     full table) are latched in the index and reported by smetric_status.
+ *   - Nothing here allocates device memory except smetric_index_create.
+ */
+#ifndef SMETRIC_H
+#define SMETRIC_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* smetric_stream_t;
+
+typedef struct smetric_index smetric_index; /* opaque, library-owned */
+
+enum {
+  SMETRIC_OK = 0,
+  SMETRIC_ERR_INVALID_ARG = -1, /* bad argument, offsets, tier or key */
+  SMETRIC_ERR_OOM = -2,         /* device allocation failed at create */
+  SMETRIC_ERR_TABLE_FULL = -3,  /* an insert found no free slot */
+  SMETRIC_ERR_CUDA = -4,        /* a CUDA runtime call failed */
+  SMETRIC_ERR_OVERFLOW = -5     /* a load or prompt length outside the exact int64 range */
+};
+
+/* Instance limit and the limits that keep every cost exact in int64:
+ * |cost| < 3 * 2^20 * 2^40 < 2^63. */
+#define SMETRIC_MAX_INSTANCES 256
+#define SMETRIC_MAX_WEIGHT (1LL << 20)
+#define SMETRIC_MAX_LOAD (1LL << 40)
+/* An insert that probes this many slots without finding its key or a free
+ * slot reports SMETRIC_ERR_TABLE_FULL; lookups stop after as many probes. */
+#define SMETRIC_MAX_PROBE 65536
+
+/* smetric_index_config.flags */
+#define SMETRIC_FLAG_HOST_STAGING 1 /* allocate device staging buffers for smetric_route_batch_host */
+
+typedef struct {
+  int32_t num_instances;      /* N, 1..SMETRIC_MAX_INSTANCES (local tiers 0..N-1) */
+  int32_t block_size;         /* B, even, 2..256 tokens */
+  int32_t session_blocks;     /* S >= 1: blocks that form the session key */
+  int32_t flags;              /* SMETRIC_FLAG_* */
+  uint64_t capacity_slots;    /* index slots, >= 1; size for a load factor <= 0.7 */
+  uint64_t hash_seed;         /* seed of the chain hash */
+  int64_t max_batch_requests; /* largest n_requests a route call accepts */
+  int64_t max_batch_tokens;   /* largest n_tokens a route call accepts */
+} smetric_index_config;
+
+/* Integer cost weights, each in [0, SMETRIC_MAX_WEIGHT]. */
+typedef struct {
+  int64_t w_load; /* per queued token of the instance (Figure 10(c): q_i) */
+  int64_t w_miss; /* per token the instance must prefill */
+  int64_t w_glob; /* per token fetched from the global tier (Section 1: slower, limited bandwidth) */
+} smetric_weights;
+
+/* Create an empty index and its route scratch on the current device.
+ * The table holds capacity_slots entries of 16, 32 or 64 bytes (key plus
+ * ceil((N+1)/64) tier-mask words, padded to a power of two); the scratch
+ * holds max_batch_tokens/B + max_batch_requests + 1 64-bit words.
+ * Returns SMETRIC_ERR_INVALID_ARG for an out-of-range field and
+ * SMETRIC_ERR_OOM when a device allocation fails; *out is NULL then. */
+int smetric_index_create(const smetric_index_config* cfg, smetric_index** out);
+
+/* Free the index and its device memory. Waits for the device first.
+ * NULL is accepted. */
+int smetric_index_destroy(smetric_index* idx);
+
+/* Empty every tier (Section 2, Figure 2: the KV$ store's contents). */
+int smetric_index_clear(smetric_index* idx, smetric_stream_t stream);
+
+/* Tier membership updates (Section 2: the local tier of each instance and the
+ * global tier each cache KV$ blocks; the serving side reports which blocks
+ * each tier holds). For each j < n: add key d_keys[j] to tier d_tiers[j]
+ * (0..N-1 = local tier of that instance, -1 = global tier). Keys are block
+ * hashes (>= 2). Set semantics: idempotent and order-independent within a
+ * call. Errors latched: a key < 2 or tier out of range (INVALID_ARG, that
+ * pair skipped), no free slot (TABLE_FULL). */
+int smetric_index_insert(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers,
+                         int64_t n, smetric_stream_t stream);
+
+/* Remove key d_keys[j] from tier d_tiers[j]; absent pairs are ignored. A key
+ * that leaves its last tier keeps its slot and matches no tier. */
+int smetric_index_evict(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers,
+                        int64_t n, smetric_stream_t stream);
+
+/* Tier masks of n keys: d_masks[j*W + w] is word w of key j's tier set
+ * (bit i < N: local tier of instance i; bit N: global tier; zeros for an
+ * absent key), W = smetric_index_mask_words(idx). */
+int smetric_index_lookup(smetric_index* idx, const uint64_t* d_keys, int64_t n,
+                         uint64_t* d_masks, smetric_stream_t stream);
+
+/* W = ceil((N+1)/64), the number of 64-bit tier-mask words per key; 0 for NULL. */
+int32_t smetric_index_mask_words(const smetric_index* idx);
+
+/* The routing step (Figure 6 and Figure 10: per request, the local hit c of
+ * every instance, then argmin over instances of the cost).
+ *   d_tokens   int32 [n_tokens], 16-byte aligned; request r is
+ *              d_tokens[d_offsets[r] .. d_offsets[r+1]).
+ *   d_offsets  int64 [n_requests+1], non-decreasing, d_offsets[0] >= 0,
+ *              d_offsets[n_requests] <= n_tokens, every length < 2^31.
+ *   d_load     int64 [N], each in [0, SMETRIC_MAX_LOAD].
+ *   outputs    int32 d_instance[r] = i*, d_local_hit[r] = B*c_{i*},
+ *              d_global_hit[r] = B*(max(c_{i*},g) - c_{i*}),
+ *              uint64 d_session_key[r] = sk_r.
+ *   d_block_hashes  NULL, or uint64 [hashes_cap] receiving every request's
+ *              full-block hashes h_0..h_{n_r-1}, request after request;
+ *              hashes_cap must be >= n_tokens / B.
+ * 0 <= n_requests <= max_batch_requests and 0 <= n_tokens <= max_batch_tokens.
+ * With invalid offsets or loads the call latches INVALID_ARG or OVERFLOW and
+ * writes instance -1, zero hits and key 0 for every request. */
+int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                        const int64_t* d_offsets, int32_t n_requests, const int64_t* d_load,
+                        smetric_weights w, int32_t* d_instance, int32_t* d_local_hit,
+                        int32_t* d_global_hit, uint64_t* d_session_key,
+                        uint64_t* d_block_hashes, int64_t hashes_cap, smetric_stream_t stream);
+
+/* Step (a)-(b) alone: block hashes and session keys of a batch, without
+ * index lookups (Appendix A: a request's block-hash sequence starts with its
+ * parent's). Same argument rules as smetric_route_batch; d_block_hashes is
+ * required here. */
+int smetric_block_hashes(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                         const int64_t* d_offsets, int32_t n_requests, uint64_t* d_session_key,
+                         uint64_t* d_block_hashes, int64_t hashes_cap, smetric_stream_t stream);
+
+/* smetric_route_batch from host buffers: copies tokens, offsets and load to
+ * the index's staging buffers (the index must have been created with
+ * SMETRIC_FLAG_HOST_STAGING), routes, copies the four outputs back and waits
+ * for the stream. Returns the call's status including any error the device
+ * latched, which it clears. */
+int smetric_route_batch_host(smetric_index* idx, const int32_t* h_tokens, int64_t n_tokens,
+                             const int64_t* h_offsets, int32_t n_requests, const int64_t* h_load,
+                             smetric_weights w, int32_t* h_instance, int32_t* h_local_hit,
+                             int32_t* h_global_hit, uint64_t* h_session_key,
+                             smetric_stream_t stream);
+
+/* Wait for `stream`, then return and clear the first error the device latched
+ * for this index since the last call (SMETRIC_OK if none). */
+int smetric_status(smetric_index* idx, smetric_stream_t stream);
+
+/* Static description of an error code. */
+const char* smetric_strerror(int code);
+
+/* Observability. With profiling on, each route records CUDA events around
+ * each of its kernels on the launch stream. smetric_profile_read waits for
+ * them and returns, per kernel k < min(max_kernels, count), the summed device
+ * milliseconds ms[k] and launches[k] since the previous read, then resets;
+ * it returns the number of kernels a route launches (or a negative error).
+ * smetric_profile_kernel_name(k) names kernel k. */
+int smetric_profile_enable(smetric_index* idx, int32_t on);
+int smetric_profile_read(smetric_index* idx, int32_t max_kernels, double* ms, int64_t* launches);
+const char* smetric_profile_kernel_name(int32_t k);
+
+/* Kernels this index has launched since it was created. */
+int64_t smetric_launch_count(const smetric_index* idx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SMETRIC_H */

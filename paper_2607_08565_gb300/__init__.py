@@ -1,0 +1,338 @@
+"""Python binding of libsmetric.so, the GB300 batched routing path of
+balanced session-centric scheduling (SMetric, arXiv 2607.08565).
+
+Functions carry the C ABI's names and only marshal arguments: device arrays
+may be passed as torch tensors or raw device pointers (ints); streams as a
+torch.cuda.Stream, a raw cudaStream_t (int) or None for torch's current
+stream. Every computation runs in the library's CUDA kernels; there is no
+CPU fallback, and using the binding without the built library raises.
+
+SMetricIndex wraps one index and allocates output tensors for convenience.
+"""
+
+from __future__ import annotations
+
+import ctypes as C
+import os
+from typing import Optional
+
+from .build_lib import LIB as _LIB_PATH
+
+SMETRIC_OK = 0
+SMETRIC_ERR_INVALID_ARG = -1
+SMETRIC_ERR_OOM = -2
+SMETRIC_ERR_TABLE_FULL = -3
+SMETRIC_ERR_CUDA = -4
+SMETRIC_ERR_OVERFLOW = -5
+SMETRIC_MAX_INSTANCES = 256
+SMETRIC_MAX_WEIGHT = 1 << 20
+SMETRIC_MAX_LOAD = 1 << 40
+SMETRIC_MAX_PROBE = 65536
+SMETRIC_FLAG_HOST_STAGING = 1
+
+EXPORTED = (
+    "smetric_index_create", "smetric_index_destroy", "smetric_index_clear",
+    "smetric_index_insert", "smetric_index_evict", "smetric_index_lookup",
+    "smetric_index_mask_words", "smetric_route_batch", "smetric_block_hashes",
+    "smetric_route_batch_host", "smetric_status", "smetric_strerror",
+    "smetric_profile_enable", "smetric_profile_read", "smetric_profile_kernel_name",
+    "smetric_launch_count",
+)
+
+
+class SmetricError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {smetric_strerror(code)} ({code})")
+
+
+class smetric_index_config(C.Structure):
+    _fields_ = [
+        ("num_instances", C.c_int32),
+        ("block_size", C.c_int32),
+        ("session_blocks", C.c_int32),
+        ("flags", C.c_int32),
+        ("capacity_slots", C.c_uint64),
+        ("hash_seed", C.c_uint64),
+        ("max_batch_requests", C.c_int64),
+        ("max_batch_tokens", C.c_int64),
+    ]
+
+
+class smetric_weights(C.Structure):
+    _fields_ = [("w_load", C.c_int64), ("w_miss", C.c_int64), ("w_glob", C.c_int64)]
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def lib():
+    """The loaded libsmetric.so. Raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError(
+                f"libsmetric.so is not built ({_LIB_PATH}); run __graft_entry__.build() "
+                "or python -m paper_2607_08565_gb300.build_lib")
+        L = C.CDLL(_LIB_PATH)
+        P, I32, I64, U64 = C.c_void_p, C.c_int32, C.c_int64, C.c_uint64
+        sig = {
+            "smetric_index_create": (C.c_int, [C.POINTER(smetric_index_config), C.POINTER(P)]),
+            "smetric_index_destroy": (C.c_int, [P]),
+            "smetric_index_clear": (C.c_int, [P, P]),
+            "smetric_index_insert": (C.c_int, [P, P, P, I64, P]),
+            "smetric_index_evict": (C.c_int, [P, P, P, I64, P]),
+            "smetric_index_lookup": (C.c_int, [P, P, I64, P, P]),
+            "smetric_index_mask_words": (I32, [P]),
+            "smetric_route_batch": (C.c_int, [P, P, I64, P, I32, P, smetric_weights, P, P, P, P, P,
+                                              I64, P]),
+            "smetric_block_hashes": (C.c_int, [P, P, I64, P, I32, P, P, I64, P]),
+            "smetric_route_batch_host": (C.c_int, [P, P, I64, P, I32, P, smetric_weights, P, P, P,
+                                                   P, P]),
+            "smetric_status": (C.c_int, [P, P]),
+            "smetric_strerror": (C.c_char_p, [C.c_int]),
+            "smetric_profile_enable": (C.c_int, [P, I32]),
+            "smetric_profile_read": (C.c_int, [P, I32, P, P]),
+            "smetric_profile_kernel_name": (C.c_char_p, [I32]),
+            "smetric_launch_count": (I64, [P]),
+        }
+        for name, (res, args) in sig.items():
+            f = getattr(L, name)
+            f.restype, f.argtypes = res, args
+        _lib = L
+    return _lib
+
+
+# ---------------------------------------------------------------------------
+# marshalling helpers
+# ---------------------------------------------------------------------------
+
+def _ptr(x) -> Optional[int]:
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        if not x.is_contiguous():
+            raise ValueError("arrays must be contiguous")
+        return x.data_ptr() if x.numel() > 0 else None
+    if hasattr(x, "ctypes"):  # numpy array (host memory)
+        return x.ctypes.data if x.size > 0 else None
+    raise TypeError(f"cannot pass {type(x)} as a pointer")
+
+
+def _stream(s) -> Optional[int]:
+    if s is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+def _check(rc: int, where: str):
+    if rc != SMETRIC_OK:
+        raise SmetricError(rc, where)
+
+
+def _weights(w) -> smetric_weights:
+    if isinstance(w, smetric_weights):
+        return w
+    a, b, c = w
+    return smetric_weights(int(a), int(b), int(c))
+
+
+# ---------------------------------------------------------------------------
+# C ABI, one function per entry point
+# ---------------------------------------------------------------------------
+
+def smetric_index_create(cfg: smetric_index_config) -> int:
+    h = C.c_void_p()
+    _check(lib().smetric_index_create(C.byref(cfg), C.byref(h)), "smetric_index_create")
+    return h.value
+
+
+def smetric_index_destroy(idx: int) -> None:
+    _check(lib().smetric_index_destroy(idx), "smetric_index_destroy")
+
+
+def smetric_index_clear(idx: int, stream=None) -> None:
+    _check(lib().smetric_index_clear(idx, _stream(stream)), "smetric_index_clear")
+
+
+def smetric_index_insert(idx: int, d_keys, d_tiers, n: int, stream=None) -> None:
+    _check(lib().smetric_index_insert(idx, _ptr(d_keys), _ptr(d_tiers), n, _stream(stream)),
+           "smetric_index_insert")
+
+
+def smetric_index_evict(idx: int, d_keys, d_tiers, n: int, stream=None) -> None:
+    _check(lib().smetric_index_evict(idx, _ptr(d_keys), _ptr(d_tiers), n, _stream(stream)),
+           "smetric_index_evict")
+
+
+def smetric_index_lookup(idx: int, d_keys, n: int, d_masks, stream=None) -> None:
+    _check(lib().smetric_index_lookup(idx, _ptr(d_keys), n, _ptr(d_masks), _stream(stream)),
+           "smetric_index_lookup")
+
+
+def smetric_index_mask_words(idx: int) -> int:
+    return int(lib().smetric_index_mask_words(idx))
+
+
+def smetric_route_batch(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int, d_load,
+                        w, d_instance, d_local_hit, d_global_hit, d_session_key,
+                        d_block_hashes=None, hashes_cap: int = 0, stream=None) -> None:
+    _check(lib().smetric_route_batch(idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests,
+                                     _ptr(d_load), _weights(w), _ptr(d_instance), _ptr(d_local_hit),
+                                     _ptr(d_global_hit), _ptr(d_session_key), _ptr(d_block_hashes),
+                                     hashes_cap, _stream(stream)), "smetric_route_batch")
+
+
+def smetric_block_hashes(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int,
+                         d_session_key, d_block_hashes, hashes_cap: int, stream=None) -> None:
+    _check(lib().smetric_block_hashes(idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests,
+                                      _ptr(d_session_key), _ptr(d_block_hashes), hashes_cap,
+                                      _stream(stream)), "smetric_block_hashes")
+
+
+def smetric_route_batch_host(idx: int, h_tokens, n_tokens: int, h_offsets, n_requests: int, h_load,
+                             w, h_instance, h_local_hit, h_global_hit, h_session_key,
+                             stream=None) -> int:
+    """Returns the call's status (device-latched errors included)."""
+    return int(lib().smetric_route_batch_host(idx, _ptr(h_tokens), n_tokens, _ptr(h_offsets),
+                                              n_requests, _ptr(h_load), _weights(w),
+                                              _ptr(h_instance), _ptr(h_local_hit),
+                                              _ptr(h_global_hit), _ptr(h_session_key),
+                                              _stream(stream)))
+
+
+def smetric_status(idx: int, stream=None) -> int:
+    return int(lib().smetric_status(idx, _stream(stream)))
+
+
+def smetric_strerror(code: int) -> str:
+    return lib().smetric_strerror(code).decode()
+
+
+def smetric_profile_enable(idx: int, on: bool) -> None:
+    _check(lib().smetric_profile_enable(idx, 1 if on else 0), "smetric_profile_enable")
+
+
+def smetric_profile_read(idx: int):
+    """{kernel name: (milliseconds, launches)} since the previous read."""
+    ms = (C.c_double * 8)()
+    ln = (C.c_int64 * 8)()
+    k = lib().smetric_profile_read(idx, 8, ms, ln)
+    if k < 0:
+        raise SmetricError(k, "smetric_profile_read")
+    return {smetric_profile_kernel_name(i): (ms[i], ln[i]) for i in range(k)}
+
+
+def smetric_profile_kernel_name(k: int) -> str:
+    return lib().smetric_profile_kernel_name(k).decode()
+
+
+def smetric_launch_count(idx: int) -> int:
+    return int(lib().smetric_launch_count(idx))
+
+
+# ---------------------------------------------------------------------------
+# convenience wrapper
+# ---------------------------------------------------------------------------
+
+class SMetricIndex:
+    """One two-tier index on the current CUDA device, with torch outputs."""
+
+    def __init__(self, num_instances: int, block_size: int, session_blocks: int,
+                 capacity_slots: int, max_batch_requests: int, max_batch_tokens: int,
+                 hash_seed: int = 0, host_staging: bool = False):
+        self.cfg = smetric_index_config(num_instances, block_size, session_blocks,
+                                        SMETRIC_FLAG_HOST_STAGING if host_staging else 0,
+                                        capacity_slots, hash_seed & 0xFFFFFFFFFFFFFFFF,
+                                        max_batch_requests, max_batch_tokens)
+        self.handle = smetric_index_create(self.cfg)
+        self.N, self.B, self.S = num_instances, block_size, session_blocks
+        self.W = smetric_index_mask_words(self.handle)
+
+    def close(self):
+        if getattr(self, "handle", None):
+            smetric_index_destroy(self.handle)
+            self.handle = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *a):
+        self.close()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _tiers(self, keys, tiers):
+        import torch
+        if isinstance(tiers, int):
+            tiers = torch.full(keys.shape, tiers, dtype=torch.int32, device=keys.device)
+        return tiers
+
+    def insert(self, keys, tiers, stream=None):
+        tiers = self._tiers(keys, tiers)
+        smetric_index_insert(self.handle, keys, tiers, keys.numel(), stream)
+
+    def evict(self, keys, tiers, stream=None):
+        tiers = self._tiers(keys, tiers)
+        smetric_index_evict(self.handle, keys, tiers, keys.numel(), stream)
+
+    def clear(self, stream=None):
+        smetric_index_clear(self.handle, stream)
+
+    def lookup(self, keys, stream=None):
+        import torch
+        out = torch.empty((keys.numel(), self.W), dtype=torch.uint64, device=keys.device)
+        smetric_index_lookup(self.handle, keys, keys.numel(), out, stream)
+        return out
+
+    def route_batch(self, tokens, offsets, load, weights=(1, 4, 2), want_hashes=False,
+                    out=None, stream=None):
+        """Returns dict(instance, local_hit, global_hit, session_key[, block_hashes])."""
+        import torch
+        n = offsets.numel() - 1
+        dev = offsets.device
+        if out is None:
+            out = dict(instance=torch.empty(n, dtype=torch.int32, device=dev),
+                       local_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                       global_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                       session_key=torch.empty(n, dtype=torch.uint64, device=dev))
+            if want_hashes:
+                out["block_hashes"] = torch.empty(max(tokens.numel() // self.B, 1),
+                                                  dtype=torch.uint64, device=dev)
+        hb = out.get("block_hashes")
+        smetric_route_batch(self.handle, tokens, tokens.numel(), offsets, n, load, weights,
+                            out["instance"], out["local_hit"], out["global_hit"],
+                            out["session_key"], hb, hb.numel() if hb is not None else 0, stream)
+        return out
+
+    def block_hashes(self, tokens, offsets, stream=None):
+        """Returns (block_hashes, session_key) as device tensors."""
+        import torch
+        n = offsets.numel() - 1
+        dev = offsets.device
+        hb = torch.empty(max(tokens.numel() // self.B, 1), dtype=torch.uint64, device=dev)
+        sk = torch.empty(max(n, 1), dtype=torch.uint64, device=dev)
+        smetric_block_hashes(self.handle, tokens, tokens.numel(), offsets, n, sk, hb, hb.numel(),
+                             stream)
+        return hb, sk[:n]
+
+    def status(self, stream=None) -> int:
+        return smetric_status(self.handle, stream)
+
+    def check(self, stream=None):
+        rc = self.status(stream)
+        if rc != SMETRIC_OK:
+            raise SmetricError(rc, "device")

@@ -1,0 +1,280 @@
+// Two-tier KV$ index on the GPU: one open-addressing table, key -> tier mask.
+//
+// The paper's KV$ store has a local tier per serving instance and a global
+// tier shared by the cluster (Section 2, Figures 1-2); the router needs, per
+// block hash, which tiers hold the block. One table serves all tiers: an
+// entry is the 64-bit block hash followed by W = ceil((N+1)/64) mask words,
+// bit i < N = local tier of instance i, bit N = global tier. Linear probing
+// from home_slot(key); key 0 marks a never-used slot. Keys are never removed:
+// an evicted key keeps its slot with a cleared bit, so lookups never see
+// tombstones and concurrent inserts cannot create duplicates.
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <new>
+
+#include "smetric_impl.cuh"
+
+using namespace smetric;
+
+namespace smetric {
+
+int cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return SMETRIC_OK;
+  (void)cudaGetLastError();
+  return SMETRIC_ERR_CUDA;
+}
+
+int check_device(const smetric_index* idx) {
+  if (!idx) return SMETRIC_ERR_INVALID_ARG;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return cuda_status(cudaErrorInvalidDevice);
+  return dev == idx->device ? SMETRIC_OK : SMETRIC_ERR_INVALID_ARG;
+}
+
+}  // namespace smetric
+
+namespace {
+
+enum Op { kInsert = 0, kEvict = 1 };
+
+// One thread per (key, tier) pair, grid-stride. Insert: find the key or claim
+// the first empty slot with a CAS on the key word, then set the tier bit with
+// an atomic OR. Evict: find the key and clear the bit; stop at an empty slot.
+// A probe is bounded by SMETRIC_MAX_PROBE slots.
+template <int OP>
+__global__ void k_update(uint64_t* __restrict__ table, uint64_t cap, int ew, int N,
+                         const uint64_t* __restrict__ keys, const int32_t* __restrict__ tiers,
+                         int64_t n, int32_t* status) {
+  const uint64_t max_probe = cap < SMETRIC_MAX_PROBE ? cap : SMETRIC_MAX_PROBE;
+  for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < n;
+       j += (int64_t)gridDim.x * blockDim.x) {
+    const uint64_t key = keys[j];
+    const int32_t tier = tiers[j];
+    if (key < 2 || tier < -1 || tier >= N) {
+      latch_error(status, SMETRIC_ERR_INVALID_ARG);
+      continue;
+    }
+    const int bit = tier < 0 ? N : tier;
+    const uint64_t m = 1ull << (bit & 63);
+    uint64_t s = home_slot(key, cap);
+    bool done = false;
+    for (uint64_t t = 0; t < max_probe; ++t) {
+      unsigned long long* e = reinterpret_cast<unsigned long long*>(table + s * ew);
+      uint64_t k = *reinterpret_cast<volatile unsigned long long*>(e);
+      if (k == kEmpty) {
+        if (OP == kEvict) { done = true; break; }
+        k = atomicCAS(e, (unsigned long long)kEmpty, (unsigned long long)key);
+        if (k == kEmpty) k = key;
+      }
+      if (k == key) {
+        if (OP == kInsert) atomicOr(e + 1 + (bit >> 6), (unsigned long long)m);
+        else atomicAnd(e + 1 + (bit >> 6), ~(unsigned long long)m);
+        done = true;
+        break;
+      }
+      if (++s == cap) s = 0;
+    }
+    if (!done && OP == kInsert) latch_error(status, SMETRIC_ERR_TABLE_FULL);
+  }
+}
+
+__global__ void k_lookup(const uint64_t* __restrict__ table, uint64_t cap, int ew, int W,
+                         const uint64_t* __restrict__ keys, int64_t n, uint64_t* __restrict__ out) {
+  const uint64_t max_probe = cap < SMETRIC_MAX_PROBE ? cap : SMETRIC_MAX_PROBE;
+  for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < n;
+       j += (int64_t)gridDim.x * blockDim.x) {
+    const uint64_t key = keys[j];
+    const uint64_t* hit = nullptr;
+    if (key >= 2) {
+      uint64_t s = home_slot(key, cap);
+      for (uint64_t t = 0; t < max_probe; ++t) {
+        const uint64_t* e = table + s * ew;
+        const uint64_t k = e[0];
+        if (k == key) { hit = e; break; }
+        if (k == kEmpty) break;
+        if (++s == cap) s = 0;
+      }
+    }
+    for (int w = 0; w < W; ++w) out[j * W + w] = hit ? hit[1 + w] : 0;
+  }
+}
+
+int grid_for(const smetric_index* idx, int64_t n, int threads) {
+  int64_t want = (n + threads - 1) / threads;
+  int64_t cap = (int64_t)idx->num_sms * 8;
+  return (int)(want < cap ? (want > 0 ? want : 1) : cap);
+}
+
+int update(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers, int64_t n,
+           smetric_stream_t stream, int op) {
+  int rc = check_device(idx);
+  if (rc) return rc;
+  if (n < 0 || (n > 0 && (!d_keys || !d_tiers))) return SMETRIC_ERR_INVALID_ARG;
+  if (n == 0) return SMETRIC_OK;
+  const int threads = 256;
+  int grid = grid_for(idx, n, threads);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (op == kInsert)
+    k_update<kInsert><<<grid, threads, 0, s>>>(idx->table, idx->cfg.capacity_slots, idx->EW,
+                                               idx->cfg.num_instances, d_keys, d_tiers, n,
+                                               idx->status);
+  else
+    k_update<kEvict><<<grid, threads, 0, s>>>(idx->table, idx->cfg.capacity_slots, idx->EW,
+                                              idx->cfg.num_instances, d_keys, d_tiers, n,
+                                              idx->status);
+  idx->launches++;
+  return cuda_status(cudaGetLastError());
+}
+
+void free_all(smetric_index* x) {
+  cudaFree(x->table);
+  cudaFree(x->status);
+  cudaFree(x->block_off);
+  cudaFree(x->digest);
+  cudaFree(x->batch_ok);
+  cudaFree(x->st_tokens);
+  cudaFree(x->st_offsets);
+  cudaFree(x->st_load);
+  cudaFree(x->st_out32);
+  cudaFree(x->st_sk);
+  for (auto& p : x->prof_pool)
+    for (auto& e : p.ev) cudaEventDestroy(e);
+  for (auto& p : x->prof_used)
+    for (auto& e : p.ev) cudaEventDestroy(e);
+}
+
+}  // namespace
+
+extern "C" {
+
+int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
+  if (!out) return SMETRIC_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg) return SMETRIC_ERR_INVALID_ARG;
+  const smetric_index_config c = *cfg;
+  if (c.num_instances < 1 || c.num_instances > SMETRIC_MAX_INSTANCES) return SMETRIC_ERR_INVALID_ARG;
+  if (c.block_size < 2 || c.block_size > 256 || (c.block_size & 1)) return SMETRIC_ERR_INVALID_ARG;
+  if (c.session_blocks < 1 || c.capacity_slots < 1) return SMETRIC_ERR_INVALID_ARG;
+  if (c.max_batch_requests < 0 || c.max_batch_requests > INT32_MAX - 1) return SMETRIC_ERR_INVALID_ARG;
+  if (c.max_batch_tokens < 0) return SMETRIC_ERR_INVALID_ARG;
+  if (c.flags & ~SMETRIC_FLAG_HOST_STAGING) return SMETRIC_ERR_INVALID_ARG;
+  const int W = (c.num_instances + 1 + 63) / 64;
+  // capacity * entry bytes must not overflow
+  if (c.capacity_slots > (UINT64_MAX / 8) / (uint64_t)entry_words(W)) return SMETRIC_ERR_INVALID_ARG;
+
+  smetric_index* x = new (std::nothrow) smetric_index();
+  if (!x) return SMETRIC_ERR_OOM;
+  x->cfg = c;
+  x->W = W;
+  x->EW = entry_words(W);
+  if (cudaGetDevice(&x->device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&x->num_sms, cudaDevAttrMultiProcessorCount, x->device) != cudaSuccess) {
+    delete x;
+    return cuda_status(cudaErrorInvalidDevice);
+  }
+  const size_t table_bytes = (size_t)c.capacity_slots * x->EW * sizeof(uint64_t);
+  const size_t max_blocks = (size_t)(c.max_batch_tokens / c.block_size);
+  const size_t R = (size_t)c.max_batch_requests;
+  bool ok = cudaMalloc(&x->table, table_bytes) == cudaSuccess &&
+            cudaMalloc(&x->status, sizeof(int32_t)) == cudaSuccess &&
+            cudaMalloc(&x->block_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
+            cudaMalloc(&x->digest, (max_blocks > 0 ? max_blocks : 1) * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&x->batch_ok, sizeof(int32_t)) == cudaSuccess;
+  if (ok && (c.flags & SMETRIC_FLAG_HOST_STAGING)) {
+    const size_t T = (size_t)(c.max_batch_tokens > 0 ? c.max_batch_tokens : 1);
+    ok = cudaMalloc(&x->st_tokens, T * sizeof(int32_t)) == cudaSuccess &&
+         cudaMalloc(&x->st_offsets, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
+         cudaMalloc(&x->st_load, (size_t)c.num_instances * sizeof(int64_t)) == cudaSuccess &&
+         cudaMalloc(&x->st_out32, (3 * R + 1) * sizeof(int32_t)) == cudaSuccess &&
+         cudaMalloc(&x->st_sk, (R + 1) * sizeof(uint64_t)) == cudaSuccess;
+  }
+  if (ok) ok = cudaMemset(x->table, 0, table_bytes) == cudaSuccess &&
+               cudaMemset(x->status, 0, sizeof(int32_t)) == cudaSuccess &&
+               cudaDeviceSynchronize() == cudaSuccess;
+  if (!ok) {
+    (void)cudaGetLastError();
+    free_all(x);
+    delete x;
+    return SMETRIC_ERR_OOM;
+  }
+  *out = x;
+  return SMETRIC_OK;
+}
+
+int smetric_index_destroy(smetric_index* idx) {
+  if (!idx) return SMETRIC_OK;
+  int dev = -1;
+  cudaGetDevice(&dev);
+  if (dev != idx->device) cudaSetDevice(idx->device);
+  cudaDeviceSynchronize();
+  free_all(idx);
+  int rc = cuda_status(cudaGetLastError());
+  if (dev >= 0 && dev != idx->device) cudaSetDevice(dev);
+  delete idx;
+  return rc;
+}
+
+int smetric_index_clear(smetric_index* idx, smetric_stream_t stream) {
+  int rc = check_device(idx);
+  if (rc) return rc;
+  return cuda_status(cudaMemsetAsync(idx->table, 0,
+                                     (size_t)idx->cfg.capacity_slots * idx->EW * sizeof(uint64_t),
+                                     reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int smetric_index_insert(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers,
+                         int64_t n, smetric_stream_t stream) {
+  return update(idx, d_keys, d_tiers, n, stream, kInsert);
+}
+
+int smetric_index_evict(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers,
+                        int64_t n, smetric_stream_t stream) {
+  return update(idx, d_keys, d_tiers, n, stream, kEvict);
+}
+
+int smetric_index_lookup(smetric_index* idx, const uint64_t* d_keys, int64_t n, uint64_t* d_masks,
+                         smetric_stream_t stream) {
+  int rc = check_device(idx);
+  if (rc) return rc;
+  if (n < 0 || (n > 0 && (!d_keys || !d_masks))) return SMETRIC_ERR_INVALID_ARG;
+  if (n == 0) return SMETRIC_OK;
+  const int threads = 256;
+  k_lookup<<<grid_for(idx, n, threads), threads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      idx->table, idx->cfg.capacity_slots, idx->EW, idx->W, d_keys, n, d_masks);
+  idx->launches++;
+  return cuda_status(cudaGetLastError());
+}
+
+int32_t smetric_index_mask_words(const smetric_index* idx) { return idx ? idx->W : 0; }
+
+int smetric_status(smetric_index* idx, smetric_stream_t stream) {
+  int rc = check_device(idx);
+  if (rc) return rc;
+  if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return cuda_status(cudaErrorUnknown);
+  int32_t h = 0;
+  if (cudaMemcpy(&h, idx->status, sizeof(h), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return cuda_status(cudaErrorUnknown);
+  if (h != 0 && cudaMemset(idx->status, 0, sizeof(int32_t)) != cudaSuccess)
+    return cuda_status(cudaErrorUnknown);
+  return h;
+}
+
+const char* smetric_strerror(int code) {
+  switch (code) {
+    case SMETRIC_OK: return "ok";
+    case SMETRIC_ERR_INVALID_ARG: return "invalid argument";
+    case SMETRIC_ERR_OOM: return "device allocation failed";
+    case SMETRIC_ERR_TABLE_FULL: return "index table full";
+    case SMETRIC_ERR_CUDA: return "CUDA runtime error";
+    case SMETRIC_ERR_OVERFLOW: return "value outside the exact integer range";
+    default: return "unknown error";
+  }
+}
+
+int64_t smetric_launch_count(const smetric_index* idx) { return idx ? idx->launches : 0; }
+
+}  // extern "C"

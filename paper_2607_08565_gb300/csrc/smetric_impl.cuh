@@ -1,0 +1,80 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <vector>
+
+#include "smetric.h"
+
+namespace smetric {
+
+constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;
+constexpr uint64_t kEmpty = 0;  // key of a never-used slot
+
+// SplitMix64 output function (Steele, Lea & Flood, OOPSLA 2014; Stafford's
+// Mix13 multipliers). Two xor-shift-multiply rounds and a final xor-shift.
+__host__ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Home slot of a key: the high 64 bits of key * capacity, uniform over
+// [0, capacity) for uniformly distributed keys (Lemire's range reduction).
+__device__ __forceinline__ uint64_t home_slot(uint64_t key, uint64_t cap) {
+  return __umul64hi(key, cap);
+}
+
+// First error wins; later ones are dropped until the host reads and clears.
+__device__ __forceinline__ void latch_error(int32_t* status, int32_t code) {
+  atomicCAS(reinterpret_cast<int*>(status), 0, code);
+}
+
+// Entry stride in 64-bit words for W mask words: key + W words, rounded up to
+// a power of two so that no entry straddles a 32-byte sector (W = 1: 16 B,
+// W = 2..3: 32 B, W = 4..7: 64 B).
+__host__ __device__ constexpr int entry_words(int W) { return W == 1 ? 2 : (W <= 3 ? 4 : 8); }
+
+// Route kernels, in launch order; names returned by smetric_profile_kernel_name.
+enum RouteKernel { kPrep = 0, kDigest = 1, kWalk = 2, kNumRouteKernels = 3 };
+
+struct ProfileSlot {
+  cudaEvent_t ev[kNumRouteKernels + 1];
+};
+
+}  // namespace smetric
+
+struct smetric_index {
+  smetric_index_config cfg;
+  int device;
+  int num_sms;
+  int W;   // tier-mask words per key
+  int EW;  // entry stride in 64-bit words
+  uint64_t* table;  // cfg.capacity_slots * EW words
+  int32_t* status;  // device: first latched error
+  // route scratch
+  int64_t* block_off;  // max_batch_requests + 1: first block of each request
+  uint64_t* digest;    // max_batch_tokens / B: per-block digests d_b
+  int32_t* batch_ok;   // device flag written by the prep kernel
+  // staging for smetric_route_batch_host
+  int32_t* st_tokens;
+  int64_t* st_offsets;
+  int64_t* st_load;
+  int32_t* st_out32;    // 3 * max_batch_requests
+  uint64_t* st_sk;      // max_batch_requests
+  int digest_occ;  // resident digest CTAs per SM (0 until the first route)
+  // observability
+  int64_t launches;
+  bool profiling;
+  std::vector<smetric::ProfileSlot> prof_pool;  // free event sets
+  std::vector<smetric::ProfileSlot> prof_used;  // recorded, not yet read
+};
+
+namespace smetric {
+// Returns SMETRIC_OK if the index is usable from the current device.
+int check_device(const smetric_index* idx);
+// Maps a CUDA error to SMETRIC_ERR_CUDA (clearing the sticky-free error state).
+int cuda_status(cudaError_t e);
+}  // namespace smetric

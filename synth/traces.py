@@ -16,6 +16,8 @@ request resending its session's cached prefix plus a small fresh suffix.
 from __future__ import annotations
 
 import math
+import os
+from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass, field
 from typing import Iterator, List, Optional, Sequence
 
@@ -23,7 +25,7 @@ import numpy as np
 
 VOCAB = 151936
 
-# Distinct stream tags so that no two generator purposes share a Philox key.
+# Distinct stream tags so that no two generator purposes share a stream.
 _TAG_PREFIX = 0x5E55_0001
 _TAG_TAIL = 0x5E55_0002
 _TAG_BATCH = 0x5E55_0003
@@ -65,26 +67,47 @@ class Batch:
         return np.diff(self.offsets)
 
 
-def _philox(*key: int) -> np.random.Generator:
-    k = np.array([key[0] & 0xFFFFFFFFFFFFFFFF,
-                  (key[1] if len(key) > 1 else 0) & 0xFFFFFFFFFFFFFFFF],
-                 dtype=np.uint64)
-    return np.random.Generator(np.random.Philox(key=k))
+def _stream(*key: int) -> np.random.Generator:
+    """An independent PCG64 stream for a tuple of non-negative integer keys."""
+    return np.random.Generator(np.random.PCG64(np.random.SeedSequence([int(k) for k in key])))
 
 
 def _tokens(rng: np.random.Generator, n: int) -> np.ndarray:
     return rng.integers(0, VOCAB, size=int(n), dtype=np.int32)
 
 
-def pack(requests: Sequence[np.ndarray]) -> tuple[np.ndarray, np.ndarray]:
-    """Concatenate per-request token arrays into (tokens, offsets)."""
+def _parallel(fn, n_items: int, threads: int = 0):
+    """Run fn(lo, hi) over [0, n_items) split into contiguous ranges on a
+    thread pool (numpy releases the GIL while generating and copying)."""
+    threads = threads or min(16, os.cpu_count() or 1)
+    if n_items == 0:
+        return
+    step = max(1, (n_items + threads * 4 - 1) // (threads * 4))
+    ranges = [(lo, min(n_items, lo + step)) for lo in range(0, n_items, step)]
+    if threads == 1 or len(ranges) == 1:
+        for lo, hi in ranges:
+            fn(lo, hi)
+        return
+    with ThreadPoolExecutor(threads) as ex:
+        for f in [ex.submit(fn, lo, hi) for lo, hi in ranges]:
+            f.result()
+
+
+def pack(requests: Sequence[np.ndarray], out: Optional[np.ndarray] = None
+         ) -> tuple[np.ndarray, np.ndarray]:
+    """Concatenate per-request token arrays into (tokens, offsets). With `out`
+    (an int32 buffer at least as long as the total), tokens is a view of it,
+    which avoids touching fresh memory for every batch."""
     lens = np.fromiter((len(r) for r in requests), dtype=np.int64, count=len(requests))
     offsets = np.zeros(len(requests) + 1, dtype=np.int64)
     np.cumsum(lens, out=offsets[1:])
-    if len(requests):
-        tokens = np.concatenate([np.asarray(r, dtype=np.int32) for r in requests])
+    total = int(offsets[-1])
+    if out is not None and len(out) >= total:
+        tokens = out[:total]
     else:
-        tokens = np.zeros(0, dtype=np.int32)
+        tokens = np.empty(total, dtype=np.int32)
+    for r, a in enumerate(requests):
+        tokens[offsets[r]:offsets[r + 1]] = a
     return tokens, offsets
 
 
@@ -244,11 +267,14 @@ class BurstTrace:
         self.cdf = np.cumsum(w) / w.sum()
 
     # -- sessions -----------------------------------------------------------
+    def _gen_prefix(self, s: int) -> np.ndarray:
+        return _tokens(_stream(_TAG_PREFIX, self.seed, int(s)), self.prefix_len[int(s)])
+
     def session_prefix(self, s: int) -> np.ndarray:
         s = int(s)
         got = self._cache.get(s)
         if got is None:
-            got = _tokens(_philox(_TAG_PREFIX ^ (self.seed << 32), s), self.prefix_len[s])
+            got = self._gen_prefix(s)
             if len(self._cache) < 16384:
                 self._cache[s] = got
         return got
@@ -262,16 +288,27 @@ class BurstTrace:
             t.append(int(self.second[s]))
         return t
 
-    def prepopulation(self, sessions: Optional[np.ndarray] = None, chunk: int = 2048):
+    def prepopulation(self, sessions: Optional[np.ndarray] = None, chunk: int = 2048,
+                      out: Optional[np.ndarray] = None):
         """Yield (session ids, tokens, offsets) chunks covering `sessions`
         (default: all). The consumer hashes each prefix and inserts its full
-        blocks into session_tiers(s)."""
+        blocks into session_tiers(s). With `out`, every chunk's tokens are a
+        view of that one buffer, valid until the next chunk."""
         if sessions is None:
             sessions = np.arange(self.n_sessions)
         sessions = np.asarray(sessions, dtype=np.int64)
         for c0 in range(0, len(sessions), chunk):
             ids = sessions[c0:c0 + chunk]
-            tokens, offsets = pack([self.session_prefix(s) for s in ids])
+            offsets = np.zeros(len(ids) + 1, dtype=np.int64)
+            np.cumsum(self.prefix_len[ids], out=offsets[1:])
+            total = int(offsets[-1])
+            tokens = out[:total] if out is not None and len(out) >= total else np.empty(total, np.int32)
+
+            def fill(lo, hi):
+                for j in range(lo, hi):
+                    tokens[offsets[j]:offsets[j + 1]] = self._gen_prefix(ids[j])
+
+            _parallel(fill, len(ids))
             yield ids, tokens, offsets
 
     def n_prefix_blocks(self, sessions: Optional[np.ndarray] = None) -> int:
@@ -281,35 +318,51 @@ class BurstTrace:
     # -- batches ------------------------------------------------------------
     def batch_sessions(self, k: int, batch_size: Optional[int] = None) -> np.ndarray:
         bs = self.batch_size if batch_size is None else batch_size
-        rng = _philox(_TAG_BATCH ^ (self.seed << 32), k)
+        rng = _stream(_TAG_BATCH, self.seed, k)
         u = rng.random(bs)
         rank = np.minimum(np.searchsorted(self.cdf, u, side="right"), self.n_sessions - 1)
         return self.perm[rank].astype(np.int64)
 
-    def batch(self, k: int, batch_size: Optional[int] = None) -> Batch:
+    def batch(self, k: int, batch_size: Optional[int] = None,
+              out: Optional[np.ndarray] = None) -> Batch:
         bs = self.batch_size if batch_size is None else batch_size
         sess = self.batch_sessions(k, bs)
-        rng = _philox(_TAG_BATCH ^ (self.seed << 32), k)
+        rng = _stream(_TAG_BATCH, self.seed, k)
         rng.random(bs)  # skip the session draws (same stream as batch_sessions)
         load = rng.integers(0, self.load_hi + 1, size=self.params.num_instances).astype(np.int64)
-        tail_rng = _philox(_TAG_TAIL ^ (self.seed << 32), k)
+        tail_rng = _stream(_TAG_TAIL, self.seed, k)
         tails = self.session_len[sess] - self.prefix_len[sess]
         fresh = _tokens(tail_rng, int(tails.sum()))
         cut = np.concatenate([[0], np.cumsum(tails)])
-        reqs = []
-        for r, s in enumerate(sess):
-            reqs.append(self.session_prefix(s))
-            reqs.append(fresh[cut[r]:cut[r + 1]])
-        tokens = np.concatenate(reqs) if reqs else np.zeros(0, dtype=np.int32)
         offsets = np.zeros(bs + 1, dtype=np.int64)
         np.cumsum(self.session_len[sess], out=offsets[1:])
+        total = int(offsets[-1])
+        tokens = out[:total] if out is not None and len(out) >= total else np.empty(total, np.int32)
+        uniq = np.unique(sess)
+        prefixes = {}
+
+        def gen(lo, hi):
+            for j in range(lo, hi):
+                prefixes[int(uniq[j])] = self.session_prefix(uniq[j])
+
+        _parallel(gen, len(uniq))
+
+        def fill(lo, hi):
+            for r in range(lo, hi):
+                a = offsets[r]
+                s = int(sess[r])
+                pl = int(self.prefix_len[s])
+                tokens[a:a + pl] = prefixes[s]
+                tokens[a + pl:offsets[r + 1]] = fresh[cut[r]:cut[r + 1]]
+
+        _parallel(fill, bs)
         return Batch(tokens=tokens, offsets=offsets, sessions=sess,
                      turns=np.ones(bs, dtype=np.int32), load=load)
 
     def filler_keys(self, n: int, k: int = 0):
         """n random 64-bit keys (>= 2) with random tiers, for padding a table
         to a target size (config 5). Returns (keys uint64, tiers int32)."""
-        rng = _philox(_TAG_FILL ^ (self.seed << 32), k)
+        rng = _stream(_TAG_FILL, self.seed, k)
         keys = rng.integers(2, np.iinfo(np.uint64).max, size=n, dtype=np.uint64, endpoint=True)
         tiers = rng.integers(-1, self.params.num_instances, size=n).astype(np.int32)
         return keys, tiers

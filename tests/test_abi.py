@@ -1,0 +1,78 @@
+"""The C-ABI library loads and exports every symbol include/smetric.h
+declares; host-side argument checks reject bad input before any CUDA call
+(no GPU needed)."""
+
+import ctypes as C
+import os
+import re
+
+import pytest
+
+import paper_2607_08565_gb300 as pkg
+from paper_2607_08565_gb300 import build_lib
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "smetric.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(smetric_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    build_lib.build()
+    return pkg.lib()
+
+
+def test_header_declares_the_binding_names():
+    assert _declared() == sorted(pkg.EXPORTED)
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in _declared():
+        assert hasattr(L, name), name
+
+
+def test_library_links_no_python_or_torch():
+    import subprocess
+    out = subprocess.run(["ldd", build_lib.LIB], capture_output=True, text=True).stdout
+    assert "torch" not in out and "python" not in out
+
+
+def test_strerror_and_kernel_names(L):
+    assert pkg.smetric_strerror(pkg.SMETRIC_ERR_TABLE_FULL) == "index table full"
+    assert pkg.smetric_strerror(12345) == "unknown error"
+    assert [pkg.smetric_profile_kernel_name(k) for k in range(3)] == ["k_prep", "k_digest", "k_walk"]
+
+
+def _create(L, **kw):
+    base = dict(num_instances=4, block_size=16, session_blocks=2, flags=0, capacity_slots=64,
+                hash_seed=0, max_batch_requests=8, max_batch_tokens=1024)
+    base.update(kw)
+    cfg = pkg.smetric_index_config(**base)
+    h = C.c_void_p()
+    return L.smetric_index_create(C.byref(cfg), C.byref(h)), h.value
+
+
+@pytest.mark.parametrize("bad", [
+    dict(num_instances=0), dict(num_instances=257), dict(block_size=7), dict(block_size=0),
+    dict(block_size=258), dict(session_blocks=0), dict(capacity_slots=0),
+    dict(max_batch_requests=-1), dict(max_batch_tokens=-5), dict(flags=8),
+    dict(capacity_slots=(1 << 64) - 1),
+])
+def test_create_rejects_bad_config_on_host(L, bad):
+    rc, h = _create(L, **bad)
+    assert rc == pkg.SMETRIC_ERR_INVALID_ARG and not h
+
+
+def test_null_handles_are_rejected(L):
+    assert L.smetric_index_create(None, None) == pkg.SMETRIC_ERR_INVALID_ARG
+    assert L.smetric_index_destroy(None) == pkg.SMETRIC_OK
+    assert L.smetric_index_insert(None, None, None, 0, None) == pkg.SMETRIC_ERR_INVALID_ARG
+    assert L.smetric_route_batch(None, None, 0, None, 0, None, pkg.smetric_weights(1, 4, 2),
+                                 None, None, None, None, None, 0, None) == pkg.SMETRIC_ERR_INVALID_ARG
+    assert L.smetric_status(None, None) == pkg.SMETRIC_ERR_INVALID_ARG
+    assert L.smetric_index_mask_words(None) == 0
+    assert L.smetric_launch_count(None) == 0

@@ -1,0 +1,163 @@
+"""The trace configurations end to end on the GPU against the CPU oracle.
+
+Configs 1-3 are multi-batch replays: after every batch each side inserts the
+routed blocks into its own index, evicts by LRU and drains its load, so the
+two replays stay identical only if every batch's outputs are bit-exact.
+Config 4 runs at full size in the launch configuration the benchmark times
+(65,536 sessions, 64 instances, B = 32, a batch of 8,192 requests): the
+oracle recomputes a sample of requests one by one, and invariants that hold
+at any size are checked on every request.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2607_08565_gb300 as pkg
+from synth import agent_trace, burst_trace
+from gpu_util import T, assert_outputs_equal, gpu_route, make_index, replay_both
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+
+
+def test_replay_config1_full():
+    st = replay_both(agent_trace("c1_tiny"))
+    assert st["batches"] == 8 and st["requests"] == 512
+    assert st["local"] > 0  # later turns hit the instance that served earlier ones
+
+
+def test_replay_config2_reduced_with_eviction():
+    tr = agent_trace("c2_medium", scale=0.1, seed=2)
+    tr.n_turns = 6
+    tr.local_cap = 3000  # small enough that LRU eviction runs every batch
+    st = replay_both(tr)
+    assert st["evicted"] > 0 and st["glob"] > 0
+
+
+def test_replay_config3_reduced_with_truncation_and_eviction():
+    tr = agent_trace("c3_long", scale=0.05, seed=3)
+    tr.n_turns = 6
+    tr.local_cap = 400
+    tr.global_cap = 3000
+    st = replay_both(tr)
+    assert st["evicted"] > 0
+
+
+def test_replay_config3_first_batches_full_size():
+    """Config 3 at full size (4096 sessions, batches of 1024): its first two
+    turn waves, both replays compared batch by batch."""
+    st = replay_both(agent_trace("c3_long"), n_batches=8)
+    assert st["requests"] == 8 * 1024
+
+
+def _populate_c4(ix, tr, chunk=4096):
+    """Hash every session prefix on the GPU and insert its blocks into the
+    global tier and the session's local tiers."""
+    p = tr.params
+    B = p.block_size
+    buf = np.empty(int(tr.prefix_len.max()) * chunk, np.int32)
+    for ids, tok, off in tr.prepopulation(chunk=chunk, out=buf):
+        hb, _ = ix.block_hashes(T(tok), T(off))
+        nb = torch.from_numpy(tr.prefix_len[ids] // B).to(hb.device)
+        total = int(nb.sum())
+        hb = hb[:total]
+        owner = torch.repeat_interleave(torch.arange(len(ids), device=hb.device), nb)
+        sess = torch.from_numpy(ids).to(hb.device)[owner]
+        ix.insert(hb, -1)
+        home = torch.from_numpy(tr.home).to(hb.device)[sess]
+        m = torch.from_numpy(tr.in_home).to(hb.device)[sess]
+        ix.insert(hb[m].contiguous(), home[m].contiguous())
+        sec = torch.from_numpy(tr.second).to(hb.device)[sess]
+        m2 = torch.from_numpy(tr.in_second).to(hb.device)[sess]
+        ix.insert(hb[m2].contiguous(), sec[m2].contiguous())
+    ix.check()
+
+
+def test_config4_full_size_sampled():
+    tr = burst_trace()
+    p = tr.params
+    N, B = p.num_instances, p.block_size
+    nkeys = tr.n_prefix_blocks()
+    bt = tr.batch(0)
+    ix = make_index(N, B, p.session_blocks, cap=int(nkeys / 0.7) + 1,
+                    max_req=bt.n_requests, max_tok=bt.n_tokens)
+    _populate_c4(ix, tr)
+    w = (p.w_load, p.w_miss, p.w_glob)
+    g = gpu_route(ix, bt.tokens, bt.offsets, bt.load, w, want_hashes=False)
+
+    # invariants on every request
+    lens = bt.lengths()
+    assert np.all((g["instance"] >= 0) & (g["instance"] < N))
+    assert np.all(g["local_hit"] + g["global_hit"] <= (lens // B) * B)
+    assert np.all(g["local_hit"] % B == 0) and np.all(g["global_hit"] % B == 0)
+    # every request of a session carries the session's cached prefix, which
+    # the global tier holds in full
+    reach = (g["local_hit"] + g["global_hit"]) // B
+    assert np.all(reach == tr.prefix_len[bt.sessions] // B)
+    # the session key is a function of the session (identical leading blocks)
+    keys = {}
+    for s, k in zip(bt.sessions.tolist(), g["session_key"].tolist()):
+        assert keys.setdefault(s, k) == k
+    assert len(set(keys.values())) == len(keys)
+
+    # the oracle on a sample, one request at a time, with an index holding
+    # the sampled sessions' prefixes
+    rng = np.random.default_rng(0)
+    sample = np.sort(rng.choice(bt.n_requests, size=96, replace=False))
+    sessions = np.unique(bt.sessions[sample])
+    ox = oracle.OracleIndex(N)
+    for s in sessions.tolist():
+        h = oracle.block_hashes(tr.session_prefix(s), B, p.hash_seed)
+        for t in tr.session_tiers(s):
+            ox.insert(h, t)
+    for r in sample.tolist():
+        a, b = bt.offsets[r], bt.offsets[r + 1]
+        o = ox.route_batch(B, p.session_blocks, p.hash_seed, bt.tokens[a:b],
+                           np.array([0, b - a], np.int64), bt.load, *w)
+        one = {f: g[f][r:r + 1] for f in ("instance", "local_hit", "global_hit", "session_key")}
+        assert_outputs_equal(one, o, fields=("instance", "local_hit", "global_hit", "session_key"),
+                             ctx=f"config 4 request {r}")
+    ix.close()
+
+
+@pytest.mark.parametrize("N,B", [(8, 64), (256, 16)])
+def test_config5_corner_points_sampled(N, B):
+    """Two corners of the config-5 sweep (fewest instances with the largest
+    blocks; most instances with the smallest), with filler keys packing the
+    table, at reduced session count."""
+    tr = burst_trace("c5_sweep", num_instances=N, block_size=B, n_sessions=2048, batch_size=2048)
+    p = tr.params
+    nkeys = tr.n_prefix_blocks()
+    n_fill = nkeys // 2
+    bt = tr.batch(3)
+    ix = make_index(N, B, 4, cap=int((nkeys + n_fill) / 0.7) + 1, max_req=bt.n_requests,
+                    max_tok=bt.n_tokens)
+    _populate_c4(ix, tr, chunk=1024)
+    fk, ft = tr.filler_keys(n_fill)
+    ix.insert(T(fk), T(ft))
+    ix.check()
+    g = gpu_route(ix, bt.tokens, bt.offsets, bt.load, (1, 4, 2), want_hashes=False)
+    rng = np.random.default_rng(1)
+    sample = np.sort(rng.choice(bt.n_requests, size=48, replace=False))
+    ox = oracle.OracleIndex(N)
+    for s in np.unique(bt.sessions[sample]).tolist():
+        h = oracle.block_hashes(tr.session_prefix(s), B)
+        for t in tr.session_tiers(s):
+            ox.insert(h, t)
+    ox.insert(fk, ft)
+    tok, off = bt.tokens, bt.offsets
+    sub = [tok[off[r]:off[r + 1]] for r in sample]
+    from synth.traces import pack
+    st, so = pack(sub)
+    o = ox.route_batch(B, 4, 0, st, so, bt.load, 1, 4, 2)
+    sel = {f: g[f][sample] for f in ("instance", "local_hit", "global_hit", "session_key")}
+    assert_outputs_equal(sel, o, fields=("instance", "local_hit", "global_hit", "session_key"))
+    ix.close()
