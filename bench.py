@@ -49,6 +49,9 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sessions", type=int, default=65536,
+                    help="sessions of the burst workload (smaller values: profiling cases)")
+    ap.add_argument("--batch", type=int, default=8192, help="requests per batch")
     return ap.parse_args()
 
 
@@ -148,9 +151,18 @@ def ncu_traffic(kernel: str):
 # workload
 # ---------------------------------------------------------------------------
 
-def c4_trace():
+def c4_trace(args=None):
     from synth import burst_trace
-    return burst_trace()
+    if args is None:
+        return burst_trace()
+    return burst_trace(n_sessions=args.sessions, batch_size=args.batch)
+
+
+def workload_name(args):
+    if args.sessions == 65536 and args.batch == 8192:
+        return WORKLOAD
+    return (f"c4_burst generator reduced to {args.sessions} sessions and batches of "
+            f"{args.batch} requests (a profiling case, not the benchmark workload)")
 
 
 def populate_index(ix, tr, device, chunk=4096):
@@ -160,7 +172,7 @@ def populate_index(ix, tr, device, chunk=4096):
     for ids, tok, off in tr.prepopulation(chunk=chunk, out=buf):
         hb, _ = ix.block_hashes(torch.from_numpy(tok).to(device), torch.from_numpy(off).to(device))
         nb = torch.from_numpy(tr.prefix_len[ids] // B).to(device)
-        hb = hb[:int(nb.sum())]
+        hb = hb[:int(nb.sum())].view(torch.int64)  # CUDA mask indexing has no uint64 kernels
         owner = torch.repeat_interleave(torch.arange(len(ids), device=device), nb)
         sess = torch.from_numpy(ids).to(device)[owner]
         ix.insert(hb, -1)
@@ -172,17 +184,23 @@ def populate_index(ix, tr, device, chunk=4096):
 
 
 def algorithmic_bytes(lens, local_hit, global_hit, B, W):
-    """Per-kernel algorithmic bytes of one route call: digest reads 4 B per
-    hashed token; walk reads one index entry (key + W
-    mask words) per probed block, P_r = min(n_r, reach_r + 1), plus offsets
-    and outputs; prep reads offsets and loads."""
+    """Per-kernel bytes of one route call. k_digest: 4 B per hashed token (the
+    method must read every token of every full block). k_probe: one index
+    entry (key + W mask words) per probed block, P_r = min(n_r, reach_r + 1)
+    (the method's probes; the kernel probes every block). k_chain, k_walk:
+    their reads and writes of this kernel split's intermediates (digests,
+    hashes, masks), which the method itself does not need, plus offsets and
+    outputs. k_prep: offsets and loads. path: the method's bytes per request,
+    4 L_r + P_r (8 + 8W) + 8 + 20."""
     nb = lens // B
     reach = (local_hit.astype(np.int64) + global_hit) // B
     probes = np.minimum(nb, reach + 1)
     n = len(lens)
     return {
         "k_digest": int(4 * B * nb.sum()),
-        "k_walk": int(probes.sum() * (8 + 8 * W) + 16 * n + 20 * n),
+        "k_chain": int(16 * nb.sum() + 24 * n),
+        "k_probe": int(probes.sum() * (8 + 8 * W)),
+        "k_walk": int(8 * W * probes.sum() + 28 * n),
         "k_prep": int(16 * n),
         "path": int(4 * lens.sum() + probes.sum() * (8 + 8 * W) + 8 * (n + 1) + 20 * n),
     }
@@ -231,7 +249,7 @@ def run_reference(args, rank, world, dist):
         return
     import oracle
     oracle.build()
-    tr = c4_trace()
+    tr = c4_trace(args)
     threads = os.cpu_count() or 1
     batches = [tr.batch(k) for k in range(N_DISTINCT_BATCHES)]
     ox = oracle_index_for(tr, batches)
@@ -246,14 +264,15 @@ def run_reference(args, rank, world, dist):
         toks += int(bt.offsets[m])
     total = sum(times)
     rps = args.steps * m / total
-    sample = (f"first {m} of the 8192 requests of a config-4 batch per step (4 batches rotated), "
+    sample = (f"first {m} of the {batches[0].n_requests} requests of a config-4 batch per step "
+              f"(4 batches rotated), "
               f"oracle index holding those batches' sessions, {threads} threads")
     line = {
         "impl": "reference", "metric": METRIC, "value": rps, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u64",
         "data": "synthetic", "tokens_per_s": toks / total,
-        "config": {"workload": WORKLOAD, "l2": "host run"},
+        "config": {"workload": workload_name(args), "l2": "host run"},
         "cpu_baseline": {"value": rps, "unit": UNIT, "cores": threads, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": rps, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -276,19 +295,20 @@ def run_ours(args, rank, world, local, dist):
         dist.barrier()
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
-    tr = c4_trace()
+    tr = c4_trace(args)
     p = tr.params
     N, B = p.num_instances, p.block_size
 
     # this rank's batches: ids rank, rank + world, ... (distinct across ranks)
     ids = [rank + world * i for i in range(N_DISTINCT_BATCHES)]
     host = [tr.batch(k) for k in ids]
-    max_tok = max(b.n_tokens for b in host)
     nkeys = tr.n_prefix_blocks()
+    chunk = 4096  # sessions hashed per pre-population call
+    max_tok = max(max(b.n_tokens for b in host), chunk * int(tr.prefix_len.max()))
     ix = pkg.SMetricIndex(N, B, p.session_blocks, capacity_slots=int(nkeys / 0.7) + 1,
-                          max_batch_requests=tr.batch_size, max_batch_tokens=max_tok,
+                          max_batch_requests=max(tr.batch_size, chunk), max_batch_tokens=max_tok,
                           hash_seed=p.hash_seed, host_staging=True)
-    populate_index(ix, tr, device)
+    populate_index(ix, tr, device, chunk)
     dev_b = []
     for b in host:
         dev_b.append(dict(tok=torch.from_numpy(b.tokens).to(device),
@@ -421,7 +441,7 @@ def run_ours(args, rank, world, local, dist):
         ox = oracle_index_for(tr, host[:1])
         m, dt = oracle_calibrate(tr, ox, host[0], args.cpu_seconds, threads)
         cpu = {"value": m / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
-               "sample": f"first {m} of the 8192 requests of config-4 batch {ids[0]} "
+               "sample": f"first {m} of the {host[0].n_requests} requests of config-4 batch {ids[0]} "
                          f"({dt:.1f} s on {threads} threads), oracle index holding that batch's "
                          f"sessions", "tokens_per_s": float(host[0].offsets[m]) / dt}
 
@@ -431,7 +451,7 @@ def run_ours(args, rank, world, local, dist):
             "warmup": args.warmup, "ms_per_step": path_ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
             "tokens_per_s": tokens_per_s,
-            "config": {"workload": WORKLOAD, "batch": int(reqs_per_step),
+            "config": {"workload": workload_name(args), "batch": int(reqs_per_step),
                        "num_instances": N, "block_size": B, "index_keys": nkeys,
                        "l2": f"inputs larger than L2: {N_DISTINCT_BATCHES} distinct batches of "
                              f"{toks_per_step * 4 / 1e6:.0f} MB rotated"},

@@ -98,9 +98,11 @@ typedef struct {
 } smetric_weights;
 
 /* Create an empty index and its route scratch on the current device.
- * The table holds capacity_slots entries of 16, 32 or 64 bytes (key plus
- * ceil((N+1)/64) tier-mask words, padded to a power of two); the scratch
- * holds max_batch_tokens/B + max_batch_requests + 1 64-bit words.
+ * The table holds capacity_slots (rounded up to a multiple of 16) entries of
+ * 16, 32 or 64 bytes (key plus ceil((N+1)/64) tier-mask words, padded to a
+ * power of two) and one tag byte per slot; the scratch holds
+ * (2 + W) * (max_batch_tokens/B) + max_batch_requests + 1 64-bit words,
+ * W = ceil((N+1)/64).
  * Returns SMETRIC_ERR_INVALID_ARG for an out-of-range field and
  * SMETRIC_ERR_OOM when a device allocation fails; *out is NULL then. */
 int smetric_index_create(const smetric_index_config* cfg, smetric_index** out);

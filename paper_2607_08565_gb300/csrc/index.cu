@@ -1,13 +1,16 @@
-// Two-tier KV$ index on the GPU: one open-addressing table, key -> tier mask.
+// Two-tier KV$ index on the GPU: one bucketed hash table, key -> tier mask.
 //
 // The paper's KV$ store has a local tier per serving instance and a global
 // tier shared by the cluster (Section 2, Figures 1-2); the router needs, per
 // block hash, which tiers hold the block. One table serves all tiers: an
 // entry is the 64-bit block hash followed by W = ceil((N+1)/64) mask words,
-// bit i < N = local tier of instance i, bit N = global tier. Linear probing
-// from home_slot(key); key 0 marks a never-used slot. Keys are never removed:
-// an evicted key keeps its slot with a cleared bit, so lookups never see
-// tombstones and concurrent inserts cannot create duplicates.
+// bit i < N = local tier of instance i, bit N = global tier. Slots are grouped
+// in buckets of kBucket; a one-byte tag per slot (0 = empty, else 0x80 | low
+// 7 key bits) lives in a separate tag array so that a lookup reads one
+// 16-byte tag group and then only the entry whose tag matches. Inserts take
+// the first empty slot in bucket order from the key's home bucket. Keys are
+// never removed: an evicted key keeps its slot with a cleared tier bit, so
+// lookups never meet tombstones and concurrent inserts cannot duplicate a key.
 
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -40,15 +43,88 @@ namespace {
 
 enum Op { kInsert = 0, kEvict = 1 };
 
-// One thread per (key, tier) pair, grid-stride. Insert: find the key or claim
-// the first empty slot with a CAS on the key word, then set the tier bit with
-// an atomic OR. Evict: find the key and clear the bit; stop at an empty slot.
-// A probe is bounded by SMETRIC_MAX_PROBE slots.
+__device__ __forceinline__ uint64_t max_buckets(uint64_t n_buckets) {
+  const uint64_t m = SMETRIC_MAX_PROBE / kBucket;
+  return n_buckets < m ? n_buckets : m;
+}
+
+__device__ __forceinline__ uint4 load_tags_volatile(const uint8_t* p) {
+  const volatile uint32_t* q = reinterpret_cast<const volatile uint32_t*>(p);
+  return make_uint4(q[0], q[1], q[2], q[3]);
+}
+
+// Slot of `key`, or -1 when absent (at most SMETRIC_MAX_PROBE slots probed).
+// Used by kernels that do not run concurrently with inserts.
+__device__ __forceinline__ int64_t find_slot(const uint8_t* __restrict__ tags,
+                                             const uint64_t* __restrict__ table, int ew,
+                                             uint64_t n_buckets, uint64_t key) {
+  const uint32_t tg = key_tag(key);
+  uint64_t b = home_bucket(key, n_buckets);
+  const uint64_t mb = max_buckets(n_buckets);
+  for (uint64_t t = 0; t < mb; ++t) {
+    const uint4 tv = *reinterpret_cast<const uint4*>(tags + b * kBucket);
+    uint32_t cand = tag_match(tv, tg);
+    while (cand) {
+      const int sl = __ffs(cand) - 1;
+      cand &= cand - 1;
+      const uint64_t slot = b * kBucket + sl;
+      if (table[slot * ew] == key) return (int64_t)slot;
+    }
+    if (tag_match(tv, 0)) return -1;  // the bucket still has an empty slot
+    if (++b == n_buckets) b = 0;
+  }
+  return -1;
+}
+
+// Insert: set tier bit (word, m) of `key`, claiming the first empty slot in
+// bucket order if the key is new. A slot is claimed by a CAS on its key word
+// and published by setting its tag after a fence; a concurrent inserter of the
+// same key that meets the claimed-but-untagged slot sees its key in the failed
+// CAS and uses that slot. Returns false when no slot was found.
+__device__ bool insert_key(uint8_t* tags, uint64_t* table, int ew, uint64_t n_buckets,
+                           uint64_t key, int word, unsigned long long m) {
+  const uint32_t tg = key_tag(key);
+  uint64_t b = home_bucket(key, n_buckets);
+  const uint64_t mb = max_buckets(n_buckets);
+  for (uint64_t t = 0; t < mb; ++t) {
+    const uint4 tv = load_tags_volatile(tags + b * kBucket);
+    uint32_t cand = tag_match(tv, tg);
+    while (cand) {
+      const int sl = __ffs(cand) - 1;
+      cand &= cand - 1;
+      unsigned long long* e = reinterpret_cast<unsigned long long*>(table + (b * kBucket + sl) * ew);
+      if (*reinterpret_cast<volatile unsigned long long*>(e) == key) {
+        atomicOr(e + 1 + word, m);
+        return true;
+      }
+    }
+    uint32_t empty = tag_match(tv, 0);
+    while (empty) {
+      const int sl = __ffs(empty) - 1;
+      empty &= empty - 1;
+      unsigned long long* e = reinterpret_cast<unsigned long long*>(table + (b * kBucket + sl) * ew);
+      const unsigned long long old = atomicCAS(e, (unsigned long long)kEmpty, (unsigned long long)key);
+      if (old == kEmpty) {
+        __threadfence();
+        atomicOr(reinterpret_cast<unsigned int*>(tags + b * kBucket) + (sl >> 2), tg << (8 * (sl & 3)));
+        atomicOr(e + 1 + word, m);
+        return true;
+      }
+      if (old == key) {
+        atomicOr(e + 1 + word, m);
+        return true;
+      }
+    }
+    if (++b == n_buckets) b = 0;
+  }
+  return false;
+}
+
+// One thread per (key, tier) pair, grid-stride.
 template <int OP>
-__global__ void k_update(uint64_t* __restrict__ table, uint64_t cap, int ew, int N,
-                         const uint64_t* __restrict__ keys, const int32_t* __restrict__ tiers,
-                         int64_t n, int32_t* status) {
-  const uint64_t max_probe = cap < SMETRIC_MAX_PROBE ? cap : SMETRIC_MAX_PROBE;
+__global__ void k_update(uint8_t* __restrict__ tags, uint64_t* __restrict__ table, uint64_t n_buckets,
+                         int ew, int N, const uint64_t* __restrict__ keys,
+                         const int32_t* __restrict__ tiers, int64_t n, int32_t* status) {
   for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < n;
        j += (int64_t)gridDim.x * blockDim.x) {
     const uint64_t key = keys[j];
@@ -58,47 +134,26 @@ __global__ void k_update(uint64_t* __restrict__ table, uint64_t cap, int ew, int
       continue;
     }
     const int bit = tier < 0 ? N : tier;
-    const uint64_t m = 1ull << (bit & 63);
-    uint64_t s = home_slot(key, cap);
-    bool done = false;
-    for (uint64_t t = 0; t < max_probe; ++t) {
-      unsigned long long* e = reinterpret_cast<unsigned long long*>(table + s * ew);
-      uint64_t k = *reinterpret_cast<volatile unsigned long long*>(e);
-      if (k == kEmpty) {
-        if (OP == kEvict) { done = true; break; }
-        k = atomicCAS(e, (unsigned long long)kEmpty, (unsigned long long)key);
-        if (k == kEmpty) k = key;
-      }
-      if (k == key) {
-        if (OP == kInsert) atomicOr(e + 1 + (bit >> 6), (unsigned long long)m);
-        else atomicAnd(e + 1 + (bit >> 6), ~(unsigned long long)m);
-        done = true;
-        break;
-      }
-      if (++s == cap) s = 0;
+    const unsigned long long m = 1ull << (bit & 63);
+    if (OP == kInsert) {
+      if (!insert_key(tags, table, ew, n_buckets, key, bit >> 6, m))
+        latch_error(status, SMETRIC_ERR_TABLE_FULL);
+    } else {
+      const int64_t slot = find_slot(tags, table, ew, n_buckets, key);
+      if (slot >= 0)
+        atomicAnd(reinterpret_cast<unsigned long long*>(table + slot * ew) + 1 + (bit >> 6), ~m);
     }
-    if (!done && OP == kInsert) latch_error(status, SMETRIC_ERR_TABLE_FULL);
   }
 }
 
-__global__ void k_lookup(const uint64_t* __restrict__ table, uint64_t cap, int ew, int W,
-                         const uint64_t* __restrict__ keys, int64_t n, uint64_t* __restrict__ out) {
-  const uint64_t max_probe = cap < SMETRIC_MAX_PROBE ? cap : SMETRIC_MAX_PROBE;
+__global__ void k_lookup(const uint8_t* __restrict__ tags, const uint64_t* __restrict__ table,
+                         uint64_t n_buckets, int ew, int W, const uint64_t* __restrict__ keys,
+                         int64_t n, uint64_t* __restrict__ out) {
   for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < n;
        j += (int64_t)gridDim.x * blockDim.x) {
     const uint64_t key = keys[j];
-    const uint64_t* hit = nullptr;
-    if (key >= 2) {
-      uint64_t s = home_slot(key, cap);
-      for (uint64_t t = 0; t < max_probe; ++t) {
-        const uint64_t* e = table + s * ew;
-        const uint64_t k = e[0];
-        if (k == key) { hit = e; break; }
-        if (k == kEmpty) break;
-        if (++s == cap) s = 0;
-      }
-    }
-    for (int w = 0; w < W; ++w) out[j * W + w] = hit ? hit[1 + w] : 0;
+    const int64_t slot = key >= 2 ? find_slot(tags, table, ew, n_buckets, key) : -1;
+    for (int w = 0; w < W; ++w) out[j * W + w] = slot >= 0 ? table[slot * ew + 1 + w] : 0;
   }
 }
 
@@ -118,11 +173,11 @@ int update(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers, i
   int grid = grid_for(idx, n, threads);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (op == kInsert)
-    k_update<kInsert><<<grid, threads, 0, s>>>(idx->table, idx->cfg.capacity_slots, idx->EW,
+    k_update<kInsert><<<grid, threads, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->EW,
                                                idx->cfg.num_instances, d_keys, d_tiers, n,
                                                idx->status);
   else
-    k_update<kEvict><<<grid, threads, 0, s>>>(idx->table, idx->cfg.capacity_slots, idx->EW,
+    k_update<kEvict><<<grid, threads, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->EW,
                                               idx->cfg.num_instances, d_keys, d_tiers, n,
                                               idx->status);
   idx->launches++;
@@ -131,9 +186,12 @@ int update(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers, i
 
 void free_all(smetric_index* x) {
   cudaFree(x->table);
+  cudaFree(x->tags);
   cudaFree(x->status);
   cudaFree(x->block_off);
   cudaFree(x->digest);
+  cudaFree(x->hashes);
+  cudaFree(x->masks);
   cudaFree(x->batch_ok);
   cudaFree(x->st_tokens);
   cudaFree(x->st_offsets);
@@ -162,26 +220,31 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
   if (c.max_batch_tokens < 0) return SMETRIC_ERR_INVALID_ARG;
   if (c.flags & ~SMETRIC_FLAG_HOST_STAGING) return SMETRIC_ERR_INVALID_ARG;
   const int W = (c.num_instances + 1 + 63) / 64;
-  // capacity * entry bytes must not overflow
-  if (c.capacity_slots > (UINT64_MAX / 8) / (uint64_t)entry_words(W)) return SMETRIC_ERR_INVALID_ARG;
+  // slots (rounded up to whole buckets) * entry bytes must not overflow
+  if (c.capacity_slots > (UINT64_MAX / 16) / (uint64_t)entry_words(W)) return SMETRIC_ERR_INVALID_ARG;
 
   smetric_index* x = new (std::nothrow) smetric_index();
   if (!x) return SMETRIC_ERR_OOM;
   x->cfg = c;
   x->W = W;
   x->EW = entry_words(W);
+  x->n_buckets = (c.capacity_slots + kBucket - 1) / kBucket;
   if (cudaGetDevice(&x->device) != cudaSuccess ||
       cudaDeviceGetAttribute(&x->num_sms, cudaDevAttrMultiProcessorCount, x->device) != cudaSuccess) {
     delete x;
     return cuda_status(cudaErrorInvalidDevice);
   }
-  const size_t table_bytes = (size_t)c.capacity_slots * x->EW * sizeof(uint64_t);
+  const size_t slots = (size_t)x->n_buckets * kBucket;
+  const size_t table_bytes = slots * x->EW * sizeof(uint64_t);
   const size_t max_blocks = (size_t)(c.max_batch_tokens / c.block_size);
   const size_t R = (size_t)c.max_batch_requests;
   bool ok = cudaMalloc(&x->table, table_bytes) == cudaSuccess &&
+            cudaMalloc(&x->tags, slots) == cudaSuccess &&
             cudaMalloc(&x->status, sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->block_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
             cudaMalloc(&x->digest, (max_blocks > 0 ? max_blocks : 1) * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&x->hashes, (max_blocks > 0 ? max_blocks : 1) * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&x->masks, (max_blocks > 0 ? max_blocks : 1) * W * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->batch_ok, sizeof(int32_t)) == cudaSuccess;
   if (ok && (c.flags & SMETRIC_FLAG_HOST_STAGING)) {
     const size_t T = (size_t)(c.max_batch_tokens > 0 ? c.max_batch_tokens : 1);
@@ -192,6 +255,7 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
          cudaMalloc(&x->st_sk, (R + 1) * sizeof(uint64_t)) == cudaSuccess;
   }
   if (ok) ok = cudaMemset(x->table, 0, table_bytes) == cudaSuccess &&
+               cudaMemset(x->tags, 0, slots) == cudaSuccess &&
                cudaMemset(x->status, 0, sizeof(int32_t)) == cudaSuccess &&
                cudaDeviceSynchronize() == cudaSuccess;
   if (!ok) {
@@ -220,9 +284,11 @@ int smetric_index_destroy(smetric_index* idx) {
 int smetric_index_clear(smetric_index* idx, smetric_stream_t stream) {
   int rc = check_device(idx);
   if (rc) return rc;
-  return cuda_status(cudaMemsetAsync(idx->table, 0,
-                                     (size_t)idx->cfg.capacity_slots * idx->EW * sizeof(uint64_t),
-                                     reinterpret_cast<cudaStream_t>(stream)));
+  const size_t slots = (size_t)idx->n_buckets * kBucket;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(idx->table, 0, slots * idx->EW * sizeof(uint64_t), s) != cudaSuccess)
+    return cuda_status(cudaErrorUnknown);
+  return cuda_status(cudaMemsetAsync(idx->tags, 0, slots, s));
 }
 
 int smetric_index_insert(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers,
@@ -243,7 +309,7 @@ int smetric_index_lookup(smetric_index* idx, const uint64_t* d_keys, int64_t n, 
   if (n == 0) return SMETRIC_OK;
   const int threads = 256;
   k_lookup<<<grid_for(idx, n, threads), threads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-      idx->table, idx->cfg.capacity_slots, idx->EW, idx->W, d_keys, n, d_masks);
+      idx->tags, idx->table, idx->n_buckets, idx->EW, idx->W, d_keys, n, d_masks);
   idx->launches++;
   return cuda_status(cudaGetLastError());
 }

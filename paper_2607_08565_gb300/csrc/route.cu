@@ -2,20 +2,25 @@
 // match, integer cost and argmin (Figure 6 and Figure 10 of the paper, with
 // every request of the batch routed against one snapshot of index and load).
 //
-// Three kernels per batch, in stream order:
+// Five kernels per batch, in stream order:
 //   k_prep    one CTA: validates offsets and loads, exclusive-scans the
 //             per-request full-block counts into block_off.
-//   k_digest  HBM-bound: one warp per 32 consecutive blocks of the flattened
-//             batch. The warp stages the tokens of its 32 blocks into shared
-//             memory with coalesced 8-byte cp.async copies (evict-first in
-//             L2), laid out with one pad word per row so that lane j reading
-//             word k of block j hits a distinct bank; then lane j folds its
-//             block's B/2 words into the digest d_b. Two stages per warp let
-//             the next chunk's copy overlap this chunk's arithmetic.
-//   k_walk    one thread per request: the serial chain h_b over the digests,
-//             home-slot probes issued eight blocks at a time, the running
-//             AND of local-tier masks and the global-tier run, then the cost
-//             of every instance and the lowest-id argmin.
+//   k_digest  HBM-bound: each warp owns a contiguous range of 32-block chunks
+//             of the flattened batch. A chunk whose blocks belong to one
+//             request is one contiguous span: the warp loads it with
+//             coalesced 16-byte loads into registers one chunk ahead and
+//             scatters it into shared memory, one row per block padded to a
+//             16-byte multiple so that lane j reading word k of block j hits
+//             a distinct bank pair; lane j folds block j's B/2 words into d_b.
+//   k_chain   one thread per request: the serial chain h_b over its digests
+//             (sixteen digests prefetched ahead) and the session key.
+//   k_probe   one thread per block: the tier masks of h_b from the index
+//             (16 tags of the home bucket, then the matching entry).
+//   k_walk    one warp per request, lanes = 32 consecutive blocks: an AND-scan
+//             of the local-tier masks across lanes, the block where each
+//             instance's run ends located by ballot, the global-tier run;
+//             then lanes = instances for the cost and a shuffle argmin with
+//             ties to the lowest id.
 
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -30,12 +35,11 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kChunk = 32;        // blocks per digest task (one per lane)
-constexpr int kDigestWarps = 8;   // most warps per digest CTA (fewer for large B)
-constexpr size_t kDigestSmem = 200 * 1024;  // shared-memory budget of one digest CTA
+constexpr int kDigestWarps = 8;   // most warps per digest CTA
 constexpr int kStages = 2;        // shared-memory stages per warp
-constexpr int kSpanBlocks = 36;   // staged span: 32 blocks + room for request tails
-constexpr int kWalkThreads = 64;  // requests per walk CTA
-constexpr int kGroup = 8;         // probes issued together per request
+constexpr int kChainThreads = 128;
+constexpr int kChainAhead = 16;   // digests prefetched per request
+constexpr int kMatchWarps = 8;    // warps per walk CTA
 
 // ---------------------------------------------------------------------------
 // prep
@@ -103,10 +107,10 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
 // digest
 // ---------------------------------------------------------------------------
 
-// Largest r in [0, n) with block_off[r] <= f, given block_off[0] <= f < block_off[n].
-__device__ __forceinline__ int32_t find_request(const int64_t* __restrict__ block_off, int32_t n,
-                                                int64_t f) {
-  int32_t lo = 0, hi = n;
+// Largest r in [lo, n) with block_off[r] <= f, given block_off[lo] <= f < block_off[n].
+__device__ __forceinline__ int32_t find_request(const int64_t* __restrict__ block_off, int32_t lo,
+                                                int32_t n, int64_t f) {
+  int32_t hi = n;
   while (hi - lo > 1) {
     const int32_t mid = (lo + hi) >> 1;
     if (__ldg(block_off + mid) <= f) lo = mid; else hi = mid;
@@ -114,80 +118,24 @@ __device__ __forceinline__ int32_t find_request(const int64_t* __restrict__ bloc
   return lo;
 }
 
-struct Chunk {
-  int64_t tok0;  // first token of this lane's block
-  int64_t u_lo;  // first staged 64-bit word (warp-uniform)
-  int32_t nq;    // staged words (warp-uniform)
-  bool valid;    // this lane has a block
-  bool fast;     // the chunk is staged through shared memory (warp-uniform)
-};
-
-__device__ __forceinline__ void locate(Chunk& ch, int64_t c, int64_t total,
-                                       const int64_t* __restrict__ off,
-                                       const int64_t* __restrict__ block_off, int32_t n, int B,
-                                       int lane, int q_max) {
-  const int64_t f = c * kChunk + lane;
-  ch.valid = f < total;
-  int64_t t0 = 0;
-  if (ch.valid) {
-    const int32_t r = find_request(block_off, n, f);
-    t0 = __ldg(off + r) + (f - __ldg(block_off + r)) * B;
-  }
-  ch.tok0 = t0;
-  const unsigned vm = __ballot_sync(kFull, ch.valid);
-  const int last = 31 - __clz(vm);
-  const int64_t lo = __shfl_sync(kFull, t0, 0);
-  const int64_t hi = __shfl_sync(kFull, t0, last) + B;  // end of the last block
-  ch.u_lo = lo >> 1;
-  const int64_t u_hi = (hi + 1) >> 1;  // one extra word when blocks start on odd tokens
-  const int64_t nq = u_hi - ch.u_lo;
-  ch.fast = nq <= q_max;
-  ch.nq = ch.fast ? (int32_t)nq : 0;
-}
-
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
-__device__ __forceinline__ void stage_copy(const Chunk& ch, const int32_t* __restrict__ tokens,
-                                           int64_t n_tokens, uint64_t* stage, int rowshift,
-                                           int lane, uint64_t policy) {
-  const uint32_t base = smem_u32(stage);
-  for (int q = lane; q < ch.nq; q += 32) {
-    const int64_t t = 2 * (ch.u_lo + q);  // first token of this word
-    const uint32_t dst = base + 8u * (uint32_t)(q + (q >> rowshift));
-    const int32_t* src = tokens + t;
-    if (t + 1 < n_tokens) {
-      asm volatile("cp.async.ca.shared.global.L2::cache_hint [%0], [%1], 8, %2;\n" ::"r"(dst),
-                   "l"(src), "l"(policy));
-    } else if (t < n_tokens) {
-      asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(dst), "l"(src));
-    }
-  }
-}
-
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
-
-// Digest of one block from the staged words. HB = B/2 when known at compile
-// time (0: runtime hb).
+// Digest of one block from its shared-memory row. `row` points at the 8-byte
+// word holding the block's first token (its low half when the block starts on
+// an even token, its high half when on an odd one).
 template <int HB>
-__device__ __forceinline__ uint64_t digest_staged(const uint64_t* stage, int q0, bool odd, int hb,
-                                                  int rowshift, uint64_t d) {
+__device__ __forceinline__ uint64_t digest_row(const uint64_t* row, bool odd, int hb, uint64_t d) {
   const int n = HB > 0 ? HB : hb;
   if (!odd) {
-#pragma unroll 8
-    for (int k = 0; k < n; ++k) {
-      const int q = q0 + k;
-      d = mix64(d ^ stage[q + (q >> rowshift)]);
-    }
+#pragma unroll 16
+    for (int k = 0; k < n; ++k) d = mix64(d ^ row[k]);
   } else {
-    uint64_t x = stage[q0 + (q0 >> rowshift)];
-#pragma unroll 8
+    uint64_t x = row[0];
+#pragma unroll 16
     for (int k = 0; k < n; ++k) {
-      const int q = q0 + k + 1;
-      const uint64_t y = stage[q + (q >> rowshift)];
+      const uint64_t y = row[k + 1];
       d = mix64(d ^ ((x >> 32) | (y << 32)));
       x = y;
     }
@@ -195,295 +143,401 @@ __device__ __forceinline__ uint64_t digest_staged(const uint64_t* stage, int q0,
   return d;
 }
 
-__device__ __forceinline__ uint64_t digest_global(const int32_t* __restrict__ tokens, int64_t t0,
-                                                  int hb, uint64_t d) {
-  for (int k = 0; k < hb; ++k) {
-    const uint64_t lo = (uint32_t)__ldg(tokens + t0 + 2 * k);
-    const uint64_t hi = (uint32_t)__ldg(tokens + t0 + 2 * k + 1);
-    d = mix64(d ^ (lo | (hi << 32)));
-  }
-  return d;
+// 16 bytes of the token buffer at byte offset `a`, of which only the first
+// `avail` bytes (a multiple of 4) are read when fewer than 16 remain.
+__device__ __forceinline__ uint4 load_piece(const char* base, int64_t a, int64_t avail) {
+  if (avail >= 16) return __ldg(reinterpret_cast<const uint4*>(base + a));
+  uint32_t w[4] = {0, 0, 0, 0};
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+    if (4 * q < avail) w[q] = __ldg(reinterpret_cast<const uint32_t*>(base + a) + q);
+  return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
+// Row layout shared by both digest kernels: row j holds the bytes of block j
+// rounded out to 16-byte boundaries, [a_j, a_j + 16*NP) with
+// a_j = (4*first token) & ~15, so lane j reading word k of its own block hits
+// bank group (row stride * j + 8k) mod 128 and rows of 16*NP bytes keep the
+// 32 lanes spread over the banks.
+
+// B = 2*HB with B % 4 == 0 (HB even). A chunk whose 32 blocks belong to one
+// request is one contiguous byte span; the warp loads it with coalesced
+// 16-byte loads (piece p = lane + 32 i) into registers one chunk ahead, and
+// scatters each piece into the row(s) that contain it: piece p lies in row
+// p / PB and, when it starts a block, also ends row p / PB - 1.
 template <int HB>
 __global__ void __launch_bounds__(kDigestWarps * 32)
     k_digest(const int32_t* __restrict__ tokens, int64_t n_tokens, const int64_t* __restrict__ off,
-             const int64_t* __restrict__ block_off, int32_t n, int B, uint64_t d_init,
-             int rowshift, int q_max, int stage_words, const int32_t* __restrict__ batch_ok,
-             uint64_t* __restrict__ digest) {
-  extern __shared__ uint64_t dsm[];
+             const int64_t* __restrict__ block_off, int32_t n, uint64_t d_init,
+             const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ digest) {
+  constexpr int B = 2 * HB;
+  constexpr int PB = HB / 2;  // 16-byte pieces per block
+  constexpr int NP = PB + 1;  // pieces per row (the block plus its misalignment)
+  extern __shared__ uint4 dsm[];
   if (!*batch_ok) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, warps = blockDim.x >> 5;
   const int64_t total = block_off[n];
   const int64_t n_chunks = (total + kChunk - 1) / kChunk;
   const int64_t tw = (int64_t)gridDim.x * warps;
-  int64_t c = (int64_t)blockIdx.x * warps + warp;
-  if (c >= n_chunks) return;
-  uint64_t* const stages = dsm + (size_t)warp * kStages * stage_words;  // this warp's stages
-  uint64_t policy;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;\n" : "=l"(policy));
-  const int hb = B >> 1;
+  const int64_t per = (n_chunks + tw - 1) / tw;
+  const int64_t c_lo = ((int64_t)blockIdx.x * warps + warp) * per;
+  const int64_t c_hi = min(n_chunks, c_lo + per);
+  if (c_lo >= c_hi) return;
+  uint4* const st = dsm + (size_t)warp * kChunk * NP;
+  const int64_t token_bytes = 4 * n_tokens;
+  const char* const tb = reinterpret_cast<const char*>(tokens);
+
+  int32_t r = find_request(block_off, 0, n, min(c_lo * kChunk + lane, total - 1));
+
+  struct Chunk {
+    int64_t tok0;  // this lane's first token
+    int64_t a0;    // byte offset of piece 0 (fast path)
+    int nv;        // valid lanes (a prefix of the warp)
+    bool valid, fast;
+  };
+  uint4 buf[NP];
+  // locate chunk c and load its bytes into registers
+  auto load = [&](int64_t c, Chunk& ch) {
+    const int64_t f = c * kChunk + lane;
+    ch.valid = f < total;
+    if (ch.valid) {
+      if (__ldg(block_off + r + 1) <= f) r = find_request(block_off, r + 1, n, f);
+      ch.tok0 = __ldg(off + r) + (f - __ldg(block_off + r)) * B;
+    } else {
+      ch.tok0 = 0;
+    }
+    ch.nv = __popc(__ballot_sync(kFull, ch.valid));
+    const int32_t r0 = __shfl_sync(kFull, r, 0);
+    ch.a0 = (4 * __shfl_sync(kFull, ch.tok0, 0)) & ~(int64_t)15;
+    const int npieces = ch.nv * PB + 1;
+    ch.fast = __all_sync(kFull, !ch.valid || r == r0) && ch.a0 + 16 * (int64_t)npieces <= token_bytes;
+    if (ch.fast) {
+#pragma unroll
+      for (int i = 0; i < NP; ++i) {
+        const int p = lane + 32 * i;
+        if (p < npieces) buf[i] = __ldg(reinterpret_cast<const uint4*>(tb + ch.a0) + p);
+      }
+    } else if (ch.valid) {
+      const int64_t a = (4 * ch.tok0) & ~(int64_t)15;
+#pragma unroll
+      for (int i = 0; i < NP; ++i) buf[i] = load_piece(tb, a + 16 * i, token_bytes - (a + 16 * i));
+    }
+  };
+  auto store = [&](const Chunk& ch) {
+    if (ch.fast) {
+      const int npieces = ch.nv * PB + 1;
+#pragma unroll
+      for (int i = 0; i < NP; ++i) {
+        const int p = lane + 32 * i;
+        if (p < npieces) {
+          const int j = p / PB, q = p - j * PB;
+          if (j < ch.nv) st[j * NP + q] = buf[i];
+          if (q == 0 && j >= 1) st[(j - 1) * NP + PB] = buf[i];
+        }
+      }
+    } else if (ch.valid) {
+#pragma unroll
+      for (int i = 0; i < NP; ++i) st[lane * NP + i] = buf[i];
+    }
+  };
 
   Chunk cur, nxt;
-  locate(cur, c, total, off, block_off, n, B, lane, q_max);
-  stage_copy(cur, tokens, n_tokens, stages, rowshift, lane, policy);
-  cp_async_commit();
-  for (int it = 0; c < n_chunks; ++it, c += tw) {
-    const int64_t cn = c + tw;
-    if (cn < n_chunks) {
-      locate(nxt, cn, total, off, block_off, n, B, lane, q_max);
-      stage_copy(nxt, tokens, n_tokens, stages + ((it + 1) & 1) * stage_words, rowshift, lane, policy);
-    }
-    cp_async_commit();
-    cp_async_wait<1>();
+  load(c_lo, cur);
+  for (int64_t c = c_lo; c < c_hi; ++c) {
+    store(cur);
     __syncwarp();
+    if (c + 1 < c_hi) load(c + 1, nxt);  // in flight during this chunk's arithmetic
     if (cur.valid) {
-      uint64_t d;
-      if (cur.fast) {
-        const int64_t rel = cur.tok0 - 2 * cur.u_lo;
-        d = digest_staged<HB>(stages + (it & 1) * stage_words, (int)(rel >> 1), (rel & 1) != 0, hb,
-                                 rowshift, d_init);
-      } else {
-        d = digest_global(tokens, cur.tok0, hb, d_init);
-      }
-      digest[c * kChunk + lane] = d;
+      const int delta = (int)((cur.tok0 * 4) & 15);  // 0, 4, 8 or 12
+      const uint64_t* row = reinterpret_cast<const uint64_t*>(st + lane * NP) + (delta >> 3);
+      digest[c * kChunk + lane] = digest_row<HB>(row, (delta & 4) != 0, HB, d_init);
     }
     __syncwarp();
     cur = nxt;
   }
-  cp_async_wait<0>();
 }
 
-// ---------------------------------------------------------------------------
-// walk
-// ---------------------------------------------------------------------------
-
-// Tier masks of key h whose home slot s holds (k0, m0) in its first 16 bytes.
-template <int W>
-__device__ __forceinline__ void resolve(const uint64_t* __restrict__ table, uint64_t cap, uint64_t h,
-                                        uint64_t s, uint64_t k0, uint64_t m0, uint64_t (&M)[W]) {
-  constexpr int EW = entry_words(W);
-  const uint64_t max_probe = cap < SMETRIC_MAX_PROBE ? cap : SMETRIC_MAX_PROBE;
-  uint64_t k = k0, t = 0;
-  const uint64_t* e = table + s * EW;
-  while (true) {
-    if (k == h) {
-      M[0] = t == 0 ? m0 : __ldg(e + 1);
-#pragma unroll
-      for (int w = 1; w < W; ++w) M[w] = __ldg(e + 1 + w);
-      return;
-    }
-    if (k == kEmpty || ++t >= max_probe) break;
-    if (++s == cap) s = 0;
-    e = table + s * EW;
-    k = __ldg(e);
+// Any even B: each lane copies its own row straight from global memory.
+__global__ void __launch_bounds__(kDigestWarps * 32)
+    k_digest_any(const int32_t* __restrict__ tokens, int64_t n_tokens, const int64_t* __restrict__ off,
+                 const int64_t* __restrict__ block_off, int32_t n, int B, int nch, uint64_t d_init,
+                 const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ digest) {
+  extern __shared__ uint4 dsm[];
+  if (!*batch_ok) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, warps = blockDim.x >> 5;
+  const int64_t total = block_off[n];
+  const int64_t n_chunks = (total + kChunk - 1) / kChunk;
+  const int64_t tw = (int64_t)gridDim.x * warps;
+  const int64_t per = (n_chunks + tw - 1) / tw;
+  const int64_t c_lo = ((int64_t)blockIdx.x * warps + warp) * per;
+  const int64_t c_hi = min(n_chunks, c_lo + per);
+  if (c_lo >= c_hi) return;
+  uint4* const row = dsm + ((size_t)warp * kChunk + lane) * nch;
+  const int64_t token_bytes = 4 * n_tokens;
+  const char* const tb = reinterpret_cast<const char*>(tokens);
+  int32_t r = find_request(block_off, 0, n, min(c_lo * kChunk + lane, total - 1));
+  for (int64_t c = c_lo; c < c_hi; ++c) {
+    const int64_t f = c * kChunk + lane;
+    if (f >= total) continue;
+    if (__ldg(block_off + r + 1) <= f) r = find_request(block_off, r + 1, n, f);
+    const int64_t tok0 = __ldg(off + r) + (f - __ldg(block_off + r)) * B;
+    const int64_t a = (4 * tok0) & ~(int64_t)15;
+    for (int i = 0; i < nch; ++i) row[i] = load_piece(tb, a + 16 * i, token_bytes - (a + 16 * i));
+    const int delta = (int)((tok0 * 4) & 15);
+    digest[f] = digest_row<0>(reinterpret_cast<const uint64_t*>(row) + (delta >> 3), (delta & 4) != 0,
+                              B >> 1, d_init);
   }
-#pragma unroll
-  for (int w = 0; w < W; ++w) M[w] = 0;
 }
 
-template <int W, bool PROBE>
-__global__ void __launch_bounds__(kWalkThreads)
-    k_walk(const uint64_t* __restrict__ table, uint64_t cap, int N, int B, int S, uint64_t h_init,
-           const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n,
-           const int64_t* __restrict__ load, int64_t w_load, int64_t w_miss, int64_t w_glob,
-           const uint64_t* __restrict__ digest, const int32_t* __restrict__ batch_ok,
-           int32_t* __restrict__ inst_out, int32_t* __restrict__ lhit_out,
-           int32_t* __restrict__ ghit_out, uint64_t* __restrict__ sk_out,
-           uint64_t* __restrict__ hash_out) {
-  constexpr int EW = entry_words(W);
-  extern __shared__ int64_t wsm[];
-  int64_t* load_s = wsm;                                    // [N]
-  int32_t* death = reinterpret_cast<int32_t*>(wsm + N);     // [N][kWalkThreads]
-  const int tid = threadIdx.x;
-  if (PROBE)
-    for (int i = tid; i < N; i += blockDim.x) load_s[i] = load[i];
-  __syncthreads();
-  const int32_t r = blockIdx.x * kWalkThreads + tid;
+// ---------------------------------------------------------------------------
+// chain
+// ---------------------------------------------------------------------------
+
+__global__ void __launch_bounds__(kChainThreads)
+    k_chain(const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n, int B,
+            int S, uint64_t h_init, const int32_t* __restrict__ batch_ok,
+            const uint64_t* __restrict__ digest, uint64_t* __restrict__ hashes,
+            uint64_t* __restrict__ sk_out) {
+  const int32_t r = blockIdx.x * kChainThreads + threadIdx.x;
   if (r >= n) return;
-  if (!*batch_ok) {
-    if (PROBE) { inst_out[r] = -1; lhit_out[r] = 0; ghit_out[r] = 0; }
-    sk_out[r] = 0;
-    return;
-  }
-  const int64_t L = off[r + 1] - off[r];
-  const int64_t nb = L / B;
+  if (!*batch_ok) { sk_out[r] = 0; return; }
+  const int64_t nb = (off[r + 1] - off[r]) / B;
   const int64_t bo = block_off[r];
+  const uint64_t* const d = digest + bo;
+  uint64_t* const hout = hashes + bo;
   const int64_t kS = (nb < S ? nb : S) - 1;
-
-  uint64_t alive[W];  // local tiers still holding every block so far
-#pragma unroll
-  for (int w = 0; w < W; ++w) {
-    const int lo = w * 64;
-    alive[w] = N >= lo + 64 ? ~0ull : (N > lo ? (1ull << (N - lo)) - 1 : 0ull);
-  }
-  int64_t g = 0;
-  bool galive = PROBE;
-  bool walking = PROBE && nb > 0;
   uint64_t h = h_init, sk = 0;
-  const int gword = N >> 6;                  // mask word holding the global-tier bit
-  const uint64_t gbit = 1ull << (N & 63);
-
-  for (int64_t b0 = 0; b0 < nb; b0 += kGroup) {
-    const int cnt = (int)min((int64_t)kGroup, nb - b0);
-    uint64_t hs[kGroup];
+  uint64_t cur[kChainAhead], nxt[kChainAhead];
 #pragma unroll
-    for (int j = 0; j < kGroup; ++j) {
-      if (j < cnt) {
-        h = mix64((h + kGamma) ^ __ldg(digest + bo + b0 + j));
+  for (int j = 0; j < kChainAhead; ++j) cur[j] = j < nb ? __ldg(d + j) : 0;
+  for (int64_t b0 = 0; b0 < nb; b0 += kChainAhead) {
+#pragma unroll
+    for (int j = 0; j < kChainAhead; ++j)
+      nxt[j] = b0 + kChainAhead + j < nb ? __ldg(d + b0 + kChainAhead + j) : 0;
+#pragma unroll
+    for (int j = 0; j < kChainAhead; ++j) {
+      if (b0 + j < nb) {
+        h = mix64((h + kGamma) ^ cur[j]);
         if (h < 2) h |= 2;
-        hs[j] = h;
-        if (hash_out) hash_out[bo + b0 + j] = h;
+        hout[b0 + j] = h;
         if (b0 + j == kS) sk = h;
       }
     }
-    if (PROBE && walking) {
-      uint64_t slot[kGroup], k0[kGroup], m0[kGroup];
 #pragma unroll
-      for (int j = 0; j < kGroup; ++j) {
-        if (j < cnt) {
-          slot[j] = home_slot(hs[j], cap);
-          const ulonglong2 v = __ldg(reinterpret_cast<const ulonglong2*>(table + slot[j] * EW));
-          k0[j] = v.x;
-          m0[j] = v.y;
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < kGroup; ++j) {
-        if (j < cnt && walking) {
-          uint64_t M[W];
-          resolve<W>(table, cap, hs[j], slot[j], k0[j], m0[j], M);
-          const int32_t b = (int32_t)(b0 + j);
-          bool any = false;
-#pragma unroll
-          for (int w = 0; w < W; ++w) {
-            uint64_t dead = alive[w] & ~M[w];
-            while (dead) {
-              const int i = w * 64 + __ffsll((long long)dead) - 1;
-              death[i * kWalkThreads + tid] = b;
-              dead &= dead - 1;
-            }
-            alive[w] &= M[w];
-            any |= alive[w] != 0;
-          }
-          if (galive) {
-            uint64_t mg = 0;
-#pragma unroll
-            for (int w = 0; w < W; ++w) if (w == gword) mg = M[w];
-            if (mg & gbit) g = b + 1;
-            else galive = false;
-          }
-          walking = any || galive;
-        }
-      }
-    }
-    if (!walking && !hash_out && b0 + cnt > kS) break;
+    for (int j = 0; j < kChainAhead; ++j) cur[j] = nxt[j];
   }
   sk_out[r] = nb > 0 ? sk : 0;
-  if (!PROBE) return;
+}
 
-  int32_t best = 0;
-  int64_t best_cost = INT64_MAX, best_c = 0;
+// ---------------------------------------------------------------------------
+// match
+// ---------------------------------------------------------------------------
+
+// Tier masks of key h (zeros when absent) from the read-only table: the home
+// bucket's 16 tags, then the entry of each tag match, then later buckets while
+// every slot of the bucket so far was full.
+template <int W>
+__device__ __forceinline__ void probe_one(const uint8_t* __restrict__ tags, const uint64_t* __restrict__ table,
+                                          uint64_t n_buckets, uint64_t h, uint64_t (&M)[W]) {
+  constexpr int EW = entry_words(W);
+  constexpr int NV = (W + 2) / 2;  // 16-byte loads covering key + W mask words
 #pragma unroll
-  for (int w = 0; w < W; ++w) {
-    const uint64_t aw = alive[w];
-    const int iend = N < 64 * (w + 1) ? N : 64 * (w + 1);
-    for (int i = 64 * w; i < iend; ++i) {
-      const int64_t ci = ((aw >> (i - 64 * w)) & 1) ? nb : (int64_t)death[i * kWalkThreads + tid];
+  for (int w = 0; w < W; ++w) M[w] = 0;
+  const uint32_t tg = key_tag(h);
+  uint64_t b = home_bucket(h, n_buckets);
+  const uint64_t mb = n_buckets < SMETRIC_MAX_PROBE / kBucket ? n_buckets : SMETRIC_MAX_PROBE / kBucket;
+  for (uint64_t t = 0; t < mb; ++t) {
+    const uint4 tv = __ldg(reinterpret_cast<const uint4*>(tags + b * kBucket));
+    uint32_t cand = tag_match(tv, tg);
+    while (cand) {
+      const int sl = __ffs(cand) - 1;
+      cand &= cand - 1;
+      const ulonglong2* e = reinterpret_cast<const ulonglong2*>(table + (b * kBucket + sl) * EW);
+      ulonglong2 v[NV];
+#pragma unroll
+      for (int q = 0; q < NV; ++q) v[q] = __ldg(e + q);
+      if (v[0].x == h) {
+#pragma unroll
+        for (int w = 0; w < W; ++w) M[w] = (w & 1) ? v[(w + 1) >> 1].x : v[(w + 1) >> 1].y;
+        return;
+      }
+    }
+    if (tag_match(tv, 0)) return;
+    if (++b == n_buckets) b = 0;
+  }
+}
+
+// One thread per block of the batch: the tier masks of every block hash.
+template <int W>
+__global__ void __launch_bounds__(256)
+    k_probe(const uint8_t* __restrict__ tags, const uint64_t* __restrict__ table, uint64_t n_buckets,
+            const int64_t* __restrict__ block_off, int32_t n, const uint64_t* __restrict__ H,
+            const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ masks) {
+  if (!*batch_ok) return;
+  const int64_t total = block_off[n];
+  for (int64_t f = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; f < total;
+       f += (int64_t)gridDim.x * blockDim.x) {
+    uint64_t M[W];
+    probe_one<W>(tags, table, n_buckets, __ldg(H + f), M);
+#pragma unroll
+    for (int w = 0; w < W; ++w) masks[f * W + w] = M[w];
+  }
+}
+
+// One warp per request, lanes = 32 consecutive blocks: the running AND of the
+// local-tier masks (a shuffle scan across lanes), the block where each
+// instance's run ends (ballot + ffs, recorded in shared memory), the
+// global-tier run; then lanes = instances for the cost and a shuffle argmin
+// with ties to the lowest id.
+template <int W>
+__global__ void __launch_bounds__(kMatchWarps * 32)
+    k_walk(int N, int B, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n,
+           const int64_t* __restrict__ load, int64_t w_load, int64_t w_miss, int64_t w_glob,
+           const uint64_t* __restrict__ masks, const int32_t* __restrict__ batch_ok,
+           int32_t* __restrict__ inst_out, int32_t* __restrict__ lhit_out,
+           int32_t* __restrict__ ghit_out) {
+  extern __shared__ int64_t msm[];
+  int64_t* load_s = msm;                                                     // [N]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  int32_t* death = reinterpret_cast<int32_t*>(msm + N) + warp * N;           // [warps][N]
+  for (int i = threadIdx.x; i < N; i += blockDim.x) load_s[i] = load[i];
+  __syncthreads();
+  const bool ok = *batch_ok != 0;
+  const int gword = N >> 6;
+  const uint64_t gbit = 1ull << (N & 63);
+  const int64_t tw = (int64_t)gridDim.x * kMatchWarps;
+
+  for (int64_t r = (int64_t)blockIdx.x * kMatchWarps + warp; r < n; r += tw) {
+    if (!ok) {
+      if (lane == 0) { inst_out[r] = -1; lhit_out[r] = 0; ghit_out[r] = 0; }
+      continue;
+    }
+    const int64_t L = off[r + 1] - off[r];
+    const int64_t nb = L / B;
+    const uint64_t* const m_r = masks + block_off[r] * W;
+    uint64_t A[W];  // local tiers holding every block so far (warp-uniform)
+#pragma unroll
+    for (int w = 0; w < W; ++w) {
+      const int lo = w * 64;
+      A[w] = N >= lo + 64 ? ~0ull : (N > lo ? (1ull << (N - lo)) - 1 : 0ull);
+    }
+    bool galive = true;
+    int64_t g = 0;
+    uint64_t nx[W];
+#pragma unroll
+    for (int w = 0; w < W; ++w) nx[w] = lane < nb ? __ldg(m_r + lane * W + w) : 0;
+    for (int64_t base = 0; base < nb; base += 32) {
+      const bool valid = base + lane < nb;
+      uint64_t M[W];
+#pragma unroll
+      for (int w = 0; w < W; ++w) {
+        M[w] = nx[w];
+        nx[w] = base + 32 + lane < nb ? __ldg(m_r + (base + 32 + lane) * W + w) : 0;
+      }
+      // global-tier run: first lane whose block the global tier lacks
+      if (galive) {
+        uint64_t mg = 0;
+#pragma unroll
+        for (int w = 0; w < W; ++w) if (w == gword) mg = M[w];
+        const unsigned miss = __ballot_sync(kFull, !(valid && (mg & gbit)));
+        if (miss) { g = base + __ffs(miss) - 1; galive = false; }
+        else g = base + 32;
+      }
+      // local runs: inclusive AND-scan of the masks across lanes
+      bool any = false;
+#pragma unroll
+      for (int w = 0; w < W; ++w) {
+        uint64_t x = valid ? M[w] : 0;
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+          const uint64_t y = __shfl_up_sync(kFull, x, d);
+          if (lane >= d) x &= y;
+        }
+        x &= A[w];                                   // held through block base + lane
+        const uint64_t last = __shfl_sync(kFull, x, 31);
+        uint64_t dead = A[w] & ~last;                // runs that end in this chunk
+        while (dead) {
+          const int bit = __ffsll((long long)dead) - 1;
+          dead &= dead - 1;
+          const unsigned gone = __ballot_sync(kFull, !((x >> bit) & 1));
+          if (lane == 0) death[w * 64 + bit] = (int32_t)(base + __ffs(gone) - 1);
+        }
+        A[w] = last;
+        any |= last != 0;
+      }
+      if (!any && !galive) break;
+    }
+    __syncwarp();
+    // cost of every instance; lanes = instances
+    int64_t best_cost = INT64_MAX;
+    int32_t best = N;
+    for (int i = lane; i < N; i += 32) {
+      uint64_t aw = 0;
+#pragma unroll
+      for (int w = 0; w < W; ++w) if (w == (i >> 6)) aw = A[w];
+      const int64_t ci = ((aw >> (i & 63)) & 1) ? nb : (int64_t)death[i];
       const int64_t gi = ci > g ? ci : g;
       const int64_t cost = w_load * load_s[i] + w_miss * (L - B * gi) + w_glob * B * (gi - ci);
-      if (cost < best_cost) { best_cost = cost; best = i; best_c = ci; }
+      if (cost < best_cost) { best_cost = cost; best = i; }
     }
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) {
+      const int64_t oc = __shfl_xor_sync(kFull, best_cost, d);
+      const int32_t oi = __shfl_xor_sync(kFull, best, d);
+      if (oc < best_cost || (oc == best_cost && oi < best)) { best_cost = oc; best = oi; }
+    }
+    if (lane == 0) {
+      uint64_t aw = 0;
+#pragma unroll
+      for (int w = 0; w < W; ++w) if (w == (best >> 6)) aw = A[w];
+      const int64_t cb = ((aw >> (best & 63)) & 1) ? nb : (int64_t)death[best];
+      const int64_t gb = cb > g ? cb : g;
+      inst_out[r] = best;
+      lhit_out[r] = (int32_t)(B * cb);
+      ghit_out[r] = (int32_t)(B * (gb - cb));
+    }
+    __syncwarp();
   }
-  const int64_t gb = best_c > g ? best_c : g;
-  inst_out[r] = best;
-  lhit_out[r] = (int32_t)(B * best_c);
-  ghit_out[r] = (int32_t)(B * (gb - best_c));
 }
 
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 
-int log2_floor(int x) { int s = 0; while ((1 << (s + 1)) <= x) ++s; return s; }
-
-struct DigestPlan {
-  int rowshift, q_max, stage_words, warps;
-  size_t smem;
-};
-
-DigestPlan digest_plan(int B) {
-  DigestPlan p;
-  const int hb = B / 2;
-  const bool pow2 = (hb & (hb - 1)) == 0;
-  p.rowshift = (pow2 && hb >= 4) ? log2_floor(hb) : 4;
-  p.q_max = kSpanBlocks * hb + 2;
-  p.stage_words = p.q_max + (p.q_max >> p.rowshift) + 2;
-  const size_t per_warp = (size_t)kStages * p.stage_words * sizeof(uint64_t);
-  p.warps = (int)std::max<size_t>(1, std::min<size_t>(kDigestWarps, kDigestSmem / per_warp));
-  p.smem = (size_t)p.warps * per_warp;
-  return p;
-}
+void profile_mark(smetric_index* idx, int k, cudaStream_t s);
 
 template <int HB>
 int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
                   const int64_t* d_offsets, int32_t n, cudaStream_t s) {
   const int B = idx->cfg.block_size;
-  const DigestPlan p = digest_plan(B);
-  auto kern = k_digest<HB>;
+  // rows of 16*nch bytes: a block's 4B bytes start at most 12 bytes past a
+  // 16-byte boundary
+  const int nch = HB > 0 ? HB / 2 + 1 : (4 * B + 12 + 15) / 16;
+  const size_t per_warp = (size_t)kChunk * nch * 16;
+  const int warps = (int)std::max<size_t>(1, std::min<size_t>(kDigestWarps, (200 * 1024) / per_warp));
+  const size_t smem = (size_t)warps * per_warp;
+  auto kern = HB > 0 ? k_digest<HB> : nullptr;
+  const void* fn = HB > 0 ? (const void*)kern : (const void*)k_digest_any;
   if (idx->digest_occ == 0) {  // once per index: B, and so the plan, is fixed
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem) != cudaSuccess)
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
       return cuda_status(cudaErrorInvalidValue);
     int occ = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, p.warps * 32, p.smem) != cudaSuccess)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fn, warps * 32, smem) != cudaSuccess)
       return cuda_status(cudaErrorInvalidValue);
     idx->digest_occ = occ < 1 ? 1 : occ;
   }
-  const int occ = idx->digest_occ;
   const int64_t max_chunks = (n_tokens / B + kChunk - 1) / kChunk;
-  const int64_t want = (max_chunks + p.warps - 1) / p.warps;
-  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * occ));
+  const int64_t want = (max_chunks + warps - 1) / warps;
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * idx->digest_occ));
   const uint64_t d_init = mix64(idx->cfg.hash_seed ^ (uint64_t)B);
-  kern<<<(unsigned)grid, p.warps * 32, p.smem, s>>>(d_tokens, n_tokens, d_offsets, idx->block_off, n, B,
-                                                          d_init, p.rowshift, p.q_max, p.stage_words,
-                                                          idx->batch_ok, idx->digest);
+  if (HB > 0)
+    kern<<<(unsigned)grid, warps * 32, smem, s>>>(d_tokens, n_tokens, d_offsets, idx->block_off, n, d_init,
+                                                  idx->batch_ok, idx->digest);
+  else
+    k_digest_any<<<(unsigned)grid, warps * 32, smem, s>>>(d_tokens, n_tokens, d_offsets, idx->block_off, n, B,
+                                                          nch, d_init, idx->batch_ok, idx->digest);
   idx->launches++;
   return cuda_status(cudaGetLastError());
-}
-
-template <int W, bool PROBE>
-int launch_walk(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
-                smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, uint64_t* sk,
-                uint64_t* hashes, cudaStream_t s) {
-  const int N = idx->cfg.num_instances;
-  const size_t smem = PROBE ? (size_t)N * sizeof(int64_t) + (size_t)N * kWalkThreads * sizeof(int32_t) : 0;
-  auto kern = k_walk<W, PROBE>;
-  if (smem > 48 * 1024 &&
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
-    return cuda_status(cudaErrorInvalidValue);
-  const unsigned grid = (unsigned)((n + kWalkThreads - 1) / kWalkThreads);
-  const uint64_t h_init = mix64(idx->cfg.hash_seed + kGamma);
-  kern<<<grid, kWalkThreads, smem, s>>>(idx->table, idx->cfg.capacity_slots, N, idx->cfg.block_size,
-                                        idx->cfg.session_blocks, h_init, d_offsets, idx->block_off, n,
-                                        d_load, w.w_load, w.w_miss, w.w_glob, idx->digest, idx->batch_ok,
-                                        inst, lhit, ghit, sk, hashes);
-  idx->launches++;
-  return cuda_status(cudaGetLastError());
-}
-
-template <bool PROBE>
-int dispatch_walk(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
-                  smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, uint64_t* sk,
-                  uint64_t* hashes, cudaStream_t s) {
-  if (!PROBE) return launch_walk<1, false>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, sk, hashes, s);
-  switch (idx->W) {
-    case 1: return launch_walk<1, PROBE>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, sk, hashes, s);
-    case 2: return launch_walk<2, PROBE>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, sk, hashes, s);
-    case 3: return launch_walk<3, PROBE>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, sk, hashes, s);
-    case 4: return launch_walk<4, PROBE>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, sk, hashes, s);
-    case 5: return launch_walk<5, PROBE>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, sk, hashes, s);
-    default: return SMETRIC_ERR_INVALID_ARG;
-  }
 }
 
 int dispatch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
@@ -496,19 +550,72 @@ int dispatch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_token
   }
 }
 
-ProfileSlot* profile_begin(smetric_index* idx, cudaStream_t s) {
-  if (!idx->profiling) return nullptr;
+int launch_chain(smetric_index* idx, const int64_t* d_offsets, int32_t n, uint64_t* hashes,
+                 uint64_t* sk, cudaStream_t s) {
+  const unsigned grid = (unsigned)((n + kChainThreads - 1) / kChainThreads);
+  const uint64_t h_init = mix64(idx->cfg.hash_seed + kGamma);
+  k_chain<<<grid, kChainThreads, 0, s>>>(d_offsets, idx->block_off, n, idx->cfg.block_size,
+                                         idx->cfg.session_blocks, h_init, idx->batch_ok, idx->digest,
+                                         hashes ? hashes : idx->hashes, sk);
+  idx->launches++;
+  return cuda_status(cudaGetLastError());
+}
+
+template <int W>
+int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
+                 smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, const uint64_t* H,
+                 int64_t max_blocks, cudaStream_t s) {
+  const int N = idx->cfg.num_instances;
+  // probe: one thread per block, grid sized to the largest possible batch
+  {
+    const int64_t want = (max_blocks + 255) / 256;
+    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
+    k_probe<W><<<(unsigned)grid, 256, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->block_off, n, H,
+                                              idx->batch_ok, idx->masks);
+    idx->launches++;
+    int rc = cuda_status(cudaGetLastError());
+    if (rc) return rc;
+  }
+  profile_mark(idx, kProbe, s);
+  const size_t smem = (size_t)N * sizeof(int64_t) + (size_t)kMatchWarps * N * sizeof(int32_t);
+  auto kern = k_walk<W>;
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+    return cuda_status(cudaErrorInvalidValue);
+  const int64_t want = ((int64_t)n + kMatchWarps - 1) / kMatchWarps;
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
+  kern<<<(unsigned)grid, kMatchWarps * 32, smem, s>>>(N, idx->cfg.block_size, d_offsets, idx->block_off, n,
+                                                      d_load, w.w_load, w.w_miss, w.w_glob, idx->masks,
+                                                      idx->batch_ok, inst, lhit, ghit);
+  idx->launches++;
+  return cuda_status(cudaGetLastError());
+}
+
+int dispatch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
+                   smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, const uint64_t* H,
+                   int64_t max_blocks, cudaStream_t s) {
+  switch (idx->W) {
+    case 1: return launch_match<1>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, H, max_blocks, s);
+    case 2: return launch_match<2>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, H, max_blocks, s);
+    case 3: return launch_match<3>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, H, max_blocks, s);
+    case 4: return launch_match<4>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, H, max_blocks, s);
+    case 5: return launch_match<5>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, H, max_blocks, s);
+    default: return SMETRIC_ERR_INVALID_ARG;
+  }
+}
+
+void profile_begin(smetric_index* idx, cudaStream_t s) {
+  if (!idx->profiling) return;
   ProfileSlot slot;
   if (!idx->prof_pool.empty()) {
     slot = idx->prof_pool.back();
     idx->prof_pool.pop_back();
   } else {
     for (auto& e : slot.ev)
-      if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+      if (cudaEventCreate(&e) != cudaSuccess) return;
   }
   idx->prof_used.push_back(slot);
   cudaEventRecord(idx->prof_used.back().ev[0], s);
-  return &idx->prof_used.back();
 }
 
 void profile_mark(smetric_index* idx, int k, cudaStream_t s) {
@@ -546,7 +653,13 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
     if ((rc = dispatch_digest(idx, d_tokens, n_tokens, d_offsets, n, s))) return rc;
   }
   profile_mark(idx, kDigest, s);
-  if ((rc = dispatch_walk<PROBE>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, sk, hashes, s))) return rc;
+  if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, s))) return rc;
+  profile_mark(idx, kChain, s);
+  if (PROBE) {
+    if ((rc = dispatch_match(idx, d_offsets, n, d_load, w, inst, lhit, ghit,
+                             hashes ? hashes : idx->hashes, n_tokens / c.block_size, s)))
+      return rc;
+  }
   profile_mark(idx, kWalk, s);
   return SMETRIC_OK;
 }
@@ -642,6 +755,8 @@ const char* smetric_profile_kernel_name(int32_t k) {
   switch (k) {
     case kPrep: return "k_prep";
     case kDigest: return "k_digest";
+    case kChain: return "k_chain";
+    case kProbe: return "k_probe";
     case kWalk: return "k_walk";
     default: return "";
   }

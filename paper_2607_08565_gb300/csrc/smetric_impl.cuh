@@ -21,10 +21,36 @@ __host__ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
   return z ^ (z >> 31);
 }
 
-// Home slot of a key: the high 64 bits of key * capacity, uniform over
-// [0, capacity) for uniformly distributed keys (Lemire's range reduction).
-__device__ __forceinline__ uint64_t home_slot(uint64_t key, uint64_t cap) {
-  return __umul64hi(key, cap);
+// The table is an array of buckets of kBucket slots. Each slot has a one-byte
+// tag (0: empty; otherwise 0x80 | low 7 key bits) in a separate tag array and
+// an entry (key + tier-mask words) in the entry array. A key's home bucket is
+// the high 64 bits of key * n_buckets (Lemire's range reduction); inserts
+// take the first empty slot in bucket order from the home bucket (linear
+// probing over buckets). At load factor 0.7, 98.6% of keys sit in their home
+// bucket, so a lookup is one tag read plus one entry read.
+constexpr int kBucket = 16;
+
+__device__ __forceinline__ uint64_t home_bucket(uint64_t key, uint64_t n_buckets) {
+  return __umul64hi(key, n_buckets);
+}
+
+__host__ __device__ __forceinline__ uint32_t key_tag(uint64_t key) {
+  return 0x80u | (uint32_t)(key & 0x7Fu);
+}
+
+// Bit s of the result is set where byte s of the 16 tag bytes equals `tag`.
+__device__ __forceinline__ uint32_t tag_match(uint4 t, uint32_t tag) {
+  const uint32_t rep = tag * 0x01010101u;
+  uint32_t m = 0;
+  const uint32_t w[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t eq = __vcmpeq4(w[i], rep);  // 0xff in each equal byte
+    // gather the top bit of each byte into 4 bits
+    const uint32_t b = ((eq >> 7) & 1u) | ((eq >> 14) & 2u) | ((eq >> 21) & 4u) | ((eq >> 28) & 8u);
+    m |= b << (4 * i);
+  }
+  return m;
 }
 
 // First error wins; later ones are dropped until the host reads and clears.
@@ -38,7 +64,7 @@ __device__ __forceinline__ void latch_error(int32_t* status, int32_t code) {
 __host__ __device__ constexpr int entry_words(int W) { return W == 1 ? 2 : (W <= 3 ? 4 : 8); }
 
 // Route kernels, in launch order; names returned by smetric_profile_kernel_name.
-enum RouteKernel { kPrep = 0, kDigest = 1, kWalk = 2, kNumRouteKernels = 3 };
+enum RouteKernel { kPrep = 0, kDigest = 1, kChain = 2, kProbe = 3, kWalk = 4, kNumRouteKernels = 5 };
 
 struct ProfileSlot {
   cudaEvent_t ev[kNumRouteKernels + 1];
@@ -52,11 +78,15 @@ struct smetric_index {
   int num_sms;
   int W;   // tier-mask words per key
   int EW;  // entry stride in 64-bit words
-  uint64_t* table;  // cfg.capacity_slots * EW words
+  uint64_t n_buckets;  // ceil(capacity_slots / kBucket)
+  uint64_t* table;     // n_buckets * kBucket entries of EW words
+  uint8_t* tags;       // n_buckets * kBucket tag bytes
   int32_t* status;  // device: first latched error
   // route scratch
   int64_t* block_off;  // max_batch_requests + 1: first block of each request
   uint64_t* digest;    // max_batch_tokens / B: per-block digests d_b
+  uint64_t* hashes;    // max_batch_tokens / B: per-block chain hashes h_b
+  uint64_t* masks;     // W * max_batch_tokens / B: per-block tier masks
   int32_t* batch_ok;   // device flag written by the prep kernel
   // staging for smetric_route_batch_host
   int32_t* st_tokens;

@@ -68,16 +68,14 @@ def _populate_c4(ix, tr, chunk=4096):
         hb, _ = ix.block_hashes(T(tok), T(off))
         nb = torch.from_numpy(tr.prefix_len[ids] // B).to(hb.device)
         total = int(nb.sum())
-        hb = hb[:total]
+        hb = hb[:total].view(torch.int64)  # CUDA mask indexing has no uint64 kernels
         owner = torch.repeat_interleave(torch.arange(len(ids), device=hb.device), nb)
         sess = torch.from_numpy(ids).to(hb.device)[owner]
         ix.insert(hb, -1)
-        home = torch.from_numpy(tr.home).to(hb.device)[sess]
-        m = torch.from_numpy(tr.in_home).to(hb.device)[sess]
-        ix.insert(hb[m].contiguous(), home[m].contiguous())
-        sec = torch.from_numpy(tr.second).to(hb.device)[sess]
-        m2 = torch.from_numpy(tr.in_second).to(hb.device)[sess]
-        ix.insert(hb[m2].contiguous(), sec[m2].contiguous())
+        for tier_of, member in ((tr.home, tr.in_home), (tr.second, tr.in_second)):
+            m = torch.from_numpy(member).to(hb.device)[sess]
+            t = torch.from_numpy(tier_of).to(hb.device)[sess]
+            ix.insert(hb[m].contiguous(), t[m].contiguous())
     ix.check()
 
 
