@@ -186,11 +186,10 @@ def populate_index(ix, tr, device, chunk=4096):
 def algorithmic_bytes(lens, local_hit, global_hit, B, W):
     """Per-kernel bytes of one route call. k_digest: 4 B per hashed token (the
     method must read every token of every full block). k_probe: one index
-    entry (key + W mask words) per probed block, P_r = min(n_r, reach_r + 1)
-    (the method's probes; the kernel probes every block). k_chain, k_walk:
-    their reads and writes of this kernel split's intermediates (digests,
-    hashes, masks), which the method itself does not need, plus offsets and
-    outputs. k_prep: offsets and loads. path: the method's bytes per request,
+    entry (key + W mask words) per probed block, P_r = min(n_r, reach_r + 1).
+    k_chain: the digests it reads and hashes it writes (intermediates of this
+    kernel split). k_walk: the masks it reads, offsets and outputs. k_prep:
+    offsets and loads. path: the method's bytes per request,
     4 L_r + P_r (8 + 8W) + 8 + 20."""
     nb = lens // B
     reach = (local_hit.astype(np.int64) + global_hit) // B

@@ -17,15 +17,17 @@
 //   k_probe   one thread per block: the tier masks of h_b from the index
 //             (16 tags of the home bucket, then the matching entry).
 //   k_walk    one warp per request, lanes = 32 consecutive blocks: an AND-scan
-//             of the local-tier masks across lanes, the block where each
-//             instance's run ends located by ballot, the global-tier run;
-//             then lanes = instances for the cost and a shuffle argmin with
-//             ties to the lowest id.
+//             of the local-tier masks across lanes gives each lane the set of
+//             instances whose run ends at its block (an event), the global
+//             run is located by ballot; then lanes = instances for the cost
+//             and a shuffle argmin with ties to the lowest id.
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
 #include <algorithm>
+#include <cstring>
 
 #include "smetric_impl.cuh"
 
@@ -257,6 +259,165 @@ __global__ void __launch_bounds__(kDigestWarps * 32)
   }
 }
 
+// ---- TMA tensor path -------------------------------------------------------
+//
+// For B % 4 == 0, block j of a request starts 4B*j bytes after block 0, so the
+// rows a_j = (4*first token of block j) & ~15 of one request form a strided
+// 2D region: rows of 4B+16 bytes at stride 4B. A 2D tensor map per 16-byte
+// phase k (base = tokens + 16k) with row stride 4B and row length 4B+16 lets
+// one TMA tile load of 32 rows bring a whole chunk into the padded layout.
+// Rows past the end of the map are zero-filled by the TMA unit; a chunk that
+// needs such a row, or whose blocks span two requests, is copied by its lanes
+// instead.
+
+constexpr int kMaxPhases = 16;  // 4B / 16 for B <= 64
+constexpr uint32_t kSpinLimit = 1u << 22;  // bounded mbarrier waits
+
+struct TokenMaps {
+  CUtensorMap map[kMaxPhases];
+  uint32_t rows[kMaxPhases];  // rows addressable through map k
+};
+
+__device__ __forceinline__ void mbar_init(uint32_t mbar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(mbar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t mbar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(mbar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t mbar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(done) : "r"(mbar), "r"(parity) : "memory");
+  return done != 0;
+}
+// Bounded wait for the phase with the given parity; false on timeout.
+__device__ __forceinline__ bool mbar_wait(uint32_t mbar, uint32_t parity) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i)
+    if (mbar_try_wait(mbar, parity)) return true;
+  return false;
+}
+__device__ __forceinline__ void tma_rows(uint32_t dst, const CUtensorMap* map, int32_t y, uint32_t mbar,
+                                         uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;\n" ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(0),
+      "r"(y), "r"(mbar), "l"(policy)
+      : "memory");
+}
+
+template <int HB, int STAGES>
+__global__ void __launch_bounds__(kDigestWarps * 32)
+    k_digest_tma(const __grid_constant__ TokenMaps maps, const int32_t* __restrict__ tokens,
+                 int64_t n_tokens, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off,
+                 int32_t n, uint64_t d_init, const int32_t* __restrict__ batch_ok,
+                 uint64_t* __restrict__ digest, int32_t* status) {
+  constexpr int B = 2 * HB;
+  constexpr int NP = HB / 2 + 1;           // 16-byte pieces per row
+  constexpr uint32_t ROW = 16u * NP;       // = 4B + 16
+  constexpr uint32_t STAGE = kChunk * ROW;
+  extern __shared__ __align__(128) unsigned char dsm_raw[];
+  if (!*batch_ok) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, warps = blockDim.x >> 5;
+  const int64_t total = block_off[n];
+  const int64_t n_chunks = (total + kChunk - 1) / kChunk;
+  const int64_t tw = (int64_t)gridDim.x * warps;
+  const int64_t per = (n_chunks + tw - 1) / tw;
+  const int64_t c_lo = ((int64_t)blockIdx.x * warps + warp) * per;
+  const int64_t c_hi = min(n_chunks, c_lo + per);
+  if (c_lo >= c_hi) return;
+  unsigned char* const stages = dsm_raw + (size_t)warp * STAGES * STAGE;
+  const uint32_t mbar0 = smem_u32(dsm_raw + (size_t)warps * STAGES * STAGE) + 8u * STAGES * (uint32_t)warp;
+  if (lane == 0) {
+#pragma unroll
+    for (int s = 0; s < STAGES; ++s) mbar_init(mbar0 + 8u * s, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+  }
+  __syncwarp();
+  uint64_t policy;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;\n" : "=l"(policy));
+  const int64_t token_bytes = 4 * n_tokens;
+  const char* const tb = reinterpret_cast<const char*>(tokens);
+  int32_t r = find_request(block_off, 0, n, min(c_lo * kChunk + lane, total - 1));
+
+  // Start the copy of chunk c into stage s; returns this lane's first token.
+  auto issue = [&](int64_t c, int s, bool& valid) -> int64_t {
+    const int64_t f = c * kChunk + lane;
+    valid = f < total;
+    int64_t tok0 = 0;
+    if (valid) {
+      if (__ldg(block_off + r + 1) <= f) r = find_request(block_off, r + 1, n, f);
+      tok0 = __ldg(off + r) + (f - __ldg(block_off + r)) * B;
+    }
+    const int nv = __popc(__ballot_sync(kFull, valid));
+    const int32_t r0 = __shfl_sync(kFull, r, 0);
+    const int64_t a0 = (4 * __shfl_sync(kFull, tok0, 0)) & ~(int64_t)15;
+    const int k = (int)((a0 % (4 * B)) >> 4);
+    const int64_t y0 = a0 / (4 * B);
+    const bool one_request = __all_sync(kFull, !valid || r == r0);
+    unsigned char* const st = stages + (size_t)s * STAGE;
+    const uint32_t mbar = mbar0 + 8u * (uint32_t)s;
+    if (one_request && y0 + nv <= (int64_t)maps.rows[k]) {
+      if (lane == 0) {
+        asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+        mbar_arrive_expect_tx(mbar, STAGE);
+        tma_rows(smem_u32(st), &maps.map[k], (int32_t)y0, mbar, policy);
+      }
+    } else {
+      // lanes copy their own rows; the stage's barrier completes on lane 0's
+      // arrival with no bytes expected
+      if (valid) {
+        const int64_t a = (4 * tok0) & ~(int64_t)15;
+        uint4* row = reinterpret_cast<uint4*>(st + lane * ROW);
+#pragma unroll
+        for (int i = 0; i < NP; ++i) row[i] = load_piece(tb, a + 16 * i, token_bytes - (a + 16 * i));
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive_expect_tx(mbar, 0);
+    }
+    return tok0;
+  };
+
+  uint32_t phase = 0;
+  bool failed = false;
+  bool v[STAGES];
+  int64_t t[STAGES];
+#pragma unroll
+  for (int s = 0; s < STAGES; ++s)
+    if (c_lo + s < c_hi) t[s] = issue(c_lo + s, s, v[s]);
+  int s = 0;
+  for (int64_t c = c_lo; c < c_hi; ++c) {
+    if (!mbar_wait(mbar0 + 8u * (uint32_t)s, (phase >> s) & 1)) { failed = true; break; }
+    phase ^= 1u << s;
+    bool vc = false;
+    int64_t tc = 0;
+#pragma unroll
+    for (int q = 0; q < STAGES; ++q) if (q == s) { vc = v[q]; tc = t[q]; }
+    if (vc) {
+      const int delta = (int)((tc * 4) & 15);  // 0, 4, 8 or 12
+      const uint64_t* row = reinterpret_cast<const uint64_t*>(stages + (size_t)s * STAGE + lane * ROW) + (delta >> 3);
+      digest[c * kChunk + lane] = digest_row<HB>(row, (delta & 4) != 0, HB, d_init);
+    }
+    __syncwarp();
+    if (c + STAGES < c_hi) {
+      bool vn;
+      const int64_t tn = issue(c + STAGES, s, vn);
+#pragma unroll
+      for (int q = 0; q < STAGES; ++q) if (q == s) { v[q] = vn; t[q] = tn; }
+    }
+    s = s + 1 == STAGES ? 0 : s + 1;
+  }
+  if (failed) {
+    // a copy never completed: report it and give copies in flight a bounded
+    // chance to land before the shared memory is released
+    if (lane == 0) latch_error(status, SMETRIC_ERR_CUDA);
+#pragma unroll
+    for (int q = 0; q < STAGES; ++q) mbar_wait(mbar0 + 8u * q, (phase >> q) & 1);
+  }
+}
+
 // Any even B: each lane copies its own row straight from global memory.
 __global__ void __launch_bounds__(kDigestWarps * 32)
     k_digest_any(const int32_t* __restrict__ tokens, int64_t n_tokens, const int64_t* __restrict__ off,
@@ -384,11 +545,15 @@ __global__ void __launch_bounds__(256)
   }
 }
 
-// One warp per request, lanes = 32 consecutive blocks: the running AND of the
-// local-tier masks (a shuffle scan across lanes), the block where each
-// instance's run ends (ballot + ffs, recorded in shared memory), the
-// global-tier run; then lanes = instances for the cost and a shuffle argmin
-// with ties to the lowest id.
+// One warp per request, lanes = 32 consecutive blocks. The masks are
+// AND-scanned across lanes; lane j's "death set" is the local tiers held
+// through block j-1 but not through block j. Lanes with a non-empty death set
+// append an event (block, set) to the warp's list in shared memory; a request
+// has at most one event per instance and usually two or three in all. The
+// global-tier run is the first lane whose block the global tier lacks. Then
+// lanes = instances: c_i = the block of the first event containing i (or n_r
+// if i held every block), the cost, and a shuffle argmin with ties to the
+// lowest id.
 template <int W>
 __global__ void __launch_bounds__(kMatchWarps * 32)
     k_walk(int N, int B, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n,
@@ -399,13 +564,16 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
   extern __shared__ int64_t msm[];
   int64_t* load_s = msm;                                                     // [N]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  int32_t* death = reinterpret_cast<int32_t*>(msm + N) + warp * N;           // [warps][N]
+  // per warp: N events of (block, W mask words)
+  uint64_t* ev_mask = reinterpret_cast<uint64_t*>(msm + N) + (size_t)warp * N * W;
+  int64_t* ev_pos = msm + N + (size_t)kMatchWarps * N * W + (size_t)warp * N;
   for (int i = threadIdx.x; i < N; i += blockDim.x) load_s[i] = load[i];
   __syncthreads();
   const bool ok = *batch_ok != 0;
   const int gword = N >> 6;
   const uint64_t gbit = 1ull << (N & 63);
   const int64_t tw = (int64_t)gridDim.x * kMatchWarps;
+  const unsigned lt = (1u << lane) - 1;
 
   for (int64_t r = (int64_t)blockIdx.x * kMatchWarps + warp; r < n; r += tw) {
     if (!ok) {
@@ -423,78 +591,85 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
     }
     bool galive = true;
     int64_t g = 0;
+    int ne = 0;
     uint64_t nx[W];
 #pragma unroll
     for (int w = 0; w < W; ++w) nx[w] = lane < nb ? __ldg(m_r + lane * W + w) : 0;
     for (int64_t base = 0; base < nb; base += 32) {
       const bool valid = base + lane < nb;
-      uint64_t M[W];
+      uint64_t x[W];
 #pragma unroll
       for (int w = 0; w < W; ++w) {
-        M[w] = nx[w];
+        x[w] = valid ? nx[w] : 0;
         nx[w] = base + 32 + lane < nb ? __ldg(m_r + (base + 32 + lane) * W + w) : 0;
       }
-      // global-tier run: first lane whose block the global tier lacks
       if (galive) {
         uint64_t mg = 0;
 #pragma unroll
-        for (int w = 0; w < W; ++w) if (w == gword) mg = M[w];
-        const unsigned miss = __ballot_sync(kFull, !(valid && (mg & gbit)));
+        for (int w = 0; w < W; ++w) if (w == gword) mg = x[w];
+        const unsigned miss = __ballot_sync(kFull, !(mg & gbit));
         if (miss) { g = base + __ffs(miss) - 1; galive = false; }
         else g = base + 32;
       }
-      // local runs: inclusive AND-scan of the masks across lanes
-      bool any = false;
+      bool dies = false, any = false;
+      uint64_t X[W];
 #pragma unroll
       for (int w = 0; w < W; ++w) {
-        uint64_t x = valid ? M[w] : 0;
+        uint64_t v = x[w];
 #pragma unroll
-        for (int d = 1; d < 32; d <<= 1) {
-          const uint64_t y = __shfl_up_sync(kFull, x, d);
-          if (lane >= d) x &= y;
+        for (int dd = 1; dd < 32; dd <<= 1) {
+          const uint64_t y = __shfl_up_sync(kFull, v, dd);
+          if (lane >= dd) v &= y;
         }
-        x &= A[w];                                   // held through block base + lane
-        const uint64_t last = __shfl_sync(kFull, x, 31);
-        uint64_t dead = A[w] & ~last;                // runs that end in this chunk
-        while (dead) {
-          const int bit = __ffsll((long long)dead) - 1;
-          dead &= dead - 1;
-          const unsigned gone = __ballot_sync(kFull, !((x >> bit) & 1));
-          if (lane == 0) death[w * 64 + bit] = (int32_t)(base + __ffs(gone) - 1);
-        }
-        A[w] = last;
-        any |= last != 0;
+        v &= A[w];                                     // held through block base + lane
+        const uint64_t prev = __shfl_up_sync(kFull, v, 1);
+        X[w] = (lane ? prev : A[w]) & ~v;              // runs that end at block base + lane
+        dies |= X[w] != 0;
+        A[w] = __shfl_sync(kFull, v, 31);
+        any |= A[w] != 0;
       }
+      const unsigned ev = __ballot_sync(kFull, dies);
+      if (dies) {
+        const int at = ne + __popc(ev & lt);
+        ev_pos[at] = base + lane;
+#pragma unroll
+        for (int w = 0; w < W; ++w) ev_mask[at * W + w] = X[w];
+      }
+      ne += __popc(ev);
       if (!any && !galive) break;
     }
     __syncwarp();
     // cost of every instance; lanes = instances
     int64_t best_cost = INT64_MAX;
     int32_t best = N;
+    int64_t best_c = 0;
     for (int i = lane; i < N; i += 32) {
+      const int wi = i >> 6;
+      const uint64_t bi = 1ull << (i & 63);
       uint64_t aw = 0;
 #pragma unroll
-      for (int w = 0; w < W; ++w) if (w == (i >> 6)) aw = A[w];
-      const int64_t ci = ((aw >> (i & 63)) & 1) ? nb : (int64_t)death[i];
+      for (int w = 0; w < W; ++w) if (w == wi) aw = A[w];
+      int64_t ci = nb;
+      if (!(aw & bi)) {
+        for (int e = 0; e < ne; ++e)
+          if (ev_mask[e * W + wi] & bi) { ci = ev_pos[e]; break; }
+      }
       const int64_t gi = ci > g ? ci : g;
       const int64_t cost = w_load * load_s[i] + w_miss * (L - B * gi) + w_glob * B * (gi - ci);
-      if (cost < best_cost) { best_cost = cost; best = i; }
+      if (cost < best_cost) { best_cost = cost; best = i; best_c = ci; }
     }
 #pragma unroll
-    for (int d = 16; d > 0; d >>= 1) {
-      const int64_t oc = __shfl_xor_sync(kFull, best_cost, d);
-      const int32_t oi = __shfl_xor_sync(kFull, best, d);
-      if (oc < best_cost || (oc == best_cost && oi < best)) { best_cost = oc; best = oi; }
+    for (int dd = 16; dd > 0; dd >>= 1) {
+      const int64_t oc = __shfl_xor_sync(kFull, best_cost, dd);
+      const int32_t oi = __shfl_xor_sync(kFull, best, dd);
+      const int64_t ocb = __shfl_xor_sync(kFull, best_c, dd);
+      if (oc < best_cost || (oc == best_cost && oi < best)) { best_cost = oc; best = oi; best_c = ocb; }
     }
     if (lane == 0) {
-      uint64_t aw = 0;
-#pragma unroll
-      for (int w = 0; w < W; ++w) if (w == (best >> 6)) aw = A[w];
-      const int64_t cb = ((aw >> (best & 63)) & 1) ? nb : (int64_t)death[best];
-      const int64_t gb = cb > g ? cb : g;
+      const int64_t gb = best_c > g ? best_c : g;
       inst_out[r] = best;
-      lhit_out[r] = (int32_t)(B * cb);
-      ghit_out[r] = (int32_t)(B * (gb - cb));
+      lhit_out[r] = (int32_t)(B * best_c);
+      ghit_out[r] = (int32_t)(B * (gb - best_c));
     }
     __syncwarp();
   }
@@ -506,13 +681,85 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
 
 void profile_mark(smetric_index* idx, int k, cudaStream_t s);
 
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*,
+                                  CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                  CUtensorMapFloatOOBfill);
+
+EncodeTiledFn tensor_map_encoder() {
+  static EncodeTiledFn fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", reinterpret_cast<void**>(&fn), 12000,
+                                         cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      fn = nullptr;
+  }
+  return fn;
+}
+
+// One map per 16-byte phase k of a row start: base tokens + 16k, rows of
+// 4B+16 bytes at stride 4B, as many rows as fit inside the token buffer.
+bool make_token_maps(TokenMaps& m, const int32_t* tokens, int64_t n_tokens, int B) {
+  EncodeTiledFn enc = tensor_map_encoder();
+  if (!enc) return false;
+  memset(&m, 0, sizeof(m));
+  const int64_t bytes = 4 * n_tokens, row = 4 * B + 16, stride = 4 * B;
+  for (int k = 0; k < B / 4; ++k) {
+    const int64_t base = 16 * k;
+    if (bytes < base + row) continue;  // rows[k] = 0: chunks fall back to lane copies
+    int64_t rows = (bytes - base - row) / stride + 1;
+    if (rows > INT32_MAX) rows = INT32_MAX;
+    const cuuint64_t dims[2] = {(cuuint64_t)(B + 4), (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)stride};
+    const cuuint32_t box[2] = {(cuuint32_t)(B + 4), (cuuint32_t)kChunk};
+    const cuuint32_t es[2] = {1, 1};
+    if (enc(&m.map[k], CU_TENSOR_MAP_DATA_TYPE_UINT32, 2,
+            const_cast<char*>(reinterpret_cast<const char*>(tokens)) + base, dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return false;
+    m.rows[k] = (uint32_t)rows;
+  }
+  return true;
+}
+
+constexpr int kTmaStages = 2;
+
 template <int HB>
 int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
                   const int64_t* d_offsets, int32_t n, cudaStream_t s) {
   const int B = idx->cfg.block_size;
+  const uint64_t d_init = mix64(idx->cfg.hash_seed ^ (uint64_t)B);
+  const int64_t max_chunks = (n_tokens / B + kChunk - 1) / kChunk;
   // rows of 16*nch bytes: a block's 4B bytes start at most 12 bytes past a
   // 16-byte boundary
   const int nch = HB > 0 ? HB / 2 + 1 : (4 * B + 12 + 15) / 16;
+  if (HB > 0 && B / 4 <= kMaxPhases) {
+    static thread_local TokenMaps maps;
+    if (make_token_maps(maps, d_tokens, n_tokens, B)) {
+      auto kern = k_digest_tma<(HB > 0 ? HB : 2), kTmaStages>;
+      const size_t per_warp = (size_t)kTmaStages * kChunk * nch * 16 + 8 * kTmaStages;
+      const int warps = kDigestWarps;
+      const size_t smem = (size_t)warps * per_warp;
+      if (idx->digest_occ == 0) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+          return cuda_status(cudaErrorInvalidValue);
+        int occ = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, warps * 32, smem) != cudaSuccess)
+          return cuda_status(cudaErrorInvalidValue);
+        idx->digest_occ = occ < 1 ? 1 : occ;
+      }
+      const int64_t want = (max_chunks + warps - 1) / warps;
+      const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * idx->digest_occ));
+      kern<<<(unsigned)grid, warps * 32, smem, s>>>(maps, d_tokens, n_tokens, d_offsets, idx->block_off, n,
+                                                    d_init, idx->batch_ok, idx->digest, idx->status);
+      idx->launches++;
+      return cuda_status(cudaGetLastError());
+    }
+  }
   const size_t per_warp = (size_t)kChunk * nch * 16;
   const int warps = (int)std::max<size_t>(1, std::min<size_t>(kDigestWarps, (200 * 1024) / per_warp));
   const size_t smem = (size_t)warps * per_warp;
@@ -526,10 +773,8 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
       return cuda_status(cudaErrorInvalidValue);
     idx->digest_occ = occ < 1 ? 1 : occ;
   }
-  const int64_t max_chunks = (n_tokens / B + kChunk - 1) / kChunk;
   const int64_t want = (max_chunks + warps - 1) / warps;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * idx->digest_occ));
-  const uint64_t d_init = mix64(idx->cfg.hash_seed ^ (uint64_t)B);
   if (HB > 0)
     kern<<<(unsigned)grid, warps * 32, smem, s>>>(d_tokens, n_tokens, d_offsets, idx->block_off, n, d_init,
                                                   idx->batch_ok, idx->digest);
@@ -563,21 +808,23 @@ int launch_chain(smetric_index* idx, const int64_t* d_offsets, int32_t n, uint64
 
 template <int W>
 int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
-                 smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, const uint64_t* H,
-                 int64_t max_blocks, cudaStream_t s) {
+                 smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, uint64_t* hashes,
+                 uint64_t* sk, int64_t max_blocks, cudaStream_t s) {
   const int N = idx->cfg.num_instances;
-  // probe: one thread per block, grid sized to the largest possible batch
+  int rc = launch_chain(idx, d_offsets, n, hashes, sk, s);
+  if (rc) return rc;
+  profile_mark(idx, kChain, s);
   {
+    // probe: one thread per block, grid sized to the largest possible batch
     const int64_t want = (max_blocks + 255) / 256;
     const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
-    k_probe<W><<<(unsigned)grid, 256, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->block_off, n, H,
-                                              idx->batch_ok, idx->masks);
+    k_probe<W><<<(unsigned)grid, 256, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->block_off, n,
+                                              hashes ? hashes : idx->hashes, idx->batch_ok, idx->masks);
     idx->launches++;
-    int rc = cuda_status(cudaGetLastError());
-    if (rc) return rc;
+    if ((rc = cuda_status(cudaGetLastError()))) return rc;
   }
   profile_mark(idx, kProbe, s);
-  const size_t smem = (size_t)N * sizeof(int64_t) + (size_t)kMatchWarps * N * sizeof(int32_t);
+  const size_t smem = (size_t)N * sizeof(int64_t) + (size_t)kMatchWarps * N * (W + 1) * sizeof(uint64_t);
   auto kern = k_walk<W>;
   if (smem > 48 * 1024 &&
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
@@ -592,14 +839,14 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
 }
 
 int dispatch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
-                   smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, const uint64_t* H,
-                   int64_t max_blocks, cudaStream_t s) {
+                   smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, uint64_t* hashes,
+                   uint64_t* sk, int64_t max_blocks, cudaStream_t s) {
   switch (idx->W) {
-    case 1: return launch_match<1>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, H, max_blocks, s);
-    case 2: return launch_match<2>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, H, max_blocks, s);
-    case 3: return launch_match<3>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, H, max_blocks, s);
-    case 4: return launch_match<4>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, H, max_blocks, s);
-    case 5: return launch_match<5>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, H, max_blocks, s);
+    case 1: return launch_match<1>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, s);
+    case 2: return launch_match<2>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, s);
+    case 3: return launch_match<3>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, s);
+    case 4: return launch_match<4>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, s);
+    case 5: return launch_match<5>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, s);
     default: return SMETRIC_ERR_INVALID_ARG;
   }
 }
@@ -653,12 +900,14 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
     if ((rc = dispatch_digest(idx, d_tokens, n_tokens, d_offsets, n, s))) return rc;
   }
   profile_mark(idx, kDigest, s);
-  if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, s))) return rc;
-  profile_mark(idx, kChain, s);
   if (PROBE) {
-    if ((rc = dispatch_match(idx, d_offsets, n, d_load, w, inst, lhit, ghit,
-                             hashes ? hashes : idx->hashes, n_tokens / c.block_size, s)))
+    if ((rc = dispatch_match(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk,
+                             n_tokens / c.block_size, s)))
       return rc;
+  } else {
+    if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, s))) return rc;
+    profile_mark(idx, kChain, s);
+    profile_mark(idx, kProbe, s);
   }
   profile_mark(idx, kWalk, s);
   return SMETRIC_OK;
