@@ -192,6 +192,8 @@ void free_all(smetric_index* x) {
   cudaFree(x->digest);
   cudaFree(x->hashes);
   cudaFree(x->masks);
+  cudaFree(x->groups);
+  cudaFree(x->lead);
   cudaFree(x->batch_ok);
   cudaFree(x->st_tokens);
   cudaFree(x->st_offsets);
@@ -238,6 +240,8 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
   const size_t table_bytes = slots * x->EW * sizeof(uint64_t);
   const size_t max_blocks = (size_t)(c.max_batch_tokens / c.block_size);
   const size_t R = (size_t)c.max_batch_requests;
+  x->group_slots = 64;
+  while (x->group_slots < 2 * (uint64_t)R) x->group_slots <<= 1;
   bool ok = cudaMalloc(&x->table, table_bytes) == cudaSuccess &&
             cudaMalloc(&x->tags, slots) == cudaSuccess &&
             cudaMalloc(&x->status, sizeof(int32_t)) == cudaSuccess &&
@@ -245,7 +249,10 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
             cudaMalloc(&x->digest, (max_blocks > 0 ? max_blocks : 1) * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->hashes, (max_blocks > 0 ? max_blocks : 1) * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->masks, (max_blocks > 0 ? max_blocks : 1) * W * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&x->groups, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&x->lead, 2 * (R + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->batch_ok, sizeof(int32_t)) == cudaSuccess;
+  if (ok) x->share = x->lead + (R + 1);
   if (ok && (c.flags & SMETRIC_FLAG_HOST_STAGING)) {
     const size_t T = (size_t)(c.max_batch_tokens > 0 ? c.max_batch_tokens : 1);
     ok = cudaMalloc(&x->st_tokens, T * sizeof(int32_t)) == cudaSuccess &&

@@ -38,7 +38,6 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kChunk = 32;        // blocks per digest task (one per lane)
 constexpr int kDigestWarps = 8;   // most warps per digest CTA
-constexpr int kStages = 2;        // shared-memory stages per warp
 constexpr int kChainThreads = 128;
 constexpr int kChainAhead = 16;   // digests prefetched per request
 constexpr int kMatchWarps = 8;    // warps per walk CTA
@@ -59,7 +58,8 @@ __device__ __forceinline__ int64_t warp_incl_scan(int64_t v, int lane) {
 __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, int32_t n,
                                               int64_t n_tokens, int B, const int64_t* __restrict__ load,
                                               int n_load, int64_t* __restrict__ block_off,
-                                              int32_t* batch_ok, int32_t* status) {
+                                              int32_t* batch_ok, int32_t* status,
+                                              uint4* __restrict__ groups, int64_t group_vecs) {
   __shared__ int64_t warp_tot[32];
   __shared__ int bad_all;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -96,6 +96,7 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
     if (a >= 0 && b >= a && b - a <= (int64_t)INT32_MAX) run += (b - a) / B;
   }
   if (tid == (int)blockDim.x - 1) block_off[n] = warp_tot[warp] + incl;
+  for (int64_t i = tid; i < group_vecs; i += blockDim.x) groups[i] = make_uint4(0, 0, 0, 0);
   __syncthreads();
   if (tid == 0) {
     const int ba = bad_all;
@@ -173,7 +174,7 @@ __global__ void __launch_bounds__(kDigestWarps * 32)
              const int64_t* __restrict__ block_off, int32_t n, uint64_t d_init,
              const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ digest) {
   constexpr int B = 2 * HB;
-  constexpr int PB = HB / 2;  // 16-byte pieces per block
+  constexpr int PB = HB > 0 ? HB / 2 : 1;  // 16-byte pieces per block (k_digest<0> is never launched)
   constexpr int NP = PB + 1;  // pieces per row (the block plus its misalignment)
   extern __shared__ uint4 dsm[];
   if (!*batch_ok) return;
@@ -454,11 +455,28 @@ __global__ void __launch_bounds__(kDigestWarps * 32)
 // chain
 // ---------------------------------------------------------------------------
 
+// Requests whose first block hashes are equal form a group; its leader is
+// the lowest request id. Table of (key, INT32_MAX - leader) word pairs,
+// key 0 = empty (block hashes are >= 2), linear probing, at most half full.
+__device__ __forceinline__ void group_insert(uint64_t* __restrict__ groups, uint64_t gmask, uint64_t key,
+                                             int32_t r) {
+  uint64_t s = key & gmask;
+  for (uint64_t t = 0; t <= gmask; ++t) {
+    unsigned long long* const slot = reinterpret_cast<unsigned long long*>(groups + 2 * s);
+    const unsigned long long k = atomicCAS(slot, 0ull, (unsigned long long)key);
+    if (k == 0ull || k == key) {
+      atomicMax(slot + 1, (unsigned long long)(INT32_MAX - r));
+      return;
+    }
+    s = (s + 1) & gmask;
+  }
+}
+
 __global__ void __launch_bounds__(kChainThreads)
     k_chain(const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n, int B,
             int S, uint64_t h_init, const int32_t* __restrict__ batch_ok,
             const uint64_t* __restrict__ digest, uint64_t* __restrict__ hashes,
-            uint64_t* __restrict__ sk_out) {
+            uint64_t* __restrict__ sk_out, uint64_t* __restrict__ groups, uint64_t gmask) {
   const int32_t r = blockIdx.x * kChainThreads + threadIdx.x;
   if (r >= n) return;
   if (!*batch_ok) { sk_out[r] = 0; return; }
@@ -467,7 +485,7 @@ __global__ void __launch_bounds__(kChainThreads)
   const uint64_t* const d = digest + bo;
   uint64_t* const hout = hashes + bo;
   const int64_t kS = (nb < S ? nb : S) - 1;
-  uint64_t h = h_init, sk = 0;
+  uint64_t h = h_init, sk = 0, h0 = 0;
   uint64_t cur[kChainAhead], nxt[kChainAhead];
 #pragma unroll
   for (int j = 0; j < kChainAhead; ++j) cur[j] = j < nb ? __ldg(d + j) : 0;
@@ -482,12 +500,67 @@ __global__ void __launch_bounds__(kChainThreads)
         if (h < 2) h |= 2;
         hout[b0 + j] = h;
         if (b0 + j == kS) sk = h;
+        if (b0 + j == 0) h0 = h;
       }
     }
 #pragma unroll
     for (int j = 0; j < kChainAhead; ++j) cur[j] = nxt[j];
   }
   sk_out[r] = nb > 0 ? sk : 0;
+  if (groups && nb > 0) group_insert(groups, gmask, h0, r);
+}
+
+// ---------------------------------------------------------------------------
+// group
+// ---------------------------------------------------------------------------
+
+// One warp per request: its leader (the group table's entry for its first
+// block hash) and share = the number of leading blocks whose hashes equal the
+// leader's. Both sides look up the same finished table, so a request that
+// leads a group finds itself (share 0) and its masks cover all its blocks;
+// a member's mask for block b < share is the leader's, which is exact because
+// a block's tier masks are a function of its hash alone.
+__global__ void __launch_bounds__(256)
+    k_group(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
+            const uint64_t* __restrict__ groups, uint64_t gmask, const uint64_t* __restrict__ H,
+            int32_t* __restrict__ lead, int32_t* __restrict__ share) {
+  if (!*batch_ok) return;
+  const int lane = threadIdx.x & 31;
+  const int64_t tw = (int64_t)gridDim.x * (blockDim.x >> 5);
+  for (int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n; r += tw) {
+    const int64_t bo = block_off[r], nb = block_off[r + 1] - bo;
+    int32_t l = (int32_t)r;
+    int64_t sh = 0;
+    if (nb > 0) {
+      const uint64_t key = __ldg(H + bo);
+      const uint64_t s0 = key & gmask;
+      for (uint64_t t = 0; t <= gmask; t += 32) {
+        const uint64_t sl = (s0 + t + lane) & gmask;
+        const uint64_t k = groups[2 * sl];
+        const unsigned hit = __ballot_sync(kFull, k == key), emp = __ballot_sync(kFull, k == 0);
+        const unsigned stop = hit | emp;
+        if (stop) {
+          const int first = __ffs(stop) - 1;
+          if (hit & (1u << first))
+            l = INT32_MAX - (int32_t)groups[2 * ((s0 + t + first) & gmask) + 1];
+          break;
+        }
+      }
+      if (l != (int32_t)r && l >= 0 && l < n) {
+        const int64_t lo = block_off[l], nl = block_off[l + 1] - lo;
+        const int64_t m = nb < nl ? nb : nl;
+        sh = m;
+        for (int64_t b = 0; b < m; b += 32) {
+          const bool ne = b + lane < m && __ldg(H + bo + b + lane) != __ldg(H + lo + b + lane);
+          const unsigned x = __ballot_sync(kFull, ne);
+          if (x) { sh = b + __ffs(x) - 1; break; }
+        }
+      } else {
+        l = (int32_t)r;
+      }
+    }
+    if (lane == 0) { lead[r] = l; share[r] = (int32_t)sh; }
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -533,11 +606,15 @@ template <int W>
 __global__ void __launch_bounds__(256)
     k_probe(const uint8_t* __restrict__ tags, const uint64_t* __restrict__ table, uint64_t n_buckets,
             const int64_t* __restrict__ block_off, int32_t n, const uint64_t* __restrict__ H,
-            const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ masks) {
+            const int32_t* __restrict__ batch_ok, const int32_t* __restrict__ share,
+            uint64_t* __restrict__ masks) {
   if (!*batch_ok) return;
   const int64_t total = block_off[n];
+  int32_t r = 0;
   for (int64_t f = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; f < total;
        f += (int64_t)gridDim.x * blockDim.x) {
+    r = find_request(block_off, r, n, f);
+    if (f - __ldg(block_off + r) < __ldg(share + r)) continue;  // the leader's mask serves
     uint64_t M[W];
     probe_one<W>(tags, table, n_buckets, __ldg(H + f), M);
 #pragma unroll
@@ -559,6 +636,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
     k_walk(int N, int B, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n,
            const int64_t* __restrict__ load, int64_t w_load, int64_t w_miss, int64_t w_glob,
            const uint64_t* __restrict__ masks, const int32_t* __restrict__ batch_ok,
+           const int32_t* __restrict__ lead, const int32_t* __restrict__ share,
            int32_t* __restrict__ inst_out, int32_t* __restrict__ lhit_out,
            int32_t* __restrict__ ghit_out) {
   extern __shared__ int64_t msm[];
@@ -583,6 +661,8 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
     const int64_t L = off[r + 1] - off[r];
     const int64_t nb = L / B;
     const uint64_t* const m_r = masks + block_off[r] * W;
+    const uint64_t* const m_l = masks + block_off[lead[r]] * W;
+    const int64_t sh = share[r];
     uint64_t A[W];  // local tiers holding every block so far (warp-uniform)
 #pragma unroll
     for (int w = 0; w < W; ++w) {
@@ -594,14 +674,15 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
     int ne = 0;
     uint64_t nx[W];
 #pragma unroll
-    for (int w = 0; w < W; ++w) nx[w] = lane < nb ? __ldg(m_r + lane * W + w) : 0;
+    for (int w = 0; w < W; ++w) nx[w] = lane < nb ? __ldg((lane < sh ? m_l : m_r) + lane * W + w) : 0;
     for (int64_t base = 0; base < nb; base += 32) {
       const bool valid = base + lane < nb;
       uint64_t x[W];
 #pragma unroll
       for (int w = 0; w < W; ++w) {
         x[w] = valid ? nx[w] : 0;
-        nx[w] = base + 32 + lane < nb ? __ldg(m_r + (base + 32 + lane) * W + w) : 0;
+        const int64_t bn = base + 32 + lane;
+        nx[w] = bn < nb ? __ldg((bn < sh ? m_l : m_r) + bn * W + w) : 0;
       }
       if (galive) {
         uint64_t mg = 0;
@@ -795,13 +876,21 @@ int dispatch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_token
   }
 }
 
+// Group-table slots a batch of n requests uses: a power of two >= 2n.
+uint64_t group_slots_for(int32_t n) {
+  uint64_t g = 64;
+  while (g < 2 * (uint64_t)n) g <<= 1;
+  return g;
+}
+
 int launch_chain(smetric_index* idx, const int64_t* d_offsets, int32_t n, uint64_t* hashes,
-                 uint64_t* sk, cudaStream_t s) {
+                 uint64_t* sk, bool group, cudaStream_t s) {
   const unsigned grid = (unsigned)((n + kChainThreads - 1) / kChainThreads);
   const uint64_t h_init = mix64(idx->cfg.hash_seed + kGamma);
   k_chain<<<grid, kChainThreads, 0, s>>>(d_offsets, idx->block_off, n, idx->cfg.block_size,
                                          idx->cfg.session_blocks, h_init, idx->batch_ok, idx->digest,
-                                         hashes ? hashes : idx->hashes, sk);
+                                         hashes ? hashes : idx->hashes, sk, group ? idx->groups : nullptr,
+                                         group_slots_for(n) - 1);
   idx->launches++;
   return cuda_status(cudaGetLastError());
 }
@@ -811,15 +900,25 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
                  smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, uint64_t* hashes,
                  uint64_t* sk, int64_t max_blocks, cudaStream_t s) {
   const int N = idx->cfg.num_instances;
-  int rc = launch_chain(idx, d_offsets, n, hashes, sk, s);
+  const uint64_t* H = hashes ? hashes : idx->hashes;
+  int rc = launch_chain(idx, d_offsets, n, hashes, sk, true, s);
   if (rc) return rc;
   profile_mark(idx, kChain, s);
+  {
+    const int64_t want = ((int64_t)n + 7) / 8;
+    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
+    k_group<<<(unsigned)grid, 256, 0, s>>>(idx->block_off, n, idx->batch_ok, idx->groups,
+                                           group_slots_for(n) - 1, H, idx->lead, idx->share);
+    idx->launches++;
+    if ((rc = cuda_status(cudaGetLastError()))) return rc;
+  }
+  profile_mark(idx, kGroup, s);
   {
     // probe: one thread per block, grid sized to the largest possible batch
     const int64_t want = (max_blocks + 255) / 256;
     const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
-    k_probe<W><<<(unsigned)grid, 256, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->block_off, n,
-                                              hashes ? hashes : idx->hashes, idx->batch_ok, idx->masks);
+    k_probe<W><<<(unsigned)grid, 256, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->block_off, n, H,
+                                              idx->batch_ok, idx->share, idx->masks);
     idx->launches++;
     if ((rc = cuda_status(cudaGetLastError()))) return rc;
   }
@@ -833,7 +932,7 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
   kern<<<(unsigned)grid, kMatchWarps * 32, smem, s>>>(N, idx->cfg.block_size, d_offsets, idx->block_off, n,
                                                       d_load, w.w_load, w.w_miss, w.w_glob, idx->masks,
-                                                      idx->batch_ok, inst, lhit, ghit);
+                                                      idx->batch_ok, idx->lead, idx->share, inst, lhit, ghit);
   idx->launches++;
   return cuda_status(cudaGetLastError());
 }
@@ -892,7 +991,8 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
 
   profile_begin(idx, s);
   k_prep<<<1, 1024, 0, s>>>(d_offsets, n, n_tokens, c.block_size, d_load, PROBE ? c.num_instances : 0,
-                            idx->block_off, idx->batch_ok, idx->status);
+                            idx->block_off, idx->batch_ok, idx->status, reinterpret_cast<uint4*>(idx->groups),
+                            PROBE ? (int64_t)group_slots_for(n) : 0);
   idx->launches++;
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   profile_mark(idx, kPrep, s);
@@ -905,8 +1005,9 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
                              n_tokens / c.block_size, s)))
       return rc;
   } else {
-    if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, s))) return rc;
+    if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, false, s))) return rc;
     profile_mark(idx, kChain, s);
+    profile_mark(idx, kGroup, s);
     profile_mark(idx, kProbe, s);
   }
   profile_mark(idx, kWalk, s);
@@ -1005,6 +1106,7 @@ const char* smetric_profile_kernel_name(int32_t k) {
     case kPrep: return "k_prep";
     case kDigest: return "k_digest";
     case kChain: return "k_chain";
+    case kGroup: return "k_group";
     case kProbe: return "k_probe";
     case kWalk: return "k_walk";
     default: return "";

@@ -178,6 +178,53 @@ def test_route_matches_oracle_tiny_alphabet(N, B):
         ix.close()
 
 
+def test_route_requests_sharing_leading_blocks():
+    """Requests with equal first blocks share their leader's probes up to the
+    first differing block: members that are prefixes of the leader, extend
+    it, diverge at block 0, 1, in the middle or only in the partial tail, a
+    hot group of hundreds of members, a leader shorter than its members,
+    empty and sub-block requests, all interleaved in one batch."""
+    rng = np.random.default_rng(31)
+    N, B = 64, 16
+    bases = [rng.integers(0, 151936, size=int(rng.integers(20, 60)) * B + 7, dtype=np.int32)
+             for _ in range(6)]
+    reqs = []
+    for i, base in enumerate(bases):
+        nb = len(base) // B
+        reqs.append(base[:B * 3])                                        # shortest: the leader when first
+        reqs.append(base.copy())
+        for cut in (0, 1, 2, nb // 2, nb - 1, nb):
+            tail = rng.integers(0, 151936, size=int(rng.integers(0, 5 * B)), dtype=np.int32)
+            reqs.append(np.concatenate([base[:cut * B], tail]))
+        reqs.append(np.concatenate([base, rng.integers(0, 151936, size=3 * B, dtype=np.int32)]))
+        reqs.append(base[:len(base) - 3])                                # differs only in the tail
+        if i == 0:
+            for _ in range(300):                                          # hot group
+                k = int(rng.integers(1, nb + 1))
+                reqs.append(np.concatenate([base[:k * B],
+                                            rng.integers(0, 151936, size=int(rng.integers(0, 40)),
+                                                         dtype=np.int32)]))
+    reqs += [np.zeros(0, np.int32), bases[1][:B - 1], bases[2][:B]]
+    order = np.concatenate([[0, 1], 2 + rng.permutation(len(reqs) - 2)])  # a short leader stays first
+    reqs = [reqs[j] for j in order]
+    stored = {}
+    for t in range(-1, N):
+        picks = rng.choice(len(bases), size=int(rng.integers(0, 3)), replace=False)
+        stored[t] = [bases[j][:int(rng.integers(0, len(bases[j]) + 1))] for j in picks]
+    ix = make_index(N, B, 2, cap=1 << 15)
+    ox = oracle.OracleIndex(N)
+    populate_both(ix, ox, stored, B)
+    tok, off = pack(reqs)
+    hits = np.zeros(2, np.int64)
+    for load in (rng.integers(0, 50, size=N), np.zeros(N, np.int64), rng.integers(0, 10**6, size=N)):
+        g = gpu_route(ix, tok, off, load, (1, 4, 2))
+        o = ox.route_batch(B, 2, 0, tok, off, load, 1, 4, 2, want_hashes=True)
+        assert_outputs_equal(g, o, ctx="shared leading blocks")
+        hits += [g["local_hit"].max(), g["global_hit"].max()]
+    assert hits.min() > 0  # both tiers contribute somewhere
+    ix.close()
+
+
 def test_route_special_cases():
     rng = np.random.default_rng(21)
     N, B = 9, 8
@@ -265,7 +312,7 @@ def test_profile_and_launch_count():
     for _ in range(3):
         gpu_route(ix, tok, off, np.zeros(4), (1, 4, 2))
     prof = pkg.smetric_profile_read(ix.handle)
-    assert set(prof) == {"k_prep", "k_digest", "k_chain", "k_probe", "k_walk"}
+    assert set(prof) == {"k_prep", "k_digest", "k_chain", "k_group", "k_probe", "k_walk"}
     assert all(v[1] == 3 and v[0] > 0 for v in prof.values())
-    assert pkg.smetric_launch_count(ix.handle) - before == 15
+    assert pkg.smetric_launch_count(ix.handle) - before == 18
     pkg.smetric_profile_enable(ix.handle, False)
