@@ -64,7 +64,8 @@ enum {
   SMETRIC_ERR_OOM = -2,         /* device allocation failed at create */
   SMETRIC_ERR_TABLE_FULL = -3,  /* an insert found no free slot */
   SMETRIC_ERR_CUDA = -4,        /* a CUDA runtime call failed */
-  SMETRIC_ERR_OVERFLOW = -5     /* a load or prompt length outside the exact int64 range */
+  SMETRIC_ERR_OVERFLOW = -5,    /* a load or prompt length outside the exact int64 range */
+  SMETRIC_ERR_TOO_LARGE = -6    /* batch larger than smetric_block_hashes_noalloc's fixed scratch */
 };
 
 /* Instance limit and the limits that keep every cost exact in int64:
@@ -167,6 +168,52 @@ int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_t
 int smetric_block_hashes(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
                          const int64_t* d_offsets, int32_t n_requests, uint64_t* d_session_key,
                          uint64_t* d_block_hashes, int64_t hashes_cap, smetric_stream_t stream);
+
+/* Limits of smetric_block_hashes_noalloc's fixed scratch. */
+#define SMETRIC_NOALLOC_MAX_REQUESTS 4096
+#define SMETRIC_NOALLOC_MAX_BLOCKS 32768
+
+/* smetric_block_hashes without an index and without allocating anything.
+ * The paper has no counterpart: this is a library convenience.
+ *
+ * Who needs it: a caller that must not allocate device memory at call time
+ * and has no index -- for example a request front-end that computes session
+ * keys and block hashes on a GPU whose memory a serving engine has already
+ * reserved in its own pools, or a latency-critical loop in which the device
+ * synchronisation that cudaMalloc/cudaFree imply would stall other streams.
+ * smetric_block_hashes needs an index, and smetric_index_create allocates the
+ * table and per-batch scratch; this call allocates nothing: no cudaMalloc,
+ * no cudaFree, no allocating library call.
+ *
+ * Scratch: one statically sized device array compiled into the library
+ * (request offsets and per-block digests, 295,424 bytes, one copy per device,
+ * existing from module load). The first call on each device, with that
+ * device current, looks up the array's device address once
+ * (cudaGetSymbolAddress) and caches it; make that first call before any
+ * stream capture on the device.
+ *
+ * Limits: n_requests <= SMETRIC_NOALLOC_MAX_REQUESTS and
+ * n_tokens / block_size <= SMETRIC_NOALLOC_MAX_BLOCKS; a larger batch returns
+ * SMETRIC_ERR_TOO_LARGE with nothing enqueued.
+ *
+ * Arguments are those of smetric_block_hashes, with the index configuration
+ * given directly (block_size B even in 2..256, session_blocks S >= 1, the
+ * hash seed) and one more:
+ *   d_status   int32 in device memory, owned by the caller; it MUST be 0 when
+ *              the call's kernels start. Invalid offsets latch
+ *              SMETRIC_ERR_INVALID_ARG and lengths of 2^31 or more latch
+ *              SMETRIC_ERR_OVERFLOW into it (first error wins); session keys
+ *              are then 0 and no hash is written.
+ * Host-detectable errors return immediately with nothing enqueued.
+ *
+ * Concurrency: every call on one device uses the same scratch. Calls whose
+ * kernels overlap (different streams or host threads without ordering
+ * between them) race on it and produce wrong results; order them on one
+ * stream or with events. */
+int smetric_block_hashes_noalloc(const int32_t* d_tokens, int64_t n_tokens, const int64_t* d_offsets,
+                                 int32_t n_requests, int32_t block_size, int32_t session_blocks,
+                                 uint64_t hash_seed, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                                 int64_t hashes_cap, int32_t* d_status, smetric_stream_t stream);
 
 /* smetric_route_batch from host buffers: copies tokens, offsets and load to
  * the index's staging buffers (the index must have been created with

@@ -24,6 +24,9 @@ SMETRIC_ERR_OOM = -2
 SMETRIC_ERR_TABLE_FULL = -3
 SMETRIC_ERR_CUDA = -4
 SMETRIC_ERR_OVERFLOW = -5
+SMETRIC_ERR_TOO_LARGE = -6
+SMETRIC_NOALLOC_MAX_REQUESTS = 4096
+SMETRIC_NOALLOC_MAX_BLOCKS = 32768
 SMETRIC_MAX_INSTANCES = 256
 SMETRIC_MAX_WEIGHT = 1 << 20
 SMETRIC_MAX_LOAD = 1 << 40
@@ -36,7 +39,7 @@ EXPORTED = (
     "smetric_index_mask_words", "smetric_route_batch", "smetric_block_hashes",
     "smetric_route_batch_host", "smetric_status", "smetric_strerror",
     "smetric_profile_enable", "smetric_profile_read", "smetric_profile_kernel_name",
-    "smetric_launch_count",
+    "smetric_launch_count", "smetric_block_hashes_noalloc",
 )
 
 
@@ -91,6 +94,8 @@ def lib():
             "smetric_route_batch": (C.c_int, [P, P, I64, P, I32, P, smetric_weights, P, P, P, P, P,
                                               I64, P]),
             "smetric_block_hashes": (C.c_int, [P, P, I64, P, I32, P, P, I64, P]),
+            "smetric_block_hashes_noalloc": (C.c_int, [P, I64, P, I32, I32, I32, C.c_uint64, P, P, I64,
+                                                      P, P]),
             "smetric_route_batch_host": (C.c_int, [P, P, I64, P, I32, P, smetric_weights, P, P, P,
                                                    P, P]),
             "smetric_status": (C.c_int, [P, P]),
@@ -197,6 +202,18 @@ def smetric_block_hashes(idx: int, d_tokens, n_tokens: int, d_offsets, n_request
     _check(lib().smetric_block_hashes(idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests,
                                       _ptr(d_session_key), _ptr(d_block_hashes), hashes_cap,
                                       _stream(stream)), "smetric_block_hashes")
+
+
+def smetric_block_hashes_noalloc(d_tokens, n_tokens: int, d_offsets, n_requests: int,
+                                 block_size: int, session_blocks: int, hash_seed: int,
+                                 d_session_key, d_block_hashes, hashes_cap: int, d_status,
+                                 stream=None) -> int:
+    """Returns the call's host-side status code (SMETRIC_ERR_TOO_LARGE for a
+    batch beyond the fixed scratch); device-detected errors land in d_status."""
+    return int(lib().smetric_block_hashes_noalloc(_ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests,
+                                                  block_size, session_blocks, hash_seed,
+                                                  _ptr(d_session_key), _ptr(d_block_hashes), hashes_cap,
+                                                  _ptr(d_status), _stream(stream)))
 
 
 def smetric_route_batch_host(idx: int, h_tokens, n_tokens: int, h_offsets, n_requests: int, h_load,

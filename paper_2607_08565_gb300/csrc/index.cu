@@ -344,6 +344,7 @@ const char* smetric_strerror(int code) {
     case SMETRIC_ERR_TABLE_FULL: return "index table full";
     case SMETRIC_ERR_CUDA: return "CUDA runtime error";
     case SMETRIC_ERR_OVERFLOW: return "value outside the exact integer range";
+    case SMETRIC_ERR_TOO_LARGE: return "batch larger than the fixed no-allocation scratch";
     default: return "unknown error";
   }
 }

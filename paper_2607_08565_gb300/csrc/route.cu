@@ -27,6 +27,7 @@
 #include <stdint.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cstring>
 
 #include "smetric_impl.cuh"
@@ -1114,3 +1115,111 @@ const char* smetric_profile_kernel_name(int32_t k) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// block hashes with fixed scratch and no allocation
+// ---------------------------------------------------------------------------
+
+namespace {
+
+// Word layout of the fixed scratch: the batch-valid flag, the per-request
+// first-block offsets, the per-block digests. Each part starts on a 256-byte
+// boundary. Nothing in it needs an initial value: every call writes the flag
+// and the offsets before any kernel reads them, and the digests of exactly
+// the blocks the chain reads.
+constexpr int64_t kNaFlagWords = 32;
+constexpr int64_t kNaOffWords = (SMETRIC_NOALLOC_MAX_REQUESTS + 1 + 31) / 32 * 32;
+constexpr int64_t kNaWords = kNaFlagWords + kNaOffWords + SMETRIC_NOALLOC_MAX_BLOCKS;
+static_assert(kNaWords * 8 == 295424, "the header states the scratch size");
+
+static __device__ __align__(256) uint64_t na_scratch[kNaWords];
+
+constexpr int kNaMaxDevices = 64;
+std::atomic<uint64_t*> na_addr[kNaMaxDevices];
+
+// Device address of na_scratch on the current device, looked up once per
+// device (the first call on a device should not be under stream capture).
+int na_scratch_for(int dev, uint64_t** out) {
+  if (dev < 0 || dev >= kNaMaxDevices) return SMETRIC_ERR_INVALID_ARG;
+  uint64_t* p = na_addr[dev].load(std::memory_order_acquire);
+  if (!p) {
+    if (cudaGetSymbolAddress(reinterpret_cast<void**>(&p), na_scratch) != cudaSuccess)
+      return cuda_status(cudaErrorInvalidSymbol);
+    na_addr[dev].store(p, std::memory_order_release);
+  }
+  *out = p;
+  return SMETRIC_OK;
+}
+
+template <int HB>
+int na_digest(const int32_t* d_tokens, int64_t n_tokens, const int64_t* d_offsets, const int64_t* block_off,
+              int32_t n, int B, int num_sms, uint64_t d_init, const int32_t* ok, uint64_t* digest,
+              cudaStream_t s) {
+  const int64_t max_chunks = (n_tokens / B + kChunk - 1) / kChunk;
+  const int nch = HB > 0 ? HB / 2 + 1 : (4 * B + 12 + 15) / 16;
+  const size_t per_warp = (size_t)kChunk * nch * 16;
+  const int warps = (int)std::max<size_t>(1, std::min<size_t>(kDigestWarps, (200 * 1024) / per_warp));
+  const size_t smem = (size_t)warps * per_warp;
+  const void* fn = HB > 0 ? (const void*)k_digest<(HB > 0 ? HB : 2)> : (const void*)k_digest_any;
+  int occ = 0;
+  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fn, warps * 32, smem) != cudaSuccess)
+    return cuda_status(cudaErrorInvalidValue);
+  const int64_t want = (max_chunks + warps - 1) / warps;
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)num_sms * std::max(occ, 1)));
+  if (HB > 0)
+    k_digest<(HB > 0 ? HB : 2)><<<(unsigned)grid, warps * 32, smem, s>>>(d_tokens, n_tokens, d_offsets,
+                                                                        block_off, n, d_init, ok, digest);
+  else
+    k_digest_any<<<(unsigned)grid, warps * 32, smem, s>>>(d_tokens, n_tokens, d_offsets, block_off, n, B, nch,
+                                                          d_init, ok, digest);
+  return cuda_status(cudaGetLastError());
+}
+
+}  // namespace
+
+extern "C" int smetric_block_hashes_noalloc(const int32_t* d_tokens, int64_t n_tokens,
+                                            const int64_t* d_offsets, int32_t n_requests, int32_t block_size,
+                                            int32_t session_blocks, uint64_t hash_seed,
+                                            uint64_t* d_session_key, uint64_t* d_block_hashes,
+                                            int64_t hashes_cap, int32_t* d_status, smetric_stream_t stream) {
+  const int B = block_size;
+  if (B < 2 || B > 256 || (B & 1) || session_blocks < 1 || n_requests < 0 || n_tokens < 0)
+    return SMETRIC_ERR_INVALID_ARG;
+  if (n_requests > SMETRIC_NOALLOC_MAX_REQUESTS || n_tokens / B > SMETRIC_NOALLOC_MAX_BLOCKS)
+    return SMETRIC_ERR_TOO_LARGE;
+  if (n_requests == 0) return SMETRIC_OK;
+  if (!d_offsets || !d_session_key || !d_block_hashes || !d_status || (n_tokens > 0 && !d_tokens))
+    return SMETRIC_ERR_INVALID_ARG;
+  if (d_tokens && (reinterpret_cast<uintptr_t>(d_tokens) & 15)) return SMETRIC_ERR_INVALID_ARG;
+  if (hashes_cap < n_tokens / B) return SMETRIC_ERR_INVALID_ARG;
+  int dev = 0, num_sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return cuda_status(cudaErrorInvalidDevice);
+  uint64_t* scratch = nullptr;
+  int rc = na_scratch_for(dev, &scratch);
+  if (rc) return rc;
+  int32_t* ok = reinterpret_cast<int32_t*>(scratch);
+  int64_t* block_off = reinterpret_cast<int64_t*>(scratch + kNaFlagWords);
+  uint64_t* digest = scratch + kNaFlagWords + kNaOffWords;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+
+  k_prep<<<1, 1024, 0, s>>>(d_offsets, n_requests, n_tokens, B, nullptr, 0, block_off, ok, d_status, nullptr, 0);
+  if ((rc = cuda_status(cudaGetLastError()))) return rc;
+  if (n_tokens / B > 0) {
+    const uint64_t d_init = mix64(hash_seed ^ (uint64_t)B);
+    switch (B) {
+      case 16: rc = na_digest<8>(d_tokens, n_tokens, d_offsets, block_off, n_requests, B, num_sms, d_init, ok, digest, s); break;
+      case 32: rc = na_digest<16>(d_tokens, n_tokens, d_offsets, block_off, n_requests, B, num_sms, d_init, ok, digest, s); break;
+      case 64: rc = na_digest<32>(d_tokens, n_tokens, d_offsets, block_off, n_requests, B, num_sms, d_init, ok, digest, s); break;
+      default: rc = na_digest<0>(d_tokens, n_tokens, d_offsets, block_off, n_requests, B, num_sms, d_init, ok, digest, s);
+    }
+    if (rc) return rc;
+  }
+  const unsigned grid = (unsigned)((n_requests + kChainThreads - 1) / kChainThreads);
+  k_chain<<<grid, kChainThreads, 0, s>>>(d_offsets, block_off, n_requests, B, session_blocks,
+                                         mix64(hash_seed + kGamma), ok, digest, d_block_hashes, d_session_key,
+                                         nullptr, 0);
+  return cuda_status(cudaGetLastError());
+}

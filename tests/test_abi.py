@@ -77,3 +77,18 @@ def test_null_handles_are_rejected(L):
     assert L.smetric_status(None, None) == pkg.SMETRIC_ERR_INVALID_ARG
     assert L.smetric_index_mask_words(None) == 0
     assert L.smetric_launch_count(None) == 0
+
+
+def test_noalloc_hashes_refuse_on_host(L):
+    """Refusals of smetric_block_hashes_noalloc that need no device: a batch
+    beyond its fixed scratch, a bad block size, an empty batch (a no-op)."""
+    f = L.smetric_block_hashes_noalloc
+    assert f(None, 0, None, pkg.SMETRIC_NOALLOC_MAX_REQUESTS + 1, 16, 1, 0, None, None, 0, None,
+             None) == pkg.SMETRIC_ERR_TOO_LARGE
+    assert f(None, 16 * (pkg.SMETRIC_NOALLOC_MAX_BLOCKS + 1), None, 1, 16, 1, 0, None, None, 0, None,
+             None) == pkg.SMETRIC_ERR_TOO_LARGE
+    assert f(None, 0, None, 1, 7, 1, 0, None, None, 0, None, None) == pkg.SMETRIC_ERR_INVALID_ARG
+    assert f(None, 0, None, 1, 16, 0, 0, None, None, 0, None, None) == pkg.SMETRIC_ERR_INVALID_ARG
+    assert f(None, 0, None, 0, 16, 1, 0, None, None, 0, None, None) == pkg.SMETRIC_OK
+    assert pkg.smetric_strerror(pkg.SMETRIC_ERR_TOO_LARGE) == \
+        "batch larger than the fixed no-allocation scratch"
