@@ -42,6 +42,7 @@ constexpr int kDigestWarps = 8;   // most warps per digest CTA
 constexpr int kChainThreads = 128;
 constexpr int kChainAhead = 16;   // digests prefetched per request
 constexpr int kMatchWarps = 8;    // warps per walk CTA
+constexpr int kGroupAhead = 8;    // 32-block rounds of hashes a group warp compares at once
 
 // ---------------------------------------------------------------------------
 // prep
@@ -56,50 +57,72 @@ __device__ __forceinline__ int64_t warp_incl_scan(int64_t v, int lane) {
   return v;
 }
 
+constexpr int kPrepPer = 8;  // requests per thread per pass
+
 __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, int32_t n,
                                               int64_t n_tokens, int B, const int64_t* __restrict__ load,
                                               int n_load, int64_t* __restrict__ block_off,
                                               int32_t* batch_ok, int32_t* status,
                                               uint4* __restrict__ groups, int64_t group_vecs) {
   __shared__ int64_t warp_tot[32];
+  __shared__ int64_t pass_tot;
   __shared__ int bad_all;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
   if (tid == 0) bad_all = 0;
+  __syncthreads();
   int bad = 0;  // bit 0: invalid offsets, bit 1: out-of-range length or load
   for (int i = tid; i < n_load; i += blockDim.x) {
     const int64_t v = load[i];
     if (v < 0 || v > SMETRIC_MAX_LOAD) bad |= 2;
   }
-  const int per = (n + (int)blockDim.x - 1) / (int)blockDim.x;
-  const int r0 = min(n, tid * per), r1 = min(n, r0 + per);
-  int64_t sum = 0;
-  for (int r = r0; r < r1; ++r) {
-    const int64_t a = off[r], b = off[r + 1];
-    if (a < 0 || b < a || b > n_tokens) { bad |= 1; continue; }
-    if (b - a > (int64_t)INT32_MAX) { bad |= 2; continue; }
-    sum += (b - a) / B;
-  }
-  int64_t incl = warp_incl_scan(sum, lane);
-  if (lane == 31) warp_tot[warp] = incl;
-  __syncthreads();
-  if (bad) atomicOr(&bad_all, bad);
-  if (warp == 0) {
-    const int nw = blockDim.x >> 5;
-    int64_t t = lane < nw ? warp_tot[lane] : 0;
-    int64_t ti = warp_incl_scan(t, lane);
-    if (lane < nw) warp_tot[lane] = ti - t;  // exclusive
-  }
-  __syncthreads();
-  int64_t run = warp_tot[warp] + incl - sum;
-  for (int r = r0; r < r1; ++r) {
-    block_off[r] = run;
-    const int64_t a = off[r], b = off[r + 1];
-    if (a >= 0 && b >= a && b - a <= (int64_t)INT32_MAX) run += (b - a) / B;
-  }
-  if (tid == (int)blockDim.x - 1) block_off[n] = warp_tot[warp] + incl;
   for (int64_t i = tid; i < group_vecs; i += blockDim.x) groups[i] = make_uint4(0, 0, 0, 0);
+  // Passes of kPrepPer consecutive requests per thread: every offset of a
+  // pass is loaded before any is used, then one block-wide scan.
+  int64_t carry = 0;
+  for (int64_t base = 0; base < n; base += (int64_t)blockDim.x * kPrepPer) {
+    const int64_t r0 = base + (int64_t)tid * kPrepPer;
+    int64_t o[kPrepPer + 1];
+#pragma unroll
+    for (int i = 0; i <= kPrepPer; ++i) o[i] = r0 + i <= n ? off[r0 + i] : 0;
+    uint32_t nbv[kPrepPer];
+    int64_t sum = 0;
+#pragma unroll
+    for (int i = 0; i < kPrepPer; ++i) {
+      uint32_t v = 0;
+      if (r0 + i < n) {
+        const int64_t a = o[i], b = o[i + 1];
+        if (a < 0 || b < a || b > n_tokens) bad |= 1;
+        else if (b - a > (int64_t)INT32_MAX) bad |= 2;
+        else v = (uint32_t)(b - a) / (uint32_t)B;
+      }
+      nbv[i] = v;
+      sum += v;
+    }
+    const int64_t incl = warp_incl_scan(sum, lane);
+    if (lane == 31) warp_tot[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+      const int64_t t = lane < nw ? warp_tot[lane] : 0;
+      const int64_t ti = warp_incl_scan(t, lane);
+      if (lane < nw) warp_tot[lane] = ti - t;  // exclusive
+      if (lane == 31) pass_tot = ti;
+    }
+    __syncthreads();
+    int64_t run = carry + warp_tot[warp] + incl - sum;
+#pragma unroll
+    for (int i = 0; i < kPrepPer; ++i) {
+      if (r0 + i < n) {
+        block_off[r0 + i] = run;
+        run += nbv[i];
+      }
+    }
+    carry += pass_tot;
+    __syncthreads();  // warp_tot and pass_tot are rewritten by the next pass
+  }
+  if (bad) atomicOr(&bad_all, bad);
   __syncthreads();
   if (tid == 0) {
+    block_off[n] = carry;
     const int ba = bad_all;
     *batch_ok = ba == 0;
     if (ba & 1) latch_error(status, SMETRIC_ERR_INVALID_ARG);
@@ -551,10 +574,21 @@ __global__ void __launch_bounds__(256)
         const int64_t lo = block_off[l], nl = block_off[l + 1] - lo;
         const int64_t m = nb < nl ? nb : nl;
         sh = m;
-        for (int64_t b = 0; b < m; b += 32) {
-          const bool ne = b + lane < m && __ldg(H + bo + b + lane) != __ldg(H + lo + b + lane);
-          const unsigned x = __ballot_sync(kFull, ne);
-          if (x) { sh = b + __ffs(x) - 1; break; }
+        // kGroupAhead rounds of 32 blocks per iteration, all loads in flight
+        for (int64_t b = 0; b < m; b += 32 * kGroupAhead) {
+          bool ne[kGroupAhead];
+#pragma unroll
+          for (int u = 0; u < kGroupAhead; ++u) {
+            const int64_t bb = b + 32 * u + lane;
+            ne[u] = bb < m && __ldg(H + bo + bb) != __ldg(H + lo + bb);
+          }
+          int64_t first = -1;
+#pragma unroll
+          for (int u = 0; u < kGroupAhead; ++u) {
+            const unsigned x = __ballot_sync(kFull, ne[u]);
+            if (x && first < 0) first = 32 * u + __ffs(x) - 1;
+          }
+          if (first >= 0) { sh = b + first; break; }
         }
       } else {
         l = (int32_t)r;

@@ -225,6 +225,31 @@ def test_route_requests_sharing_leading_blocks():
     ix.close()
 
 
+@pytest.mark.parametrize("B", [16, 32, 64, 6])
+def test_hash_many_short_and_few_long_requests(B):
+    """Batch shapes at the edges of the digest and chain work split: many
+    short requests (several per warp, some empty), a few very long ones (one
+    request's chain much longer than the others), and a mix; B = 6 takes the
+    digest kernel for any even block size."""
+    rng = np.random.default_rng(40 + B)
+    shapes = [
+        rng.integers(0, 4 * B, size=20000),                     # many short (some empty)
+        np.array([300000, 7, 120000, 0, 2 * B]),                # few long
+        np.concatenate([rng.integers(0, 3 * B, size=3000), [250000], rng.integers(0, 60 * B, size=500)]),
+    ]
+    for lens in shapes:
+        reqs = [rng.integers(0, 151936, size=int(L), dtype=np.int32) for L in lens]
+        tok, off = pack(reqs)
+        ix = make_index(8, B, 3, max_req=len(lens), max_tok=len(tok) + 16)
+        hb, sk = gpu_hashes(ix, tok, off)
+        o = oracle.OracleIndex(8).route_batch(B, 3, 0, tok, off, np.zeros(8, np.int64), 1, 4, 2,
+                                               want_hashes=True)
+        assert np.array_equal(hb, o["block_hashes"]) and np.array_equal(sk, o["session_key"])
+        g = gpu_route(ix, tok, off, np.zeros(8, np.int64), (1, 4, 2))
+        assert_outputs_equal(g, o, ctx=f"B={B} n={len(lens)}")
+        ix.close()
+
+
 def test_route_special_cases():
     rng = np.random.default_rng(21)
     N, B = 9, 8
