@@ -42,8 +42,8 @@ N_DISTINCT_BATCHES = 4
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
-    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--e2e-steps", type=int, default=8)
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -439,10 +439,20 @@ def run_ours(args, rank, world, local, dist):
         threads = os.cpu_count() or 1
         ox = oracle_index_for(tr, host[:1])
         m, dt = oracle_calibrate(tr, ox, host[0], args.cpu_seconds, threads)
-        cpu = {"value": m / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
-               "sample": f"first {m} of the {host[0].n_requests} requests of config-4 batch {ids[0]} "
-                         f"({dt:.1f} s on {threads} threads), oracle index holding that batch's "
-                         f"sessions", "tokens_per_s": float(host[0].offsets[m]) / dt}
+        reps = 1
+        if m == host[0].n_requests and dt < args.cpu_seconds / 2:
+            # the whole batch is quicker than the target: route it repeatedly
+            reps = max(2, int(args.cpu_seconds / max(dt, 1e-3)))
+            t0 = time.perf_counter()
+            for _ in range(reps):
+                oracle_route(tr, ox, host[0], m, threads)
+            dt = time.perf_counter() - t0
+        what = (f"{reps} passes over all {m} requests" if reps > 1 else
+                f"first {m} of the {host[0].n_requests} requests")
+        cpu = {"value": reps * m / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+               "sample": f"{what} of config-4 batch {ids[0]} ({dt:.1f} s on {threads} threads), "
+                         f"oracle index holding that batch's sessions",
+               "tokens_per_s": reps * float(host[0].offsets[m]) / dt}
 
     if rank == 0:
         line = {

@@ -719,6 +719,23 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
         const int64_t bn = base + 32 + lane;
         nx[w] = bn < nb ? __ldg((bn < sh ? m_l : m_r) + bn * W + w) : 0;
       }
+      {
+        // fast path: every run alive before this round survives all of its
+        // 32 blocks (the usual case; lanes past the last block hold 0 and so
+        // always take the full path)
+        bool keep = true;
+#pragma unroll
+        for (int w = 0; w < W; ++w) {
+          const uint64_t all = (uint64_t)__reduce_and_sync(kFull, (unsigned)x[w]) |
+                               ((uint64_t)__reduce_and_sync(kFull, (unsigned)(x[w] >> 32)) << 32);
+          keep &= (all & A[w]) == A[w];
+          if (w == gword && galive) keep &= (all & gbit) != 0;
+        }
+        if (keep) {
+          if (galive) g = base + 32;
+          continue;
+        }
+      }
       if (galive) {
         uint64_t mg = 0;
 #pragma unroll
