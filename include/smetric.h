@@ -9,8 +9,8 @@
  *       index (one local tier per serving instance plus one global tier),
  *   (d) scores every instance with an integer cost and takes the argmin.
  * The paper's router scores instances per request (Section 4.1, Figure 6:
- * "route to argmin over instances of f(c_i, l_i)", with c_i the prefix hit of
- * the prompt in instance i's local KV$ and l_i its load) and keeps only
+ * each request goes to the instance minimising a function of c_i, the
+ * prompt's prefix hit in instance i's local KV$, and l_i, its load) and keeps only
  * per-instance state (Section 4.2, Challenge 1); the two-tier store is the
  * local GPU tier plus the cluster-wide global tier (Section 2, Figure 2).
  *

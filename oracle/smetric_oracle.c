@@ -27,19 +27,20 @@
  *    Only full blocks are hashed: n_r = floor(L_r / B); a partial tail block
  *    is never a hit (Section 3.1 counts reuse in whole hit blocks).
  *
- *  Session key (Section 4.2, "Basic solution": sessions are identified from
- *  the request itself, without per-session state): sk_r = h_{min(n_r,S)-1},
+ *  Session key (Section 4.2, basic solution: a session is recognised from
+ *  the request itself, with no per-session state): sk_r = h_{min(n_r,S)-1},
  *  or 0 when n_r = 0.
  *
- *  Two-tier longest prefix match (Figure 6 / Figure 10: c = kvc.hit_len(req),
- *  the per-instance local KV$ prefix hit; Section 2 and Section 4.2: a local
- *  miss can be fetched from the global tier):
+ *  Two-tier longest prefix match (Figure 6 and Figure 10: the router asks the
+ *  KV$ for the prompt's prefix hit on each instance; Section 2 and Section
+ *  4.2: a local miss can be fetched from the global tier):
  *    c_i = largest k <= n_r with h_0..h_{k-1} all in instance i's local tier,
  *    g   = largest k <= n_r with h_0..h_{k-1} all in the global tier,
  *    g_i = max(c_i, g).
  *
- *  Integer cost and argmin (Figure 6, instances.argmin(f(c, l)); Figure 10(c):
- *  load = queued prefill plus the request's own new tokens):
+ *  Integer cost and argmin (Figure 6: the request goes to the instance that
+ *  minimises a function of its hit and its load; Figure 10(c): the load is
+ *  the queued prefill plus the request's own new tokens):
  *    miss_i  = L_r - B*g_i            (tokens instance i must prefill)
  *    fetch_i = B*(g_i - c_i)          (tokens fetched from the global tier)
  *    cost_i  = w_load*load_i + w_miss*miss_i + w_glob*fetch_i   (int64)

@@ -262,8 +262,8 @@ def check_jsq_when_index_empty(L):
 
 def check_argmax_hit_when_load_ignored(L):
     """w_load = 0 and an empty global tier: cost_i = w_miss*(L - B*c_i), so
-    routing picks the instance with the longest local hit (the paper's
-    prev = argmax(c), Figure 10), ties to the lowest id."""
+    routing picks the instance with the longest local hit (the sticky choice
+    of Figure 10), ties to the lowest id."""
     rng = np.random.default_rng(10)
     B = 2
     for trial in range(30):
