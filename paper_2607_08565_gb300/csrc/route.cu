@@ -39,7 +39,8 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kChunk = 32;        // blocks per digest task (one per lane)
 constexpr int kDigestWarps = 8;   // most warps per digest CTA
-constexpr int kChainThreads = 128;
+constexpr int kTmaWarps = 16;     // warps per TMA digest CTA (one stage each)
+constexpr int kChainThreads = 32;   // one warp per CTA: chains spread over every SM
 constexpr int kChainAhead = 16;   // digests prefetched per request
 constexpr int kMatchWarps = 8;    // warps per walk CTA
 constexpr int kGroupAhead = 8;    // 32-block rounds of hashes a group warp compares at once
@@ -334,7 +335,7 @@ __device__ __forceinline__ void tma_rows(uint32_t dst, const CUtensorMap* map, i
 }
 
 template <int HB, int STAGES>
-__global__ void __launch_bounds__(kDigestWarps * 32)
+__global__ void __launch_bounds__(kTmaWarps * 32)
     k_digest_tma(const __grid_constant__ TokenMaps maps, const int32_t* __restrict__ tokens,
                  int64_t n_tokens, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off,
                  int32_t n, uint64_t d_init, const int32_t* __restrict__ batch_ok,
@@ -523,12 +524,14 @@ __global__ void __launch_bounds__(kChainThreads)
         h = mix64((h + kGamma) ^ cur[j]);
         if (h < 2) h |= 2;
         hout[b0 + j] = h;
-        if (b0 + j == kS) sk = h;
-        if (b0 + j == 0) h0 = h;
       }
     }
 #pragma unroll
     for (int j = 0; j < kChainAhead; ++j) cur[j] = nxt[j];
+  }
+  if (nb > 0) {  // read back rather than tested at every step of the serial chain
+    sk = hout[kS];
+    h0 = hout[0];
   }
   sk_out[r] = nb > 0 ? sk : 0;
   if (groups && nb > 0) group_insert(groups, gmask, h0, r);
@@ -859,7 +862,7 @@ bool make_token_maps(TokenMaps& m, const int32_t* tokens, int64_t n_tokens, int 
   return true;
 }
 
-constexpr int kTmaStages = 2;
+constexpr int kTmaStages = 1;
 
 template <int HB>
 int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
@@ -875,7 +878,7 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
     if (make_token_maps(maps, d_tokens, n_tokens, B)) {
       auto kern = k_digest_tma<(HB > 0 ? HB : 2), kTmaStages>;
       const size_t per_warp = (size_t)kTmaStages * kChunk * nch * 16 + 8 * kTmaStages;
-      const int warps = kDigestWarps;
+      const int warps = kTmaWarps;
       const size_t smem = (size_t)warps * per_warp;
       if (idx->digest_occ == 0) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
