@@ -264,6 +264,7 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
   if (ok) ok = cudaMemset(x->table, 0, table_bytes) == cudaSuccess &&
                cudaMemset(x->tags, 0, slots) == cudaSuccess &&
                cudaMemset(x->status, 0, sizeof(int32_t)) == cudaSuccess &&
+               cudaMemset(x->groups, 0, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
                cudaDeviceSynchronize() == cudaSuccess;
   if (!ok) {
     (void)cudaGetLastError();

@@ -63,8 +63,7 @@ constexpr int kPrepPer = 8;  // requests per thread per pass
 __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, int32_t n,
                                               int64_t n_tokens, int B, const int64_t* __restrict__ load,
                                               int n_load, int64_t* __restrict__ block_off,
-                                              int32_t* batch_ok, int32_t* status,
-                                              uint4* __restrict__ groups, int64_t group_vecs) {
+                                              int32_t* batch_ok, int32_t* status) {
   __shared__ int64_t warp_tot[32];
   __shared__ int64_t pass_tot;
   __shared__ int bad_all;
@@ -76,7 +75,6 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
     const int64_t v = load[i];
     if (v < 0 || v > SMETRIC_MAX_LOAD) bad |= 2;
   }
-  for (int64_t i = tid; i < group_vecs; i += blockDim.x) groups[i] = make_uint4(0, 0, 0, 0);
   // Passes of kPrepPer consecutive requests per thread: every offset of a
   // pass is loaded before any is used, then one block-wide scan.
   int64_t carry = 0;
@@ -676,7 +674,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
            const uint64_t* __restrict__ masks, const int32_t* __restrict__ batch_ok,
            const int32_t* __restrict__ lead, const int32_t* __restrict__ share,
            int32_t* __restrict__ inst_out, int32_t* __restrict__ lhit_out,
-           int32_t* __restrict__ ghit_out) {
+           int32_t* __restrict__ ghit_out, uint4* __restrict__ groups, int64_t group_vecs) {
   extern __shared__ int64_t msm[];
   int64_t* load_s = msm;                                                     // [N]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -809,6 +807,11 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
     }
     __syncwarp();
   }
+  // k_group has read the group table: empty it for the next route (it is
+  // zero from index creation before the first)
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < group_vecs;
+       i += (int64_t)gridDim.x * blockDim.x)
+    groups[i] = make_uint4(0, 0, 0, 0);
 }
 
 // ---------------------------------------------------------------------------
@@ -987,7 +990,9 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
   kern<<<(unsigned)grid, kMatchWarps * 32, smem, s>>>(N, idx->cfg.block_size, d_offsets, idx->block_off, n,
                                                       d_load, w.w_load, w.w_miss, w.w_glob, idx->masks,
-                                                      idx->batch_ok, idx->lead, idx->share, inst, lhit, ghit);
+                                                      idx->batch_ok, idx->lead, idx->share, inst, lhit, ghit,
+                                                      reinterpret_cast<uint4*>(idx->groups),
+                                                      (int64_t)group_slots_for(n));
   idx->launches++;
   return cuda_status(cudaGetLastError());
 }
@@ -1046,8 +1051,7 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
 
   profile_begin(idx, s);
   k_prep<<<1, 1024, 0, s>>>(d_offsets, n, n_tokens, c.block_size, d_load, PROBE ? c.num_instances : 0,
-                            idx->block_off, idx->batch_ok, idx->status, reinterpret_cast<uint4*>(idx->groups),
-                            PROBE ? (int64_t)group_slots_for(n) : 0);
+                            idx->block_off, idx->batch_ok, idx->status);
   idx->launches++;
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   profile_mark(idx, kPrep, s);
@@ -1259,7 +1263,7 @@ extern "C" int smetric_block_hashes_noalloc(const int32_t* d_tokens, int64_t n_t
   uint64_t* digest = scratch + kNaFlagWords + kNaOffWords;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
-  k_prep<<<1, 1024, 0, s>>>(d_offsets, n_requests, n_tokens, B, nullptr, 0, block_off, ok, d_status, nullptr, 0);
+  k_prep<<<1, 1024, 0, s>>>(d_offsets, n_requests, n_tokens, B, nullptr, 0, block_off, ok, d_status);
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   if (n_tokens / B > 0) {
     const uint64_t d_init = mix64(hash_seed ^ (uint64_t)B);
