@@ -52,6 +52,10 @@ def parse():
     ap.add_argument("--sessions", type=int, default=65536,
                     help="sessions of the burst workload (smaller values: profiling cases)")
     ap.add_argument("--batch", type=int, default=8192, help="requests per batch")
+    ap.add_argument("--sweep", action="store_true",
+                    help="config-5 stress sweep instead of the benchmark line: batch, N and B "
+                         "varied on the config-4 generator, table filled to --table-gb")
+    ap.add_argument("--table-gb", type=float, default=40.0)
     return ap.parse_args()
 
 
@@ -484,8 +488,115 @@ def run_ours(args, rank, world, local, dist):
         dist.destroy_process_group()
 
 
+# ---------------------------------------------------------------------------
+# config-5 stress sweep
+# ---------------------------------------------------------------------------
+
+SWEEP_BATCHES = (1, 4, 16, 64, 256, 1024, 4096, 8192, 16384, 32768)
+SWEEP_N = (8, 16, 32, 64, 128, 256)
+SWEEP_B = (16, 32, 64)
+
+
+def sweep_index(N, B, table_gb, max_req, max_tok, device):
+    """An index of about table_gb GB for N instances and block size B,
+    holding every config-4 session prefix plus random filler keys (random
+    tiers) up to load factor 0.7."""
+    import torch
+    import paper_2607_08565_gb300 as pkg
+    from synth import burst_trace
+    tr = burst_trace("c5_sweep", num_instances=N, block_size=B, batch_size=max_req)
+    W = (N + 1 + 63) // 64
+    entry = 16 if W == 1 else (32 if W <= 3 else 64)
+    slots = int(table_gb * 1e9 / (entry + 1))
+    chunk = 4096
+    max_tok = max(max_tok, chunk * int(tr.prefix_len.max()))
+    ix = pkg.SMetricIndex(N, B, tr.params.session_blocks, capacity_slots=slots,
+                          max_batch_requests=max(max_req, chunk), max_batch_tokens=max_tok,
+                          hash_seed=tr.params.hash_seed)
+    populate_index(ix, tr, device, chunk)
+    n_fill = int(0.7 * slots) - tr.n_prefix_blocks()
+    g = torch.Generator(device=device)
+    g.manual_seed(5 + N * 1000 + B)
+    step = 1 << 26
+    for a in range(0, max(n_fill, 0), step):
+        m = min(step, n_fill - a)
+        # full 64-bit range (home buckets come from a key's high bits); bit 1
+        # set keeps every key >= 2
+        keys = torch.randint(-(1 << 63), (1 << 63) - 1, (m,), device=device, generator=g,
+                             dtype=torch.int64) | 2
+        tiers = torch.randint(-1, N, (m,), device=device, generator=g, dtype=torch.int32)
+        ix.insert(keys, tiers)
+    ix.check()
+    return tr, ix, slots * (entry + 1), tr.n_prefix_blocks() + max(n_fill, 0)
+
+
+def sweep_point(tr, ix, batch, device):
+    """Route one config-5 batch repeatedly; per-kernel device time."""
+    import torch
+    import paper_2607_08565_gb300 as pkg
+    p = tr.params
+    bt = tr.batch(0, batch_size=batch)
+    tok = torch.from_numpy(bt.tokens).to(device)
+    off = torch.from_numpy(bt.offsets).to(device)
+    load = torch.from_numpy(bt.load).to(device)
+    w = (p.w_load, p.w_miss, p.w_glob)
+    for _ in range(3):
+        ix.route_batch(tok, off, load, w, want_hashes=False)
+    ix.check()
+    steps = max(5, min(200, int(2e6 / max(bt.n_tokens // p.block_size, 1))))
+    stream = torch.cuda.current_stream(device)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        ix.route_batch(tok, off, load, w, want_hashes=False)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    us = e0.elapsed_time(e1) * 1e3 / steps
+    pkg.smetric_profile_enable(ix.handle, True)
+    for _ in range(steps):
+        ix.route_batch(tok, off, load, w, want_hashes=False)
+    prof = pkg.smetric_profile_read(ix.handle)
+    pkg.smetric_profile_enable(ix.handle, False)
+    ix.check()
+    return {"batch": batch, "tokens": int(bt.n_tokens), "us_per_batch": us,
+            "requests_per_s": batch / us * 1e6, "tokens_per_s": bt.n_tokens / us * 1e6,
+            "kernels_us": {k: v[0] * 1e3 / max(v[1], 1) for k, v in prof.items()}, "steps": steps}
+
+
+def run_sweep(args):
+    import torch
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    from paper_2607_08565_gb300 import build_lib
+    if not build_lib.up_to_date():
+        build_lib.build()
+    combos = [(64, 32, SWEEP_BATCHES)] + [(N, 32, (8192,)) for N in SWEEP_N if N != 64] + \
+             [(64, B, (8192,)) for B in SWEEP_B if B != 32]
+    for N, B, batches in combos:
+        max_req = max(batches)
+        max_tok = 0
+        tr0 = None
+        t0 = time.perf_counter()
+        from synth import burst_trace
+        tr0 = burst_trace("c5_sweep", num_instances=N, block_size=B, batch_size=max_req)
+        max_tok = int(tr0.session_len.max()) * max_req
+        tr, ix, table_bytes, keys = sweep_index(N, B, args.table_gb, max_req, max_tok, device)
+        build_s = time.perf_counter() - t0
+        for b in batches:
+            pt = sweep_point(tr, ix, b, device)
+            pt.update({"sweep": "config-5", "num_instances": N, "block_size": B,
+                       "table_bytes": table_bytes, "index_keys": int(keys), "build_s": build_s})
+            print(json.dumps(pt), flush=True)
+        ix.close()
+        del ix
+        torch.cuda.empty_cache()
+
+
 def main():
     args = parse()
+    if args.sweep:
+        run_sweep(args)
+        return
     rank, world, local, dist = dist_setup(args)
     if args.impl == "reference":
         run_reference(args, rank, world, dist)
