@@ -495,6 +495,16 @@ __device__ __forceinline__ void group_insert(uint64_t* __restrict__ groups, uint
   }
 }
 
+// End of a request's chain: the session key and the first block's hash are
+// read back rather than tested at every serial step; the latter enters the
+// group table.
+__device__ __forceinline__ void nb_done(int32_t r, int64_t nb, const uint64_t* hout, int64_t kS,
+                                        uint64_t* __restrict__ sk_out, uint64_t* __restrict__ groups,
+                                        uint64_t gmask) {
+  sk_out[r] = nb > 0 ? hout[kS] : 0;
+  if (groups && nb > 0) group_insert(groups, gmask, hout[0], r);
+}
+
 __global__ void __launch_bounds__(kChainThreads)
     k_chain(const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n, int B,
             int S, uint64_t h_init, const int32_t* __restrict__ batch_ok,
@@ -503,36 +513,64 @@ __global__ void __launch_bounds__(kChainThreads)
   const int32_t r = blockIdx.x * kChainThreads + threadIdx.x;
   if (r >= n) return;
   if (!*batch_ok) { sk_out[r] = 0; return; }
-  const int64_t nb = (off[r + 1] - off[r]) / B;
   const int64_t bo = block_off[r];
+  const int64_t nb = block_off[r + 1] - bo;
   const uint64_t* const d = digest + bo;
   uint64_t* const hout = hashes + bo;
   const int64_t kS = (nb < S ? nb : S) - 1;
-  uint64_t h = h_init, sk = 0, h0 = 0;
-  uint64_t cur[kChainAhead], nxt[kChainAhead];
+  uint64_t h = h_init;
+  auto step = [](uint64_t hp, uint64_t db) {
+    uint64_t x = mix64((hp + kGamma) ^ db);
+    if (x < 2) x |= 2;
+    return x;
+  };
+  // Digests are read and hashes written two blocks per 16-byte access (a
+  // lane's accesses are its own request's, so they do not coalesce across
+  // the warp): at most one single block first to reach a 16-byte boundary
+  // and one last.
+  if (((reinterpret_cast<uintptr_t>(d) ^ reinterpret_cast<uintptr_t>(hout)) & 15) != 0) {
+    // the caller's hash buffer and the digests differ in 16-byte phase:
+    // one block per access
+    for (int64_t k = 0; k < nb; ++k) {
+      h = step(h, __ldg(d + k));
+      hout[k] = h;
+    }
+    nb_done(r, nb, hout, kS, sk_out, groups, gmask);
+    return;
+  }
+  int64_t b = 0;
+  if ((reinterpret_cast<uintptr_t>(d) & 15) && nb > 0) {
+    h = step(h, __ldg(d));
+    hout[0] = h;
+    b = 1;
+  }
+  const ulonglong2* const dv = reinterpret_cast<const ulonglong2*>(d + b);
+  ulonglong2* const hv = reinterpret_cast<ulonglong2*>(hout + b);
+  const int64_t np = (nb - b) >> 1;  // whole pairs
+  constexpr int P = kChainAhead / 2;
+  const ulonglong2 z2 = make_ulonglong2(0, 0);
+  ulonglong2 cur[P], nxt[P];
 #pragma unroll
-  for (int j = 0; j < kChainAhead; ++j) cur[j] = j < nb ? __ldg(d + j) : 0;
-  for (int64_t b0 = 0; b0 < nb; b0 += kChainAhead) {
+  for (int j = 0; j < P; ++j) cur[j] = j < np ? __ldg(dv + j) : z2;
+  for (int64_t p0 = 0; p0 < np; p0 += P) {
 #pragma unroll
-    for (int j = 0; j < kChainAhead; ++j)
-      nxt[j] = b0 + kChainAhead + j < nb ? __ldg(d + b0 + kChainAhead + j) : 0;
+    for (int j = 0; j < P; ++j) nxt[j] = p0 + P + j < np ? __ldg(dv + p0 + P + j) : z2;
 #pragma unroll
-    for (int j = 0; j < kChainAhead; ++j) {
-      if (b0 + j < nb) {
-        h = mix64((h + kGamma) ^ cur[j]);
-        if (h < 2) h |= 2;
-        hout[b0 + j] = h;
+    for (int j = 0; j < P; ++j) {
+      if (p0 + j < np) {
+        const uint64_t x = step(h, cur[j].x);
+        h = step(x, cur[j].y);
+        hv[p0 + j] = make_ulonglong2(x, h);
       }
     }
 #pragma unroll
-    for (int j = 0; j < kChainAhead; ++j) cur[j] = nxt[j];
+    for (int j = 0; j < P; ++j) cur[j] = nxt[j];
   }
-  if (nb > 0) {  // read back rather than tested at every step of the serial chain
-    sk = hout[kS];
-    h0 = hout[0];
+  if (b + 2 * np < nb) {
+    h = step(h, __ldg(d + nb - 1));
+    hout[nb - 1] = h;
   }
-  sk_out[r] = nb > 0 ? sk : 0;
-  if (groups && nb > 0) group_insert(groups, gmask, h0, r);
+  nb_done(r, nb, hout, kS, sk_out, groups, gmask);
 }
 
 // ---------------------------------------------------------------------------

@@ -53,6 +53,31 @@ def test_block_hashes_ragged(B, seed):
         ix.close()
 
 
+@pytest.mark.parametrize("shift", [0, 1])
+def test_block_hashes_into_caller_buffer_of_either_16_byte_phase(shift):
+    """The chain writes hashes two per 16-byte store when the caller's hash
+    buffer and the digests share a 16-byte phase, one per store when not:
+    both give the oracle's hashes and session keys."""
+    rng = np.random.default_rng(60 + shift)
+    B = 32
+    reqs = [rng.integers(0, 151936, size=int(L), dtype=np.int32) for L in rng.integers(0, 3000, 200)]
+    tok, off = pack(reqs)
+    ix = make_index(4, B, 2)
+    nb = n_blocks(off, B)
+    cap = len(tok) // B  # the call requires room for n_tokens / B hashes
+    big = torch.zeros(cap + 2, dtype=torch.int64, device="cuda")
+    hb = big[shift:shift + cap]  # shift 1: 8 bytes past a 16-byte boundary
+    sk = torch.zeros(len(off) - 1, dtype=torch.int64, device="cuda")
+    pkg.smetric_block_hashes(ix.handle, T(tok), len(tok), T(off), len(off) - 1, sk, hb, cap, None)
+    ix.check()
+    o = oracle.OracleIndex(4).route_batch(B, 2, 0, tok, off, np.zeros(4, np.int64), 1, 4, 2,
+                                           want_hashes=True)
+    got = hb[:nb].cpu().numpy().view(np.uint64)
+    assert np.array_equal(got, o["block_hashes"])
+    assert np.array_equal(sk.cpu().numpy().view(np.uint64), o["session_key"])
+    ix.close()
+
+
 def test_block_hashes_wide_gaps_between_blocks():
     """Many requests shorter than one block between full blocks: a 32-block
     chunk then spans far more tokens than it hashes."""
