@@ -495,6 +495,17 @@ __device__ __forceinline__ void group_insert(uint64_t* __restrict__ groups, uint
   }
 }
 
+// 32-byte global load (read-only path) and store of four 64-bit words; the
+// address must be 32-byte aligned.
+__device__ __forceinline__ void ld_nc_v4(const uint64_t* p, uint64_t (&v)[4]) {
+  asm volatile("ld.global.nc.v4.u64 {%0,%1,%2,%3}, [%4];\n"
+               : "=l"(v[0]), "=l"(v[1]), "=l"(v[2]), "=l"(v[3])
+               : "l"(p));
+}
+__device__ __forceinline__ void st_v4(uint64_t* p, uint64_t a, uint64_t b, uint64_t c, uint64_t d) {
+  asm volatile("st.global.v4.u64 [%0], {%1,%2,%3,%4};\n" ::"l"(p), "l"(a), "l"(b), "l"(c), "l"(d) : "memory");
+}
+
 // End of a request's chain: the session key and the first block's hash are
 // read back rather than tested at every serial step; the latter enters the
 // group table.
@@ -524,13 +535,13 @@ __global__ void __launch_bounds__(kChainThreads)
     if (x < 2) x |= 2;
     return x;
   };
-  // Digests are read and hashes written two blocks per 16-byte access (a
-  // lane's accesses are its own request's, so they do not coalesce across
-  // the warp): at most one single block first to reach a 16-byte boundary
-  // and one last.
-  if (((reinterpret_cast<uintptr_t>(d) ^ reinterpret_cast<uintptr_t>(hout)) & 15) != 0) {
-    // the caller's hash buffer and the digests differ in 16-byte phase:
-    // one block per access
+  // Digests are read and hashes written four blocks per 32-byte access (a
+  // lane's accesses are its own request's and do not coalesce across the
+  // warp, and fewer instructions shorten every serial step): single blocks
+  // up to a 32-byte boundary and after the last whole quad. A caller hash
+  // buffer in another 32-byte phase than the digests takes one block per
+  // access throughout.
+  if (((reinterpret_cast<uintptr_t>(d) ^ reinterpret_cast<uintptr_t>(hout)) & 31) != 0) {
     for (int64_t k = 0; k < nb; ++k) {
       h = step(h, __ldg(d + k));
       hout[k] = h;
@@ -539,36 +550,39 @@ __global__ void __launch_bounds__(kChainThreads)
     return;
   }
   int64_t b = 0;
-  if ((reinterpret_cast<uintptr_t>(d) & 15) && nb > 0) {
-    h = step(h, __ldg(d));
-    hout[0] = h;
-    b = 1;
+  while (b < nb && (reinterpret_cast<uintptr_t>(d + b) & 31)) {
+    h = step(h, __ldg(d + b));
+    hout[b] = h;
+    ++b;
   }
-  const ulonglong2* const dv = reinterpret_cast<const ulonglong2*>(d + b);
-  ulonglong2* const hv = reinterpret_cast<ulonglong2*>(hout + b);
-  const int64_t np = (nb - b) >> 1;  // whole pairs
-  constexpr int P = kChainAhead / 2;
-  const ulonglong2 z2 = make_ulonglong2(0, 0);
-  ulonglong2 cur[P], nxt[P];
+  const uint64_t* const dq = d + b;
+  uint64_t* const hq = hout + b;
+  const int64_t nq = (nb - b) >> 2;  // whole quads
+  constexpr int Q = kChainAhead / 4;
+  uint64_t c[Q][4], x[Q][4];
 #pragma unroll
-  for (int j = 0; j < P; ++j) cur[j] = j < np ? __ldg(dv + j) : z2;
-  for (int64_t p0 = 0; p0 < np; p0 += P) {
+  for (int j = 0; j < Q; ++j)
+    if (j < nq) ld_nc_v4(dq + 4 * j, c[j]);
+  for (int64_t q0 = 0; q0 < nq; q0 += Q) {
 #pragma unroll
-    for (int j = 0; j < P; ++j) nxt[j] = p0 + P + j < np ? __ldg(dv + p0 + P + j) : z2;
+    for (int j = 0; j < Q; ++j)
+      if (q0 + Q + j < nq) ld_nc_v4(dq + 4 * (q0 + Q + j), x[j]);
 #pragma unroll
-    for (int j = 0; j < P; ++j) {
-      if (p0 + j < np) {
-        const uint64_t x = step(h, cur[j].x);
-        h = step(x, cur[j].y);
-        hv[p0 + j] = make_ulonglong2(x, h);
+    for (int j = 0; j < Q; ++j) {
+      if (q0 + j < nq) {
+        const uint64_t a0 = step(h, c[j][0]), a1 = step(a0, c[j][1]), a2 = step(a1, c[j][2]);
+        h = step(a2, c[j][3]);
+        st_v4(hq + 4 * (q0 + j), a0, a1, a2, h);
       }
     }
 #pragma unroll
-    for (int j = 0; j < P; ++j) cur[j] = nxt[j];
+    for (int j = 0; j < Q; ++j)
+#pragma unroll
+      for (int k = 0; k < 4; ++k) c[j][k] = x[j][k];
   }
-  if (b + 2 * np < nb) {
-    h = step(h, __ldg(d + nb - 1));
-    hout[nb - 1] = h;
+  for (int64_t k = b + 4 * nq; k < nb; ++k) {
+    h = step(h, __ldg(d + k));
+    hout[k] = h;
   }
   nb_done(r, nb, hout, kS, sk_out, groups, gmask);
 }

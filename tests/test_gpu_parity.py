@@ -53,11 +53,11 @@ def test_block_hashes_ragged(B, seed):
         ix.close()
 
 
-@pytest.mark.parametrize("shift", [0, 1])
-def test_block_hashes_into_caller_buffer_of_either_16_byte_phase(shift):
-    """The chain writes hashes two per 16-byte store when the caller's hash
-    buffer and the digests share a 16-byte phase, one per store when not:
-    both give the oracle's hashes and session keys."""
+@pytest.mark.parametrize("shift", [0, 1, 2, 3])
+def test_block_hashes_into_caller_buffer_of_any_32_byte_phase(shift):
+    """The chain writes hashes four per 32-byte store when the caller's hash
+    buffer and the digests share a 32-byte phase, one per store when not:
+    every phase gives the oracle's hashes and session keys."""
     rng = np.random.default_rng(60 + shift)
     B = 32
     reqs = [rng.integers(0, 151936, size=int(L), dtype=np.int32) for L in rng.integers(0, 3000, 200)]
@@ -65,8 +65,8 @@ def test_block_hashes_into_caller_buffer_of_either_16_byte_phase(shift):
     ix = make_index(4, B, 2)
     nb = n_blocks(off, B)
     cap = len(tok) // B  # the call requires room for n_tokens / B hashes
-    big = torch.zeros(cap + 2, dtype=torch.int64, device="cuda")
-    hb = big[shift:shift + cap]  # shift 1: 8 bytes past a 16-byte boundary
+    big = torch.zeros(cap + 4, dtype=torch.int64, device="cuda")
+    hb = big[shift:shift + cap]  # shift s: 8 s bytes past a 32-byte boundary
     sk = torch.zeros(len(off) - 1, dtype=torch.int64, device="cuda")
     pkg.smetric_block_hashes(ix.handle, T(tok), len(tok), T(off), len(off) - 1, sk, hb, cap, None)
     ix.check()
