@@ -101,8 +101,11 @@ typedef struct {
 /* Create an empty index and its route scratch on the current device.
  * The table holds capacity_slots (rounded up to a multiple of 16) entries of
  * 16, 32 or 64 bytes (key plus ceil((N+1)/64) tier-mask words, padded to a
- * power of two) and one tag byte per slot; the scratch holds
- * (2 + W) * (max_batch_tokens/B) + max_batch_requests + 1 64-bit words,
+ * power of two) and one tag byte per slot. The route scratch holds, in 64-bit
+ * words, (2 + W) * (max_batch_tokens/B) for per-block digests, hashes and
+ * tier masks, 2 * (max_batch_requests + 1) for per-request offsets, group
+ * leaders and shared-block counts, and 2 * G for the group table, G the
+ * smallest power of two >= max(64, 2 * max_batch_requests);
  * W = ceil((N+1)/64).
  * Returns SMETRIC_ERR_INVALID_ARG for an out-of-range field and
  * SMETRIC_ERR_OOM when a device allocation fails; *out is NULL then. */
