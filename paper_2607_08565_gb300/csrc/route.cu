@@ -760,35 +760,9 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
     bool galive = true;
     int64_t g = 0;
     int ne = 0;
-    uint64_t nx[W];
-#pragma unroll
-    for (int w = 0; w < W; ++w) nx[w] = lane < nb ? __ldg((lane < sh ? m_l : m_r) + lane * W + w) : 0;
-    for (int64_t base = 0; base < nb; base += 32) {
-      const bool valid = base + lane < nb;
-      uint64_t x[W];
-#pragma unroll
-      for (int w = 0; w < W; ++w) {
-        x[w] = valid ? nx[w] : 0;
-        const int64_t bn = base + 32 + lane;
-        nx[w] = bn < nb ? __ldg((bn < sh ? m_l : m_r) + bn * W + w) : 0;
-      }
-      {
-        // fast path: every run alive before this round survives all of its
-        // 32 blocks (the usual case; lanes past the last block hold 0 and so
-        // always take the full path)
-        bool keep = true;
-#pragma unroll
-        for (int w = 0; w < W; ++w) {
-          const uint64_t all = (uint64_t)__reduce_and_sync(kFull, (unsigned)x[w]) |
-                               ((uint64_t)__reduce_and_sync(kFull, (unsigned)(x[w] >> 32)) << 32);
-          keep &= (all & A[w]) == A[w];
-          if (w == gword && galive) keep &= (all & gbit) != 0;
-        }
-        if (keep) {
-          if (galive) g = base + 32;
-          continue;
-        }
-      }
+    // 32 blocks with lane j holding block base + j: the runs that end there
+    // become events; returns true once no run is alive
+    auto half = [&](int64_t base, const uint64_t (&x)[W]) -> bool {
       if (galive) {
         uint64_t mg = 0;
 #pragma unroll
@@ -822,7 +796,43 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
         for (int w = 0; w < W; ++w) ev_mask[at * W + w] = X[w];
       }
       ne += __popc(ev);
-      if (!any && !galive) break;
+      return !any && !galive;
+    };
+    auto mask_at = [&](int64_t bb, int w) -> uint64_t {
+      return bb < nb ? __ldg((bb < sh ? m_l : m_r) + bb * W + w) : 0;
+    };
+    // rounds of 64 blocks, lane j holding blocks base + j and base + 32 + j,
+    // the next round's masks in flight
+    uint64_t n0[W], n1[W];
+#pragma unroll
+    for (int w = 0; w < W; ++w) { n0[w] = mask_at(lane, w); n1[w] = mask_at(32 + lane, w); }
+    for (int64_t base = 0; base < nb; base += 64) {
+      uint64_t x0[W], x1[W];
+#pragma unroll
+      for (int w = 0; w < W; ++w) {
+        x0[w] = n0[w];
+        x1[w] = n1[w];
+        n0[w] = mask_at(base + 64 + lane, w);
+        n1[w] = mask_at(base + 96 + lane, w);
+      }
+      // fast path: every run alive before this round survives all of its 64
+      // blocks (the usual case; blocks past the last hold 0 and so always take
+      // the full path)
+      bool keep = true;
+#pragma unroll
+      for (int w = 0; w < W; ++w) {
+        const uint64_t both = x0[w] & x1[w];
+        const uint64_t all = (uint64_t)__reduce_and_sync(kFull, (unsigned)both) |
+                             ((uint64_t)__reduce_and_sync(kFull, (unsigned)(both >> 32)) << 32);
+        keep &= (all & A[w]) == A[w];
+        if (w == gword && galive) keep &= (all & gbit) != 0;
+      }
+      if (keep) {
+        if (galive) g = base + 64;
+        continue;
+      }
+      if (half(base, x0)) break;
+      if (half(base + 32, x1)) break;
     }
     __syncwarp();
     // cost of every instance; lanes = instances
