@@ -194,6 +194,7 @@ void free_all(smetric_index* x) {
   cudaFree(x->masks);
   cudaFree(x->groups);
   cudaFree(x->lead);
+  cudaFree(x->chunk_off);
   cudaFree(x->batch_ok);
   cudaFree(x->st_tokens);
   cudaFree(x->st_offsets);
@@ -251,6 +252,7 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
             cudaMalloc(&x->masks, (max_blocks > 0 ? max_blocks : 1) * W * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->groups, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->lead, 2 * (R + 1) * sizeof(int32_t)) == cudaSuccess &&
+            cudaMalloc(&x->chunk_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
             cudaMalloc(&x->batch_ok, sizeof(int32_t)) == cudaSuccess;
   if (ok) x->share = x->lead + (R + 1);
   if (ok && (c.flags & SMETRIC_FLAG_HOST_STAGING)) {

@@ -63,9 +63,11 @@ constexpr int kPrepPer = 8;  // requests per thread per pass
 __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, int32_t n,
                                               int64_t n_tokens, int B, const int64_t* __restrict__ load,
                                               int n_load, int64_t* __restrict__ block_off,
-                                              int32_t* batch_ok, int32_t* status) {
-  __shared__ int64_t warp_tot[32];
-  __shared__ int64_t pass_tot;
+                                              int64_t* __restrict__ chunk_off, int32_t* batch_ok,
+                                              int32_t* status) {
+  constexpr int NS = 2;  // scans: full blocks, and 32-block chunks (when chunk_off is wanted)
+  __shared__ int64_t warp_tot[NS][32];
+  __shared__ int64_t pass_tot[NS];
   __shared__ int bad_all;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
   if (tid == 0) bad_all = 0;
@@ -76,15 +78,14 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
     if (v < 0 || v > SMETRIC_MAX_LOAD) bad |= 2;
   }
   // Passes of kPrepPer consecutive requests per thread: every offset of a
-  // pass is loaded before any is used, then one block-wide scan.
-  int64_t carry = 0;
+  // pass is loaded before any is used, then one block-wide scan per count.
+  int64_t carry[NS] = {0, 0};
   for (int64_t base = 0; base < n; base += (int64_t)blockDim.x * kPrepPer) {
     const int64_t r0 = base + (int64_t)tid * kPrepPer;
     int64_t o[kPrepPer + 1];
 #pragma unroll
     for (int i = 0; i <= kPrepPer; ++i) o[i] = r0 + i <= n ? off[r0 + i] : 0;
     uint32_t nbv[kPrepPer];
-    int64_t sum = 0;
 #pragma unroll
     for (int i = 0; i < kPrepPer; ++i) {
       uint32_t v = 0;
@@ -95,33 +96,49 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
         else v = (uint32_t)(b - a) / (uint32_t)B;
       }
       nbv[i] = v;
-      sum += v;
     }
-    const int64_t incl = warp_incl_scan(sum, lane);
-    if (lane == 31) warp_tot[warp] = incl;
+    auto cnt = [&](int k, int i) -> int64_t { return k == 0 ? nbv[i] : (nbv[i] + 31) >> 5; };
+    int64_t sum[NS], incl[NS];
+#pragma unroll
+    for (int k = 0; k < NS; ++k) {
+      sum[k] = 0;
+#pragma unroll
+      for (int i = 0; i < kPrepPer; ++i) sum[k] += cnt(k, i);
+      incl[k] = warp_incl_scan(sum[k], lane);
+      if (lane == 31) warp_tot[k][warp] = incl[k];
+    }
     __syncthreads();
     if (warp == 0) {
-      const int64_t t = lane < nw ? warp_tot[lane] : 0;
-      const int64_t ti = warp_incl_scan(t, lane);
-      if (lane < nw) warp_tot[lane] = ti - t;  // exclusive
-      if (lane == 31) pass_tot = ti;
-    }
-    __syncthreads();
-    int64_t run = carry + warp_tot[warp] + incl - sum;
 #pragma unroll
-    for (int i = 0; i < kPrepPer; ++i) {
-      if (r0 + i < n) {
-        block_off[r0 + i] = run;
-        run += nbv[i];
+      for (int k = 0; k < NS; ++k) {
+        const int64_t t = lane < nw ? warp_tot[k][lane] : 0;
+        const int64_t ti = warp_incl_scan(t, lane);
+        if (lane < nw) warp_tot[k][lane] = ti - t;  // exclusive
+        if (lane == 31) pass_tot[k] = ti;
       }
     }
-    carry += pass_tot;
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < NS; ++k) {
+      int64_t* const dst = k == 0 ? block_off : chunk_off;
+      if (!dst) continue;
+      int64_t run = carry[k] + warp_tot[k][warp] + incl[k] - sum[k];
+#pragma unroll
+      for (int i = 0; i < kPrepPer; ++i) {
+        if (r0 + i < n) {
+          dst[r0 + i] = run;
+          run += cnt(k, i);
+        }
+      }
+      carry[k] += pass_tot[k];
+    }
     __syncthreads();  // warp_tot and pass_tot are rewritten by the next pass
   }
   if (bad) atomicOr(&bad_all, bad);
   __syncthreads();
   if (tid == 0) {
-    block_off[n] = carry;
+    block_off[n] = carry[0];
+    if (chunk_off) chunk_off[n] = carry[1];
     const int ba = bad_all;
     *batch_ok = ba == 0;
     if (ba & 1) latch_error(status, SMETRIC_ERR_INVALID_ARG);
@@ -336,7 +353,7 @@ template <int HB, int STAGES>
 __global__ void __launch_bounds__(kTmaWarps * 32)
     k_digest_tma(const __grid_constant__ TokenMaps maps, const int32_t* __restrict__ tokens,
                  int64_t n_tokens, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off,
-                 int32_t n, uint64_t d_init, const int32_t* __restrict__ batch_ok,
+                 const int64_t* __restrict__ chunk_off, int32_t n, uint64_t d_init, const int32_t* __restrict__ batch_ok,
                  uint64_t* __restrict__ digest, int32_t* status) {
   constexpr int B = 2 * HB;
   constexpr int NP = HB / 2 + 1;           // 16-byte pieces per row
@@ -345,8 +362,9 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
   extern __shared__ __align__(128) unsigned char dsm_raw[];
   if (!*batch_ok) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, warps = blockDim.x >> 5;
-  const int64_t total = block_off[n];
-  const int64_t n_chunks = (total + kChunk - 1) / kChunk;
+  // chunk c is chunk q of request r: its blocks 32q .. 32q+31, so a chunk
+  // never spans two requests
+  const int64_t n_chunks = chunk_off[n];
   const int64_t tw = (int64_t)gridDim.x * warps;
   const int64_t per = (n_chunks + tw - 1) / tw;
   const int64_t c_lo = ((int64_t)blockIdx.x * warps + warp) * per;
@@ -364,26 +382,24 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;\n" : "=l"(policy));
   const int64_t token_bytes = 4 * n_tokens;
   const char* const tb = reinterpret_cast<const char*>(tokens);
-  int32_t r = find_request(block_off, 0, n, min(c_lo * kChunk + lane, total - 1));
+  int32_t r = find_request(chunk_off, 0, n, c_lo);  // warp-uniform
 
-  // Start the copy of chunk c into stage s; returns this lane's first token.
-  auto issue = [&](int64_t c, int s, bool& valid) -> int64_t {
-    const int64_t f = c * kChunk + lane;
-    valid = f < total;
-    int64_t tok0 = 0;
-    if (valid) {
-      if (__ldg(block_off + r + 1) <= f) r = find_request(block_off, r + 1, n, f);
-      tok0 = __ldg(off + r) + (f - __ldg(block_off + r)) * B;
-    }
-    const int nv = __popc(__ballot_sync(kFull, valid));
-    const int32_t r0 = __shfl_sync(kFull, r, 0);
+  // Start the copy of chunk c into stage s; returns this lane's first token
+  // and sets its digest index.
+  auto issue = [&](int64_t c, int s, bool& valid, int64_t& gidx) -> int64_t {
+    if (__ldg(chunk_off + r + 1) <= c) r = find_request(chunk_off, r + 1, n, c);
+    const int64_t bo = __ldg(block_off + r), nbr = __ldg(block_off + r + 1) - bo;
+    const int64_t b = (c - __ldg(chunk_off + r)) * kChunk + lane;  // block of request r
+    valid = b < nbr;
+    const int64_t tok0 = __ldg(off + r) + b * B;
+    gidx = bo + b;
+    const int nv = (int)min((int64_t)kChunk, nbr - (b - lane));
     const int64_t a0 = (4 * __shfl_sync(kFull, tok0, 0)) & ~(int64_t)15;
     const int k = (int)((a0 % (4 * B)) >> 4);
     const int64_t y0 = a0 / (4 * B);
-    const bool one_request = __all_sync(kFull, !valid || r == r0);
     unsigned char* const st = stages + (size_t)s * STAGE;
     const uint32_t mbar = mbar0 + 8u * (uint32_t)s;
-    if (one_request && y0 + nv <= (int64_t)maps.rows[k]) {
+    if (y0 + nv <= (int64_t)maps.rows[k]) {
       if (lane == 0) {
         asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
         mbar_arrive_expect_tx(mbar, STAGE);
@@ -407,29 +423,30 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
   uint32_t phase = 0;
   bool failed = false;
   bool v[STAGES];
-  int64_t t[STAGES];
+  int64_t t[STAGES], gi[STAGES];
 #pragma unroll
   for (int s = 0; s < STAGES; ++s)
-    if (c_lo + s < c_hi) t[s] = issue(c_lo + s, s, v[s]);
+    if (c_lo + s < c_hi) t[s] = issue(c_lo + s, s, v[s], gi[s]);
   int s = 0;
   for (int64_t c = c_lo; c < c_hi; ++c) {
     if (!mbar_wait(mbar0 + 8u * (uint32_t)s, (phase >> s) & 1)) { failed = true; break; }
     phase ^= 1u << s;
     bool vc = false;
-    int64_t tc = 0;
+    int64_t tc = 0, gc = 0;
 #pragma unroll
-    for (int q = 0; q < STAGES; ++q) if (q == s) { vc = v[q]; tc = t[q]; }
+    for (int q = 0; q < STAGES; ++q) if (q == s) { vc = v[q]; tc = t[q]; gc = gi[q]; }
     if (vc) {
       const int delta = (int)((tc * 4) & 15);  // 0, 4, 8 or 12
       const uint64_t* row = reinterpret_cast<const uint64_t*>(stages + (size_t)s * STAGE + lane * ROW) + (delta >> 3);
-      digest[c * kChunk + lane] = digest_row<HB>(row, (delta & 4) != 0, HB, d_init);
+      digest[gc] = digest_row<HB>(row, (delta & 4) != 0, HB, d_init);
     }
     __syncwarp();
     if (c + STAGES < c_hi) {
       bool vn;
-      const int64_t tn = issue(c + STAGES, s, vn);
+      int64_t gn = 0;
+      const int64_t tn = issue(c + STAGES, s, vn, gn);
 #pragma unroll
-      for (int q = 0; q < STAGES; ++q) if (q == s) { v[q] = vn; t[q] = tn; }
+      for (int q = 0; q < STAGES; ++q) if (q == s) { v[q] = vn; t[q] = tn; gi[q] = gn; }
     }
     s = s + 1 == STAGES ? 0 : s + 1;
   }
@@ -934,7 +951,8 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
                   const int64_t* d_offsets, int32_t n, cudaStream_t s) {
   const int B = idx->cfg.block_size;
   const uint64_t d_init = mix64(idx->cfg.hash_seed ^ (uint64_t)B);
-  const int64_t max_chunks = (n_tokens / B + kChunk - 1) / kChunk;
+  // request-aligned chunks (TMA kernel) number at most blocks / 32 + n
+  const int64_t max_chunks = (n_tokens / B + kChunk - 1) / kChunk + (HB > 0 ? n : 0);
   // rows of 16*nch bytes: a block's 4B bytes start at most 12 bytes past a
   // 16-byte boundary
   const int nch = HB > 0 ? HB / 2 + 1 : (4 * B + 12 + 15) / 16;
@@ -955,8 +973,9 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
       }
       const int64_t want = (max_chunks + warps - 1) / warps;
       const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * idx->digest_occ));
-      kern<<<(unsigned)grid, warps * 32, smem, s>>>(maps, d_tokens, n_tokens, d_offsets, idx->block_off, n,
-                                                    d_init, idx->batch_ok, idx->digest, idx->status);
+      kern<<<(unsigned)grid, warps * 32, smem, s>>>(maps, d_tokens, n_tokens, d_offsets, idx->block_off,
+                                                    idx->chunk_off, n, d_init, idx->batch_ok, idx->digest,
+                                                    idx->status);
       idx->launches++;
       return cuda_status(cudaGetLastError());
     }
@@ -1113,7 +1132,7 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
 
   profile_begin(idx, s);
   k_prep<<<1, 1024, 0, s>>>(d_offsets, n, n_tokens, c.block_size, d_load, PROBE ? c.num_instances : 0,
-                            idx->block_off, idx->batch_ok, idx->status);
+                            idx->block_off, idx->chunk_off, idx->batch_ok, idx->status);
   idx->launches++;
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   profile_mark(idx, kPrep, s);
@@ -1325,7 +1344,7 @@ extern "C" int smetric_block_hashes_noalloc(const int32_t* d_tokens, int64_t n_t
   uint64_t* digest = scratch + kNaFlagWords + kNaOffWords;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
-  k_prep<<<1, 1024, 0, s>>>(d_offsets, n_requests, n_tokens, B, nullptr, 0, block_off, ok, d_status);
+  k_prep<<<1, 1024, 0, s>>>(d_offsets, n_requests, n_tokens, B, nullptr, 0, block_off, nullptr, ok, d_status);
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   if (n_tokens / B > 0) {
     const uint64_t d_init = mix64(hash_seed ^ (uint64_t)B);
