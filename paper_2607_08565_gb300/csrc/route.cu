@@ -27,6 +27,7 @@
 #include <stdint.h>
 
 #include <algorithm>
+#include <utility>
 #include <atomic>
 #include <cstring>
 
@@ -37,6 +38,13 @@ using namespace smetric;
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
+
+// Programmatic dependent launch: a route kernel launched with programmatic
+// stream serialisation is set up while its predecessor still runs and waits
+// here until that predecessor has finished and its writes are visible (a
+// no-op for an ordinary launch). No kernel triggers its successor early:
+// successors waiting on the SMs during a kernel's run measured slower.
+__device__ __forceinline__ void pdl_enter() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
 constexpr int kChunk = 32;        // blocks per digest task (one per lane)
 constexpr int kDigestWarps = 8;   // most warps per digest CTA
 constexpr int kTmaWarps = 16;     // warps per TMA digest CTA (one stage each)
@@ -213,6 +221,7 @@ __global__ void __launch_bounds__(kDigestWarps * 32)
     k_digest(const int32_t* __restrict__ tokens, int64_t n_tokens, const int64_t* __restrict__ off,
              const int64_t* __restrict__ block_off, int32_t n, uint64_t d_init,
              const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ digest) {
+  pdl_enter();
   constexpr int B = 2 * HB;
   constexpr int PB = HB > 0 ? HB / 2 : 1;  // 16-byte pieces per block (k_digest<0> is never launched)
   constexpr int NP = PB + 1;  // pieces per row (the block plus its misalignment)
@@ -355,6 +364,7 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
                  int64_t n_tokens, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off,
                  const int64_t* __restrict__ chunk_off, int32_t n, uint64_t d_init, const int32_t* __restrict__ batch_ok,
                  uint64_t* __restrict__ digest, int32_t* status) {
+  pdl_enter();
   constexpr int B = 2 * HB;
   constexpr int NP = HB / 2 + 1;           // 16-byte pieces per row
   constexpr uint32_t ROW = 16u * NP;       // = 4B + 16
@@ -464,6 +474,7 @@ __global__ void __launch_bounds__(kDigestWarps * 32)
     k_digest_any(const int32_t* __restrict__ tokens, int64_t n_tokens, const int64_t* __restrict__ off,
                  const int64_t* __restrict__ block_off, int32_t n, int B, int nch, uint64_t d_init,
                  const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ digest) {
+  pdl_enter();
   extern __shared__ uint4 dsm[];
   if (!*batch_ok) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, warps = blockDim.x >> 5;
@@ -538,6 +549,7 @@ __global__ void __launch_bounds__(kChainThreads)
             int S, uint64_t h_init, const int32_t* __restrict__ batch_ok,
             const uint64_t* __restrict__ digest, uint64_t* __restrict__ hashes,
             uint64_t* __restrict__ sk_out, uint64_t* __restrict__ groups, uint64_t gmask) {
+  pdl_enter();
   const int32_t r = blockIdx.x * kChainThreads + threadIdx.x;
   if (r >= n) return;
   if (!*batch_ok) { sk_out[r] = 0; return; }
@@ -618,6 +630,7 @@ __global__ void __launch_bounds__(256)
     k_group(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
             const uint64_t* __restrict__ groups, uint64_t gmask, const uint64_t* __restrict__ H,
             int32_t* __restrict__ lead, int32_t* __restrict__ share) {
+  pdl_enter();
   if (!*batch_ok) return;
   const int lane = threadIdx.x & 31;
   const int64_t tw = (int64_t)gridDim.x * (blockDim.x >> 5);
@@ -713,6 +726,7 @@ __global__ void __launch_bounds__(256)
             const int64_t* __restrict__ block_off, int32_t n, const uint64_t* __restrict__ H,
             const int32_t* __restrict__ batch_ok, const int32_t* __restrict__ share,
             uint64_t* __restrict__ masks) {
+  pdl_enter();
   if (!*batch_ok) return;
   const int64_t total = block_off[n];
   int32_t r = 0;
@@ -744,6 +758,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
            const int32_t* __restrict__ lead, const int32_t* __restrict__ share,
            int32_t* __restrict__ inst_out, int32_t* __restrict__ lhit_out,
            int32_t* __restrict__ ghit_out, uint4* __restrict__ groups, int64_t group_vecs) {
+  pdl_enter();
   extern __shared__ int64_t msm[];
   int64_t* load_s = msm;                                                     // [N]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -899,6 +914,24 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
 
 void profile_mark(smetric_index* idx, int k, cudaStream_t s);
 
+// Launches a route kernel; with pdl the launch may begin while the previous
+// kernel on the stream is still running (the kernel waits in pdl_enter).
+template <typename... KArgs, typename... Args>
+int launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl,
+             Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = pdl ? attr : nullptr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cuda_status(cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...));
+}
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*,
                                   CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
@@ -973,11 +1006,10 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
       }
       const int64_t want = (max_chunks + warps - 1) / warps;
       const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * idx->digest_occ));
-      kern<<<(unsigned)grid, warps * 32, smem, s>>>(maps, d_tokens, n_tokens, d_offsets, idx->block_off,
-                                                    idx->chunk_off, n, d_init, idx->batch_ok, idx->digest,
-                                                    idx->status);
       idx->launches++;
-      return cuda_status(cudaGetLastError());
+      return launch_k(kern, dim3((unsigned)grid), dim3(warps * 32), smem, s, !idx->profiling, maps, d_tokens,
+                      n_tokens, d_offsets, (const int64_t*)idx->block_off, (const int64_t*)idx->chunk_off, n, d_init,
+                      (const int32_t*)idx->batch_ok, idx->digest, idx->status);
     }
   }
   const size_t per_warp = (size_t)kChunk * nch * 16;
@@ -995,14 +1027,14 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
   }
   const int64_t want = (max_chunks + warps - 1) / warps;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * idx->digest_occ));
-  if (HB > 0)
-    kern<<<(unsigned)grid, warps * 32, smem, s>>>(d_tokens, n_tokens, d_offsets, idx->block_off, n, d_init,
-                                                  idx->batch_ok, idx->digest);
-  else
-    k_digest_any<<<(unsigned)grid, warps * 32, smem, s>>>(d_tokens, n_tokens, d_offsets, idx->block_off, n, B,
-                                                          nch, d_init, idx->batch_ok, idx->digest);
   idx->launches++;
-  return cuda_status(cudaGetLastError());
+  if (HB > 0)
+    return launch_k(kern, dim3((unsigned)grid), dim3(warps * 32), smem, s, !idx->profiling, d_tokens, n_tokens,
+                    d_offsets, (const int64_t*)idx->block_off, n, d_init, (const int32_t*)idx->batch_ok,
+                    idx->digest);
+  return launch_k(k_digest_any, dim3((unsigned)grid), dim3(warps * 32), smem, s, !idx->profiling, d_tokens,
+                  n_tokens, d_offsets, (const int64_t*)idx->block_off, n, B, nch, d_init,
+                  (const int32_t*)idx->batch_ok, idx->digest);
 }
 
 int dispatch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
@@ -1026,12 +1058,10 @@ int launch_chain(smetric_index* idx, const int64_t* d_offsets, int32_t n, uint64
                  uint64_t* sk, bool group, cudaStream_t s) {
   const unsigned grid = (unsigned)((n + kChainThreads - 1) / kChainThreads);
   const uint64_t h_init = mix64(idx->cfg.hash_seed + kGamma);
-  k_chain<<<grid, kChainThreads, 0, s>>>(d_offsets, idx->block_off, n, idx->cfg.block_size,
-                                         idx->cfg.session_blocks, h_init, idx->batch_ok, idx->digest,
-                                         hashes ? hashes : idx->hashes, sk, group ? idx->groups : nullptr,
-                                         group_slots_for(n) - 1);
   idx->launches++;
-  return cuda_status(cudaGetLastError());
+  return launch_k(k_chain, dim3(grid), dim3(kChainThreads), 0, s, !idx->profiling, d_offsets, idx->block_off, n,
+                  idx->cfg.block_size, idx->cfg.session_blocks, h_init, idx->batch_ok, idx->digest,
+                  hashes ? hashes : idx->hashes, sk, group ? idx->groups : nullptr, group_slots_for(n) - 1);
 }
 
 template <int W>
@@ -1046,20 +1076,20 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
   {
     const int64_t want = ((int64_t)n + 7) / 8;
     const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
-    k_group<<<(unsigned)grid, 256, 0, s>>>(idx->block_off, n, idx->batch_ok, idx->groups,
-                                           group_slots_for(n) - 1, H, idx->lead, idx->share);
     idx->launches++;
-    if ((rc = cuda_status(cudaGetLastError()))) return rc;
+    if ((rc = launch_k(k_group, dim3((unsigned)grid), dim3(256), 0, s, !idx->profiling, idx->block_off, n,
+                       idx->batch_ok, idx->groups, group_slots_for(n) - 1, H, idx->lead, idx->share)))
+      return rc;
   }
   profile_mark(idx, kGroup, s);
   {
     // probe: one thread per block, grid sized to the largest possible batch
     const int64_t want = (max_blocks + 255) / 256;
     const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
-    k_probe<W><<<(unsigned)grid, 256, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->block_off, n, H,
-                                              idx->batch_ok, idx->share, idx->masks);
     idx->launches++;
-    if ((rc = cuda_status(cudaGetLastError()))) return rc;
+    if ((rc = launch_k(k_probe<W>, dim3((unsigned)grid), dim3(256), 0, s, !idx->profiling, idx->tags, idx->table,
+                       idx->n_buckets, idx->block_off, n, H, idx->batch_ok, idx->share, idx->masks)))
+      return rc;
   }
   profile_mark(idx, kProbe, s);
   const size_t smem = (size_t)N * sizeof(int64_t) + (size_t)kMatchWarps * N * (W + 1) * sizeof(uint64_t);
@@ -1069,13 +1099,11 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
     return cuda_status(cudaErrorInvalidValue);
   const int64_t want = ((int64_t)n + kMatchWarps - 1) / kMatchWarps;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
-  kern<<<(unsigned)grid, kMatchWarps * 32, smem, s>>>(N, idx->cfg.block_size, d_offsets, idx->block_off, n,
-                                                      d_load, w.w_load, w.w_miss, w.w_glob, idx->masks,
-                                                      idx->batch_ok, idx->lead, idx->share, inst, lhit, ghit,
-                                                      reinterpret_cast<uint4*>(idx->groups),
-                                                      (int64_t)group_slots_for(n));
   idx->launches++;
-  return cuda_status(cudaGetLastError());
+  return launch_k(kern, dim3((unsigned)grid), dim3(kMatchWarps * 32), smem, s, !idx->profiling, N,
+                  idx->cfg.block_size, d_offsets, idx->block_off, n, d_load, w.w_load, w.w_miss, w.w_glob,
+                  idx->masks, idx->batch_ok, idx->lead, idx->share, inst, lhit, ghit,
+                  reinterpret_cast<uint4*>(idx->groups), (int64_t)group_slots_for(n));
 }
 
 int dispatch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
