@@ -560,7 +560,7 @@ __global__ void __launch_bounds__(kChainThreads)
   const int64_t kS = (nb < S ? nb : S) - 1;
   uint64_t h = h_init;
   auto step = [](uint64_t hp, uint64_t db) {
-    uint64_t x = mix64((hp + kGamma) ^ db);
+    uint64_t x = mix64_halves((hp + kGamma) ^ db);
     if (x < 2) x |= 2;
     return x;
   };

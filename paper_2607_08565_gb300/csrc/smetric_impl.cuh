@@ -30,6 +30,29 @@ __host__ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
 // bucket, so a lookup is one tag read plus one entry read.
 constexpr int kBucket = 16;
 
+// mix64 on 32-bit halves, for the serial chain where only latency counts:
+// the high word of each product is one three-input sum of the low-by-low
+// high half and the two cross products. Same value as mix64.
+__device__ __forceinline__ uint64_t mix64_halves(uint64_t z) {
+  uint32_t lo = (uint32_t)z, hi = (uint32_t)(z >> 32);
+  auto xs = [&](int s) {
+    lo ^= __funnelshift_r(lo, hi, s);
+    hi ^= hi >> s;
+  };
+  auto mul = [&](uint64_t c) {
+    const uint32_t cl = (uint32_t)c, ch = (uint32_t)(c >> 32);
+    const uint32_t x1 = lo * ch, x2 = hi * cl;
+    hi = __umulhi(lo, cl) + x1 + x2;
+    lo = lo * cl;
+  };
+  xs(30);
+  mul(0xBF58476D1CE4E5B9ull);
+  xs(27);
+  mul(0x94D049BB133111EBull);
+  xs(31);
+  return ((uint64_t)hi << 32) | lo;
+}
+
 __device__ __forceinline__ uint64_t home_bucket(uint64_t key, uint64_t n_buckets) {
   return __umul64hi(key, n_buckets);
 }
