@@ -159,3 +159,48 @@ def test_config5_corner_points_sampled(N, B):
     sel = {f: g[f][sample] for f in ("instance", "local_hit", "global_hit", "session_key")}
     assert_outputs_equal(sel, o, fields=("instance", "local_hit", "global_hit", "session_key"))
     ix.close()
+
+
+@pytest.mark.parametrize("N,B,batch", [(256, 16, 8192), (8, 64, 8192), (64, 32, 32768)])
+def test_config5_full_size_points_sampled(N, B, batch):
+    """Config-5 sweep points at the full session count, in the benchmark's
+    launch configuration: the most instances with the smallest blocks, the
+    fewest with the largest, and the largest batch. Random filler keys with
+    random tiers pad the table to load factor 0.7 of its capacity; the
+    oracle recomputes a sample of requests one by one and invariants are
+    checked on every request."""
+    tr = burst_trace("c5_sweep", num_instances=N, block_size=B, batch_size=batch)
+    p = tr.params
+    nkeys = tr.n_prefix_blocks()
+    n_fill = nkeys // 2
+    bt = tr.batch(1)
+    ix = make_index(N, B, p.session_blocks, cap=int((nkeys + n_fill) / 0.7) + 1,
+                    max_req=max(bt.n_requests, 4096), max_tok=bt.n_tokens)
+    _populate_c4(ix, tr)
+    fk, ft = tr.filler_keys(n_fill)
+    ix.insert(T(fk.view(np.int64)), T(ft))
+    ix.check()
+    w = (p.w_load, p.w_miss, p.w_glob)
+    g = gpu_route(ix, bt.tokens, bt.offsets, bt.load, w, want_hashes=False)
+    lens = bt.lengths()
+    assert np.all((g["instance"] >= 0) & (g["instance"] < N))
+    assert np.all(g["local_hit"] + g["global_hit"] <= (lens // B) * B)
+    rng = np.random.default_rng(N + B)
+    sample = np.sort(rng.choice(bt.n_requests, size=48, replace=False))
+    ox = oracle.OracleIndex(N)
+    sample_hashes = []
+    for s in np.unique(bt.sessions[sample]).tolist():
+        h = oracle.block_hashes(tr.session_prefix(s), B, p.hash_seed)
+        sample_hashes.append(h)
+        for t in tr.session_tiers(s):
+            ox.insert(h, t)
+    from synth.traces import pack
+    st, so = pack([bt.tokens[bt.offsets[r]:bt.offsets[r + 1]] for r in sample])
+    o = ox.route_batch(B, p.session_blocks, p.hash_seed, st, so, bt.load, *w, want_hashes=True)
+    # the oracle leaves out the filler keys (tens of millions): exact as long
+    # as none of them equals a block hash of the sample, which is checked
+    assert not np.isin(np.concatenate(sample_hashes + [o["block_hashes"]]), fk).any()
+    sel = {f: g[f][sample] for f in ("instance", "local_hit", "global_hit", "session_key")}
+    assert_outputs_equal(sel, o, fields=("instance", "local_hit", "global_hit", "session_key"),
+                         ctx=f"config 5 N={N} B={B} batch={batch}")
+    ix.close()
