@@ -534,21 +534,18 @@ __device__ __forceinline__ void st_v4(uint64_t* p, uint64_t a, uint64_t b, uint6
   asm volatile("st.global.v4.u64 [%0], {%1,%2,%3,%4};\n" ::"l"(p), "l"(a), "l"(b), "l"(c), "l"(d) : "memory");
 }
 
-// End of a request's chain: the session key and the first block's hash are
-// read back rather than tested at every serial step; the latter enters the
-// group table.
+// End of a request's chain: the session key is read back rather than tested
+// at every serial step.
 __device__ __forceinline__ void nb_done(int32_t r, int64_t nb, const uint64_t* hout, int64_t kS,
-                                        uint64_t* __restrict__ sk_out, uint64_t* __restrict__ groups,
-                                        uint64_t gmask) {
+                                        uint64_t* __restrict__ sk_out) {
   sk_out[r] = nb > 0 ? hout[kS] : 0;
-  if (groups && nb > 0) group_insert(groups, gmask, hout[0], r);
 }
 
 __global__ void __launch_bounds__(kChainThreads)
     k_chain(const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n, int B,
             int S, uint64_t h_init, const int32_t* __restrict__ batch_ok,
             const uint64_t* __restrict__ digest, uint64_t* __restrict__ hashes,
-            uint64_t* __restrict__ sk_out, uint64_t* __restrict__ groups, uint64_t gmask) {
+            uint64_t* __restrict__ sk_out) {
   pdl_enter();
   const int32_t r = blockIdx.x * kChainThreads + threadIdx.x;
   if (r >= n) return;
@@ -575,7 +572,7 @@ __global__ void __launch_bounds__(kChainThreads)
       h = step(h, __ldg(d + k));
       hout[k] = h;
     }
-    nb_done(r, nb, hout, kS, sk_out, groups, gmask);
+    nb_done(r, nb, hout, kS, sk_out);
     return;
   }
   int64_t b = 0;
@@ -613,24 +610,44 @@ __global__ void __launch_bounds__(kChainThreads)
     h = step(h, __ldg(d + k));
     hout[k] = h;
   }
-  nb_done(r, nb, hout, kS, sk_out, groups, gmask);
+  nb_done(r, nb, hout, kS, sk_out);
 }
 
 // ---------------------------------------------------------------------------
 // group
 // ---------------------------------------------------------------------------
 
+// The group stage works from the digests, so that it runs beside the chain:
+// a request's first-block hash h_0 = chain step from h_init over d_0 is the
+// group key, and the shared-prefix length is the number of leading blocks
+// whose digests equal the leader's. Equal digests from equal previous hashes
+// give equal hashes, so the leader's masks serve those blocks exactly.
+__device__ __forceinline__ uint64_t first_hash(uint64_t h_init, uint64_t d0) {
+  uint64_t h = mix64((h_init + kGamma) ^ d0);
+  return h < 2 ? (h | 2) : h;
+}
+
+// One thread per request: its first-block hash into the group table.
+__global__ void __launch_bounds__(256)
+    k_group_insert(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
+                   const uint64_t* __restrict__ digest, uint64_t h_init, uint64_t* __restrict__ groups,
+                   uint64_t gmask) {
+  const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= n || !*batch_ok) return;
+  const int64_t bo = block_off[r];
+  if (block_off[r + 1] > bo) group_insert(groups, gmask, first_hash(h_init, __ldg(digest + bo)), (int32_t)r);
+}
+
 // One warp per request: its leader (the group table's entry for its first
-// block hash) and share = the number of leading blocks whose hashes equal the
-// leader's. Both sides look up the same finished table, so a request that
-// leads a group finds itself (share 0) and its masks cover all its blocks;
-// a member's mask for block b < share is the leader's, which is exact because
+// block hash) and share = the number of leading blocks whose digests equal
+// the leader's. Both sides look up the same finished table, so a request
+// that leads a group finds itself (share 0) and its masks cover all its
+// blocks; a member's mask for block b < share is the leader's, exact because
 // a block's tier masks are a function of its hash alone.
 __global__ void __launch_bounds__(256)
     k_group(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
-            const uint64_t* __restrict__ groups, uint64_t gmask, const uint64_t* __restrict__ H,
-            int32_t* __restrict__ lead, int32_t* __restrict__ share) {
-  pdl_enter();
+            const uint64_t* __restrict__ groups, uint64_t gmask, const uint64_t* __restrict__ D,
+            uint64_t h_init, int32_t* __restrict__ lead, int32_t* __restrict__ share) {
   if (!*batch_ok) return;
   const int lane = threadIdx.x & 31;
   const int64_t tw = (int64_t)gridDim.x * (blockDim.x >> 5);
@@ -639,7 +656,7 @@ __global__ void __launch_bounds__(256)
     int32_t l = (int32_t)r;
     int64_t sh = 0;
     if (nb > 0) {
-      const uint64_t key = __ldg(H + bo);
+      const uint64_t key = first_hash(h_init, __ldg(D + bo));
       const uint64_t s0 = key & gmask;
       for (uint64_t t = 0; t <= gmask; t += 32) {
         const uint64_t sl = (s0 + t + lane) & gmask;
@@ -663,7 +680,7 @@ __global__ void __launch_bounds__(256)
 #pragma unroll
           for (int u = 0; u < kGroupAhead; ++u) {
             const int64_t bb = b + 32 * u + lane;
-            ne[u] = bb < m && __ldg(H + bo + bb) != __ldg(H + lo + bb);
+            ne[u] = bb < m && __ldg(D + bo + bb) != __ldg(D + lo + bb);
           }
           int64_t first = -1;
 #pragma unroll
@@ -1055,13 +1072,30 @@ uint64_t group_slots_for(int32_t n) {
 }
 
 int launch_chain(smetric_index* idx, const int64_t* d_offsets, int32_t n, uint64_t* hashes,
-                 uint64_t* sk, bool group, cudaStream_t s) {
+                 uint64_t* sk, bool pdl, cudaStream_t s) {
   const unsigned grid = (unsigned)((n + kChainThreads - 1) / kChainThreads);
   const uint64_t h_init = mix64(idx->cfg.hash_seed + kGamma);
   idx->launches++;
-  return launch_k(k_chain, dim3(grid), dim3(kChainThreads), 0, s, !idx->profiling, d_offsets, idx->block_off, n,
+  return launch_k(k_chain, dim3(grid), dim3(kChainThreads), 0, s, pdl, d_offsets, idx->block_off, n,
                   idx->cfg.block_size, idx->cfg.session_blocks, h_init, idx->batch_ok, idx->digest,
-                  hashes ? hashes : idx->hashes, sk, group ? idx->groups : nullptr, group_slots_for(n) - 1);
+                  hashes ? hashes : idx->hashes, sk);
+}
+
+// The group stage (k_group_insert, then k_group) on stream s.
+int launch_group(smetric_index* idx, int32_t n, cudaStream_t s) {
+  const uint64_t h_init = mix64(idx->cfg.hash_seed + kGamma);
+  const uint64_t gmask = group_slots_for(n) - 1;
+  k_group_insert<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(idx->block_off, n, idx->batch_ok, idx->digest, h_init,
+                                                             idx->groups, gmask);
+  idx->launches++;
+  int rc = cuda_status(cudaGetLastError());
+  if (rc) return rc;
+  const int64_t want = ((int64_t)n + 7) / 8;
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
+  k_group<<<(unsigned)grid, 256, 0, s>>>(idx->block_off, n, idx->batch_ok, idx->groups, gmask, idx->digest, h_init,
+                                         idx->lead, idx->share);
+  idx->launches++;
+  return cuda_status(cudaGetLastError());
 }
 
 template <int W>
@@ -1070,24 +1104,29 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
                  uint64_t* sk, int64_t max_blocks, cudaStream_t s) {
   const int N = idx->cfg.num_instances;
   const uint64_t* H = hashes ? hashes : idx->hashes;
-  int rc = launch_chain(idx, d_offsets, n, hashes, sk, true, s);
-  if (rc) return rc;
-  profile_mark(idx, kChain, s);
-  {
-    const int64_t want = ((int64_t)n + 7) / 8;
-    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
-    idx->launches++;
-    if ((rc = launch_k(k_group, dim3((unsigned)grid), dim3(256), 0, s, !idx->profiling, idx->block_off, n,
-                       idx->batch_ok, idx->groups, group_slots_for(n) - 1, H, idx->lead, idx->share)))
-      return rc;
+  int rc;
+  if (idx->profiling) {  // one stream, so that each kernel's events bracket it alone
+    if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, false, s))) return rc;
+    profile_mark(idx, kChain, s);
+    if ((rc = launch_group(idx, n, s))) return rc;
+    profile_mark(idx, kGroup, s);
+  } else {
+    // the group stage needs only the digests: it runs on the side stream
+    // beside the latency-bound chain
+    if (cudaEventRecord(idx->fork_ev, s) != cudaSuccess || cudaStreamWaitEvent(idx->side, idx->fork_ev, 0) != cudaSuccess)
+      return cuda_status(cudaErrorUnknown);
+    if ((rc = launch_group(idx, n, idx->side))) return rc;
+    if (cudaEventRecord(idx->join_ev, idx->side) != cudaSuccess) return cuda_status(cudaErrorUnknown);
+    if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, false, s))) return rc;
+    if (cudaStreamWaitEvent(s, idx->join_ev, 0) != cudaSuccess) return cuda_status(cudaErrorUnknown);
   }
-  profile_mark(idx, kGroup, s);
   {
     // probe: one thread per block, grid sized to the largest possible batch
     const int64_t want = (max_blocks + 255) / 256;
     const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
     idx->launches++;
-    if ((rc = launch_k(k_probe<W>, dim3((unsigned)grid), dim3(256), 0, s, !idx->profiling, idx->tags, idx->table,
+    // an ordinary launch: it follows the wait for the side stream
+    if ((rc = launch_k(k_probe<W>, dim3((unsigned)grid), dim3(256), 0, s, false, idx->tags, idx->table,
                        idx->n_buckets, idx->block_off, n, H, idx->batch_ok, idx->share, idx->masks)))
       return rc;
   }
@@ -1173,7 +1212,7 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
                              n_tokens / c.block_size, s)))
       return rc;
   } else {
-    if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, false, s))) return rc;
+    if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, !idx->profiling, s))) return rc;
     profile_mark(idx, kChain, s);
     profile_mark(idx, kGroup, s);
     profile_mark(idx, kProbe, s);
@@ -1386,7 +1425,6 @@ extern "C" int smetric_block_hashes_noalloc(const int32_t* d_tokens, int64_t n_t
   }
   const unsigned grid = (unsigned)((n_requests + kChainThreads - 1) / kChainThreads);
   k_chain<<<grid, kChainThreads, 0, s>>>(d_offsets, block_off, n_requests, B, session_blocks,
-                                         mix64(hash_seed + kGamma), ok, digest, d_block_hashes, d_session_key,
-                                         nullptr, 0);
+                                         mix64(hash_seed + kGamma), ok, digest, d_block_hashes, d_session_key);
   return cuda_status(cudaGetLastError());
 }

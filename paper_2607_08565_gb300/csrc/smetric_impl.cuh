@@ -117,6 +117,8 @@ struct smetric_index {
   int32_t* lead;       // max_batch_requests: the request whose masks a request shares
   int32_t* share;      // max_batch_requests: leading blocks taken from the leader
   int64_t* chunk_off;  // max_batch_requests + 1: first 32-block chunk of each request
+  cudaStream_t side;   // runs the group stage beside the chain
+  cudaEvent_t fork_ev, join_ev;
   int32_t* batch_ok;   // device flag written by the prep kernel
   // staging for smetric_route_batch_host
   int32_t* st_tokens;
