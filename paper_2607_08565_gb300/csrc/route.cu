@@ -66,7 +66,7 @@ __device__ __forceinline__ int64_t warp_incl_scan(int64_t v, int lane) {
   return v;
 }
 
-constexpr int kPrepPer = 8;  // requests per thread per pass
+constexpr int kPrepRounds = 8;  // rounds of 32 consecutive requests per warp per pass
 
 __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, int32_t n,
                                               int64_t n_tokens, int B, const int64_t* __restrict__ load,
@@ -74,6 +74,7 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
                                               int64_t* __restrict__ chunk_off, int32_t* batch_ok,
                                               int32_t* status) {
   constexpr int NS = 2;  // scans: full blocks, and 32-block chunks (when chunk_off is wanted)
+  constexpr int R = kPrepRounds;
   __shared__ int64_t warp_tot[NS][32];
   __shared__ int64_t pass_tot[NS];
   __shared__ int bad_all;
@@ -85,35 +86,40 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
     const int64_t v = load[i];
     if (v < 0 || v > SMETRIC_MAX_LOAD) bad |= 2;
   }
-  // Passes of kPrepPer consecutive requests per thread: every offset of a
-  // pass is loaded before any is used, then one block-wide scan per count.
+  // A pass gives each warp R rounds of 32 consecutive requests (lane = request),
+  // so that offsets are loaded and both outputs stored coalesced. Every offset
+  // of the pass is loaded before any is used; the counts stay in registers
+  // between the warp sums and the scans that write the outputs.
   int64_t carry[NS] = {0, 0};
-  for (int64_t base = 0; base < n; base += (int64_t)blockDim.x * kPrepPer) {
-    const int64_t r0 = base + (int64_t)tid * kPrepPer;
-    int64_t o[kPrepPer + 1];
+  for (int64_t base = 0; base < n; base += (int64_t)blockDim.x * R) {
+    const int64_t seg = base + (int64_t)warp * 32 * R + lane;
+    int64_t a[R], b[R];
 #pragma unroll
-    for (int i = 0; i <= kPrepPer; ++i) o[i] = r0 + i <= n ? off[r0 + i] : 0;
-    uint32_t nbv[kPrepPer];
+    for (int i = 0; i < R; ++i) {
+      const int64_t r = seg + 32 * i;
+      a[i] = r < n ? off[r] : 0;
+      b[i] = r < n ? off[r + 1] : 0;
+    }
+    uint32_t nbv[R];
 #pragma unroll
-    for (int i = 0; i < kPrepPer; ++i) {
+    for (int i = 0; i < R; ++i) {
       uint32_t v = 0;
-      if (r0 + i < n) {
-        const int64_t a = o[i], b = o[i + 1];
-        if (a < 0 || b < a || b > n_tokens) bad |= 1;
-        else if (b - a > (int64_t)INT32_MAX) bad |= 2;
-        else v = (uint32_t)(b - a) / (uint32_t)B;
+      if (seg + 32 * i < n) {
+        if (a[i] < 0 || b[i] < a[i] || b[i] > n_tokens) bad |= 1;
+        else if (b[i] - a[i] > (int64_t)INT32_MAX) bad |= 2;
+        else v = (uint32_t)(b[i] - a[i]) / (uint32_t)B;
       }
       nbv[i] = v;
     }
     auto cnt = [&](int k, int i) -> int64_t { return k == 0 ? nbv[i] : (nbv[i] + 31) >> 5; };
-    int64_t sum[NS], incl[NS];
 #pragma unroll
     for (int k = 0; k < NS; ++k) {
-      sum[k] = 0;
+      int64_t t = 0;
 #pragma unroll
-      for (int i = 0; i < kPrepPer; ++i) sum[k] += cnt(k, i);
-      incl[k] = warp_incl_scan(sum[k], lane);
-      if (lane == 31) warp_tot[k][warp] = incl[k];
+      for (int i = 0; i < R; ++i) t += cnt(k, i);
+#pragma unroll
+      for (int d = 16; d > 0; d >>= 1) t += __shfl_xor_sync(kFull, t, d);
+      if (lane == 0) warp_tot[k][warp] = t;
     }
     __syncthreads();
     if (warp == 0) {
@@ -130,13 +136,14 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
     for (int k = 0; k < NS; ++k) {
       int64_t* const dst = k == 0 ? block_off : chunk_off;
       if (!dst) continue;
-      int64_t run = carry[k] + warp_tot[k][warp] + incl[k] - sum[k];
+      int64_t run = carry[k] + warp_tot[k][warp];  // exclusive start of this warp's rounds
 #pragma unroll
-      for (int i = 0; i < kPrepPer; ++i) {
-        if (r0 + i < n) {
-          dst[r0 + i] = run;
-          run += cnt(k, i);
-        }
+      for (int i = 0; i < R; ++i) {
+        const int64_t c = cnt(k, i);
+        const int64_t incl = warp_incl_scan(c, lane);
+        const int64_t r = seg + 32 * i;
+        if (r < n) dst[r] = run + incl - c;
+        run += __shfl_sync(kFull, incl, 31);
       }
       carry[k] += pass_tot[k];
     }
