@@ -137,6 +137,21 @@ def peak_hbm():
         return 6800.0, "fallback"
 
 
+def section_sha(section: str) -> str:
+    """Hash of one kernel's source: its section of route.cu (from its
+    `// <section>` banner to the next banner) plus the shared device header."""
+    csrc = os.path.join(ROOT, "paper_2607_08565_gb300", "csrc")
+    text = open(os.path.join(csrc, "route.cu")).read()
+    banner = "// " + "-" * 75 + "\n"
+    parts = text.split(banner)
+    body = next((parts[i + 1] for i in range(len(parts) - 1) if parts[i].rstrip("\n").endswith("// " + section)), None)
+    if body is None:
+        return ""
+    h = hashlib.sha256(body.encode())
+    h.update(open(os.path.join(csrc, "smetric_impl.cuh"), "rb").read())
+    return h.hexdigest()[:16]
+
+
 def ncu_traffic(kernel: str):
     """Per-launch DRAM bytes of `kernel` from the committed ncu summary, if
     that summary was taken on the current kernel source; else None."""
@@ -146,9 +161,8 @@ def ncu_traffic(kernel: str):
             rec = json.load(f)[kernel]
     except (OSError, KeyError, ValueError):
         return None
-    src = os.path.join(ROOT, "paper_2607_08565_gb300", "csrc", rec["source"])
-    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-    return rec["bytes_per_launch"] if sha == rec["source_sha"] else None
+    sha = section_sha(rec["section"]) if "section" in rec else ""
+    return rec["bytes_per_launch"] if sha and sha == rec["source_sha"] else None
 
 
 # ---------------------------------------------------------------------------
