@@ -192,6 +192,9 @@ void free_all(smetric_index* x) {
   cudaFree(x->digest);
   cudaFree(x->hashes);
   cudaFree(x->masks);
+  cudaFree(x->summ);
+  cudaFree(x->chunk_and);
+  cudaFree(x->order);
   cudaFree(x->groups);
   cudaFree(x->lead);
   cudaFree(x->chunk_off);
@@ -253,9 +256,12 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
             cudaMalloc(&x->digest, (max_blocks > 0 ? max_blocks : 1) * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->hashes, (max_blocks > 0 ? max_blocks : 1) * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->masks, (max_blocks > 0 ? max_blocks : 1) * W * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&x->chunk_and, (max_blocks / 32 + 1) * W * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->groups, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->lead, 2 * (R + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->chunk_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
+            cudaMalloc(&x->order, (R + 2) * sizeof(int32_t)) == cudaSuccess &&
+            cudaMalloc(&x->summ, (R > 0 ? R : 1) * ((size_t)c.num_instances + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->batch_ok, sizeof(int32_t)) == cudaSuccess;
   if (ok) x->share = x->lead + (R + 1);
   if (ok)

@@ -638,8 +638,9 @@ __device__ __forceinline__ uint64_t first_hash(uint64_t h_init, uint64_t d0) {
 __global__ void __launch_bounds__(256)
     k_group_insert(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
                    const uint64_t* __restrict__ digest, uint64_t h_init, uint64_t* __restrict__ groups,
-                   uint64_t gmask) {
+                   uint64_t gmask, int32_t* __restrict__ counts) {
   const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (r == 0) { counts[0] = 0; counts[1] = 0; }  // k_group's leader and member counts
   if (r >= n || !*batch_ok) return;
   const int64_t bo = block_off[r];
   if (block_off[r + 1] > bo) group_insert(groups, gmask, first_hash(h_init, __ldg(digest + bo)), (int32_t)r);
@@ -654,7 +655,8 @@ __global__ void __launch_bounds__(256)
 __global__ void __launch_bounds__(256)
     k_group(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
             const uint64_t* __restrict__ groups, uint64_t gmask, const uint64_t* __restrict__ D,
-            uint64_t h_init, int32_t* __restrict__ lead, int32_t* __restrict__ share) {
+            uint64_t h_init, int32_t* __restrict__ lead, int32_t* __restrict__ share,
+            int32_t* __restrict__ order, int32_t* __restrict__ counts) {
   if (!*batch_ok) return;
   const int lane = threadIdx.x & 31;
   const int64_t tw = (int64_t)gridDim.x * (blockDim.x >> 5);
@@ -701,7 +703,13 @@ __global__ void __launch_bounds__(256)
         l = (int32_t)r;
       }
     }
-    if (lane == 0) { lead[r] = l; share[r] = (int32_t)sh; }
+    if (lane == 0) {
+      lead[r] = l;
+      share[r] = (int32_t)sh;
+      // leaders listed from the front, members from the back (any order)
+      if (l == (int32_t)r) order[atomicAdd(counts, 1)] = (int32_t)r;
+      else order[n - 1 - atomicAdd(counts + 1, 1)] = (int32_t)r;
+    }
   }
 }
 
@@ -744,24 +752,46 @@ __device__ __forceinline__ void probe_one(const uint8_t* __restrict__ tags, cons
 }
 
 // One thread per block of the batch: the tier masks of every block hash.
+// Each warp also stores the AND of its 32 blocks' masks (blocks 32k..32k+31
+// of the batch, a block the kernel skips counting as all ones): for a chunk
+// that lies wholly inside one request's probed blocks this is the set of
+// tiers holding every block of the chunk, which lets the walk cross such a
+// chunk in one step.
 template <int W>
 __global__ void __launch_bounds__(256)
     k_probe(const uint8_t* __restrict__ tags, const uint64_t* __restrict__ table, uint64_t n_buckets,
             const int64_t* __restrict__ block_off, int32_t n, const uint64_t* __restrict__ H,
             const int32_t* __restrict__ batch_ok, const int32_t* __restrict__ share,
-            uint64_t* __restrict__ masks) {
+            uint64_t* __restrict__ masks, uint64_t* __restrict__ chunk_and) {
   pdl_enter();
   if (!*batch_ok) return;
   const int64_t total = block_off[n];
+  const int lane = threadIdx.x & 31;
   int32_t r = 0;
-  for (int64_t f = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; f < total;
-       f += (int64_t)gridDim.x * blockDim.x) {
-    r = find_request(block_off, r, n, f);
-    if (f - __ldg(block_off + r) < __ldg(share + r)) continue;  // the leader's mask serves
+  // warp-uniform loop over 32-aligned chunks (the stride is a multiple of 32)
+  for (int64_t f0 = blockIdx.x * (int64_t)blockDim.x + (threadIdx.x & ~31); f0 < total;
+       f0 += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t f = f0 + lane;
     uint64_t M[W];
-    probe_one<W>(tags, table, n_buckets, __ldg(H + f), M);
+    bool act = f < total;
+    if (act) {
+      r = find_request(block_off, r, n, f);
+      act = f - __ldg(block_off + r) >= __ldg(share + r);  // else the leader's mask serves
+    }
+    if (act) {
+      probe_one<W>(tags, table, n_buckets, __ldg(H + f), M);
 #pragma unroll
-    for (int w = 0; w < W; ++w) masks[f * W + w] = M[w];
+      for (int w = 0; w < W; ++w) masks[f * W + w] = M[w];
+    } else {
+#pragma unroll
+      for (int w = 0; w < W; ++w) M[w] = ~0ull;
+    }
+#pragma unroll
+    for (int w = 0; w < W; ++w) {
+      const uint64_t a = (uint64_t)__reduce_and_sync(kFull, (unsigned)M[w]) |
+                         ((uint64_t)__reduce_and_sync(kFull, (unsigned)(M[w] >> 32)) << 32);
+      if (lane == w) chunk_and[(f0 >> 5) * W + w] = a;
+    }
   }
 }
 
@@ -774,12 +804,22 @@ __global__ void __launch_bounds__(256)
 // lanes = instances: c_i = the block of the first event containing i (or n_r
 // if i held every block), the cost, and a shuffle argmin with ties to the
 // lowest id.
-template <int W>
+//
+// Two passes. The first walks the group leaders over their own masks and
+// records each leader's run ends (c_i for every instance, then g) in `summ`.
+// The second walks the members: a member's blocks before `share` are the
+// leader's, so a run that ended there ended at the same block, and a run
+// alive through share - 1 continues over the member's own masks from block
+// `share` on. Members therefore start at `share` instead of re-reading the
+// leader's masks from block 0.
+template <int W, bool MEMBERS>
 __global__ void __launch_bounds__(kMatchWarps * 32)
     k_walk(int N, int B, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n,
            const int64_t* __restrict__ load, int64_t w_load, int64_t w_miss, int64_t w_glob,
-           const uint64_t* __restrict__ masks, const int32_t* __restrict__ batch_ok,
-           const int32_t* __restrict__ lead, const int32_t* __restrict__ share,
+           const uint64_t* __restrict__ masks, const uint64_t* __restrict__ chunk_and,
+           const int32_t* __restrict__ batch_ok,
+           const int32_t* __restrict__ lead, const int32_t* __restrict__ share, int32_t* __restrict__ summ,
+           const int32_t* __restrict__ order, const int32_t* __restrict__ counts,
            int32_t* __restrict__ inst_out, int32_t* __restrict__ lhit_out,
            int32_t* __restrict__ ghit_out, uint4* __restrict__ groups, int64_t group_vecs) {
   pdl_enter();
@@ -797,35 +837,70 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
   const int64_t tw = (int64_t)gridDim.x * kMatchWarps;
   const unsigned lt = (1u << lane) - 1;
 
-  for (int64_t r = (int64_t)blockIdx.x * kMatchWarps + warp; r < n; r += tw) {
-    if (!ok) {
+  if (!ok && !MEMBERS)
+    for (int64_t r = (int64_t)blockIdx.x * kMatchWarps + warp; r < n; r += tw)
       if (lane == 0) { inst_out[r] = -1; lhit_out[r] = 0; ghit_out[r] = 0; }
-      continue;
-    }
+  // k_group's lists: leaders from the front of `order`, members from the back
+  const int64_t count = !ok ? 0 : MEMBERS ? counts[1] : counts[0];
+  for (int64_t k = (int64_t)blockIdx.x * kMatchWarps + warp; k < count; k += tw) {
+    const int64_t r = MEMBERS ? order[n - 1 - k] : order[k];
+    const int32_t l = lead[r];
     const int64_t L = off[r + 1] - off[r];
     const int64_t nb = L / B;
-    const uint64_t* const m_r = masks + block_off[r] * W;
-    const uint64_t* const m_l = masks + block_off[lead[r]] * W;
-    const int64_t sh = share[r];
-    uint64_t A[W];  // local tiers holding every block so far (warp-uniform)
+    const int64_t bo = block_off[r];
+    const int64_t sh = MEMBERS ? share[r] : 0;
+    const int32_t* const cl = summ + (int64_t)l * (N + 1);  // the leader's run ends
+    // the first step's loads (see below) go out with the leader's run ends
+    int64_t f = bo + sh;
+    const int64_t F1 = bo + nb;
+    const bool head_single = (f & 31) || F1 - f < 32;
+    uint64_t pre[W];
 #pragma unroll
     for (int w = 0; w < W; ++w) {
-      const int lo = w * 64;
-      A[w] = N >= lo + 64 ? ~0ull : (N > lo ? (1ull << (N - lo)) - 1 : 0ull);
+      if (head_single) {
+        const int64_t len = min((int64_t)(32 - (f & 31)), F1 - f);
+        pre[w] = lane < len ? __ldg(masks + (f + lane) * W + w) : ~0ull;
+      } else {
+        pre[w] = lane < ((F1 - f) >> 5) ? __ldg(chunk_and + ((f >> 5) + lane) * W + w) : 0;
+      }
     }
+    constexpr int CT = 2 * W;  // groups of 32 covering the N + 1 <= 64 W run ends
+    int32_t cv[CT];            // cv[t] = the leader's run end of tier 32 t + lane (g at tier N)
+    uint64_t A[W];  // local tiers holding every block so far (warp-uniform)
     bool galive = true;
     int64_t g = 0;
+    if (!MEMBERS) {
+#pragma unroll
+      for (int w = 0; w < W; ++w) {
+        const int lo = w * 64;
+        A[w] = N >= lo + 64 ? ~0ull : (N > lo ? (1ull << (N - lo)) - 1 : 0ull);
+      }
+    } else {
+#pragma unroll
+      for (int t = 0; t < CT; ++t) cv[t] = 32 * t + lane <= N ? __ldg(cl + 32 * t + lane) : 0;
+      int32_t gl = 0;
+#pragma unroll
+      for (int t = 0; t < CT; ++t) {
+        const unsigned alive = __ballot_sync(kFull, 32 * t + lane < N && cv[t] >= sh);
+        if ((t & 1) == 0) A[t >> 1] = alive;
+        else A[t >> 1] |= (uint64_t)alive << 32;
+        if (t == (N >> 5)) gl = __shfl_sync(kFull, cv[t], N & 31);
+      }
+      galive = gl >= sh;
+      g = galive ? sh : gl;
+    }
     int ne = 0;
-    // 32 blocks with lane j holding block base + j: the runs that end there
+    // `len` consecutive blocks from request block `base`, lane j < len holding
+    // block base + j (lanes past len hold all ones): the runs that end there
     // become events; returns true once no run is alive
-    auto half = [&](int64_t base, const uint64_t (&x)[W]) -> bool {
+    auto span = [&](int64_t base, int len, const uint64_t (&x)[W]) -> bool {
       if (galive) {
         uint64_t mg = 0;
 #pragma unroll
         for (int w = 0; w < W; ++w) if (w == gword) mg = x[w];
         const unsigned miss = __ballot_sync(kFull, !(mg & gbit));
         if (miss) { g = base + __ffs(miss) - 1; galive = false; }
-        else g = base + 32;
+        else g = base + len;
       }
       bool dies = false, any = false;
       uint64_t X[W];
@@ -854,62 +929,77 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
       ne += __popc(ev);
       return !any && !galive;
     };
-    auto mask_at = [&](int64_t bb, int w) -> uint64_t {
-      return bb < nb ? __ldg((bb < sh ? m_l : m_r) + bb * W + w) : 0;
-    };
-    // rounds of 64 blocks, lane j holding blocks base + j and base + 32 + j,
-    // the next round's masks in flight
-    uint64_t n0[W], n1[W];
+    bool dead = !galive;
 #pragma unroll
-    for (int w = 0; w < W; ++w) { n0[w] = mask_at(lane, w); n1[w] = mask_at(32 + lane, w); }
-    for (int64_t base = 0; base < nb; base += 64) {
-      uint64_t x0[W], x1[W];
+    for (int w = 0; w < W; ++w) dead &= A[w] == 0;
+    // From block sh: single blocks up to a 32-aligned batch position, then
+    // 32 chunks per step from their AND summaries (lane = chunk); the first
+    // chunk that ends an alive run is walked block by block, and the request's
+    // last partial chunk too. The first step uses the loads issued above.
+    bool first = true;
+    while (!dead && f < F1) {
+      uint64_t x[W];
+      if ((f & 31) || F1 - f < 32) {
+        const int len = (int)min((int64_t)(32 - (f & 31)), F1 - f);
 #pragma unroll
-      for (int w = 0; w < W; ++w) {
-        x0[w] = n0[w];
-        x1[w] = n1[w];
-        n0[w] = mask_at(base + 64 + lane, w);
-        n1[w] = mask_at(base + 96 + lane, w);
-      }
-      // fast path: every run alive before this round survives all of its 64
-      // blocks (the usual case; blocks past the last hold 0 and so always take
-      // the full path)
-      bool keep = true;
-#pragma unroll
-      for (int w = 0; w < W; ++w) {
-        const uint64_t both = x0[w] & x1[w];
-        const uint64_t all = (uint64_t)__reduce_and_sync(kFull, (unsigned)both) |
-                             ((uint64_t)__reduce_and_sync(kFull, (unsigned)(both >> 32)) << 32);
-        keep &= (all & A[w]) == A[w];
-        if (w == gword && galive) keep &= (all & gbit) != 0;
-      }
-      if (keep) {
-        if (galive) g = base + 64;
+        for (int w = 0; w < W; ++w)
+          x[w] = first ? pre[w] : lane < len ? __ldg(masks + (f + lane) * W + w) : ~0ull;
+        first = false;
+        dead = span(f - bo, len, x);
+        f += len;
         continue;
       }
-      if (half(base, x0)) break;
-      if (half(base + 32, x1)) break;
+      const int64_t nfull = (F1 - f) >> 5;
+#pragma unroll
+      for (int w = 0; w < W; ++w)
+        x[w] = first ? pre[w] : lane < nfull ? __ldg(chunk_and + ((f >> 5) + lane) * W + w) : 0;
+      first = false;
+      bool stop = lane >= nfull;
+#pragma unroll
+      for (int w = 0; w < W; ++w) {
+        stop |= (x[w] & A[w]) != A[w];
+        if (w == gword && galive) stop |= !(x[w] & gbit);
+      }
+      const unsigned sm = __ballot_sync(kFull, stop);
+      const int j = sm ? __ffs(sm) - 1 : 32;
+      f += 32 * (int64_t)j;  // chunks that keep every alive run
+      if (galive) g = f - bo;
+      if (j < nfull && j < 32) {
+#pragma unroll
+        for (int w = 0; w < W; ++w) x[w] = __ldg(masks + (f + lane) * W + w);
+        dead = span(f - bo, 32, x);
+        f += 32;
+      }
     }
+    if (galive) g = nb;  // the global run reaches the last block
     __syncwarp();
     // cost of every instance; lanes = instances
     int64_t best_cost = INT64_MAX;
     int32_t best = N;
     int64_t best_c = 0;
-    for (int i = lane; i < N; i += 32) {
+    int32_t* const out_c = summ + r * (N + 1);
+#pragma unroll
+    for (int t = 0; t < CT; ++t) {
+      const int i = 32 * t + lane;
+      if (i >= N) break;
       const int wi = i >> 6;
       const uint64_t bi = 1ull << (i & 63);
       uint64_t aw = 0;
 #pragma unroll
       for (int w = 0; w < W; ++w) if (w == wi) aw = A[w];
       int64_t ci = nb;
-      if (!(aw & bi)) {
+      if (MEMBERS && cv[t] < sh) {
+        ci = cv[t];  // ended on the shared blocks, as in the leader
+      } else if (!(aw & bi)) {
         for (int e = 0; e < ne; ++e)
           if (ev_mask[e * W + wi] & bi) { ci = ev_pos[e]; break; }
       }
+      if (!MEMBERS) out_c[i] = (int32_t)ci;
       const int64_t gi = ci > g ? ci : g;
       const int64_t cost = w_load * load_s[i] + w_miss * (L - B * gi) + w_glob * B * (gi - ci);
       if (cost < best_cost) { best_cost = cost; best = i; best_c = ci; }
     }
+    if (!MEMBERS && lane == 0) out_c[N] = (int32_t)g;
 #pragma unroll
     for (int dd = 16; dd > 0; dd >>= 1) {
       const int64_t oc = __shfl_xor_sync(kFull, best_cost, dd);
@@ -925,11 +1015,13 @@ __global__ void __launch_bounds__(kMatchWarps * 32)
     }
     __syncwarp();
   }
-  // k_group has read the group table: empty it for the next route (it is
-  // zero from index creation before the first)
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < group_vecs;
-       i += (int64_t)gridDim.x * blockDim.x)
-    groups[i] = make_uint4(0, 0, 0, 0);
+  if (MEMBERS) {
+    // k_group has read the group table: empty it for the next route (it is
+    // zero from index creation before the first)
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < group_vecs;
+         i += (int64_t)gridDim.x * blockDim.x)
+      groups[i] = make_uint4(0, 0, 0, 0);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -1092,15 +1184,17 @@ int launch_chain(smetric_index* idx, const int64_t* d_offsets, int32_t n, uint64
 int launch_group(smetric_index* idx, int32_t n, cudaStream_t s) {
   const uint64_t h_init = mix64(idx->cfg.hash_seed + kGamma);
   const uint64_t gmask = group_slots_for(n) - 1;
+  int32_t* const counts = idx->order + idx->cfg.max_batch_requests;
   k_group_insert<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(idx->block_off, n, idx->batch_ok, idx->digest, h_init,
-                                                             idx->groups, gmask);
+                                                             idx->groups, gmask, counts);
   idx->launches++;
   int rc = cuda_status(cudaGetLastError());
   if (rc) return rc;
   const int64_t want = ((int64_t)n + 7) / 8;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
   k_group<<<(unsigned)grid, 256, 0, s>>>(idx->block_off, n, idx->batch_ok, idx->groups, gmask, idx->digest, h_init,
-                                         idx->lead, idx->share);
+                                         idx->lead, idx->share,
+                                         idx->order, counts);
   idx->launches++;
   return cuda_status(cudaGetLastError());
 }
@@ -1134,22 +1228,28 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
     idx->launches++;
     // an ordinary launch: it follows the wait for the side stream
     if ((rc = launch_k(k_probe<W>, dim3((unsigned)grid), dim3(256), 0, s, false, idx->tags, idx->table,
-                       idx->n_buckets, idx->block_off, n, H, idx->batch_ok, idx->share, idx->masks)))
+                       idx->n_buckets, idx->block_off, n, H, idx->batch_ok, idx->share, idx->masks,
+                       idx->chunk_and)))
       return rc;
   }
   profile_mark(idx, kProbe, s);
   const size_t smem = (size_t)N * sizeof(int64_t) + (size_t)kMatchWarps * N * (W + 1) * sizeof(uint64_t);
-  auto kern = k_walk<W>;
-  if (smem > 48 * 1024 &&
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
-    return cuda_status(cudaErrorInvalidValue);
   const int64_t want = ((int64_t)n + kMatchWarps - 1) / kMatchWarps;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
-  idx->launches++;
-  return launch_k(kern, dim3((unsigned)grid), dim3(kMatchWarps * 32), smem, s, !idx->profiling, N,
-                  idx->cfg.block_size, d_offsets, idx->block_off, n, d_load, w.w_load, w.w_miss, w.w_glob,
-                  idx->masks, idx->batch_ok, idx->lead, idx->share, inst, lhit, ghit,
-                  reinterpret_cast<uint4*>(idx->groups), (int64_t)group_slots_for(n));
+  // leaders, then members (which read the leaders' run ends)
+  for (auto kern : {k_walk<W, false>, k_walk<W, true>}) {
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+      return cuda_status(cudaErrorInvalidValue);
+    idx->launches++;
+    if ((rc = launch_k(kern, dim3((unsigned)grid), dim3(kMatchWarps * 32), smem, s, !idx->profiling, N,
+                       idx->cfg.block_size, d_offsets, idx->block_off, n, d_load, w.w_load, w.w_miss, w.w_glob,
+                       idx->masks, idx->chunk_and, idx->batch_ok, idx->lead, idx->share, idx->summ, idx->order,
+                       idx->order + idx->cfg.max_batch_requests, inst, lhit, ghit,
+                       reinterpret_cast<uint4*>(idx->groups), (int64_t)group_slots_for(n))))
+      return rc;
+  }
+  return SMETRIC_OK;
 }
 
 int dispatch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,

@@ -112,10 +112,13 @@ struct smetric_index {
   uint64_t* digest;    // max_batch_tokens / B: per-block digests d_b
   uint64_t* hashes;    // max_batch_tokens / B: per-block chain hashes h_b
   uint64_t* masks;     // W * max_batch_tokens / B: per-block tier masks
+  uint64_t* chunk_and; // W * ceil(max_batch_tokens / B / 32): AND of each 32-block chunk's masks
   uint64_t* groups;    // 2 * group_slots: (first-block hash, INT32_MAX - leader) pairs
   uint64_t group_slots;  // power of two >= 2 * max_batch_requests
   int32_t* lead;       // max_batch_requests: the request whose masks a request shares
   int32_t* share;      // max_batch_requests: leading blocks taken from the leader
+  int32_t* summ;       // max_batch_requests * (num_instances + 1): a leader's run ends c_i, then g
+  int32_t* order;      // max_batch_requests + 2: leaders from the front, members from the back, then both counts
   int64_t* chunk_off;  // max_batch_requests + 1: first 32-block chunk of each request
   cudaStream_t side;   // runs the group stage beside the chain
   cudaEvent_t fork_ev, join_ev;

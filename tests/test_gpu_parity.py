@@ -364,5 +364,5 @@ def test_profile_and_launch_count():
     prof = pkg.smetric_profile_read(ix.handle)
     assert set(prof) == {"k_prep", "k_digest", "k_chain", "k_group", "k_probe", "k_walk"}
     assert all(v[1] == 3 and v[0] > 0 for v in prof.values())
-    assert pkg.smetric_launch_count(ix.handle) - before == 21  # 7 kernels per route
+    assert pkg.smetric_launch_count(ix.handle) - before == 24  # 8 kernels per route
     pkg.smetric_profile_enable(ix.handle, False)
