@@ -382,10 +382,13 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
   // chunk c is chunk q of request r: its blocks 32q .. 32q+31, so a chunk
   // never spans two requests
   const int64_t n_chunks = chunk_off[n];
-  const int64_t tw = (int64_t)gridDim.x * warps;
-  const int64_t per = (n_chunks + tw - 1) / tw;
-  const int64_t c_lo = ((int64_t)blockIdx.x * warps + warp) * per;
-  const int64_t c_hi = min(n_chunks, c_lo + per);
+  // A CTA takes a contiguous range of chunks and its warps interleave over it
+  // (warp w: chunks w, w + warps, ...), so that the copies a CTA has in flight
+  // cover one stretch of consecutive tokens.
+  const int64_t per = (n_chunks + gridDim.x - 1) / gridDim.x;  // chunks per CTA
+  const int64_t k_lo = (int64_t)blockIdx.x * per;
+  const int64_t c_hi = min(n_chunks, k_lo + per);
+  const int64_t c_lo = k_lo + warp;  // then every warps-th chunk of the CTA's range
   if (c_lo >= c_hi) return;
   unsigned char* const stages = dsm_raw + (size_t)warp * STAGES * STAGE;
   const uint32_t mbar0 = smem_u32(dsm_raw + (size_t)warps * STAGES * STAGE) + 8u * STAGES * (uint32_t)warp;
@@ -404,6 +407,7 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
   // Start the copy of chunk c into stage s; returns this lane's first token
   // and sets its digest index.
   auto issue = [&](int64_t c, int s, bool& valid, int64_t& gidx) -> int64_t {
+    for (int i = 0; i < 4 && __ldg(chunk_off + r + 1) <= c; ++i) ++r;  // usually a step or two
     if (__ldg(chunk_off + r + 1) <= c) r = find_request(chunk_off, r + 1, n, c);
     const int64_t bo = __ldg(block_off + r), nbr = __ldg(block_off + r + 1) - bo;
     const int64_t b = (c - __ldg(chunk_off + r)) * kChunk + lane;  // block of request r
@@ -443,9 +447,9 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
   int64_t t[STAGES], gi[STAGES];
 #pragma unroll
   for (int s = 0; s < STAGES; ++s)
-    if (c_lo + s < c_hi) t[s] = issue(c_lo + s, s, v[s], gi[s]);
+    if (c_lo + s * warps < c_hi) t[s] = issue(c_lo + s * warps, s, v[s], gi[s]);
   int s = 0;
-  for (int64_t c = c_lo; c < c_hi; ++c) {
+  for (int64_t c = c_lo; c < c_hi; c += warps) {
     if (!mbar_wait(mbar0 + 8u * (uint32_t)s, (phase >> s) & 1)) { failed = true; break; }
     phase ^= 1u << s;
     bool vc = false;
@@ -458,10 +462,10 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
       digest[gc] = digest_row<HB>(row, (delta & 4) != 0, HB, d_init);
     }
     __syncwarp();
-    if (c + STAGES < c_hi) {
+    if (c + STAGES * warps < c_hi) {
       bool vn;
       int64_t gn = 0;
-      const int64_t tn = issue(c + STAGES, s, vn, gn);
+      const int64_t tn = issue(c + STAGES * warps, s, vn, gn);
 #pragma unroll
       for (int q = 0; q < STAGES; ++q) if (q == s) { v[q] = vn; t[q] = tn; gi[q] = gn; }
     }
