@@ -139,7 +139,8 @@ def peak_hbm():
 
 def section_sha(section: str) -> str:
     """Hash of one kernel's source: its section of route.cu (from its
-    `// <section>` banner to the next banner) plus the shared device header."""
+    `// <section>` banner to the next banner), the file's preamble of launch
+    constants, and the shared device header."""
     csrc = os.path.join(ROOT, "paper_2607_08565_gb300", "csrc")
     text = open(os.path.join(csrc, "route.cu")).read()
     banner = "// " + "-" * 75 + "\n"
@@ -147,7 +148,7 @@ def section_sha(section: str) -> str:
     body = next((parts[i + 1] for i in range(len(parts) - 1) if parts[i].rstrip("\n").endswith("// " + section)), None)
     if body is None:
         return ""
-    h = hashlib.sha256(body.encode())
+    h = hashlib.sha256(parts[0].encode() + body.encode())
     h.update(open(os.path.join(csrc, "smetric_impl.cuh"), "rb").read())
     return h.hexdigest()[:16]
 

@@ -47,7 +47,8 @@ constexpr unsigned kFull = 0xffffffffu;
 __device__ __forceinline__ void pdl_enter() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
 constexpr int kChunk = 32;        // blocks per digest task (one per lane)
 constexpr int kDigestWarps = 8;   // most warps per digest CTA
-constexpr int kTmaWarps = 16;     // warps per TMA digest CTA (one stage each)
+constexpr int kTmaWarps = 24;     // warps per TMA digest CTA (two CTAs per SM)
+constexpr int kTmaStages = 1;     // copy stages per TMA digest warp
 constexpr int kChainThreads = 32;   // one warp per CTA: chains spread over every SM
 constexpr int kChainAhead = 16;   // digests prefetched per request
 constexpr int kMatchWarps = 8;    // warps per walk CTA
@@ -1096,8 +1097,6 @@ bool make_token_maps(TokenMaps& m, const int32_t* tokens, int64_t n_tokens, int 
   }
   return true;
 }
-
-constexpr int kTmaStages = 1;
 
 template <int HB>
 int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
