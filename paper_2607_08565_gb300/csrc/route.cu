@@ -818,7 +818,7 @@ __global__ void __launch_bounds__(256)
 // `share` on. Members therefore start at `share` instead of re-reading the
 // leader's masks from block 0.
 template <int W, bool MEMBERS>
-__global__ void __launch_bounds__(kMatchWarps * 32)
+__global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 1)  // members: 5 CTAs (40 warps) per SM
     k_walk(int N, int B, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n,
            const int64_t* __restrict__ load, int64_t w_load, int64_t w_miss, int64_t w_glob,
            const uint64_t* __restrict__ masks, const uint64_t* __restrict__ chunk_and,

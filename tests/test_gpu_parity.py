@@ -319,6 +319,38 @@ def test_route_rejects_bad_offsets_and_loads():
                                 T(np.zeros(3, np.uint64)))
 
 
+def test_batch_of_3100_requests_parity_and_late_errors():
+    """A batch of 3,100 requests (several passes of the offset scan's warps):
+    outputs equal the oracle's, an invalid offset early, in the middle or at
+    the end of the batch, or a bad load, is caught, and the next good batch is
+    unaffected."""
+    rng = np.random.default_rng(31)
+    N, B, S = 5, 8, 2
+    stored, reqs = tiny_alphabet_case(rng, N, B, n_req=3100, max_blocks=12)
+    ix = make_index(N, B, S, cap=1 << 15, max_req=4096)
+    ox = oracle.OracleIndex(N)
+    populate_both(ix, ox, stored, B)
+    tok, off = pack(reqs)
+    load = rng.integers(0, 50, size=N)
+    before = pkg.smetric_launch_count(ix.handle)
+    g = gpu_route(ix, tok, off, load, (1, 4, 2))
+    assert pkg.smetric_launch_count(ix.handle) - before == 8
+    o = ox.route_batch(B, S, 0, tok, off, load, 1, 4, 2, want_hashes=True)
+    assert_outputs_equal(g, o, ctx="3100 requests")
+    for r in (0, 1500, 2600, 3099):  # ranges of the first, a middle and the last CTA
+        bad = off.copy()
+        bad[r + 1] = bad[r] - 1 if bad[r] > 0 else len(tok) + 1
+        out = ix.route_batch(T(tok), T(bad), T(load), (1, 4, 2))
+        assert ix.status() == pkg.SMETRIC_ERR_INVALID_ARG, r
+        assert np.all(out["instance"].cpu().numpy() == -1)
+    out = ix.route_batch(T(tok), T(off), T(np.array([0, 0, -1, 0, 0])), (1, 4, 2))
+    assert ix.status() == pkg.SMETRIC_ERR_OVERFLOW
+    assert np.all(out["instance"].cpu().numpy() == -1)
+    g = gpu_route(ix, tok, off, load, (1, 4, 2))  # the next good batch is unaffected
+    assert_outputs_equal(g, o, ctx="after errors")
+    ix.close()
+
+
 def test_empty_batch_and_token_free_batch():
     ix = make_index(3, 16, 1)
     out = ix.route_batch(T(np.zeros(0, np.int32)), T(np.zeros(1, np.int64)),
