@@ -133,21 +133,26 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
       }
     }
     __syncthreads();
+    // both scans side by side, so that their shuffle chains overlap; rounds
+    // past the last request are skipped (the test is warp-uniform)
+    int64_t run[NS];
 #pragma unroll
-    for (int k = 0; k < NS; ++k) {
-      int64_t* const dst = k == 0 ? block_off : chunk_off;
-      if (!dst) continue;
-      int64_t run = carry[k] + warp_tot[k][warp];  // exclusive start of this warp's rounds
+    for (int k = 0; k < NS; ++k) run[k] = carry[k] + warp_tot[k][warp];  // this warp's exclusive start
 #pragma unroll
-      for (int i = 0; i < R; ++i) {
-        const int64_t c = cnt(k, i);
-        const int64_t incl = warp_incl_scan(c, lane);
-        const int64_t r = seg + 32 * i;
-        if (r < n) dst[r] = run + incl - c;
-        run += __shfl_sync(kFull, incl, 31);
+    for (int i = 0; i < R; ++i) {
+      if (seg - lane + 32 * i >= n) break;
+      const int64_t r = seg + 32 * i;
+      const int64_t c0 = cnt(0, i), c1 = cnt(1, i);
+      const int64_t i0 = warp_incl_scan(c0, lane), i1 = warp_incl_scan(c1, lane);
+      if (r < n) {
+        block_off[r] = run[0] + i0 - c0;
+        if (chunk_off) chunk_off[r] = run[1] + i1 - c1;
       }
-      carry[k] += pass_tot[k];
+      run[0] += __shfl_sync(kFull, i0, 31);
+      run[1] += __shfl_sync(kFull, i1, 31);
     }
+#pragma unroll
+    for (int k = 0; k < NS; ++k) carry[k] += pass_tot[k];
     __syncthreads();  // warp_tot and pass_tot are rewritten by the next pass
   }
   if (bad) atomicOr(&bad_all, bad);
