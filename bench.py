@@ -140,7 +140,7 @@ def peak_hbm():
 def section_sha(section: str) -> str:
     """Hash of one kernel's source: its section of route.cu (from its
     `// <section>` banner to the next banner), the file's preamble of launch
-    constants, and the shared device header."""
+    constants, and the shared device header, comments left out."""
     csrc = os.path.join(ROOT, "paper_2607_08565_gb300", "csrc")
     text = open(os.path.join(csrc, "route.cu")).read()
     banner = "// " + "-" * 75 + "\n"
@@ -148,8 +148,16 @@ def section_sha(section: str) -> str:
     body = next((parts[i + 1] for i in range(len(parts) - 1) if parts[i].rstrip("\n").endswith("// " + section)), None)
     if body is None:
         return ""
-    h = hashlib.sha256(parts[0].encode() + body.encode())
-    h.update(open(os.path.join(csrc, "smetric_impl.cuh"), "rb").read())
+    def code(t):  # comments and blank lines do not change a kernel
+        out = []
+        for line in t.splitlines():
+            line = line.split("//")[0].rstrip()
+            if line:
+                out.append(line)
+        return "\n".join(out).encode()
+
+    h = hashlib.sha256(code(parts[0]) + code(body))
+    h.update(code(open(os.path.join(csrc, "smetric_impl.cuh")).read()))
     return h.hexdigest()[:16]
 
 

@@ -2,25 +2,32 @@
 // match, integer cost and argmin (Figure 6 and Figure 10 of the paper, with
 // every request of the batch routed against one snapshot of index and load).
 //
-// Five kernels per batch, in stream order:
-//   k_prep    one CTA: validates offsets and loads, exclusive-scans the
-//             per-request full-block counts into block_off.
-//   k_digest  HBM-bound: each warp owns a contiguous range of 32-block chunks
-//             of the flattened batch. A chunk whose blocks belong to one
-//             request is one contiguous span: the warp loads it with
-//             coalesced 16-byte loads into registers one chunk ahead and
-//             scatters it into shared memory, one row per block padded to a
-//             16-byte multiple so that lane j reading word k of block j hits
-//             a distinct bank pair; lane j folds block j's B/2 words into d_b.
-//   k_chain   one thread per request: the serial chain h_b over its digests
-//             (sixteen digests prefetched ahead) and the session key.
-//   k_probe   one thread per block: the tier masks of h_b from the index
-//             (16 tags of the home bucket, then the matching entry).
-//   k_walk    one warp per request, lanes = 32 consecutive blocks: an AND-scan
-//             of the local-tier masks across lanes gives each lane the set of
-//             instances whose run ends at its block (an event), the global
-//             run is located by ballot; then lanes = instances for the cost
-//             and a shuffle argmin with ties to the lowest id.
+// Kernels per batch, in stream order (the group stage on a side stream):
+//   k_prep        one CTA: validates offsets and loads; scans the per-request
+//                 full-block counts into block_off and the 32-block chunk
+//                 counts into chunk_off.
+//   k_digest_tma  HBM-bound block digests d_b: chunk q of request r is its
+//                 blocks 32q..32q+31, one 2D TMA tile of 32 overlapping rows
+//                 (each block's bytes rounded out to 16-byte boundaries); a
+//                 CTA takes a contiguous range of chunks, its warps
+//                 interleaved over it; lane j folds block j's B/2 words.
+//                 (k_digest and k_digest_any cover block sizes the tensor
+//                 maps do not.)
+//   k_group_insert, k_group   (side stream, beside k_chain) each request's
+//                 first-block hash into a group table, then its leader and
+//                 the number of leading blocks whose digests equal the
+//                 leader's.
+//   k_chain       one thread per request: the serial chain h_b over its
+//                 digests and the session key.
+//   k_probe       one thread per block not shared with the leader: the tier
+//                 masks of h_b from the index (16 tags of the home bucket,
+//                 then the matching entry), and per warp the AND of its 32
+//                 blocks' masks.
+//   k_walk        leaders, then members: one warp per request walks the runs
+//                 of the local tiers and the global tier, 32 chunks per step
+//                 from the chunk ANDs and block by block where a run ends;
+//                 then lanes = instances for the cost and a shuffle argmin
+//                 with ties to the lowest id.
 
 #include <cuda.h>
 #include <cuda_runtime.h>
