@@ -530,23 +530,6 @@ __global__ void __launch_bounds__(kDigestWarps * 32)
 // chain
 // ---------------------------------------------------------------------------
 
-// Requests whose first block hashes are equal form a group; its leader is
-// the lowest request id. Table of (key, INT32_MAX - leader) word pairs,
-// key 0 = empty (block hashes are >= 2), linear probing, at most half full.
-__device__ __forceinline__ void group_insert(uint64_t* __restrict__ groups, uint64_t gmask, uint64_t key,
-                                             int32_t r) {
-  uint64_t s = key & gmask;
-  for (uint64_t t = 0; t <= gmask; ++t) {
-    unsigned long long* const slot = reinterpret_cast<unsigned long long*>(groups + 2 * s);
-    const unsigned long long k = atomicCAS(slot, 0ull, (unsigned long long)key);
-    if (k == 0ull || k == key) {
-      atomicMax(slot + 1, (unsigned long long)(INT32_MAX - r));
-      return;
-    }
-    s = (s + 1) & gmask;
-  }
-}
-
 // 32-byte global load (read-only path) and store of four 64-bit words; the
 // address must be 32-byte aligned.
 __device__ __forceinline__ void ld_nc_v4(const uint64_t* p, uint64_t (&v)[4]) {
@@ -649,6 +632,23 @@ __global__ void __launch_bounds__(kChainThreads)
 __device__ __forceinline__ uint64_t first_hash(uint64_t h_init, uint64_t d0) {
   uint64_t h = mix64((h_init + kGamma) ^ d0);
   return h < 2 ? (h | 2) : h;
+}
+
+// Requests whose first block hashes are equal form a group; its leader is
+// the lowest request id. Table of (key, INT32_MAX - leader) word pairs,
+// key 0 = empty (block hashes are >= 2), linear probing, at most half full.
+__device__ __forceinline__ void group_insert(uint64_t* __restrict__ groups, uint64_t gmask, uint64_t key,
+                                             int32_t r) {
+  uint64_t s = key & gmask;
+  for (uint64_t t = 0; t <= gmask; ++t) {
+    unsigned long long* const slot = reinterpret_cast<unsigned long long*>(groups + 2 * s);
+    const unsigned long long k = atomicCAS(slot, 0ull, (unsigned long long)key);
+    if (k == 0ull || k == key) {
+      atomicMax(slot + 1, (unsigned long long)(INT32_MAX - r));
+      return;
+    }
+    s = (s + 1) & gmask;
+  }
 }
 
 // One thread per request: its first-block hash into the group table.
