@@ -58,6 +58,11 @@ def load_library(path: str):
     L.oracle_route_batch.argtypes = [
         C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p,
         C.c_int64, C.c_int64, C.c_int64, i32p, i32p, i32p, u64p, C.c_void_p, C.c_int32]
+    L.oracle_route_batch_policy.restype = C.c_int
+    L.oracle_route_batch_policy.argtypes = [
+        C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p, i32p, i64p,
+        C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int32,
+        i32p, i32p, i32p, i32p, u64p]
     return L
 
 
@@ -153,3 +158,29 @@ class OracleIndex:
         if want_hashes:
             out["block_hashes"] = hb[:nblk]
         return out
+
+    def route_batch_policy(self, block_size: int, session_blocks: int, seed: int, tokens, offsets,
+                           queued, turn, est_hit, c_lin: int, c_att: int, d0: int, d1: int,
+                           hit_num: int, hit_den: int, rr_base: int = 0):
+        """The session-centric policy of Figure 10. Returns dict(instance,
+        local_hit, global_hit, stick, session_key)."""
+        t = np.ascontiguousarray(tokens, dtype=np.int32)
+        o = np.ascontiguousarray(offsets, dtype=np.int64)
+        q = np.ascontiguousarray(queued, dtype=np.int64)
+        n = len(o) - 1
+        tu = np.ascontiguousarray(turn, dtype=np.int32)
+        eh = np.ascontiguousarray(est_hit, dtype=np.int64)
+        if len(q) != self.N or len(tu) != n or len(eh) != n:
+            raise ValueError("queued has one entry per instance; turn and est_hit one per request")
+        outs = [np.zeros(max(n, 1), np.int32) for _ in range(4)]
+        sk = np.zeros(max(n, 1), np.uint64)
+        rc = self._L.oracle_route_batch_policy(
+            self._h, block_size, session_blocks, seed & 0xFFFFFFFFFFFFFFFF,
+            t if len(t) else np.zeros(1, np.int32), o, n, q,
+            tu if n else np.zeros(1, np.int32), eh if n else np.zeros(1, np.int64),
+            c_lin, c_att, d0, d1, hit_num, hit_den, rr_base, *outs, sk)
+        if rc != 0:
+            raise ValueError(f"oracle_route_batch_policy: {rc}")
+        inst, lh, gh, st = outs
+        return dict(instance=inst[:n], local_hit=lh[:n], global_hit=gh[:n], stick=st[:n],
+                    session_key=sk[:n])

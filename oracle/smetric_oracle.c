@@ -49,6 +49,27 @@
  *  session_key = sk_r.
  *
  * Every request of a batch sees the same index and load (snapshot semantics).
+ *
+ * Session-centric policy (Figure 10, second epilogue over the same c_i and
+ * g; oracle_route_batch_policy). Figure 10(c), Eq. 1: the prefill cost of n
+ * new tokens in an L-token prompt is C_LIN*n + C_ATT*n*(L - n/2); here in
+ * fixed point and doubled so that it stays an integer:
+ *    n_i     = L_r - B*c_i
+ *    est2_i  = 2*q_i + 2*C_LIN*n_i + C_ATT*n_i*(2*L_r - n_i)
+ *              (= 2 * estimate_load(req, i), q_i = instance i's queued cost)
+ * Figure 10(a):
+ *    prev    = argmax_i c_i (lowest id among equals)
+ *    cached  = B*c_prev*HIT_DEN > HIT_NUM*est_hit_r   (session_cached; the
+ *              ratio HIT_RATIO = HIT_NUM/HIT_DEN, est_hit_r = the hit the
+ *              request's history leads one to expect)
+ * Figure 10(b): meets(i) = est2_i <= 2*(D0 + D1*L_r), the TTFT deadline in
+ * cost units (SLACK * PREFILL_RATE * (b + a*L)), none_meets = no i meets.
+ *    stick   = turn_r != 0 and cached and (meets(prev) or none_meets)
+ *    i*      = prev if stick, else the first minimal est2_i in the order
+ *              s, s+1, ..., N-1, 0, ..., s-1 with s = (rr_base + r) mod N
+ *              (rr_argmin: equal loads are taken in turn).
+ * Outputs: instance = i*, stick, local_hit = B*c_{i*}, global_hit =
+ * B*(max(c_{i*}, g) - c_{i*}), session_key as above.
  */
 #include <stdint.h>
 #include <stdlib.h>
@@ -295,4 +316,86 @@ int oracle_route_batch(const oracle_index* x, int32_t B, int32_t S, uint64_t see
   }
   free(before);
   return failed ? ORACLE_ERR_OOM : ORACLE_OK;
+}
+
+/* Session-centric policy (Figure 10) over the same hashes and prefix hits.
+ * Limits that keep every quantity below 2^63: L_r <= 2^24, C_LIN <= 2^20,
+ * C_ATT <= 2^12, 0 <= q_i <= 2^59, D0 <= 2^60, D1 <= 2^35,
+ * 0 <= est_hit_r < 2^31, 0 <= HIT_NUM <= HIT_DEN, 1 <= HIT_DEN <= 2^20,
+ * 0 <= rr_base < N; anything else returns ORACLE_ERR_INVALID_ARG. */
+int oracle_route_batch_policy(const oracle_index* x, int32_t B, int32_t S, uint64_t seed,
+                              const int32_t* tokens, const int64_t* offsets, int32_t n_requests,
+                              const int64_t* queued, const int32_t* turn, const int64_t* est_hit,
+                              int64_t c_lin, int64_t c_att, int64_t d0, int64_t d1, int64_t hit_num,
+                              int64_t hit_den, int32_t rr_base, int32_t* instance, int32_t* local_hit,
+                              int32_t* global_hit, int32_t* stick, uint64_t* session_key) {
+  if (!x || B < 2 || (B % 2) != 0 || S < 1 || n_requests < 0) return ORACLE_ERR_INVALID_ARG;
+  const int32_t N = x->N;
+  if (c_lin < 0 || c_lin > (1LL << 20) || c_att < 0 || c_att > (1LL << 12) || d0 < 0 ||
+      d0 > (1LL << 60) || d1 < 0 || d1 > (1LL << 35) || hit_den < 1 || hit_den > (1LL << 20) ||
+      hit_num < 0 || hit_num > hit_den || rr_base < 0 || rr_base >= N)
+    return ORACLE_ERR_INVALID_ARG;
+  for (int32_t i = 0; i < N; ++i)
+    if (queued[i] < 0 || queued[i] > (1LL << 59)) return ORACLE_ERR_INVALID_ARG;
+  for (int32_t r = 0; r < n_requests; ++r) {
+    if (offsets[r + 1] < offsets[r] || offsets[r] < 0 || offsets[r + 1] - offsets[r] > (1LL << 24))
+      return ORACLE_ERR_INVALID_ARG;
+    if (est_hit[r] < 0 || est_hit[r] >= (1LL << 31)) return ORACLE_ERR_INVALID_ARG;
+  }
+  int64_t* c = (int64_t*)malloc((size_t)N * sizeof(int64_t));
+  int64_t* est2 = (int64_t*)malloc((size_t)N * sizeof(int64_t));
+  uint64_t* h = NULL;
+  int64_t cap = 0;
+  int rc = ORACLE_OK;
+  if (!c || !est2) rc = ORACLE_ERR_OOM;
+  for (int32_t r = 0; r < n_requests && rc == ORACLE_OK; ++r) {
+    const int64_t L = offsets[r + 1] - offsets[r];
+    const int64_t n = L / B;
+    if (n + 1 > cap) {
+      free(h);
+      cap = n + 1;
+      h = (uint64_t*)malloc((size_t)cap * sizeof(uint64_t));
+      if (!h) { rc = ORACLE_ERR_OOM; break; }
+    }
+    oracle_block_hashes(tokens + offsets[r], L, B, seed, h);
+    int64_t g;
+    oracle_prefix_hits(x, h, n, c, &g);
+    /* (c) load model: doubled Eq. 1 plus the queued cost */
+    for (int32_t i = 0; i < N; ++i) {
+      const int64_t nn = L - (int64_t)B * c[i];
+      est2[i] = 2 * queued[i] + 2 * c_lin * nn + c_att * nn * (2 * L - nn);
+    }
+    /* (a) the instance that likely served the previous turn */
+    int32_t prev = 0;
+    for (int32_t i = 1; i < N; ++i)
+      if (c[i] > c[prev]) prev = i;
+    const int cached = (int64_t)B * c[prev] * hit_den > hit_num * est_hit[r];
+    /* (b) SLO checks */
+    const int64_t budget2 = 2 * (d0 + d1 * L);
+    int any_meets = 0;
+    for (int32_t i = 0; i < N; ++i)
+      if (est2[i] <= budget2) any_meets = 1;
+    const int meets_prev = est2[prev] <= budget2;
+    const int st = turn[r] != 0 && cached && (meets_prev || !any_meets);
+    int32_t to = prev;
+    if (!st) {
+      /* rr_argmin: the first minimal load in the order starting at s */
+      const int32_t s0 = (int32_t)(((int64_t)rr_base + r) % N);
+      to = s0;
+      for (int32_t k = 1; k < N; ++k) {
+        const int32_t i = (s0 + k) % N;
+        if (est2[i] < est2[to]) to = i;
+      }
+    }
+    const int64_t gt = c[to] > g ? c[to] : g;
+    instance[r] = to;
+    stick[r] = st;
+    local_hit[r] = (int32_t)((int64_t)B * c[to]);
+    global_hit[r] = (int32_t)((int64_t)B * (gt - c[to]));
+    session_key[r] = n == 0 ? 0 : h[(n < S ? n : S) - 1];
+  }
+  free(h);
+  free(c);
+  free(est2);
+  return rc;
 }

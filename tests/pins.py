@@ -380,6 +380,154 @@ def check_index_set_semantics(L):
                 assert ix.contains(key, tier) == (key in ref[tier])
 
 
+# ---------------------------------------------------------------------------
+# session-centric policy (Figure 10)
+# ---------------------------------------------------------------------------
+
+def eq1_cost(n, Lp, c_lin, c_att):
+    """Eq. 1 as printed: c_linear*n + c_attn*n*(L - n/2), exactly."""
+    return Fraction(c_lin) * n + Fraction(c_att) * n * (Lp - Fraction(n, 2))
+
+
+def _policy(ix, B, reqs, queued, turn, est_hit, c_lin=1, c_att=0, d0=1 << 60, d1=0,
+            hit_num=1, hit_den=2, rr_base=0, S=1):
+    from synth.traces import pack
+    tokens, offsets = pack(reqs)
+    return ix.route_batch_policy(B, S, 0, tokens, offsets, np.asarray(queued, np.int64),
+                                 np.asarray(turn, np.int32), np.asarray(est_hit, np.int64),
+                                 c_lin, c_att, d0, d1, hit_num, hit_den, rr_base)
+
+
+def _held(L, ix, t, B, tier_blocks):
+    h = oracle.block_hashes(t, B, 0, L)
+    for tier, k in tier_blocks.items():
+        if k:
+            ix.insert(h[:k], tier)
+
+
+def check_policy_eq1_boundary(L):
+    """Balance branch: the load model is Eq. 1 plus the queue. Instance 1
+    caches k blocks, instance 0 none; instance 1 wins exactly when
+    q_1 - q_0 < cost(L, L) - cost(L - kB, L), ties to instance 0."""
+    rng = np.random.default_rng(40)
+    for B, Lp, k, c_lin, c_att in ((4, 64, 5, 3, 1), (8, 77, 3, 1, 2), (2, 31, 9, 0, 7),
+                                   (16, 500, 17, 11, 3), (4, 9, 1, 5, 1)):
+        t = rng.integers(0, 151936, size=Lp, dtype=np.int32)
+        ix = oracle.OracleIndex(2, L)
+        _held(L, ix, t, B, {1: k})
+        T = eq1_cost(Lp, Lp, c_lin, c_att) - eq1_cost(Lp - k * B, Lp, c_lin, c_att)
+        lo, hi = T.numerator // T.denominator, -((-T.numerator) // T.denominator)
+        for D in (lo - 1, lo, hi, hi + 1):
+            q0 = 1 << 30
+            out = _policy(ix, B, [t], [q0, q0 + D], [0], [0], c_lin=c_lin, c_att=c_att)
+            want = 1 if D < T else 0
+            assert int(out["instance"][0]) == want, (B, Lp, k, D, T)
+            assert int(out["stick"][0]) == 0
+            assert int(out["local_hit"][0]) == (k * B if want else 0)
+
+
+def check_policy_first_turn_is_cost_argmin(L):
+    """First-turn requests take the balance branch; with C_ATT = 0 its load
+    q_i + C_LIN*(L - B*c_i) is the argmin cost of a3-a5 with w_load = 1,
+    w_miss = C_LIN and an empty global tier (one request, rotation from 0,
+    so ties go to the lowest id in both)."""
+    rng = np.random.default_rng(41)
+    B = 2
+    for trial in range(40):
+        N = int(rng.integers(1, 7))
+        base = rng.integers(0, 3, size=10 * B, dtype=np.int32)
+        ix = oracle.OracleIndex(N, L)
+        for i in range(N):
+            for _ in range(int(rng.integers(0, 3))):
+                ix.insert(oracle.block_hashes(_mutate(rng, base, int(rng.integers(0, 11 * B))), B, 0, L), i)
+        req = _mutate(rng, base, int(rng.integers(0, 11 * B)))
+        q = rng.integers(0, 30, size=N)
+        c_lin = int(rng.integers(0, 4))
+        a = _policy(ix, B, [req], q, [0], [0], c_lin=c_lin)
+        b = _route(ix, B, 1, [req], q, w=(1, c_lin, 0))
+        assert int(a["instance"][0]) == int(b["instance"][0])
+        assert int(a["local_hit"][0]) == int(b["local_hit"][0]) and int(a["stick"][0]) == 0
+
+
+def check_policy_sticks_to_longest_local_hit(L):
+    """A follow-up with a cached session and a loose deadline sticks to
+    prev = argmax_i c_i (lowest id among equals), whatever the loads."""
+    rng = np.random.default_rng(42)
+    B = 2
+    for trial in range(40):
+        N = int(rng.integers(1, 7))
+        base = rng.integers(0, 3, size=10 * B, dtype=np.int32)
+        stored = {i: [_mutate(rng, base, int(rng.integers(0, 11 * B)))
+                      for _ in range(int(rng.integers(0, 3)))] for i in range(N)}
+        ix = oracle.OracleIndex(N, L)
+        for i, ps in stored.items():
+            for p in ps:
+                ix.insert(oracle.block_hashes(p, B, 0, L), i)
+        req = _mutate(rng, base, int(rng.integers(0, 11 * B)))
+        c = [brute_hit(req, stored[i], B) for i in range(N)]
+        out = _policy(ix, B, [req], rng.integers(0, 1 << 20, size=N), [3], [0])
+        if max(c) > 0:
+            assert int(out["instance"][0]) == int(np.argmax(c)) and int(out["stick"][0]) == 1
+            assert int(out["local_hit"][0]) == B * max(c)
+        else:  # nothing cached: not session_cached, so balanced
+            assert int(out["stick"][0]) == 0
+
+
+def check_policy_session_cached_threshold(L):
+    """session_cached: c[prev] > HIT_RATIO * est_hit, strictly; at equality
+    the request is balanced like a first turn."""
+    rng = np.random.default_rng(43)
+    B, Lp, k = 4, 40, 6
+    t = rng.integers(0, 151936, size=Lp, dtype=np.int32)
+    ix = oracle.OracleIndex(3, L)
+    _held(L, ix, t, B, {2: k})
+    q = [0, 5, 1 << 40]  # instance 0 is the least loaded
+    for num, den in ((1, 2), (3, 4), (9, 10), (1, 1)):
+        # B*k*den == num*e exactly for e = B*k*den/num when that is an integer
+        e = Fraction(B * k * den, num)
+        if e.denominator != 1:
+            continue
+        e = int(e)
+        out = _policy(ix, B, [t, t], q, [1, 1], [e, e - 1], hit_num=num, hit_den=den)
+        assert int(out["stick"][0]) == 0 and int(out["instance"][0]) == 0
+        assert int(out["stick"][1]) == 1 and int(out["instance"][1]) == 2
+
+
+def check_policy_slo_migration(L):
+    """meets_ttft: estimate_load <= SLACK*PREFILL_RATE*(b + a*L), here the
+    budget d0 + d1*L in cost units. prev sticks while it meets the deadline
+    (inclusive), migrates to the least-loaded instance when another one meets
+    it, and sticks again when no instance meets it."""
+    rng = np.random.default_rng(44)
+    B, Lp, k, c_lin, c_att = 4, 64, 10, 2, 1
+    t = rng.integers(0, 151936, size=Lp, dtype=np.int32)
+    ix = oracle.OracleIndex(3, L)
+    _held(L, ix, t, B, {1: k})
+    q = [50, 4000, 20]
+    est = [q[i] + eq1_cost(Lp - (k * B if i == 1 else 0), Lp, c_lin, c_att) for i in range(3)]
+    assert all(e.denominator == 1 for e in est)  # n is even in every case here
+    assert est[2] < est[0] < est[1]
+    d1 = 3
+    for d0, want, stick in ((est[1] - d1 * Lp, 1, 1),       # prev meets exactly
+                            (est[1] - d1 * Lp - 1, 2, 0),   # prev misses, others meet
+                            (est[2] - d1 * Lp, 2, 0),       # only the least loaded meets
+                            (est[2] - d1 * Lp - 1, 1, 1)):  # no instance meets: stick
+        out = _policy(ix, B, [t], q, [1], [0], c_lin=c_lin, c_att=c_att, d0=int(d0), d1=d1)
+        assert (int(out["instance"][0]), int(out["stick"][0])) == (want, stick), (d0, est)
+
+
+def check_policy_round_robin_ties(L):
+    """rr_argmin: with nothing cached and equal queues every load ties, and
+    request r of the batch goes to (rr_base + r) mod N."""
+    rng = np.random.default_rng(45)
+    for N in (1, 2, 5, 8):
+        ix = oracle.OracleIndex(N, L)
+        reqs = [rng.integers(0, 151936, size=int(rng.integers(0, 90)), dtype=np.int32) for _ in range(13)]
+        for base in range(N):
+            out = _policy(ix, 4, reqs, [9] * N, [0] * 13, [0] * 13, c_lin=1, c_att=1, rr_base=base)
+            assert np.array_equal(out["instance"], (base + np.arange(13)) % N)
+
+
 ALL_CHECKS = [
     check_published_vector,
     check_bijection,
@@ -397,4 +545,10 @@ ALL_CHECKS = [
     check_hand_costs,
     check_batch_invariants,
     check_index_set_semantics,
+    check_policy_eq1_boundary,
+    check_policy_first_turn_is_cost_argmin,
+    check_policy_sticks_to_longest_local_hit,
+    check_policy_session_cached_threshold,
+    check_policy_slo_migration,
+    check_policy_round_robin_ties,
 ]

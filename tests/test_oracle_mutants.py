@@ -45,6 +45,16 @@ MUTANTS = {
                              "global_hit[r] = (int32_t)((int64_t)B * gb);"),
     "tail_block_hashed": ("int64_t n = L / B;\n  uint64_t h = oracle_mix64",
                           "int64_t n = (L + B - 1) / B;\n  uint64_t h = oracle_mix64"),
+    "policy_drops_half_term": ("c_att * nn * (2 * L - nn)", "c_att * nn * (2 * L)"),
+    "policy_drops_queue": ("est2[i] = 2 * queued[i] + ", "est2[i] = "),
+    "policy_prev_highest_id": ("if (c[i] > c[prev]) prev = i;", "if (c[i] >= c[prev]) prev = i;"),
+    "policy_cached_inclusive": ("hit_den > hit_num * est_hit[r];", "hit_den >= hit_num * est_hit[r];"),
+    "policy_meets_strict": ("const int meets_prev = est2[prev] <= budget2;",
+                            "const int meets_prev = est2[prev] < budget2;"),
+    "policy_no_last_resort": ("(meets_prev || !any_meets)", "meets_prev"),
+    "policy_ignores_turn": ("turn[r] != 0 && cached", "cached"),
+    "policy_no_rotation": ("(int32_t)(((int64_t)rr_base + r) % N)", "0"),
+    "policy_rotation_takes_last": ("if (est2[i] < est2[to]) to = i;", "if (est2[i] <= est2[to]) to = i;"),
 }
 
 
