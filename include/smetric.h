@@ -164,6 +164,65 @@ int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_t
                         int32_t* d_global_hit, uint64_t* d_session_key,
                         uint64_t* d_block_hashes, int64_t hashes_cap, smetric_stream_t stream);
 
+/* Limits of the session-centric policy's inputs (its integer arithmetic
+ * stays below 2^63 within them). */
+#define SMETRIC_POLICY_MAX_LEN (1LL << 24)     /* prompt tokens per request */
+#define SMETRIC_POLICY_MAX_QUEUED (1LL << 59)  /* an instance's queued cost */
+
+/* Parameters of the session-centric policy (Figure 10), integers:
+ *   c_lin, c_att  Eq. 1's coefficients: the prefill cost of n new tokens in
+ *                 an L-token prompt is c_lin*n + c_att*n*(L - n/2) cost units;
+ *                 c_lin in [0, 2^20], c_att in [0, 2^12].
+ *   ttft_d0, ttft_d1  the TTFT deadline in cost units,
+ *                 D(L) = ttft_d0 + ttft_d1*L (SLACK * PREFILL_RATE * the
+ *                 SLO b + a*L); ttft_d0 in [0, 2^60], ttft_d1 in [0, 2^35].
+ *   hit_num, hit_den  HIT_RATIO = hit_num / hit_den,
+ *                 0 <= hit_num <= hit_den, 1 <= hit_den <= 2^20.
+ *   rr_base       where request 0's round robin over equal loads starts,
+ *                 [0, N). */
+typedef struct smetric_policy {
+  int64_t c_lin;
+  int64_t c_att;
+  int64_t ttft_d0;
+  int64_t ttft_d1;
+  int64_t hit_num;
+  int64_t hit_den;
+  int32_t rr_base;
+  int32_t reserved; /* 0 */
+} smetric_policy;
+
+/* The routing step with the session-centric policy of Figure 10 as its
+ * decision (the second epilogue over the same local hits c_i and global run
+ * g as smetric_route_batch; Section 4.2's basic policy with SLO-aware
+ * migration). Per request r, with n_i = L - B*c_i its new tokens on
+ * instance i and est_i = d_queued[i] + c_lin*n_i + c_att*n_i*(L - n_i/2)
+ * (Figure 10(c), Eq. 1):
+ *   prev   = argmax_i c_i, lowest id among equals;
+ *   cached = B*c_prev > HIT_RATIO * d_est_hit[r]          (session_cached)
+ *   meets(i) = est_i <= D(L)                              (Figure 10(b))
+ *   stick  = d_turn[r] != 0 and cached and (meets(prev) or no i meets);
+ *   i*     = prev if stick, else the first minimal est_i scanning
+ *            i = s, s+1, ..., N-1, 0, ..., s-1 with s = (rr_base + r) mod N.
+ * All comparisons are exact (computed on 2*est_i in int64).
+ *   d_queued   int64 [N], each in [0, SMETRIC_POLICY_MAX_QUEUED]: the cost
+ *              already queued on each instance, in Eq. 1's units.
+ *   d_turn     int32 [n_requests]: 0 marks a session's first request.
+ *   d_est_hit  int64 [n_requests], each in [0, 2^31): the hit in tokens
+ *              that the request's history leads one to expect.
+ *   outputs    as smetric_route_batch for i*, plus int32 d_stick[r] = 1 when
+ *              the request stuck to prev, else 0.
+ * Other arguments and the other rules as smetric_route_batch; every prompt
+ * must be at most SMETRIC_POLICY_MAX_LEN tokens. Parameters out of range
+ * return SMETRIC_ERR_INVALID_ARG with nothing enqueued; queued costs,
+ * expected hits or prompt lengths out of range latch SMETRIC_ERR_OVERFLOW
+ * and the batch's outputs are instance -1, zero hits, stick 0 and key 0. */
+int smetric_route_batch_policy(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                               const int64_t* d_offsets, int32_t n_requests, const int64_t* d_queued,
+                               const int32_t* d_turn, const int64_t* d_est_hit, smetric_policy p,
+                               int32_t* d_instance, int32_t* d_local_hit, int32_t* d_global_hit,
+                               int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                               int64_t hashes_cap, smetric_stream_t stream);
+
 /* Step (a)-(b) alone: block hashes and session keys of a batch, without
  * index lookups (Appendix A: a request's block-hash sequence starts with its
  * parent's). Same argument rules as smetric_route_batch; d_block_hashes is

@@ -32,6 +32,8 @@ SMETRIC_MAX_WEIGHT = 1 << 20
 SMETRIC_MAX_LOAD = 1 << 40
 SMETRIC_MAX_PROBE = 65536
 SMETRIC_FLAG_HOST_STAGING = 1
+SMETRIC_POLICY_MAX_LEN = 1 << 24
+SMETRIC_POLICY_MAX_QUEUED = 1 << 59
 
 EXPORTED = (
     "smetric_index_create", "smetric_index_destroy", "smetric_index_clear",
@@ -39,7 +41,7 @@ EXPORTED = (
     "smetric_index_mask_words", "smetric_route_batch", "smetric_block_hashes",
     "smetric_route_batch_host", "smetric_status", "smetric_strerror",
     "smetric_profile_enable", "smetric_profile_read", "smetric_profile_kernel_name",
-    "smetric_launch_count", "smetric_block_hashes_noalloc",
+    "smetric_launch_count", "smetric_block_hashes_noalloc", "smetric_route_batch_policy",
 )
 
 
@@ -64,6 +66,12 @@ class smetric_index_config(C.Structure):
 
 class smetric_weights(C.Structure):
     _fields_ = [("w_load", C.c_int64), ("w_miss", C.c_int64), ("w_glob", C.c_int64)]
+
+
+class smetric_policy(C.Structure):
+    _fields_ = [("c_lin", C.c_int64), ("c_att", C.c_int64), ("ttft_d0", C.c_int64),
+                ("ttft_d1", C.c_int64), ("hit_num", C.c_int64), ("hit_den", C.c_int64),
+                ("rr_base", C.c_int32), ("reserved", C.c_int32)]
 
 
 _lib = None
@@ -93,6 +101,8 @@ def lib():
             "smetric_index_mask_words": (I32, [P]),
             "smetric_route_batch": (C.c_int, [P, P, I64, P, I32, P, smetric_weights, P, P, P, P, P,
                                               I64, P]),
+            "smetric_route_batch_policy": (C.c_int, [P, P, I64, P, I32, P, P, P, smetric_policy, P, P,
+                                                     P, P, P, P, I64, P]),
             "smetric_block_hashes": (C.c_int, [P, P, I64, P, I32, P, P, I64, P]),
             "smetric_block_hashes_noalloc": (C.c_int, [P, I64, P, I32, I32, I32, C.c_uint64, P, P, I64,
                                                       P, P]),
@@ -195,6 +205,25 @@ def smetric_route_batch(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests
                                      _ptr(d_load), _weights(w), _ptr(d_instance), _ptr(d_local_hit),
                                      _ptr(d_global_hit), _ptr(d_session_key), _ptr(d_block_hashes),
                                      hashes_cap, _stream(stream)), "smetric_route_batch")
+
+
+def _policy(p) -> smetric_policy:
+    if isinstance(p, smetric_policy):
+        return p
+    d = dict(p)
+    return smetric_policy(int(d["c_lin"]), int(d["c_att"]), int(d["ttft_d0"]), int(d["ttft_d1"]),
+                          int(d["hit_num"]), int(d["hit_den"]), int(d.get("rr_base", 0)), 0)
+
+
+def smetric_route_batch_policy(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int,
+                               d_queued, d_turn, d_est_hit, policy, d_instance, d_local_hit,
+                               d_global_hit, d_stick, d_session_key, d_block_hashes=None,
+                               hashes_cap: int = 0, stream=None) -> None:
+    _check(lib().smetric_route_batch_policy(
+        idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests, _ptr(d_queued), _ptr(d_turn),
+        _ptr(d_est_hit), _policy(policy), _ptr(d_instance), _ptr(d_local_hit), _ptr(d_global_hit),
+        _ptr(d_stick), _ptr(d_session_key), _ptr(d_block_hashes), hashes_cap, _stream(stream)),
+        "smetric_route_batch_policy")
 
 
 def smetric_block_hashes(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int,
@@ -333,6 +362,30 @@ class SMetricIndex:
         smetric_route_batch(self.handle, tokens, tokens.numel(), offsets, n, load, weights,
                             out["instance"], out["local_hit"], out["global_hit"],
                             out["session_key"], hb, hb.numel() if hb is not None else 0, stream)
+        return out
+
+    def route_batch_policy(self, tokens, offsets, queued, turn, est_hit, policy, want_hashes=False,
+                           out=None, stream=None):
+        """The session-centric policy (Figure 10). `policy` is a dict with c_lin,
+        c_att, ttft_d0, ttft_d1, hit_num, hit_den and optionally rr_base.
+        Returns dict(instance, local_hit, global_hit, stick, session_key[, block_hashes])."""
+        import torch
+        n = offsets.numel() - 1
+        dev = offsets.device
+        if out is None:
+            out = dict(instance=torch.empty(n, dtype=torch.int32, device=dev),
+                       local_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                       global_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                       stick=torch.empty(n, dtype=torch.int32, device=dev),
+                       session_key=torch.empty(n, dtype=torch.uint64, device=dev))
+            if want_hashes:
+                out["block_hashes"] = torch.empty(max(tokens.numel() // self.B, 1),
+                                                  dtype=torch.uint64, device=dev)
+        hb = out.get("block_hashes")
+        smetric_route_batch_policy(self.handle, tokens, tokens.numel(), offsets, n, queued, turn, est_hit,
+                                   policy, out["instance"], out["local_hit"], out["global_hit"],
+                                   out["stick"], out["session_key"], hb,
+                                   hb.numel() if hb is not None else 0, stream)
         return out
 
     def block_hashes(self, tokens, offsets, stream=None):

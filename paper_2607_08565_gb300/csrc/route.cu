@@ -80,7 +80,8 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
                                               int64_t n_tokens, int B, const int64_t* __restrict__ load,
                                               int n_load, int64_t* __restrict__ block_off,
                                               int64_t* __restrict__ chunk_off, int32_t* batch_ok,
-                                              int32_t* status) {
+                                              int32_t* status, int64_t max_load, int64_t max_len,
+                                              const int64_t* __restrict__ est_hit) {
   constexpr int NS = 2;  // scans: full blocks, and 32-block chunks (when chunk_off is wanted)
   constexpr int R = kPrepRounds;
   __shared__ int64_t warp_tot[NS][32];
@@ -92,8 +93,13 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
   int bad = 0;  // bit 0: invalid offsets, bit 1: out-of-range length or load
   for (int i = tid; i < n_load; i += blockDim.x) {
     const int64_t v = load[i];
-    if (v < 0 || v > SMETRIC_MAX_LOAD) bad |= 2;
+    if (v < 0 || v > max_load) bad |= 2;
   }
+  if (est_hit)  // the policy's expected hits, each in [0, 2^31)
+    for (int64_t r = tid; r < n; r += blockDim.x) {
+      const int64_t v = est_hit[r];
+      if (v < 0 || v > (int64_t)INT32_MAX) bad |= 2;
+    }
   // A pass gives each warp R rounds of 32 consecutive requests (lane = request),
   // so that offsets are loaded and both outputs stored coalesced. Every offset
   // of the pass is loaded before any is used; the counts stay in registers
@@ -114,7 +120,7 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
       uint32_t v = 0;
       if (seg + 32 * i < n) {
         if (a[i] < 0 || b[i] < a[i] || b[i] > n_tokens) bad |= 1;
-        else if (b[i] - a[i] > (int64_t)INT32_MAX) bad |= 2;
+        else if (b[i] - a[i] > max_len) bad |= 2;
         else v = (uint32_t)(b[i] - a[i]) / (uint32_t)B;
       }
       nbv[i] = v;
@@ -812,6 +818,17 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+// The session-centric policy (Figure 10) as the walk's decision; off for
+// the argmin cost of smetric_route_batch.
+struct WalkPolicy {
+  int on;
+  int64_t c_lin, c_att, d0, d1, hit_num, hit_den;
+  int32_t rr_base;
+  const int32_t* turn;
+  const int64_t* est_hit;
+  int32_t* stick;
+};
+
 // One warp per request, lanes = 32 consecutive blocks. The masks are
 // AND-scanned across lanes; lane j's "death set" is the local tiers held
 // through block j-1 but not through block j. Lanes with a non-empty death set
@@ -829,8 +846,8 @@ __global__ void __launch_bounds__(256)
 // alive through share - 1 continues over the member's own masks from block
 // `share` on. Members therefore start at `share` instead of re-reading the
 // leader's masks from block 0.
-template <int W, bool MEMBERS>
-__global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 1)  // members: 5 CTAs (40 warps) per SM
+template <int W, bool MEMBERS, bool POLICY>
+__global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (leaders) or 5 (members) CTAs per SM
     k_walk(int N, int B, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n,
            const int64_t* __restrict__ load, int64_t w_load, int64_t w_miss, int64_t w_glob,
            const uint64_t* __restrict__ masks, const uint64_t* __restrict__ chunk_and,
@@ -838,7 +855,8 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 1)  // members
            const int32_t* __restrict__ lead, const int32_t* __restrict__ share, int32_t* __restrict__ summ,
            const int32_t* __restrict__ order, const int32_t* __restrict__ counts,
            int32_t* __restrict__ inst_out, int32_t* __restrict__ lhit_out,
-           int32_t* __restrict__ ghit_out, uint4* __restrict__ groups, int64_t group_vecs) {
+           int32_t* __restrict__ ghit_out, uint4* __restrict__ groups, int64_t group_vecs,
+           const WalkPolicy pol) {
   pdl_enter();
   extern __shared__ int64_t msm[];
   int64_t* load_s = msm;                                                     // [N]
@@ -856,7 +874,10 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 1)  // members
 
   if (!ok && !MEMBERS)
     for (int64_t r = (int64_t)blockIdx.x * kMatchWarps + warp; r < n; r += tw)
-      if (lane == 0) { inst_out[r] = -1; lhit_out[r] = 0; ghit_out[r] = 0; }
+      if (lane == 0) {
+        inst_out[r] = -1; lhit_out[r] = 0; ghit_out[r] = 0;
+        if (POLICY) pol.stick[r] = 0;
+      }
   // k_group's lists: leaders from the front of `order`, members from the back
   const int64_t count = !ok ? 0 : MEMBERS ? counts[1] : counts[0];
   for (int64_t k = (int64_t)blockIdx.x * kMatchWarps + warp; k < count; k += tw) {
@@ -990,10 +1011,16 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 1)  // members
     }
     if (galive) g = nb;  // the global run reaches the last block
     __syncwarp();
-    // cost of every instance; lanes = instances
+    // per instance (lanes = instances): c_i, then the decision
     int64_t best_cost = INT64_MAX;
     int32_t best = N;
     int64_t best_c = 0;
+    // policy: prev = argmax c (lowest id), rr_argmin of 2*estimate_load
+    int64_t pc = -1, pe = INT64_MAX, pec = 0;
+    int32_t pi = N, prot = N;
+    bool meets_any = false;
+    const int32_t s0 = POLICY ? (int32_t)(((int64_t)pol.rr_base + r) % N) : 0;
+    const int64_t budget2 = POLICY ? 2 * (pol.d0 + pol.d1 * L) : 0;
     int32_t* const out_c = summ + r * (N + 1);
 #pragma unroll
     for (int t = 0; t < CT; ++t) {
@@ -1012,23 +1039,60 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 1)  // members
           if (ev_mask[e * W + wi] & bi) { ci = ev_pos[e]; break; }
       }
       if (!MEMBERS) out_c[i] = (int32_t)ci;
-      const int64_t gi = ci > g ? ci : g;
-      const int64_t cost = w_load * load_s[i] + w_miss * (L - B * gi) + w_glob * B * (gi - ci);
-      if (cost < best_cost) { best_cost = cost; best = i; best_c = ci; }
+      if (!POLICY) {
+        const int64_t gi = ci > g ? ci : g;
+        const int64_t cost = w_load * load_s[i] + w_miss * (L - B * gi) + w_glob * B * (gi - ci);
+        if (cost < best_cost) { best_cost = cost; best = i; best_c = ci; }
+      } else {
+        // Eq. 1 doubled: 2*q_i + 2*c_lin*n + c_att*n*(2L - n), n = new tokens
+        const int64_t nn = L - B * ci;
+        const int64_t est2 = 2 * load_s[i] + 2 * pol.c_lin * nn + pol.c_att * nn * (2 * L - nn);
+        meets_any |= est2 <= budget2;
+        if (ci > pc) { pc = ci; pi = i; }  // lanes see their instances in increasing order
+        const int32_t rot = (int32_t)((i - s0 + N) % N);
+        if (est2 < pe || (est2 == pe && rot < prot)) { pe = est2; prot = rot; pec = ci; }
+      }
     }
     if (!MEMBERS && lane == 0) out_c[N] = (int32_t)g;
+    if (!POLICY) {
 #pragma unroll
-    for (int dd = 16; dd > 0; dd >>= 1) {
-      const int64_t oc = __shfl_xor_sync(kFull, best_cost, dd);
-      const int32_t oi = __shfl_xor_sync(kFull, best, dd);
-      const int64_t ocb = __shfl_xor_sync(kFull, best_c, dd);
-      if (oc < best_cost || (oc == best_cost && oi < best)) { best_cost = oc; best = oi; best_c = ocb; }
-    }
-    if (lane == 0) {
-      const int64_t gb = best_c > g ? best_c : g;
-      inst_out[r] = best;
-      lhit_out[r] = (int32_t)(B * best_c);
-      ghit_out[r] = (int32_t)(B * (gb - best_c));
+      for (int dd = 16; dd > 0; dd >>= 1) {
+        const int64_t oc = __shfl_xor_sync(kFull, best_cost, dd);
+        const int32_t oi = __shfl_xor_sync(kFull, best, dd);
+        const int64_t ocb = __shfl_xor_sync(kFull, best_c, dd);
+        if (oc < best_cost || (oc == best_cost && oi < best)) { best_cost = oc; best = oi; best_c = ocb; }
+      }
+      if (lane == 0) {
+        const int64_t gb = best_c > g ? best_c : g;
+        inst_out[r] = best;
+        lhit_out[r] = (int32_t)(B * best_c);
+        ghit_out[r] = (int32_t)(B * (gb - best_c));
+      }
+    } else {
+#pragma unroll
+      for (int dd = 16; dd > 0; dd >>= 1) {
+        const int64_t oc = __shfl_xor_sync(kFull, pc, dd);
+        const int32_t oi = __shfl_xor_sync(kFull, pi, dd);
+        if (oc > pc || (oc == pc && oi < pi)) { pc = oc; pi = oi; }
+        const int64_t oe = __shfl_xor_sync(kFull, pe, dd);
+        const int32_t orot = __shfl_xor_sync(kFull, prot, dd);
+        const int64_t oec = __shfl_xor_sync(kFull, pec, dd);
+        if (oe < pe || (oe == pe && orot < prot)) { pe = oe; prot = orot; pec = oec; }
+      }
+      const bool any = __any_sync(kFull, meets_any);
+      if (lane == 0) {
+        const int64_t np = L - B * pc;
+        const int64_t est2p = 2 * load_s[pi] + 2 * pol.c_lin * np + pol.c_att * np * (2 * L - np);
+        const bool cached = B * pc * pol.hit_den > pol.hit_num * pol.est_hit[r];
+        const bool stick = pol.turn[r] != 0 && cached && (est2p <= budget2 || !any);
+        const int32_t to = stick ? pi : (int32_t)((s0 + prot) % N);
+        const int64_t ct = stick ? pc : pec;
+        const int64_t gt = ct > g ? ct : g;
+        inst_out[r] = to;
+        lhit_out[r] = (int32_t)(B * ct);
+        ghit_out[r] = (int32_t)(B * (gt - ct));
+        pol.stick[r] = stick ? 1 : 0;
+      }
     }
     __syncwarp();
   }
@@ -1217,7 +1281,7 @@ int launch_group(smetric_index* idx, int32_t n, cudaStream_t s) {
 template <int W>
 int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
                  smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, uint64_t* hashes,
-                 uint64_t* sk, int64_t max_blocks, cudaStream_t s) {
+                 uint64_t* sk, int64_t max_blocks, const WalkPolicy& pol, cudaStream_t s) {
   const int N = idx->cfg.num_instances;
   const uint64_t* H = hashes ? hashes : idx->hashes;
   int rc;
@@ -1252,7 +1316,10 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
   const int64_t want = ((int64_t)n + kMatchWarps - 1) / kMatchWarps;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
   // leaders, then members (which read the leaders' run ends)
-  for (auto kern : {k_walk<W, false>, k_walk<W, true>}) {
+  using WalkKernel = decltype(&k_walk<W, false, false>);  // every instantiation has this signature
+  const WalkKernel kerns[2] = {pol.on ? k_walk<W, false, true> : k_walk<W, false, false>,
+                               pol.on ? k_walk<W, true, true> : k_walk<W, true, false>};
+  for (const WalkKernel kern : kerns) {
     if (smem > 48 * 1024 &&
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
       return cuda_status(cudaErrorInvalidValue);
@@ -1261,7 +1328,7 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
                        idx->cfg.block_size, d_offsets, idx->block_off, n, d_load, w.w_load, w.w_miss, w.w_glob,
                        idx->masks, idx->chunk_and, idx->batch_ok, idx->lead, idx->share, idx->summ, idx->order,
                        idx->order + idx->cfg.max_batch_requests, inst, lhit, ghit,
-                       reinterpret_cast<uint4*>(idx->groups), (int64_t)group_slots_for(n))))
+                       reinterpret_cast<uint4*>(idx->groups), (int64_t)group_slots_for(n), pol)))
       return rc;
   }
   return SMETRIC_OK;
@@ -1269,13 +1336,13 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
 
 int dispatch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
                    smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, uint64_t* hashes,
-                   uint64_t* sk, int64_t max_blocks, cudaStream_t s) {
+                   uint64_t* sk, int64_t max_blocks, const WalkPolicy& pol, cudaStream_t s) {
   switch (idx->W) {
-    case 1: return launch_match<1>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, s);
-    case 2: return launch_match<2>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, s);
-    case 3: return launch_match<3>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, s);
-    case 4: return launch_match<4>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, s);
-    case 5: return launch_match<5>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, s);
+    case 1: return launch_match<1>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s);
+    case 2: return launch_match<2>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s);
+    case 3: return launch_match<3>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s);
+    case 4: return launch_match<4>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s);
+    case 5: return launch_match<5>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s);
     default: return SMETRIC_ERR_INVALID_ARG;
   }
 }
@@ -1306,7 +1373,8 @@ bool weights_ok(const smetric_weights& w) {
 template <bool PROBE>
 int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, const int64_t* d_offsets,
                  int32_t n, const int64_t* d_load, smetric_weights w, int32_t* inst, int32_t* lhit,
-                 int32_t* ghit, uint64_t* sk, uint64_t* hashes, int64_t hashes_cap, cudaStream_t s) {
+                 int32_t* ghit, uint64_t* sk, uint64_t* hashes, int64_t hashes_cap, cudaStream_t s,
+                 const WalkPolicy* pol = nullptr) {
   int rc = check_device(idx);
   if (rc) return rc;
   const smetric_index_config& c = idx->cfg;
@@ -1321,7 +1389,9 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
 
   profile_begin(idx, s);
   k_prep<<<1, 1024, 0, s>>>(d_offsets, n, n_tokens, c.block_size, d_load, PROBE ? c.num_instances : 0,
-                            idx->block_off, idx->chunk_off, idx->batch_ok, idx->status);
+                            idx->block_off, idx->chunk_off, idx->batch_ok, idx->status,
+                            pol ? SMETRIC_POLICY_MAX_QUEUED : SMETRIC_MAX_LOAD,
+                            pol ? SMETRIC_POLICY_MAX_LEN : (int64_t)INT32_MAX, pol ? pol->est_hit : nullptr);
   idx->launches++;
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   profile_mark(idx, kPrep, s);
@@ -1330,8 +1400,9 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
   }
   profile_mark(idx, kDigest, s);
   if (PROBE) {
+    const WalkPolicy off_pol = {};
     if ((rc = dispatch_match(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk,
-                             n_tokens / c.block_size, s)))
+                             n_tokens / c.block_size, pol ? *pol : off_pol, s)))
       return rc;
   } else {
     if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, !idx->profiling, s))) return rc;
@@ -1355,6 +1426,38 @@ int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_t
   return route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance,
                             d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap,
                             reinterpret_cast<cudaStream_t>(stream));
+}
+
+int smetric_route_batch_policy(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                               const int64_t* d_offsets, int32_t n_requests, const int64_t* d_queued,
+                               const int32_t* d_turn, const int64_t* d_est_hit, smetric_policy p,
+                               int32_t* d_instance, int32_t* d_local_hit, int32_t* d_global_hit,
+                               int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                               int64_t hashes_cap, smetric_stream_t stream) {
+  if (!idx) return SMETRIC_ERR_INVALID_ARG;
+  const int64_t N = idx->cfg.num_instances;
+  if (p.c_lin < 0 || p.c_lin > (1LL << 20) || p.c_att < 0 || p.c_att > (1LL << 12) || p.ttft_d0 < 0 ||
+      p.ttft_d0 > (1LL << 60) || p.ttft_d1 < 0 || p.ttft_d1 > (1LL << 35) || p.hit_den < 1 ||
+      p.hit_den > (1LL << 20) || p.hit_num < 0 || p.hit_num > p.hit_den || p.rr_base < 0 || p.rr_base >= N ||
+      p.reserved != 0)
+    return SMETRIC_ERR_INVALID_ARG;
+  if (n_requests > 0 && (!d_turn || !d_est_hit || !d_stick)) return SMETRIC_ERR_INVALID_ARG;
+  WalkPolicy pol;
+  pol.on = 1;
+  pol.c_lin = p.c_lin;
+  pol.c_att = p.c_att;
+  pol.d0 = p.ttft_d0;
+  pol.d1 = p.ttft_d1;
+  pol.hit_num = p.hit_num;
+  pol.hit_den = p.hit_den;
+  pol.rr_base = p.rr_base;
+  pol.turn = d_turn;
+  pol.est_hit = d_est_hit;
+  pol.stick = d_stick;
+  // the argmin weights are unused by the policy; any valid ones pass the checks
+  return route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_queued, smetric_weights{0, 0, 0},
+                            d_instance, d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap,
+                            reinterpret_cast<cudaStream_t>(stream), &pol);
 }
 
 int smetric_block_hashes(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
@@ -1533,7 +1636,8 @@ extern "C" int smetric_block_hashes_noalloc(const int32_t* d_tokens, int64_t n_t
   uint64_t* digest = scratch + kNaFlagWords + kNaOffWords;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
-  k_prep<<<1, 1024, 0, s>>>(d_offsets, n_requests, n_tokens, B, nullptr, 0, block_off, nullptr, ok, d_status);
+  k_prep<<<1, 1024, 0, s>>>(d_offsets, n_requests, n_tokens, B, nullptr, 0, block_off, nullptr, ok, d_status,
+                            SMETRIC_MAX_LOAD, (int64_t)INT32_MAX, nullptr);
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   if (n_tokens / B > 0) {
     const uint64_t d_init = mix64(hash_seed ^ (uint64_t)B);

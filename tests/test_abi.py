@@ -74,6 +74,9 @@ def test_null_handles_are_rejected(L):
     assert L.smetric_index_insert(None, None, None, 0, None) == pkg.SMETRIC_ERR_INVALID_ARG
     assert L.smetric_route_batch(None, None, 0, None, 0, None, pkg.smetric_weights(1, 4, 2),
                                  None, None, None, None, None, 0, None) == pkg.SMETRIC_ERR_INVALID_ARG
+    assert L.smetric_route_batch_policy(None, None, 0, None, 0, None, None, None,
+                                        pkg.smetric_policy(1, 1, 0, 0, 1, 2, 0, 0), None, None, None,
+                                        None, None, None, 0, None) == pkg.SMETRIC_ERR_INVALID_ARG
     assert L.smetric_status(None, None) == pkg.SMETRIC_ERR_INVALID_ARG
     assert L.smetric_index_mask_words(None) == 0
     assert L.smetric_launch_count(None) == 0
