@@ -56,6 +56,9 @@ def parse():
                     help="config-5 stress sweep instead of the benchmark line: batch, N and B "
                          "varied on the config-4 generator, table filled to --table-gb")
     ap.add_argument("--table-gb", type=float, default=40.0)
+    ap.add_argument("--policy", action="store_true",
+                    help="time the session-centric policy (Figure 10) instead of the argmin cost "
+                         "(one GPU; its own JSON line)")
     return ap.parse_args()
 
 
@@ -512,6 +515,183 @@ def run_ours(args, rank, world, local, dist):
 
 
 # ---------------------------------------------------------------------------
+# session-centric policy (Figure 10) on the same workload
+# ---------------------------------------------------------------------------
+
+# Eq. 1 in cost units: a 24k-token prompt with nothing cached costs ~3.1e8;
+# queues are the batch's load draws (U[0, 2M]) scaled by 256, so up to 5.1e8;
+# the TTFT deadline is 4e8 + 4,000 units per prompt token.
+POLICY = dict(c_lin=1000, c_att=1, ttft_d0=400_000_000, ttft_d1=4000, hit_num=9, hit_den=10, rr_base=0)
+QUEUED_SCALE = 256
+
+
+def policy_inputs(tr, bt, k):
+    """Per-request turn and expected hit, and per-instance queued cost, of
+    batch k: a tenth of the requests open their session (turn 0), the others
+    expect their session's cached prefix."""
+    rng = np.random.default_rng([0x5E55_0005, k])
+    turn = np.ones(bt.n_requests, np.int32)
+    turn[rng.random(bt.n_requests) < 0.1] = 0
+    est_hit = tr.prefix_len[bt.sessions].astype(np.int64)
+    queued = bt.load.astype(np.int64) * QUEUED_SCALE
+    return turn, est_hit, queued
+
+
+def run_policy(args):
+    import torch
+    import oracle
+    import paper_2607_08565_gb300 as pkg
+    from paper_2607_08565_gb300 import build_lib
+
+    build_lib.build()
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    tr = c4_trace(args)
+    p = tr.params
+    N, B = p.num_instances, p.block_size
+    ids = list(range(N_DISTINCT_BATCHES))
+    host = [tr.batch(k) for k in ids]
+    extra = [policy_inputs(tr, b, k) for b, k in zip(host, ids)]
+    nkeys = tr.n_prefix_blocks()
+    chunk = 4096
+    max_tok = max(max(b.n_tokens for b in host), chunk * int(tr.prefix_len.max()))
+    ix = pkg.SMetricIndex(N, B, p.session_blocks, capacity_slots=int(nkeys / 0.7) + 1,
+                          max_batch_requests=max(tr.batch_size, chunk), max_batch_tokens=max_tok,
+                          hash_seed=p.hash_seed)
+    populate_index(ix, tr, device, chunk)
+    T = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)
+    dev_b = [dict(tok=T(b.tokens), off=T(b.offsets), n=b.n_requests, n_tokens=b.n_tokens, turn=T(tu),
+                  est=T(eh), queued=T(q)) for b, (tu, eh, q) in zip(host, extra)]
+    n = tr.batch_size
+    outs = dict(instance=torch.empty(n, dtype=torch.int32, device=device),
+                local_hit=torch.empty(n, dtype=torch.int32, device=device),
+                global_hit=torch.empty(n, dtype=torch.int32, device=device),
+                stick=torch.empty(n, dtype=torch.int32, device=device),
+                session_key=torch.empty(n, dtype=torch.uint64, device=device))
+    stream = torch.cuda.current_stream(device)
+
+    def step(i):
+        b = dev_b[i % len(dev_b)]
+        pkg.smetric_route_batch_policy(ix.handle, b["tok"], b["n_tokens"], b["off"], b["n"], b["queued"],
+                                       b["turn"], b["est"], POLICY, outs["instance"], outs["local_hit"],
+                                       outs["global_hit"], outs["stick"], outs["session_key"], None, 0,
+                                       stream)
+
+    per_batch = []
+    for i in range(len(dev_b)):
+        step(i)
+        ix.check()
+        per_batch.append({k: v.cpu().numpy().copy() for k, v in outs.items()})
+    clocks = ClockSampler("GPU-" + str(torch.cuda.get_device_properties(0).uuid))
+    clocks.start()
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    launches0 = pkg.smetric_launch_count(ix.handle)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1)
+    launches = pkg.smetric_launch_count(ix.handle) - launches0
+    clk = clocks.stop()
+    if ix.status() != pkg.SMETRIC_OK:
+        raise RuntimeError("policy bench: device error")
+    reqs = float(np.mean([b.n_requests for b in host]))
+    value = args.steps * reqs / (ms / 1e3)
+    pkg.smetric_profile_enable(ix.handle, True)
+    for i in range(max(20, min(args.steps, 200))):
+        step(i)
+    prof = pkg.smetric_profile_read(ix.handle)
+    pkg.smetric_profile_enable(ix.handle, False)
+    algo = [algorithmic_bytes(b.lengths(), pb["local_hit"], pb["global_hit"], B, ix.W)
+            for b, pb in zip(host, per_batch)]
+    algo_mean = {k: float(np.mean([a[k] for a in algo])) for k in algo[0]}
+    peak, peak_kind = peak_hbm()
+    dom = max(prof, key=lambda k: prof[k][0])
+    dom_ms = prof[dom][0] / max(prof[dom][1], 1)
+    achieved = algo_mean[dom] / (dom_ms / 1e3) / 1e9
+
+    # end to end through the public API: pinned host inputs copied in, the
+    # policy call, outputs read back, every step
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+    hb = [dict(tok=pin(b.tokens), off=pin(b.offsets), turn=pin(tu), est=pin(eh), queued=pin(q), n=b.n_requests)
+          for b, (tu, eh, q) in zip(host[:2], extra[:2])]
+    stage = {k: torch.empty_like(v, device=device) for k, v in hb[0].items() if k != "n"}
+    hout = {k: torch.empty(n, dtype=v.dtype, pin_memory=True) for k, v in outs.items()}
+
+    def e2e_step(i):
+        b = hb[i % len(hb)]
+        for k in ("tok", "off", "turn", "est", "queued"):
+            if stage[k].numel() < b[k].numel():
+                stage[k] = torch.empty_like(b[k], device=device)
+            stage[k][:b[k].numel()].copy_(b[k], non_blocking=True)
+        pkg.smetric_route_batch_policy(ix.handle, stage["tok"], b["tok"].numel(), stage["off"], b["n"],
+                                       stage["queued"], stage["turn"], stage["est"], POLICY, outs["instance"],
+                                       outs["local_hit"], outs["global_hit"], outs["stick"],
+                                       outs["session_key"], None, 0, stream)
+        for k in hout:
+            hout[k].copy_(outs[k], non_blocking=True)
+        torch.cuda.synchronize()
+
+    for i in range(2):
+        e2e_step(i)
+    t0 = time.perf_counter()
+    for i in range(args.e2e_steps):
+        e2e_step(i)
+    e2e_s = time.perf_counter() - t0
+    last = per_batch[(args.e2e_steps - 1) % len(hb)]
+    for k in hout:
+        if not np.array_equal(hout[k].numpy(), last[k]):
+            raise RuntimeError(f"end-to-end policy route differs from the device route in {k}")
+    h2d = float(np.mean([sum(b[k].numel() * b[k].element_size() for k in ("tok", "off", "turn", "est", "queued"))
+                         for b in hb]))
+
+    cpu = None
+    if not args.no_cpu_baseline:
+        ox = oracle_index_for(tr, host[:1])
+        bt, (tu, eh, q) = host[0], extra[0]
+        m, dt = 16, 0.0
+        while True:  # the oracle's policy route runs on one thread
+            off = bt.offsets[:m + 1]
+            t0 = time.perf_counter()
+            ox.route_batch_policy(B, p.session_blocks, p.hash_seed, bt.tokens[:off[-1]], off, q, tu[:m], eh[:m],
+                                  POLICY["c_lin"], POLICY["c_att"], POLICY["ttft_d0"], POLICY["ttft_d1"],
+                                  POLICY["hit_num"], POLICY["hit_den"], POLICY["rr_base"])
+            dt = time.perf_counter() - t0
+            if dt > args.cpu_seconds / 2 or m == bt.n_requests:
+                break
+            m = min(bt.n_requests, 2 * m)
+        cpu = {"value": m / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"first {m} requests of config-4 batch 0 ({dt:.1f} s, one thread)"}
+
+    stick = float(np.mean([pb["stick"].mean() for pb in per_batch]))
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+        "config": {"workload": workload_name(args), "batch": int(reqs), "num_instances": N, "block_size": B,
+                   "decision": "session-centric policy (Figure 10, Eq. 1 in fixed point)", "policy": POLICY,
+                   "queued": f"batch load x {QUEUED_SCALE}", "first_turn_fraction": 0.1,
+                   "stick_fraction": stick,
+                   "l2": f"inputs larger than L2: {N_DISTINCT_BATCHES} distinct batches rotated"},
+        "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "peak_kind": f"{peak_kind} copy", "traffic": ncu_traffic(dom),
+                     "algorithmic_bytes_per_launch": algo_mean[dom], "ms_per_launch": dom_ms},
+        "kernels_ms_per_launch": {k: v[0] / max(v[1], 1) for k, v in prof.items()},
+        "clocks": clk,
+        "e2e": {"value": args.e2e_steps * reqs / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": float(24 * reqs), "steps": args.e2e_steps},
+        "gpu_launches": int(launches),
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    ix.close()
+
+
+# ---------------------------------------------------------------------------
 # config-5 stress sweep
 # ---------------------------------------------------------------------------
 
@@ -619,6 +799,9 @@ def main():
     args = parse()
     if args.sweep:
         run_sweep(args)
+        return
+    if args.policy:
+        run_policy(args)
         return
     rank, world, local, dist = dist_setup(args)
     if args.impl == "reference":
