@@ -223,6 +223,33 @@ int smetric_route_batch_policy(smetric_index* idx, const int32_t* d_tokens, int6
                                int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
                                int64_t hashes_cap, smetric_stream_t stream);
 
+/* Flags of smetric_index_commit_batch. */
+#define SMETRIC_COMMIT_GLOBAL 1 /* also add every block to the global tier */
+
+/* Device-side index maintenance after a routed batch, with no host round
+ * trip (the replay step between batches: Section 2, the serving side caches
+ * a request's KV$ blocks on the instance that ran it). For every request r
+ * with d_instance[r] >= 0, its full-block hashes join the local tier of
+ * d_instance[r] (and the global tier with SMETRIC_COMMIT_GLOBAL). Then, when
+ * d_load is not NULL, each instance's queue drains:
+ *   d_load[i] <- (d_load[i] + sum over r routed to i of (L_r - d_local_hit[r])) >> 1.
+ *   d_offsets      the routed batch's offsets (int64 [n_requests+1]).
+ *   d_instance, d_local_hit  the route's outputs (int32 [n_requests]).
+ *   d_block_hashes the route's block hashes (request after request, as
+ *                  smetric_route_batch writes them).
+ *   d_load         int64 [N], read and written; NULL skips the drain.
+ * Stream-ordered after the route; set semantics as smetric_index_insert
+ * (inserting a key a tier holds is a no-op). Capped tiers are the caller's
+ * to evict (smetric_index_evict): the index keeps no recency. Errors
+ * latched: invalid offsets, an instance outside [-1, N) or a local hit
+ * outside [0, L_r] (INVALID_ARG: nothing is committed and the loads are left
+ * as they were), no free slot (TABLE_FULL). d_local_hit may be NULL when
+ * d_load is. */
+int smetric_index_commit_batch(smetric_index* idx, const int64_t* d_offsets, int32_t n_requests,
+                               const int32_t* d_instance, const int32_t* d_local_hit,
+                               const uint64_t* d_block_hashes, int32_t flags, int64_t* d_load,
+                               smetric_stream_t stream);
+
 /* Step (a)-(b) alone: block hashes and session keys of a batch, without
  * index lookups (Appendix A: a request's block-hash sequence starts with its
  * parent's). Same argument rules as smetric_route_batch; d_block_hashes is

@@ -34,6 +34,7 @@ SMETRIC_MAX_PROBE = 65536
 SMETRIC_FLAG_HOST_STAGING = 1
 SMETRIC_POLICY_MAX_LEN = 1 << 24
 SMETRIC_POLICY_MAX_QUEUED = 1 << 59
+SMETRIC_COMMIT_GLOBAL = 1
 
 EXPORTED = (
     "smetric_index_create", "smetric_index_destroy", "smetric_index_clear",
@@ -42,6 +43,7 @@ EXPORTED = (
     "smetric_route_batch_host", "smetric_status", "smetric_strerror",
     "smetric_profile_enable", "smetric_profile_read", "smetric_profile_kernel_name",
     "smetric_launch_count", "smetric_block_hashes_noalloc", "smetric_route_batch_policy",
+    "smetric_index_commit_batch",
 )
 
 
@@ -103,6 +105,7 @@ def lib():
                                               I64, P]),
             "smetric_route_batch_policy": (C.c_int, [P, P, I64, P, I32, P, P, P, smetric_policy, P, P,
                                                      P, P, P, P, I64, P]),
+            "smetric_index_commit_batch": (C.c_int, [P, P, I32, P, P, P, I32, P, P]),
             "smetric_block_hashes": (C.c_int, [P, P, I64, P, I32, P, P, I64, P]),
             "smetric_block_hashes_noalloc": (C.c_int, [P, I64, P, I32, I32, I32, C.c_uint64, P, P, I64,
                                                       P, P]),
@@ -224,6 +227,13 @@ def smetric_route_batch_policy(idx: int, d_tokens, n_tokens: int, d_offsets, n_r
         _ptr(d_est_hit), _policy(policy), _ptr(d_instance), _ptr(d_local_hit), _ptr(d_global_hit),
         _ptr(d_stick), _ptr(d_session_key), _ptr(d_block_hashes), hashes_cap, _stream(stream)),
         "smetric_route_batch_policy")
+
+
+def smetric_index_commit_batch(idx: int, d_offsets, n_requests: int, d_instance, d_local_hit,
+                               d_block_hashes, flags: int = 0, d_load=None, stream=None) -> None:
+    _check(lib().smetric_index_commit_batch(idx, _ptr(d_offsets), n_requests, _ptr(d_instance),
+                                            _ptr(d_local_hit), _ptr(d_block_hashes), flags, _ptr(d_load),
+                                            _stream(stream)), "smetric_index_commit_batch")
 
 
 def smetric_block_hashes(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int,
@@ -387,6 +397,14 @@ class SMetricIndex:
                                    out["stick"], out["session_key"], hb,
                                    hb.numel() if hb is not None else 0, stream)
         return out
+
+    def commit_batch(self, offsets, out, also_global=False, load=None, stream=None):
+        """Add the routed batch's blocks (`out` from route_batch(..., want_hashes=True)
+        or route_batch_policy) to its chosen instances' local tiers (and the
+        global tier); with `load`, drain it in place."""
+        smetric_index_commit_batch(self.handle, offsets, offsets.numel() - 1, out["instance"],
+                                   out["local_hit"], out["block_hashes"],
+                                   SMETRIC_COMMIT_GLOBAL if also_global else 0, load, stream)
 
     def block_hashes(self, tokens, offsets, stream=None):
         """Returns (block_hashes, session_key) as device tensors."""

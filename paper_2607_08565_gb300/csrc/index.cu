@@ -157,6 +157,40 @@ __global__ void k_lookup(const uint8_t* __restrict__ tags, const uint64_t* __res
   }
 }
 
+// Committing a routed batch: thread per block f of the batch (request r, the
+// largest with block_off[r] <= f) adds h_f to the local tier of r's chosen
+// instance and, with `global`, to the global tier. A request routed to -1
+// (an invalid batch) adds nothing; another out-of-range instance latches
+// INVALID_ARG.
+__global__ void k_commit(uint8_t* __restrict__ tags, uint64_t* __restrict__ table, uint64_t n_buckets,
+                         int ew, int N, const int64_t* __restrict__ block_off, int32_t n,
+                         const uint64_t* __restrict__ H, const int32_t* __restrict__ instance, int global,
+                         const int32_t* __restrict__ batch_ok, int32_t* status) {
+  if (!*batch_ok) return;
+  const int64_t total = block_off[n];
+  int32_t r = 0;
+  for (int64_t f = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; f < total;
+       f += (int64_t)gridDim.x * blockDim.x) {
+    int32_t lo = r, hi = n;  // largest r with block_off[r] <= f
+    while (hi - lo > 1) {
+      const int32_t mid = (lo + hi) >> 1;
+      if (block_off[mid] <= f) lo = mid; else hi = mid;
+    }
+    r = lo;
+    const int32_t i = instance[r];
+    if (i == -1) continue;
+    const uint64_t key = H[f];
+    if (i < -1 || i >= N || key < 2) {
+      latch_error(status, SMETRIC_ERR_INVALID_ARG);
+      continue;
+    }
+    if (!insert_key(tags, table, ew, n_buckets, key, i >> 6, 1ull << (i & 63)))
+      latch_error(status, SMETRIC_ERR_TABLE_FULL);
+    if (global && !insert_key(tags, table, ew, n_buckets, key, N >> 6, 1ull << (N & 63)))
+      latch_error(status, SMETRIC_ERR_TABLE_FULL);
+  }
+}
+
 int grid_for(const smetric_index* idx, int64_t n, int threads) {
   int64_t want = (n + threads - 1) / threads;
   int64_t cap = (int64_t)idx->num_sms * 8;
@@ -183,6 +217,25 @@ int update(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers, i
   idx->launches++;
   return cuda_status(cudaGetLastError());
 }
+
+}  // namespace
+
+namespace smetric {
+
+int launch_commit(smetric_index* idx, const int32_t* d_instance, const uint64_t* d_hashes, int32_t n,
+                  int64_t max_blocks, bool global, cudaStream_t s) {
+  const int threads = 256;
+  const int grid = grid_for(idx, max_blocks, threads);
+  k_commit<<<grid, threads, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->EW, idx->cfg.num_instances,
+                                    idx->block_off, n, d_hashes, d_instance, global ? 1 : 0, idx->batch_ok,
+                                    idx->status);
+  idx->launches++;
+  return cuda_status(cudaGetLastError());
+}
+
+}  // namespace smetric
+
+namespace {
 
 void free_all(smetric_index* x) {
   cudaFree(x->table);

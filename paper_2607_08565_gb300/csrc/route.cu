@@ -1106,6 +1106,45 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
 }
 
 // ---------------------------------------------------------------------------
+// commit
+// ---------------------------------------------------------------------------
+
+// Checks of a batch to commit and the queue drain: one CTA checks every
+// request's instance (in [-1, N)) and local hit (in [0, L_r]); a bad value
+// clears the batch flag, so that nothing is committed and the loads stay as
+// they were. Otherwise, with `load`, it sums per instance the tokens each
+// request routed there must prefill or fetch (L_r - local hit) and sets
+// load_i <- (load_i + that sum) >> 1. Integer sums, so the order of the
+// atomics does not matter.
+__global__ void __launch_bounds__(1024)
+    k_drain(const int64_t* __restrict__ off, int32_t n, int N, const int32_t* __restrict__ instance,
+            const int32_t* __restrict__ local_hit, int32_t* __restrict__ batch_ok,
+            int64_t* __restrict__ load, int32_t* status) {
+  __shared__ unsigned long long acc[SMETRIC_MAX_INSTANCES];
+  __shared__ int bad;
+  if (threadIdx.x == 0) bad = 0;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) acc[i] = 0;
+  __syncthreads();
+  if (!*batch_ok) return;  // invalid offsets
+  for (int64_t r = threadIdx.x; r < n; r += blockDim.x) {
+    const int32_t i = instance[r];
+    const int64_t L = off[r + 1] - off[r], h = local_hit ? local_hit[r] : 0;
+    if (i < -1 || i >= N || h < 0 || h > L) { bad = 1; continue; }
+    if (i >= 0 && load) atomicAdd(&acc[i], (unsigned long long)(L - h));
+  }
+  __syncthreads();
+  if (bad) {
+    if (threadIdx.x == 0) {
+      *batch_ok = 0;
+      latch_error(status, SMETRIC_ERR_INVALID_ARG);
+    }
+    return;
+  }
+  if (load)
+    for (int i = threadIdx.x; i < N; i += blockDim.x) load[i] = (load[i] + (int64_t)acc[i]) >> 1;
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 
@@ -1458,6 +1497,32 @@ int smetric_route_batch_policy(smetric_index* idx, const int32_t* d_tokens, int6
   return route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_queued, smetric_weights{0, 0, 0},
                             d_instance, d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap,
                             reinterpret_cast<cudaStream_t>(stream), &pol);
+}
+
+int smetric_index_commit_batch(smetric_index* idx, const int64_t* d_offsets, int32_t n_requests,
+                               const int32_t* d_instance, const int32_t* d_local_hit,
+                               const uint64_t* d_block_hashes, int32_t flags, int64_t* d_load,
+                               smetric_stream_t stream) {
+  int rc = check_device(idx);
+  if (rc) return rc;
+  const smetric_index_config& c = idx->cfg;
+  if (n_requests < 0 || n_requests > c.max_batch_requests || (flags & ~SMETRIC_COMMIT_GLOBAL))
+    return SMETRIC_ERR_INVALID_ARG;
+  if (n_requests == 0) return SMETRIC_OK;
+  if (!d_offsets || !d_instance || !d_block_hashes || (d_load && !d_local_hit)) return SMETRIC_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // block offsets of the batch (and the offsets' checks) into the index's scratch
+  k_prep<<<1, 1024, 0, s>>>(d_offsets, n_requests, c.max_batch_tokens, c.block_size, nullptr, 0, idx->block_off,
+                            nullptr, idx->batch_ok, idx->status, SMETRIC_MAX_LOAD, (int64_t)INT32_MAX, nullptr);
+  idx->launches++;
+  if ((rc = cuda_status(cudaGetLastError()))) return rc;
+  // the checks (and the drain) first: a bad output commits nothing
+  k_drain<<<1, 1024, 0, s>>>(d_offsets, n_requests, c.num_instances, d_instance, d_local_hit, idx->batch_ok,
+                             d_load, idx->status);
+  idx->launches++;
+  if ((rc = cuda_status(cudaGetLastError()))) return rc;
+  return launch_commit(idx, d_instance, d_block_hashes, n_requests, c.max_batch_tokens / c.block_size,
+                       (flags & SMETRIC_COMMIT_GLOBAL) != 0, s);
 }
 
 int smetric_block_hashes(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,

@@ -142,4 +142,8 @@ namespace smetric {
 int check_device(const smetric_index* idx);
 // Maps a CUDA error to SMETRIC_ERR_CUDA (clearing the sticky-free error state).
 int cuda_status(cudaError_t e);
+// Inserts a routed batch's block hashes into its chosen instances' local tiers
+// (and the global tier); block_off must hold the batch's block offsets.
+int launch_commit(smetric_index* idx, const int32_t* d_instance, const uint64_t* d_hashes, int32_t n,
+                  int64_t max_blocks, bool global, cudaStream_t s);
 }  // namespace smetric
