@@ -56,6 +56,9 @@ def parse():
                     help="config-5 stress sweep instead of the benchmark line: batch, N and B "
                          "varied on the config-4 generator, table filled to --table-gb")
     ap.add_argument("--table-gb", type=float, default=40.0)
+    ap.add_argument("--commit", action="store_true",
+                    help="time device-side index maintenance (route, then commit the batch's blocks "
+                         "and drain the queues) over a config-2 replay (one GPU; its own JSON line)")
     ap.add_argument("--policy", action="store_true",
                     help="time the session-centric policy (Figure 10) instead of the argmin cost "
                          "(one GPU; its own JSON line)")
@@ -692,6 +695,67 @@ def run_policy(args):
 
 
 # ---------------------------------------------------------------------------
+# device-side index maintenance over a config-2 replay
+# ---------------------------------------------------------------------------
+
+def run_commit(args, n_batches=24):
+    import itertools
+    import torch
+    import paper_2607_08565_gb300 as pkg
+    from paper_2607_08565_gb300 import build_lib
+    from synth import ReplayDriver, agent_trace
+
+    build_lib.build()
+    torch.cuda.set_device(0)
+    tr = agent_trace("c2_medium")
+    p = tr.params
+    batches = list(itertools.islice(tr.batches(), n_batches))
+    blocks = [int((b.lengths() // p.block_size).sum()) for b in batches]
+    ix = pkg.SMetricIndex(p.num_instances, p.block_size, p.session_blocks,
+                          capacity_slots=max(1024, int(sum(blocks) * 2 / 0.5)),
+                          max_batch_requests=max(b.n_requests for b in batches),
+                          max_batch_tokens=max(b.n_tokens for b in batches), hash_seed=p.hash_seed)
+    driver = ReplayDriver(p.num_instances, p.block_size, local_cap=tr.local_cap,
+                          global_policy=tr.global_policy, global_cap=tr.global_cap)
+    load = torch.zeros(p.num_instances, dtype=torch.int64, device="cuda")
+    w = (p.w_load, p.w_miss, p.w_glob)
+    stream = torch.cuda.current_stream()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    route_ms, commit_ms, done = 0.0, 0.0, 0
+    for k, bt in enumerate(batches):
+        tok = torch.from_numpy(bt.tokens).cuda()
+        off = torch.from_numpy(bt.offsets).cuda()
+        torch.cuda.synchronize()
+        ev[0].record(stream)
+        out = ix.route_batch(tok, off, load, w, want_hashes=True)
+        ev[1].record(stream)
+        ix.commit_batch(off, out, also_global=tr.global_policy != "none", load=load)
+        ev[2].record(stream)
+        torch.cuda.synchronize()
+        ix.check()
+        if k >= 2:  # the first batches warm up
+            route_ms += ev[0].elapsed_time(ev[1])
+            commit_ms += ev[1].elapsed_time(ev[2])
+            done += blocks[k]
+        # the capped local tiers evict on the host's orders, outside the timed region
+        g = {key: v.cpu().numpy() for key, v in out.items()}
+        _, _, ek, et = driver.after_batch(bt.offsets, g["instance"], g["local_hit"],
+                                          g["block_hashes"][:blocks[k]])
+        if len(ek):
+            ix.evict(torch.from_numpy(ek).cuda(), torch.from_numpy(et).cuda())
+    timed = len(batches) - 2
+    line = {"metric": "device-side commit of routed batches (blocks into the chosen local tier and the "
+                      "global tier, queue drain)", "value": done / (commit_ms / 1e3), "unit": "blocks/s",
+            "n_gpus": 1, "steps": timed, "warmup": 2, "ms_per_step": commit_ms / timed,
+            "route_ms_per_step": route_ms / timed, "higher_is_better": True, "data": "synthetic",
+            "config": {"workload": "c2_medium agent trace (16 instances, B = 16, 256 requests per batch)",
+                       "blocks_per_batch": float(np.mean(blocks[2:])), "tiers_per_block": 2,
+                       "evictions": "host LRU driver, outside the timed region"}}
+    print(json.dumps(line), flush=True)
+    ix.close()
+
+
+# ---------------------------------------------------------------------------
 # config-5 stress sweep
 # ---------------------------------------------------------------------------
 
@@ -802,6 +866,9 @@ def main():
         return
     if args.policy:
         run_policy(args)
+        return
+    if args.commit:
+        run_commit(args)
         return
     rank, world, local, dist = dist_setup(args)
     if args.impl == "reference":
