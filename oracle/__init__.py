@@ -63,6 +63,11 @@ def load_library(path: str):
         C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p, i32p, i64p,
         C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int32,
         i32p, i32p, i32p, i32p, u64p]
+    L.oracle_route_batch_coloc.restype = C.c_int
+    L.oracle_route_batch_coloc.argtypes = [
+        C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p, i64p, i64p, i32p, i64p,
+        C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int32,
+        i32p, i32p, i32p, i32p, u64p]
     return L
 
 
@@ -181,6 +186,32 @@ class OracleIndex:
             c_lin, c_att, d0, d1, hit_num, hit_den, rr_base, *outs, sk)
         if rc != 0:
             raise ValueError(f"oracle_route_batch_policy: {rc}")
+        inst, lh, gh, st = outs
+        return dict(instance=inst[:n], local_hit=lh[:n], global_hit=gh[:n], stick=st[:n],
+                    session_key=sk[:n])
+
+    def route_batch_coloc(self, block_size: int, session_blocks: int, seed: int, tokens, offsets,
+                          queued, tpot_budget, num_requests, turn, est_hit, c_lin: int, c_att: int,
+                          d0: int, d1: int, hit_num: int, hit_den: int, rr_base: int = 0):
+        """The session-centric policy under PD colocation (Appendix B).
+        Returns dict(instance, local_hit, global_hit, stick, session_key)."""
+        t = np.ascontiguousarray(tokens, dtype=np.int32)
+        o = np.ascontiguousarray(offsets, dtype=np.int64)
+        n = len(o) - 1
+        per_inst = [np.ascontiguousarray(a, dtype=np.int64) for a in (queued, tpot_budget, num_requests)]
+        tu = np.ascontiguousarray(turn, dtype=np.int32)
+        eh = np.ascontiguousarray(est_hit, dtype=np.int64)
+        if any(len(a) != self.N for a in per_inst) or len(tu) != n or len(eh) != n:
+            raise ValueError("queued, tpot_budget, num_requests: one per instance; turn, est_hit: one per request")
+        outs = [np.zeros(max(n, 1), np.int32) for _ in range(4)]
+        sk = np.zeros(max(n, 1), np.uint64)
+        rc = self._L.oracle_route_batch_coloc(
+            self._h, block_size, session_blocks, seed & 0xFFFFFFFFFFFFFFFF,
+            t if len(t) else np.zeros(1, np.int32), o, n, *per_inst,
+            tu if n else np.zeros(1, np.int32), eh if n else np.zeros(1, np.int64),
+            c_lin, c_att, d0, d1, hit_num, hit_den, rr_base, *outs, sk)
+        if rc != 0:
+            raise ValueError(f"oracle_route_batch_coloc: {rc}")
         inst, lh, gh, st = outs
         return dict(instance=inst[:n], local_hit=lh[:n], global_hit=gh[:n], stick=st[:n],
                     session_key=sk[:n])

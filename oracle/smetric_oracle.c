@@ -70,6 +70,19 @@
  *              (rr_argmin: equal loads are taken in turn).
  * Outputs: instance = i*, stick, local_hit = B*c_{i*}, global_hit =
  * B*(max(c_{i*}, g) - c_{i*}), session_key as above.
+ *
+ * The same policy under PD colocation (Appendix B; oracle_route_batch_coloc):
+ *    cost2_i = 2*C_LIN*n_i + C_ATT*n_i*(2*L_r - n_i)   (2 * prefill_cost)
+ *    tpot(i) = cost2_i <= 2*T_i, T_i the prefill cost instance i's live
+ *              decodes can absorb within their TPOT SLO (PREFILL_RATE times
+ *              the smallest slack); cand = {i : tpot(i)}, or every instance
+ *              when no instance passes.
+ *    stick   = turn_r != 0 and cached and meets(prev) and prev in cand
+ *              (no last resort here)
+ *    i*      = prev if stick, else the first minimal est2_i * R_i over cand
+ *              in the rotation order above, R_i = the requests instance i
+ *              runs (LMetric's multiplicative score), compared exactly in
+ *              128 bits.
  */
 #include <stdint.h>
 #include <stdlib.h>
@@ -397,5 +410,96 @@ int oracle_route_batch_policy(const oracle_index* x, int32_t B, int32_t S, uint6
   free(h);
   free(c);
   free(est2);
+  return rc;
+}
+
+/* Session-centric policy under PD colocation (Appendix B). Limits as the
+ * policy above plus 0 <= T_i <= 2^60 and 0 <= R_i <= 2^20. */
+int oracle_route_batch_coloc(const oracle_index* x, int32_t B, int32_t S, uint64_t seed,
+                             const int32_t* tokens, const int64_t* offsets, int32_t n_requests,
+                             const int64_t* queued, const int64_t* tpot_budget, const int64_t* num_requests,
+                             const int32_t* turn, const int64_t* est_hit, int64_t c_lin, int64_t c_att,
+                             int64_t d0, int64_t d1, int64_t hit_num, int64_t hit_den, int32_t rr_base,
+                             int32_t* instance, int32_t* local_hit, int32_t* global_hit, int32_t* stick,
+                             uint64_t* session_key) {
+  if (!x || B < 2 || (B % 2) != 0 || S < 1 || n_requests < 0) return ORACLE_ERR_INVALID_ARG;
+  const int32_t N = x->N;
+  if (c_lin < 0 || c_lin > (1LL << 20) || c_att < 0 || c_att > (1LL << 12) || d0 < 0 ||
+      d0 > (1LL << 60) || d1 < 0 || d1 > (1LL << 35) || hit_den < 1 || hit_den > (1LL << 20) ||
+      hit_num < 0 || hit_num > hit_den || rr_base < 0 || rr_base >= N)
+    return ORACLE_ERR_INVALID_ARG;
+  for (int32_t i = 0; i < N; ++i)
+    if (queued[i] < 0 || queued[i] > (1LL << 59) || tpot_budget[i] < 0 || tpot_budget[i] > (1LL << 60) ||
+        num_requests[i] < 0 || num_requests[i] > (1LL << 20))
+      return ORACLE_ERR_INVALID_ARG;
+  for (int32_t r = 0; r < n_requests; ++r) {
+    if (offsets[r + 1] < offsets[r] || offsets[r] < 0 || offsets[r + 1] - offsets[r] > (1LL << 24))
+      return ORACLE_ERR_INVALID_ARG;
+    if (est_hit[r] < 0 || est_hit[r] >= (1LL << 31)) return ORACLE_ERR_INVALID_ARG;
+  }
+  int64_t* c = (int64_t*)malloc((size_t)N * sizeof(int64_t));
+  int64_t* cost2 = (int64_t*)malloc((size_t)N * sizeof(int64_t));
+  int64_t* est2 = (int64_t*)malloc((size_t)N * sizeof(int64_t));
+  int* cand = (int*)malloc((size_t)N * sizeof(int));
+  uint64_t* h = NULL;
+  int64_t cap = 0;
+  int rc = ORACLE_OK;
+  if (!c || !cost2 || !est2 || !cand) rc = ORACLE_ERR_OOM;
+  for (int32_t r = 0; r < n_requests && rc == ORACLE_OK; ++r) {
+    const int64_t L = offsets[r + 1] - offsets[r];
+    const int64_t n = L / B;
+    if (n + 1 > cap) {
+      free(h);
+      cap = n + 1;
+      h = (uint64_t*)malloc((size_t)cap * sizeof(uint64_t));
+      if (!h) { rc = ORACLE_ERR_OOM; break; }
+    }
+    oracle_block_hashes(tokens + offsets[r], L, B, seed, h);
+    int64_t g;
+    oracle_prefix_hits(x, h, n, c, &g);
+    for (int32_t i = 0; i < N; ++i) {
+      const int64_t nn = L - (int64_t)B * c[i];
+      cost2[i] = 2 * c_lin * nn + c_att * nn * (2 * L - nn);
+      est2[i] = 2 * queued[i] + cost2[i];
+    }
+    int32_t prev = 0;
+    for (int32_t i = 1; i < N; ++i)
+      if (c[i] > c[prev]) prev = i;
+    /* the TPOT filter: every live decode of i tolerates the new prefill */
+    int n_cand = 0;
+    for (int32_t i = 0; i < N; ++i) {
+      cand[i] = cost2[i] <= 2 * tpot_budget[i];
+      n_cand += cand[i];
+    }
+    if (n_cand == 0)
+      for (int32_t i = 0; i < N; ++i) cand[i] = 1;
+    const int cached = (int64_t)B * c[prev] * hit_den > hit_num * est_hit[r];
+    const int meets_prev = est2[prev] <= 2 * (d0 + d1 * L);
+    const int st = turn[r] != 0 && cached && meets_prev && cand[prev];
+    int32_t to = prev;
+    if (!st) {
+      /* rr_argmin over the candidates of estimate_load * num_requests */
+      const int32_t s0 = (int32_t)(((int64_t)rr_base + r) % N);
+      to = -1;
+      unsigned __int128 best = 0;
+      for (int32_t k = 0; k < N; ++k) {
+        const int32_t i = (s0 + k) % N;
+        if (!cand[i]) continue;
+        const unsigned __int128 score = (unsigned __int128)(uint64_t)est2[i] * (uint64_t)num_requests[i];
+        if (to < 0 || score < best) { to = i; best = score; }
+      }
+    }
+    const int64_t gt = c[to] > g ? c[to] : g;
+    instance[r] = to;
+    stick[r] = st;
+    local_hit[r] = (int32_t)((int64_t)B * c[to]);
+    global_hit[r] = (int32_t)((int64_t)B * (gt - c[to]));
+    session_key[r] = n == 0 ? 0 : h[(n < S ? n : S) - 1];
+  }
+  free(h);
+  free(c);
+  free(cost2);
+  free(est2);
+  free(cand);
   return rc;
 }

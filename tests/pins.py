@@ -528,6 +528,107 @@ def check_policy_round_robin_ties(L):
             assert np.array_equal(out["instance"], (base + np.arange(13)) % N)
 
 
+def _coloc(ix, B, reqs, queued, tpot, nreq, turn, est_hit, c_lin=1, c_att=0, d0=1 << 60, d1=0,
+           hit_num=1, hit_den=2, rr_base=0, S=1):
+    from synth.traces import pack
+    tokens, offsets = pack(reqs)
+    return ix.route_batch_coloc(B, S, 0, tokens, offsets, np.asarray(queued, np.int64),
+                                np.asarray(tpot, np.int64), np.asarray(nreq, np.int64),
+                                np.asarray(turn, np.int32), np.asarray(est_hit, np.int64),
+                                c_lin, c_att, d0, d1, hit_num, hit_den, rr_base)
+
+
+def check_coloc_reduces_to_disaggregated(L):
+    """Appendix B against Figure 10: with every instance passing the TPOT
+    check, one request per instance and a deadline every instance meets, the
+    colocated policy decides exactly as the disaggregated one."""
+    rng = np.random.default_rng(50)
+    B = 2
+    for trial in range(40):
+        N = int(rng.integers(1, 7))
+        base = rng.integers(0, 3, size=10 * B, dtype=np.int32)
+        ix = oracle.OracleIndex(N, L)
+        for i in range(N):
+            for _ in range(int(rng.integers(0, 3))):
+                ix.insert(oracle.block_hashes(_mutate(rng, base, int(rng.integers(0, 11 * B))), B, 0, L), i)
+        reqs = [_mutate(rng, base, int(rng.integers(0, 11 * B))) for _ in range(5)]
+        q = rng.integers(0, 50, size=N)
+        kw = dict(c_lin=int(rng.integers(0, 4)), c_att=int(rng.integers(0, 3)), rr_base=int(rng.integers(0, N)))
+        turn, est = rng.integers(0, 2, size=5), rng.integers(0, 30, size=5)
+        a = _coloc(ix, B, reqs, q, [1 << 60] * N, [1] * N, turn, est, **kw)
+        b = _policy(ix, B, reqs, q, turn, est, **kw)
+        for k in ("instance", "stick", "local_hit", "global_hit"):
+            assert np.array_equal(a[k], b[k]), (trial, k)
+
+
+def check_coloc_tpot_filter(L):
+    """An instance whose live decodes cannot absorb the prefill (2*cost_i >
+    2*T_i) is not a candidate: a cached follow-up leaves prev when prev fails
+    the check, the balance skips failing instances, and when none passes
+    every instance is a candidate again."""
+    rng = np.random.default_rng(51)
+    B, Lp, k, c_lin, c_att = 4, 48, 8, 3, 1
+    t = rng.integers(0, 151936, size=Lp, dtype=np.int32)
+    ix = oracle.OracleIndex(3, L)
+    _held(L, ix, t, B, {1: k})
+    cost = [eq1_cost(Lp - (k * B if i == 1 else 0), Lp, c_lin, c_att) for i in range(3)]
+    assert all(x.denominator == 1 for x in cost)
+    big = 1 << 50
+    q = [7, 5, 100]  # instance 0 the least loaded; queues do not count in the TPOT check
+    kw = dict(c_lin=c_lin, c_att=c_att)
+    out = _coloc(ix, B, [t], q, [big, int(cost[1]), big], [1, 1, 1], [1], [0], **kw)
+    assert (int(out["instance"][0]), int(out["stick"][0])) == (1, 1)   # prev passes exactly
+    out = _coloc(ix, B, [t], q, [big, int(cost[1]) - 1, big], [1, 1, 1], [1], [0], **kw)
+    assert (int(out["instance"][0]), int(out["stick"][0])) == (0, 0)   # prev fails: balanced
+    out = _coloc(ix, B, [t], q, [int(cost[0]) - 1, int(cost[1]) - 1, big], [1, 1, 1], [1], [0], **kw)
+    assert (int(out["instance"][0]), int(out["stick"][0])) == (2, 0)   # only instance 2 passes
+    out = _coloc(ix, B, [t], q, [0, 0, 0], [1, 1, 1], [1], [0], **kw)
+    assert (int(out["instance"][0]), int(out["stick"][0])) == (1, 1)   # none passes: all are candidates
+
+
+def check_coloc_lmetric_product(L):
+    """The balance target minimises estimate_load * num_requests (LMetric's
+    product, not a sum): it flips exactly where the products cross, an idle
+    instance (no requests) scores 0, and equal products rotate."""
+    rng = np.random.default_rng(52)
+    B, Lp, c_lin, c_att = 4, 40, 2, 1
+    t = rng.integers(0, 151936, size=Lp, dtype=np.int32)
+    ix = oracle.OracleIndex(2, L)
+    c = eq1_cost(Lp, Lp, c_lin, c_att)  # nothing cached: same prefill cost everywhere
+    assert c.denominator == 1
+    c = int(c)
+    big = [1 << 60] * 2
+    for q0, q1, r0, r1 in ((0, 0, 3, 2), (10, 0, 2, 3), (5 * c, c, 1, 3), (0, 10 ** 6, 7, 0)):
+        e0, e1 = q0 + c, q1 + c
+        want = 0 if e0 * r0 < e1 * r1 else 1 if e1 * r1 < e0 * r0 else 0  # ties: rotation from 0
+        out = _coloc(ix, B, [t], [q0, q1], big, [r0, r1], [0], [0], c_lin=c_lin, c_att=c_att)
+        assert int(out["instance"][0]) == want, (q0, q1, r0, r1)
+    out = _coloc(ix, B, [t] * 4, [0, 0], big, [2, 2], [0] * 4, [0] * 4, c_lin=c_lin, c_att=c_att, rr_base=1)
+    assert np.array_equal(out["instance"], [1, 0, 1, 0])
+    # products beyond 64 bits: est2 about 2^60 times 2^20 requests
+    out = _coloc(ix, B, [t], [(1 << 59) - 1, 1 << 59], big, [1 << 20, (1 << 20) - 1], [0], [0],
+                 c_lin=c_lin, c_att=c_att)
+    assert int(out["instance"][0]) == 1
+
+
+def check_coloc_no_last_resort(L):
+    """Under colocation a cached follow-up sticks only if prev meets the
+    deadline; when no instance meets it the request is balanced (Figure 10
+    would stick)."""
+    rng = np.random.default_rng(53)
+    B, Lp, k = 4, 64, 10
+    t = rng.integers(0, 151936, size=Lp, dtype=np.int32)
+    ix = oracle.OracleIndex(3, L)
+    _held(L, ix, t, B, {1: k})
+    q = [50, 4000, 20]
+    big = [1 << 60] * 3
+    kw = dict(c_lin=2, c_att=1, d0=0, d1=0)  # a deadline nobody meets
+    a = _coloc(ix, B, [t], q, big, [1, 1, 1], [1], [0], **kw)
+    b = _policy(ix, B, [t], q, [1], [0], **kw)
+    assert (int(b["instance"][0]), int(b["stick"][0])) == (1, 1)
+    assert int(a["stick"][0]) == 0 and int(a["instance"][0]) != 1
+
+
 ALL_CHECKS = [
     check_published_vector,
     check_bijection,
@@ -551,4 +652,8 @@ ALL_CHECKS = [
     check_policy_session_cached_threshold,
     check_policy_slo_migration,
     check_policy_round_robin_ties,
+    check_coloc_reduces_to_disaggregated,
+    check_coloc_tpot_filter,
+    check_coloc_lmetric_product,
+    check_coloc_no_last_resort,
 ]

@@ -55,6 +55,16 @@ MUTANTS = {
     "policy_ignores_turn": ("turn[r] != 0 && cached", "cached"),
     "policy_no_rotation": ("(int32_t)(((int64_t)rr_base + r) % N)", "0"),
     "policy_rotation_takes_last": ("if (est2[i] < est2[to]) to = i;", "if (est2[i] <= est2[to]) to = i;"),
+    "coloc_no_tpot_filter": ("cand[i] = cost2[i] <= 2 * tpot_budget[i];", "cand[i] = 1;"),
+    "coloc_filter_uses_load": ("cand[i] = cost2[i] <= 2 * tpot_budget[i];",
+                               "cand[i] = est2[i] <= 2 * tpot_budget[i];"),
+    "coloc_empty_filter_kept": ("for (int32_t i = 0; i < N; ++i) cand[i] = 1;", ";"),
+    "coloc_last_resort": ("meets_prev && cand[prev];", "(meets_prev || 1) && cand[prev];"),
+    "coloc_prev_not_checked": ("meets_prev && cand[prev];", "meets_prev;"),
+    "coloc_sum_not_product": ("(unsigned __int128)(uint64_t)est2[i] * (uint64_t)num_requests[i];",
+                              "(unsigned __int128)((uint64_t)est2[i] + (uint64_t)num_requests[i]);"),
+    "coloc_product_64_bit": ("(unsigned __int128)(uint64_t)est2[i] * (uint64_t)num_requests[i];",
+                             "(unsigned __int128)((uint64_t)est2[i] * (uint64_t)num_requests[i]);"),
 }
 
 
