@@ -59,6 +59,8 @@ def parse():
     ap.add_argument("--commit", action="store_true",
                     help="time device-side index maintenance (route, then commit the batch's blocks "
                          "and drain the queues) over a config-2 replay (one GPU; its own JSON line)")
+    ap.add_argument("--coloc", action="store_true",
+                    help="with --policy: the PD-colocation variant (Appendix B)")
     ap.add_argument("--policy", action="store_true",
                     help="time the session-centric policy (Figure 10) instead of the argmin cost "
                          "(one GPU; its own JSON line)")
@@ -540,6 +542,17 @@ def policy_inputs(tr, bt, k):
     return turn, est_hit, queued
 
 
+def coloc_inputs(tr, k):
+    """Per-instance TPOT budgets (a quarter of the instances run no decodes;
+    the others absorb 1e7 to 1e9 cost units of prefill) and request counts
+    (1 to 64) of batch k under PD colocation."""
+    rng = np.random.default_rng([0x5E55_0006, k])
+    N = tr.params.num_instances
+    tpot = rng.integers(10 ** 7, 10 ** 9, size=N).astype(np.int64)
+    tpot[rng.random(N) < 0.25] = 1 << 60
+    return tpot, rng.integers(1, 65, size=N).astype(np.int64)
+
+
 def run_policy(args):
     import torch
     import oracle
@@ -555,6 +568,7 @@ def run_policy(args):
     ids = list(range(N_DISTINCT_BATCHES))
     host = [tr.batch(k) for k in ids]
     extra = [policy_inputs(tr, b, k) for b, k in zip(host, ids)]
+    coloc = [coloc_inputs(tr, k) for k in ids] if args.coloc else None
     nkeys = tr.n_prefix_blocks()
     chunk = 4096
     max_tok = max(max(b.n_tokens for b in host), chunk * int(tr.prefix_len.max()))
@@ -565,6 +579,9 @@ def run_policy(args):
     T = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)
     dev_b = [dict(tok=T(b.tokens), off=T(b.offsets), n=b.n_requests, n_tokens=b.n_tokens, turn=T(tu),
                   est=T(eh), queued=T(q)) for b, (tu, eh, q) in zip(host, extra)]
+    if coloc:
+        for d, (tp, nr) in zip(dev_b, coloc):
+            d["tpot"], d["nreq"] = T(tp), T(nr)
     n = tr.batch_size
     outs = dict(instance=torch.empty(n, dtype=torch.int32, device=device),
                 local_hit=torch.empty(n, dtype=torch.int32, device=device),
@@ -575,6 +592,12 @@ def run_policy(args):
 
     def step(i):
         b = dev_b[i % len(dev_b)]
+        if coloc:
+            pkg.smetric_route_batch_policy_coloc(ix.handle, b["tok"], b["n_tokens"], b["off"], b["n"],
+                                                 b["queued"], b["tpot"], b["nreq"], b["turn"], b["est"], POLICY,
+                                                 outs["instance"], outs["local_hit"], outs["global_hit"],
+                                                 outs["stick"], outs["session_key"], None, 0, stream)
+            return
         pkg.smetric_route_batch_policy(ix.handle, b["tok"], b["n_tokens"], b["off"], b["n"], b["queued"],
                                        b["turn"], b["est"], POLICY, outs["instance"], outs["local_hit"],
                                        outs["global_hit"], outs["stick"], outs["session_key"], None, 0,
@@ -625,16 +648,29 @@ def run_policy(args):
     stage = {k: torch.empty_like(v, device=device) for k, v in hb[0].items() if k != "n"}
     hout = {k: torch.empty(n, dtype=v.dtype, pin_memory=True) for k, v in outs.items()}
 
+    if coloc:
+        for d, (tp, nr) in zip(hb, coloc[:2]):
+            d["tpot"], d["nreq"] = pin(tp), pin(nr)
+        stage["tpot"] = torch.empty_like(hb[0]["tpot"], device=device)
+        stage["nreq"] = torch.empty_like(hb[0]["nreq"], device=device)
+
     def e2e_step(i):
         b = hb[i % len(hb)]
-        for k in ("tok", "off", "turn", "est", "queued"):
+        for k in ("tok", "off", "turn", "est", "queued") + (("tpot", "nreq") if coloc else ()):
             if stage[k].numel() < b[k].numel():
                 stage[k] = torch.empty_like(b[k], device=device)
             stage[k][:b[k].numel()].copy_(b[k], non_blocking=True)
-        pkg.smetric_route_batch_policy(ix.handle, stage["tok"], b["tok"].numel(), stage["off"], b["n"],
-                                       stage["queued"], stage["turn"], stage["est"], POLICY, outs["instance"],
-                                       outs["local_hit"], outs["global_hit"], outs["stick"],
-                                       outs["session_key"], None, 0, stream)
+        if coloc:
+            pkg.smetric_route_batch_policy_coloc(ix.handle, stage["tok"], b["tok"].numel(), stage["off"], b["n"],
+                                                 stage["queued"], stage["tpot"], stage["nreq"], stage["turn"],
+                                                 stage["est"], POLICY, outs["instance"], outs["local_hit"],
+                                                 outs["global_hit"], outs["stick"], outs["session_key"], None, 0,
+                                                 stream)
+        else:
+            pkg.smetric_route_batch_policy(ix.handle, stage["tok"], b["tok"].numel(), stage["off"], b["n"],
+                                           stage["queued"], stage["turn"], stage["est"], POLICY, outs["instance"],
+                                           outs["local_hit"], outs["global_hit"], outs["stick"],
+                                           outs["session_key"], None, 0, stream)
         for k in hout:
             hout[k].copy_(outs[k], non_blocking=True)
         torch.cuda.synchronize()
@@ -649,7 +685,8 @@ def run_policy(args):
     for k in hout:
         if not np.array_equal(hout[k].numpy(), last[k]):
             raise RuntimeError(f"end-to-end policy route differs from the device route in {k}")
-    h2d = float(np.mean([sum(b[k].numel() * b[k].element_size() for k in ("tok", "off", "turn", "est", "queued"))
+    h2d = float(np.mean([sum(b[k].numel() * b[k].element_size()
+                             for k in ("tok", "off", "turn", "est", "queued") + (("tpot", "nreq") if coloc else ()))
                          for b in hb]))
 
     cpu = None
@@ -660,9 +697,13 @@ def run_policy(args):
         while True:  # the oracle's policy route runs on one thread
             off = bt.offsets[:m + 1]
             t0 = time.perf_counter()
-            ox.route_batch_policy(B, p.session_blocks, p.hash_seed, bt.tokens[:off[-1]], off, q, tu[:m], eh[:m],
-                                  POLICY["c_lin"], POLICY["c_att"], POLICY["ttft_d0"], POLICY["ttft_d1"],
-                                  POLICY["hit_num"], POLICY["hit_den"], POLICY["rr_base"])
+            pv = [POLICY[k] for k in ("c_lin", "c_att", "ttft_d0", "ttft_d1", "hit_num", "hit_den", "rr_base")]
+            if coloc:
+                ox.route_batch_coloc(B, p.session_blocks, p.hash_seed, bt.tokens[:off[-1]], off, q, coloc[0][0],
+                                     coloc[0][1], tu[:m], eh[:m], *pv)
+            else:
+                ox.route_batch_policy(B, p.session_blocks, p.hash_seed, bt.tokens[:off[-1]], off, q, tu[:m],
+                                      eh[:m], *pv)
             dt = time.perf_counter() - t0
             if dt > args.cpu_seconds / 2 or m == bt.n_requests:
                 break
@@ -676,7 +717,9 @@ def run_policy(args):
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
         "config": {"workload": workload_name(args), "batch": int(reqs), "num_instances": N, "block_size": B,
-                   "decision": "session-centric policy (Figure 10, Eq. 1 in fixed point)", "policy": POLICY,
+                   "decision": ("session-centric policy under PD colocation (Appendix B: TPOT filter, "
+                                "LMetric product)" if coloc else
+                                "session-centric policy (Figure 10, Eq. 1 in fixed point)"), "policy": POLICY,
                    "queued": f"batch load x {QUEUED_SCALE}", "first_turn_fraction": 0.1,
                    "stick_fraction": stick,
                    "l2": f"inputs larger than L2: {N_DISTINCT_BATCHES} distinct batches rotated"},

@@ -168,6 +168,8 @@ int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_t
  * stays below 2^63 within them). */
 #define SMETRIC_POLICY_MAX_LEN (1LL << 24)     /* prompt tokens per request */
 #define SMETRIC_POLICY_MAX_QUEUED (1LL << 59)  /* an instance's queued cost */
+#define SMETRIC_POLICY_MAX_TPOT (1LL << 60)    /* colocation: a TPOT budget */
+#define SMETRIC_POLICY_MAX_REQUESTS (1LL << 20) /* colocation: an instance's request count */
 
 /* Parameters of the session-centric policy (Figure 10), integers:
  *   c_lin, c_att  Eq. 1's coefficients: the prefill cost of n new tokens in
@@ -222,6 +224,31 @@ int smetric_route_batch_policy(smetric_index* idx, const int32_t* d_tokens, int6
                                int32_t* d_instance, int32_t* d_local_hit, int32_t* d_global_hit,
                                int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
                                int64_t hashes_cap, smetric_stream_t stream);
+
+/* The session-centric policy under PD colocation (Appendix B): as
+ * smetric_route_batch_policy, with two changes.
+ *   TPOT check: with cost_i = c_lin*n_i + c_att*n_i*(L - n_i/2) (the request's
+ *   own prefill on instance i), instance i is a candidate when
+ *   cost_i <= d_tpot_budget[i], the prefill the live decodes on i absorb
+ *   within their TPOT SLO (PREFILL_RATE times their smallest slack, in cost
+ *   units; SMETRIC_POLICY_MAX_TPOT for an instance with none); when no
+ *   instance passes, every instance is a candidate.
+ *   stick = d_turn[r] != 0 and cached and meets(prev) and prev is a
+ *   candidate (no last resort);
+ *   i* = prev if stick, else the first minimal est_i * d_num_requests[i]
+ *   over the candidates in the rotation order (LMetric's product, compared
+ *   exactly in 128 bits).
+ *   d_tpot_budget   int64 [N], each in [0, SMETRIC_POLICY_MAX_TPOT].
+ *   d_num_requests  int64 [N], each in [0, SMETRIC_POLICY_MAX_REQUESTS].
+ * Out-of-range values of either latch SMETRIC_ERR_OVERFLOW like the queued
+ * costs. */
+int smetric_route_batch_policy_coloc(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                                     const int64_t* d_offsets, int32_t n_requests, const int64_t* d_queued,
+                                     const int64_t* d_tpot_budget, const int64_t* d_num_requests,
+                                     const int32_t* d_turn, const int64_t* d_est_hit, smetric_policy p,
+                                     int32_t* d_instance, int32_t* d_local_hit, int32_t* d_global_hit,
+                                     int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                                     int64_t hashes_cap, smetric_stream_t stream);
 
 /* Flags of smetric_index_commit_batch. */
 #define SMETRIC_COMMIT_GLOBAL 1 /* also add every block to the global tier */

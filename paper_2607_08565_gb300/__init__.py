@@ -35,6 +35,8 @@ SMETRIC_FLAG_HOST_STAGING = 1
 SMETRIC_POLICY_MAX_LEN = 1 << 24
 SMETRIC_POLICY_MAX_QUEUED = 1 << 59
 SMETRIC_COMMIT_GLOBAL = 1
+SMETRIC_POLICY_MAX_TPOT = 1 << 60
+SMETRIC_POLICY_MAX_REQUESTS = 1 << 20
 
 EXPORTED = (
     "smetric_index_create", "smetric_index_destroy", "smetric_index_clear",
@@ -43,7 +45,7 @@ EXPORTED = (
     "smetric_route_batch_host", "smetric_status", "smetric_strerror",
     "smetric_profile_enable", "smetric_profile_read", "smetric_profile_kernel_name",
     "smetric_launch_count", "smetric_block_hashes_noalloc", "smetric_route_batch_policy",
-    "smetric_index_commit_batch",
+    "smetric_index_commit_batch", "smetric_route_batch_policy_coloc",
 )
 
 
@@ -106,6 +108,8 @@ def lib():
             "smetric_route_batch_policy": (C.c_int, [P, P, I64, P, I32, P, P, P, smetric_policy, P, P,
                                                      P, P, P, P, I64, P]),
             "smetric_index_commit_batch": (C.c_int, [P, P, I32, P, P, P, I32, P, P]),
+            "smetric_route_batch_policy_coloc": (C.c_int, [P, P, I64, P, I32, P, P, P, P, P, smetric_policy,
+                                                           P, P, P, P, P, P, I64, P]),
             "smetric_block_hashes": (C.c_int, [P, P, I64, P, I32, P, P, I64, P]),
             "smetric_block_hashes_noalloc": (C.c_int, [P, I64, P, I32, I32, I32, C.c_uint64, P, P, I64,
                                                       P, P]),
@@ -227,6 +231,17 @@ def smetric_route_batch_policy(idx: int, d_tokens, n_tokens: int, d_offsets, n_r
         _ptr(d_est_hit), _policy(policy), _ptr(d_instance), _ptr(d_local_hit), _ptr(d_global_hit),
         _ptr(d_stick), _ptr(d_session_key), _ptr(d_block_hashes), hashes_cap, _stream(stream)),
         "smetric_route_batch_policy")
+
+
+def smetric_route_batch_policy_coloc(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int,
+                                     d_queued, d_tpot_budget, d_num_requests, d_turn, d_est_hit, policy,
+                                     d_instance, d_local_hit, d_global_hit, d_stick, d_session_key,
+                                     d_block_hashes=None, hashes_cap: int = 0, stream=None) -> None:
+    _check(lib().smetric_route_batch_policy_coloc(
+        idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests, _ptr(d_queued), _ptr(d_tpot_budget),
+        _ptr(d_num_requests), _ptr(d_turn), _ptr(d_est_hit), _policy(policy), _ptr(d_instance),
+        _ptr(d_local_hit), _ptr(d_global_hit), _ptr(d_stick), _ptr(d_session_key), _ptr(d_block_hashes),
+        hashes_cap, _stream(stream)), "smetric_route_batch_policy_coloc")
 
 
 def smetric_index_commit_batch(idx: int, d_offsets, n_requests: int, d_instance, d_local_hit,
@@ -396,6 +411,27 @@ class SMetricIndex:
                                    policy, out["instance"], out["local_hit"], out["global_hit"],
                                    out["stick"], out["session_key"], hb,
                                    hb.numel() if hb is not None else 0, stream)
+        return out
+
+    def route_batch_policy_coloc(self, tokens, offsets, queued, tpot_budget, num_requests, turn, est_hit,
+                                 policy, want_hashes=False, stream=None):
+        """The session-centric policy under PD colocation (Appendix B).
+        Returns dict(instance, local_hit, global_hit, stick, session_key[, block_hashes])."""
+        import torch
+        n = offsets.numel() - 1
+        dev = offsets.device
+        out = dict(instance=torch.empty(n, dtype=torch.int32, device=dev),
+                   local_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                   global_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                   stick=torch.empty(n, dtype=torch.int32, device=dev),
+                   session_key=torch.empty(n, dtype=torch.uint64, device=dev))
+        if want_hashes:
+            out["block_hashes"] = torch.empty(max(tokens.numel() // self.B, 1), dtype=torch.uint64, device=dev)
+        hb = out.get("block_hashes")
+        smetric_route_batch_policy_coloc(self.handle, tokens, tokens.numel(), offsets, n, queued, tpot_budget,
+                                         num_requests, turn, est_hit, policy, out["instance"], out["local_hit"],
+                                         out["global_hit"], out["stick"], out["session_key"], hb,
+                                         hb.numel() if hb is not None else 0, stream)
         return out
 
     def commit_batch(self, offsets, out, also_global=False, load=None, stream=None):

@@ -81,7 +81,9 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
                                               int n_load, int64_t* __restrict__ block_off,
                                               int64_t* __restrict__ chunk_off, int32_t* batch_ok,
                                               int32_t* status, int64_t max_load, int64_t max_len,
-                                              const int64_t* __restrict__ est_hit) {
+                                              const int64_t* __restrict__ est_hit,
+                                              const int64_t* __restrict__ aux0 = nullptr, int64_t aux0_max = 0,
+                                              const int64_t* __restrict__ aux1 = nullptr, int64_t aux1_max = 0) {
   constexpr int NS = 2;  // scans: full blocks, and 32-block chunks (when chunk_off is wanted)
   constexpr int R = kPrepRounds;
   __shared__ int64_t warp_tot[NS][32];
@@ -94,6 +96,8 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
   for (int i = tid; i < n_load; i += blockDim.x) {
     const int64_t v = load[i];
     if (v < 0 || v > max_load) bad |= 2;
+    if (aux0 && (aux0[i] < 0 || aux0[i] > aux0_max)) bad |= 2;  // further per-instance inputs
+    if (aux1 && (aux1[i] < 0 || aux1[i] > aux1_max)) bad |= 2;
   }
   if (est_hit)  // the policy's expected hits, each in [0, 2^31)
     for (int64_t r = tid; r < n; r += blockDim.x) {
@@ -820,13 +824,17 @@ __global__ void __launch_bounds__(256)
 
 // The session-centric policy (Figure 10) as the walk's decision; off for
 // the argmin cost of smetric_route_batch.
+enum Decide { kArgmin = 0, kSession = 1, kColoc = 2 };
+
 struct WalkPolicy {
-  int on;
+  int on;    // a Decide value; 0 = the argmin cost
   int64_t c_lin, c_att, d0, d1, hit_num, hit_den;
   int32_t rr_base;
   const int32_t* turn;
   const int64_t* est_hit;
   int32_t* stick;
+  const int64_t* tpot;  // colocation: prefill cost each instance's live decodes absorb
+  const int64_t* nreq;  // colocation: requests each instance runs
 };
 
 // One warp per request, lanes = 32 consecutive blocks. The masks are
@@ -846,7 +854,7 @@ struct WalkPolicy {
 // alive through share - 1 continues over the member's own masks from block
 // `share` on. Members therefore start at `share` instead of re-reading the
 // leader's masks from block 0.
-template <int W, bool MEMBERS, bool POLICY>
+template <int W, bool MEMBERS, int DECIDE>
 __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (leaders) or 5 (members) CTAs per SM
     k_walk(int N, int B, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n,
            const int64_t* __restrict__ load, int64_t w_load, int64_t w_miss, int64_t w_glob,
@@ -876,7 +884,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
     for (int64_t r = (int64_t)blockIdx.x * kMatchWarps + warp; r < n; r += tw)
       if (lane == 0) {
         inst_out[r] = -1; lhit_out[r] = 0; ghit_out[r] = 0;
-        if (POLICY) pol.stick[r] = 0;
+        if (DECIDE != kArgmin) pol.stick[r] = 0;
       }
   // k_group's lists: leaders from the front of `order`, members from the back
   const int64_t count = !ok ? 0 : MEMBERS ? counts[1] : counts[0];
@@ -1015,12 +1023,21 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
     int64_t best_cost = INT64_MAX;
     int32_t best = N;
     int64_t best_c = 0;
-    // policy: prev = argmax c (lowest id), rr_argmin of 2*estimate_load
+    // policies: prev = argmax c (lowest id); the balance key per instance:
+    // 2*estimate_load (Figure 10), or the 128-bit product 2*estimate_load *
+    // requests (colocation: over the candidates passing the TPOT check, and
+    // over all instances for when none passes); ties rotate from s0
     int64_t pc = -1, pe = INT64_MAX, pec = 0;
     int32_t pi = N, prot = N;
-    bool meets_any = false;
-    const int32_t s0 = POLICY ? (int32_t)(((int64_t)pol.rr_base + r) % N) : 0;
-    const int64_t budget2 = POLICY ? 2 * (pol.d0 + pol.d1 * L) : 0;
+    bool meets_any = false, cand_any = false;
+    uint64_t ahi = ~0ull, alo = ~0ull, chi = ~0ull, clo = ~0ull;
+    int32_t arot = N, crot = N;
+    int64_t ac = 0, cc = 0;
+    auto less128 = [](uint64_t h1, uint64_t l1, int32_t r1, uint64_t h2, uint64_t l2, int32_t r2) {
+      return h1 < h2 || (h1 == h2 && (l1 < l2 || (l1 == l2 && r1 < r2)));
+    };
+    const int32_t s0 = DECIDE != kArgmin ? (int32_t)(((int64_t)pol.rr_base + r) % N) : 0;
+    const int64_t budget2 = DECIDE != kArgmin ? 2 * (pol.d0 + pol.d1 * L) : 0;
     int32_t* const out_c = summ + r * (N + 1);
 #pragma unroll
     for (int t = 0; t < CT; ++t) {
@@ -1039,22 +1056,32 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
           if (ev_mask[e * W + wi] & bi) { ci = ev_pos[e]; break; }
       }
       if (!MEMBERS) out_c[i] = (int32_t)ci;
-      if (!POLICY) {
+      if (DECIDE == kArgmin) {
         const int64_t gi = ci > g ? ci : g;
         const int64_t cost = w_load * load_s[i] + w_miss * (L - B * gi) + w_glob * B * (gi - ci);
         if (cost < best_cost) { best_cost = cost; best = i; best_c = ci; }
       } else {
-        // Eq. 1 doubled: 2*q_i + 2*c_lin*n + c_att*n*(2L - n), n = new tokens
+        // Eq. 1 doubled: 2*c_lin*n + c_att*n*(2L - n), n = new tokens, plus 2*q_i
         const int64_t nn = L - B * ci;
-        const int64_t est2 = 2 * load_s[i] + 2 * pol.c_lin * nn + pol.c_att * nn * (2 * L - nn);
+        const int64_t cost2 = 2 * pol.c_lin * nn + pol.c_att * nn * (2 * L - nn);
+        const int64_t est2 = 2 * load_s[i] + cost2;
         meets_any |= est2 <= budget2;
         if (ci > pc) { pc = ci; pi = i; }  // lanes see their instances in increasing order
         const int32_t rot = (int32_t)((i - s0 + N) % N);
-        if (est2 < pe || (est2 == pe && rot < prot)) { pe = est2; prot = rot; pec = ci; }
+        if (DECIDE == kSession) {
+          if (est2 < pe || (est2 == pe && rot < prot)) { pe = est2; prot = rot; pec = ci; }
+        } else {
+          const bool cand = cost2 <= 2 * __ldg(pol.tpot + i);
+          const uint64_t R = (uint64_t)__ldg(pol.nreq + i);
+          const uint64_t lo = (uint64_t)est2 * R, hi = __umul64hi((uint64_t)est2, R);
+          cand_any |= cand;
+          if (less128(hi, lo, rot, ahi, alo, arot)) { ahi = hi; alo = lo; arot = rot; ac = ci; }
+          if (cand && less128(hi, lo, rot, chi, clo, crot)) { chi = hi; clo = lo; crot = rot; cc = ci; }
+        }
       }
     }
     if (!MEMBERS && lane == 0) out_c[N] = (int32_t)g;
-    if (!POLICY) {
+    if (DECIDE == kArgmin) {
 #pragma unroll
       for (int dd = 16; dd > 0; dd >>= 1) {
         const int64_t oc = __shfl_xor_sync(kFull, best_cost, dd);
@@ -1074,19 +1101,43 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
         const int64_t oc = __shfl_xor_sync(kFull, pc, dd);
         const int32_t oi = __shfl_xor_sync(kFull, pi, dd);
         if (oc > pc || (oc == pc && oi < pi)) { pc = oc; pi = oi; }
-        const int64_t oe = __shfl_xor_sync(kFull, pe, dd);
-        const int32_t orot = __shfl_xor_sync(kFull, prot, dd);
-        const int64_t oec = __shfl_xor_sync(kFull, pec, dd);
-        if (oe < pe || (oe == pe && orot < prot)) { pe = oe; prot = orot; pec = oec; }
+        if (DECIDE == kSession) {
+          const int64_t oe = __shfl_xor_sync(kFull, pe, dd);
+          const int32_t orot = __shfl_xor_sync(kFull, prot, dd);
+          const int64_t oec = __shfl_xor_sync(kFull, pec, dd);
+          if (oe < pe || (oe == pe && orot < prot)) { pe = oe; prot = orot; pec = oec; }
+        } else {
+          uint64_t oh = __shfl_xor_sync(kFull, ahi, dd), ol = __shfl_xor_sync(kFull, alo, dd);
+          int32_t orot = __shfl_xor_sync(kFull, arot, dd);
+          int64_t oc2 = __shfl_xor_sync(kFull, ac, dd);
+          if (less128(oh, ol, orot, ahi, alo, arot)) { ahi = oh; alo = ol; arot = orot; ac = oc2; }
+          oh = __shfl_xor_sync(kFull, chi, dd);
+          ol = __shfl_xor_sync(kFull, clo, dd);
+          orot = __shfl_xor_sync(kFull, crot, dd);
+          oc2 = __shfl_xor_sync(kFull, cc, dd);
+          if (less128(oh, ol, orot, chi, clo, crot)) { chi = oh; clo = ol; crot = orot; cc = oc2; }
+        }
       }
       const bool any = __any_sync(kFull, meets_any);
+      const bool cands = __any_sync(kFull, cand_any);
       if (lane == 0) {
         const int64_t np = L - B * pc;
-        const int64_t est2p = 2 * load_s[pi] + 2 * pol.c_lin * np + pol.c_att * np * (2 * L - np);
+        const int64_t cost2p = 2 * pol.c_lin * np + pol.c_att * np * (2 * L - np);
+        const int64_t est2p = 2 * load_s[pi] + cost2p;
         const bool cached = B * pc * pol.hit_den > pol.hit_num * pol.est_hit[r];
-        const bool stick = pol.turn[r] != 0 && cached && (est2p <= budget2 || !any);
-        const int32_t to = stick ? pi : (int32_t)((s0 + prot) % N);
-        const int64_t ct = stick ? pc : pec;
+        bool stick;
+        int32_t to;
+        int64_t ct;
+        if (DECIDE == kSession) {
+          stick = pol.turn[r] != 0 && cached && (est2p <= budget2 || !any);
+          to = stick ? pi : (int32_t)((s0 + prot) % N);
+          ct = stick ? pc : pec;
+        } else {
+          const bool prev_cand = !cands || cost2p <= 2 * __ldg(pol.tpot + pi);
+          stick = pol.turn[r] != 0 && cached && est2p <= budget2 && prev_cand;
+          to = stick ? pi : (int32_t)((s0 + (cands ? crot : arot)) % N);
+          ct = stick ? pc : (cands ? cc : ac);
+        }
         const int64_t gt = ct > g ? ct : g;
         inst_out[r] = to;
         lhit_out[r] = (int32_t)(B * ct);
@@ -1355,9 +1406,10 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
   const int64_t want = ((int64_t)n + kMatchWarps - 1) / kMatchWarps;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
   // leaders, then members (which read the leaders' run ends)
-  using WalkKernel = decltype(&k_walk<W, false, false>);  // every instantiation has this signature
-  const WalkKernel kerns[2] = {pol.on ? k_walk<W, false, true> : k_walk<W, false, false>,
-                               pol.on ? k_walk<W, true, true> : k_walk<W, true, false>};
+  using WalkKernel = decltype(&k_walk<W, false, kArgmin>);  // every instantiation has this signature
+  const WalkKernel kerns[2] = {
+      pol.on == kColoc ? k_walk<W, false, kColoc> : pol.on == kSession ? k_walk<W, false, kSession> : k_walk<W, false, kArgmin>,
+      pol.on == kColoc ? k_walk<W, true, kColoc> : pol.on == kSession ? k_walk<W, true, kSession> : k_walk<W, true, kArgmin>};
   for (const WalkKernel kern : kerns) {
     if (smem > 48 * 1024 &&
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
@@ -1430,7 +1482,9 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
   k_prep<<<1, 1024, 0, s>>>(d_offsets, n, n_tokens, c.block_size, d_load, PROBE ? c.num_instances : 0,
                             idx->block_off, idx->chunk_off, idx->batch_ok, idx->status,
                             pol ? SMETRIC_POLICY_MAX_QUEUED : SMETRIC_MAX_LOAD,
-                            pol ? SMETRIC_POLICY_MAX_LEN : (int64_t)INT32_MAX, pol ? pol->est_hit : nullptr);
+                            pol ? SMETRIC_POLICY_MAX_LEN : (int64_t)INT32_MAX, pol ? pol->est_hit : nullptr,
+                            pol ? pol->tpot : nullptr, SMETRIC_POLICY_MAX_TPOT,
+                            pol ? pol->nreq : nullptr, SMETRIC_POLICY_MAX_REQUESTS);
   idx->launches++;
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   profile_mark(idx, kPrep, s);
@@ -1453,6 +1507,40 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
   return SMETRIC_OK;
 }
 
+int route_policy(smetric_index* idx, int mode, const int32_t* d_tokens, int64_t n_tokens,
+                 const int64_t* d_offsets, int32_t n_requests, const int64_t* d_queued,
+                 const int64_t* d_tpot, const int64_t* d_nreq, const int32_t* d_turn,
+                 const int64_t* d_est_hit, smetric_policy p, int32_t* d_instance, int32_t* d_local_hit,
+                 int32_t* d_global_hit, int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                 int64_t hashes_cap, smetric_stream_t stream) {
+  if (!idx) return SMETRIC_ERR_INVALID_ARG;
+  const int64_t N = idx->cfg.num_instances;
+  if (p.c_lin < 0 || p.c_lin > (1LL << 20) || p.c_att < 0 || p.c_att > (1LL << 12) || p.ttft_d0 < 0 ||
+      p.ttft_d0 > (1LL << 60) || p.ttft_d1 < 0 || p.ttft_d1 > (1LL << 35) || p.hit_den < 1 ||
+      p.hit_den > (1LL << 20) || p.hit_num < 0 || p.hit_num > p.hit_den || p.rr_base < 0 || p.rr_base >= N ||
+      p.reserved != 0)
+    return SMETRIC_ERR_INVALID_ARG;
+  if (n_requests > 0 && (!d_turn || !d_est_hit || !d_stick)) return SMETRIC_ERR_INVALID_ARG;
+  WalkPolicy pol;
+  pol.on = mode;
+  pol.c_lin = p.c_lin;
+  pol.c_att = p.c_att;
+  pol.d0 = p.ttft_d0;
+  pol.d1 = p.ttft_d1;
+  pol.hit_num = p.hit_num;
+  pol.hit_den = p.hit_den;
+  pol.rr_base = p.rr_base;
+  pol.turn = d_turn;
+  pol.est_hit = d_est_hit;
+  pol.stick = d_stick;
+  pol.tpot = d_tpot;
+  pol.nreq = d_nreq;
+  // the argmin weights are unused by the policy; any valid ones pass the checks
+  return route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_queued, smetric_weights{0, 0, 0},
+                            d_instance, d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap,
+                            reinterpret_cast<cudaStream_t>(stream), &pol);
+}
+
 }  // namespace
 
 extern "C" {
@@ -1467,37 +1555,30 @@ int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_t
                             reinterpret_cast<cudaStream_t>(stream));
 }
 
+int smetric_route_batch_policy_coloc(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                                     const int64_t* d_offsets, int32_t n_requests, const int64_t* d_queued,
+                                     const int64_t* d_tpot_budget, const int64_t* d_num_requests,
+                                     const int32_t* d_turn, const int64_t* d_est_hit, smetric_policy p,
+                                     int32_t* d_instance, int32_t* d_local_hit, int32_t* d_global_hit,
+                                     int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                                     int64_t hashes_cap, smetric_stream_t stream) {
+  if (!idx || !d_tpot_budget || !d_num_requests) return SMETRIC_ERR_INVALID_ARG;
+  return route_policy(idx, kColoc, d_tokens, n_tokens, d_offsets, n_requests, d_queued, d_tpot_budget,
+                      d_num_requests, d_turn, d_est_hit, p, d_instance, d_local_hit, d_global_hit, d_stick,
+                      d_session_key, d_block_hashes, hashes_cap, stream);
+}
+
 int smetric_route_batch_policy(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
                                const int64_t* d_offsets, int32_t n_requests, const int64_t* d_queued,
                                const int32_t* d_turn, const int64_t* d_est_hit, smetric_policy p,
                                int32_t* d_instance, int32_t* d_local_hit, int32_t* d_global_hit,
                                int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
                                int64_t hashes_cap, smetric_stream_t stream) {
-  if (!idx) return SMETRIC_ERR_INVALID_ARG;
-  const int64_t N = idx->cfg.num_instances;
-  if (p.c_lin < 0 || p.c_lin > (1LL << 20) || p.c_att < 0 || p.c_att > (1LL << 12) || p.ttft_d0 < 0 ||
-      p.ttft_d0 > (1LL << 60) || p.ttft_d1 < 0 || p.ttft_d1 > (1LL << 35) || p.hit_den < 1 ||
-      p.hit_den > (1LL << 20) || p.hit_num < 0 || p.hit_num > p.hit_den || p.rr_base < 0 || p.rr_base >= N ||
-      p.reserved != 0)
-    return SMETRIC_ERR_INVALID_ARG;
-  if (n_requests > 0 && (!d_turn || !d_est_hit || !d_stick)) return SMETRIC_ERR_INVALID_ARG;
-  WalkPolicy pol;
-  pol.on = 1;
-  pol.c_lin = p.c_lin;
-  pol.c_att = p.c_att;
-  pol.d0 = p.ttft_d0;
-  pol.d1 = p.ttft_d1;
-  pol.hit_num = p.hit_num;
-  pol.hit_den = p.hit_den;
-  pol.rr_base = p.rr_base;
-  pol.turn = d_turn;
-  pol.est_hit = d_est_hit;
-  pol.stick = d_stick;
-  // the argmin weights are unused by the policy; any valid ones pass the checks
-  return route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_queued, smetric_weights{0, 0, 0},
-                            d_instance, d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap,
-                            reinterpret_cast<cudaStream_t>(stream), &pol);
+  return route_policy(idx, kSession, d_tokens, n_tokens, d_offsets, n_requests, d_queued, nullptr, nullptr,
+                      d_turn, d_est_hit, p, d_instance, d_local_hit, d_global_hit, d_stick, d_session_key,
+                      d_block_hashes, hashes_cap, stream);
 }
+
 
 int smetric_index_commit_batch(smetric_index* idx, const int64_t* d_offsets, int32_t n_requests,
                                const int32_t* d_instance, const int32_t* d_local_hit,

@@ -146,3 +146,76 @@ def test_policy_rejects_prompts_longer_than_its_limit():
         assert ix.status() == code
         assert int(out["instance"].cpu()[0]) == (-1 if code else 1)  # equal loads: rotation from rr_base
     ix.close()
+
+
+# ---------------------------------------------------------------------------
+# PD colocation (Appendix B)
+# ---------------------------------------------------------------------------
+
+def gpu_coloc(ix, tok, off, queued, tpot, nreq, turn, est_hit, p):
+    out = ix.route_batch_policy_coloc(T(tok), T(off), T(np.asarray(queued, np.int64)), T(np.asarray(tpot, np.int64)),
+                                      T(np.asarray(nreq, np.int64)), T(np.asarray(turn, np.int32)),
+                                      T(np.asarray(est_hit, np.int64)), p)
+    ix.check()
+    return {k: v.cpu().numpy() for k, v in out.items()}
+
+
+def oracle_coloc(ox, B, S, tok, off, queued, tpot, nreq, turn, est_hit, p):
+    return ox.route_batch_coloc(B, S, 0, tok, off, queued, tpot, nreq, turn, est_hit, p["c_lin"], p["c_att"],
+                                p["ttft_d0"], p["ttft_d1"], p["hit_num"], p["hit_den"], p["rr_base"])
+
+
+@pytest.mark.parametrize("N,B", [(1, 4), (3, 2), (8, 16), (64, 4), (130, 2), (256, 8)])
+def test_coloc_matches_oracle_tiny_alphabet(N, B):
+    rng = np.random.default_rng(N * 977 + B)
+    for trial in range(3):
+        stored, reqs = tiny_alphabet_case(rng, N, B, n_req=300, max_blocks=12)
+        S = int(rng.integers(1, 4))
+        ix = make_index(N, B, S, cap=8192)
+        ox = oracle.OracleIndex(N)
+        populate_both(ix, ox, stored, B)
+        tok, off = pack(reqs)
+        n = len(reqs)
+        L = np.diff(off)
+        for case in range(6):
+            p = _params(rng, N, tight=case % 2 == 0)
+            queued = rng.integers(0, [1 << 59, 1 << 20, 8, 1 << 40, 3, 1 << 59][case], size=N)
+            # TPOT budgets around the prefill costs, some unlimited, some zero
+            tpot = rng.integers(0, 1 << [60, 30, 12, 45, 8, 60][case], size=N)
+            tpot[rng.random(N) < 0.2] = pkg.SMETRIC_POLICY_MAX_TPOT
+            tpot[rng.random(N) < 0.1] = 0
+            nreq = rng.integers(0, [1 << 20, 4, 64, 2, 1 << 20, 1000][case], size=N)
+            turn = rng.integers(0, 3, size=n) * (case != 5)
+            est_hit = np.minimum(rng.integers(0, 2 * L + 1), (1 << 31) - 1)
+            g = gpu_coloc(ix, tok, off, queued, tpot, nreq, turn, est_hit, p)
+            o = oracle_coloc(ox, B, S, tok, off, queued, tpot, nreq, turn, est_hit, p)
+            assert_outputs_equal(g, o, fields=FIELDS, ctx=f"coloc N={N} B={B} trial={trial} case={case}")
+        ix.close()
+
+
+def test_coloc_rejects_out_of_range_inputs():
+    rng = np.random.default_rng(79)
+    N, B = 4, 16
+    ix = make_index(N, B, 1)
+    tok = rng.integers(0, 151936, size=1000, dtype=np.int32)
+    off = np.array([0, 100, 400, 1000], np.int64)
+    good = dict(c_lin=1, c_att=1, ttft_d0=1000, ttft_d1=1, hit_num=1, hit_den=2, rr_base=0)
+    ok_t, ok_r = np.full(N, 1 << 40), np.ones(N)
+    for tpot, nreq in ((np.array([0, (1 << 60) + 1, 0, 0]), ok_r), (np.array([0, -1, 0, 0]), ok_r),
+                       (ok_t, np.array([0, (1 << 20) + 1, 0, 0])), (ok_t, np.array([-1, 0, 0, 0]))):
+        out = ix.route_batch_policy_coloc(T(tok), T(off), T(np.zeros(N, np.int64)), T(np.asarray(tpot, np.int64)),
+                                          T(np.asarray(nreq, np.int64)), T(np.ones(3, np.int32)),
+                                          T(np.zeros(3, np.int64)), good)
+        assert ix.status() == pkg.SMETRIC_ERR_OVERFLOW
+        assert np.all(out["instance"].cpu().numpy() == -1)
+    with pytest.raises(pkg.SmetricError):
+        pkg.smetric_route_batch_policy_coloc(ix.handle, T(tok), 1000, T(off), 3, T(np.zeros(N, np.int64)), None,
+                                             T(np.ones(N, np.int64)), T(np.ones(3, np.int32)),
+                                             T(np.zeros(3, np.int64)), good, T(np.zeros(3, np.int32)),
+                                             T(np.zeros(3, np.int32)), T(np.zeros(3, np.int32)),
+                                             T(np.zeros(3, np.int32)), T(np.zeros(3, np.uint64)))
+    out = ix.route_batch_policy_coloc(T(tok), T(off), T(np.zeros(N, np.int64)), T(ok_t.astype(np.int64)),
+                                      T(ok_r.astype(np.int64)), T(np.ones(3, np.int32)), T(np.zeros(3, np.int64)),
+                                      good)
+    assert ix.status() == pkg.SMETRIC_OK
+    ix.close()
