@@ -68,6 +68,8 @@ def load_library(path: str):
         C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p, i64p, i64p, i32p, i64p,
         C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int32,
         i32p, i32p, i32p, i32p, u64p]
+    L.oracle_link_sessions.restype = C.c_int
+    L.oracle_link_sessions.argtypes = [C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p, i32p, i32p, i32p]
     return L
 
 
@@ -90,6 +92,24 @@ def block_hashes(tokens: np.ndarray, block_size: int, seed: int = 0, L=None) -> 
     if n < 0:
         raise ValueError("invalid block size")
     return out[:n]
+
+
+def link_sessions(block_size: int, seed: int, tokens, offsets, users, turns, L=None):
+    """Session reconstruction (Appendix A). Returns (parent, session), int32 per request."""
+    t = np.ascontiguousarray(tokens, dtype=np.int32)
+    o = np.ascontiguousarray(offsets, dtype=np.int64)
+    n = len(o) - 1
+    u = np.ascontiguousarray(users, dtype=np.int64)
+    tu = np.ascontiguousarray(turns, dtype=np.int32)
+    parent = np.zeros(max(n, 1), np.int32)
+    session = np.zeros(max(n, 1), np.int32)
+    rc = (L or lib()).oracle_link_sessions(block_size, seed & 0xFFFFFFFFFFFFFFFF,
+                                           t if len(t) else np.zeros(1, np.int32), o, n,
+                                           u if n else np.zeros(1, np.int64), tu if n else np.zeros(1, np.int32),
+                                           parent, session)
+    if rc != 0:
+        raise ValueError(f"oracle_link_sessions: {rc}")
+    return parent[:n], session[:n]
 
 
 class OracleIndex:

@@ -83,6 +83,13 @@
  *              in the rotation order above, R_i = the requests instance i
  *              runs (LMetric's multiplicative score), compared exactly in
  *              128 bits.
+ *
+ * Session reconstruction (Appendix A; oracle_link_sessions): request r
+ * follows request p when p is earlier (p < r, requests in arrival order), of
+ * the same user, of turn turn_r - 1, and p's block-hash sequence is a prefix
+ * of r's (h_p[b] = h_r[b] for every b < n_p; the empty sequence is a prefix
+ * of every sequence). parent_r is the latest such p, or -1; session_r is the
+ * first request of r's chain of parents.
  */
 #include <stdint.h>
 #include <stdlib.h>
@@ -502,4 +509,39 @@ int oracle_route_batch_coloc(const oracle_index* x, int32_t B, int32_t S, uint64
   free(est2);
   free(cand);
   return rc;
+}
+
+/* Session reconstruction (Appendix A), by definition: every earlier request
+ * is compared in full, latest first. users and turns have n_requests
+ * entries; parent and session receive n_requests entries. */
+int oracle_link_sessions(int32_t B, uint64_t seed, const int32_t* tokens, const int64_t* offsets,
+                         int32_t n_requests, const int64_t* users, const int32_t* turns, int32_t* parent,
+                         int32_t* session) {
+  if (B < 2 || (B % 2) != 0 || n_requests < 0) return ORACLE_ERR_INVALID_ARG;
+  for (int32_t r = 0; r < n_requests; ++r)
+    if (offsets[r + 1] < offsets[r] || offsets[r] < 0) return ORACLE_ERR_INVALID_ARG;
+  int64_t* first = (int64_t*)malloc((size_t)(n_requests + 1) * sizeof(int64_t));
+  if (!first) return ORACLE_ERR_OOM;
+  first[0] = 0;
+  for (int32_t r = 0; r < n_requests; ++r) first[r + 1] = first[r] + (offsets[r + 1] - offsets[r]) / B;
+  uint64_t* h = (uint64_t*)malloc((size_t)(first[n_requests] + 1) * sizeof(uint64_t));
+  if (!h) { free(first); return ORACLE_ERR_OOM; }
+  for (int32_t r = 0; r < n_requests; ++r)
+    oracle_block_hashes(tokens + offsets[r], offsets[r + 1] - offsets[r], B, seed, h + first[r]);
+  for (int32_t r = 0; r < n_requests; ++r) {
+    const int64_t nr = first[r + 1] - first[r];
+    parent[r] = -1;
+    for (int32_t p = r - 1; p >= 0; --p) {
+      if (users[p] != users[r] || (int64_t)turns[p] != (int64_t)turns[r] - 1) continue;
+      const int64_t np = first[p + 1] - first[p];
+      if (np > nr) continue;
+      int prefix = 1;
+      for (int64_t b = 0; b < np && prefix; ++b) prefix = h[first[p] + b] == h[first[r] + b];
+      if (prefix) { parent[r] = p; break; }
+    }
+    session[r] = parent[r] < 0 ? r : session[parent[r]];  /* parents come first */
+  }
+  free(h);
+  free(first);
+  return ORACLE_OK;
 }

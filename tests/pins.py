@@ -629,6 +629,89 @@ def check_coloc_no_last_resort(L):
     assert int(a["stick"][0]) == 0 and int(a["instance"][0]) != 1
 
 
+# ---------------------------------------------------------------------------
+# session reconstruction (Appendix A)
+# ---------------------------------------------------------------------------
+
+def _link(L, B, reqs, users, turns, seed=0):
+    from synth.traces import pack
+    tokens, offsets = pack(reqs)
+    return oracle.link_sessions(B, seed, tokens, offsets, users, turns, L)
+
+
+def check_link_against_token_prefixes(L):
+    """Brute force by token comparison: r follows the latest earlier p of the
+    same user and turn_r - 1 whose full blocks are the first tokens of r."""
+    rng = np.random.default_rng(60)
+    B = 2
+    for trial in range(30):
+        base = rng.integers(0, 3, size=12 * B, dtype=np.int32)
+        n = int(rng.integers(1, 25))
+        reqs = [_mutate(rng, base, int(rng.integers(0, 12 * B))) for _ in range(n)]
+        users = rng.integers(0, 3, size=n)
+        turns = rng.integers(0, 4, size=n)
+        parent, session = _link(L, B, reqs, users, turns)
+        want_session = []
+        for r in range(n):
+            want = -1
+            for q in range(r - 1, -1, -1):
+                nq = len(reqs[q]) // B
+                if users[q] != users[r] or turns[q] != turns[r] - 1 or nq > len(reqs[r]) // B:
+                    continue
+                if np.array_equal(reqs[q][:nq * B], reqs[r][:nq * B]):
+                    want = q
+                    break
+            assert parent[r] == want, (trial, r)
+            want_session.append(r if want < 0 else want_session[want])
+            assert session[r] == want_session[r], (trial, r)
+
+
+def check_link_recovers_generated_sessions(L):
+    """A multi-turn trace without truncation, one user per session: every
+    turn extends the previous one, so the chains are the generator's
+    sessions and each session's id is its first request."""
+    from synth import agent_trace
+    from synth.traces import pack
+    tr = agent_trace("c1_tiny", scale=0.25, seed=5)
+    bs = list(tr.batches())
+    reqs, sess, turns = [], [], []
+    for bt in bs:
+        for r in range(bt.n_requests):
+            reqs.append(bt.tokens[bt.offsets[r]:bt.offsets[r + 1]])
+        sess.extend(bt.sessions.tolist())
+        turns.extend(bt.turns.tolist())
+    sess, turns = np.array(sess), np.array(turns)
+    parent, session = _link(L, tr.params.block_size, reqs, sess, turns)
+    first = {}
+    for r, s_ in enumerate(sess):
+        first.setdefault(int(s_), r)
+    assert all(int(session[r]) == first[int(s_)] for r, s_ in enumerate(sess))
+    assert np.all((parent >= 0) == (turns > 0))
+
+
+def check_link_special_cases(L):
+    """Different users or a turn gap never link; the latest of two equal
+    parents wins; a prompt shorter than a block links as the empty prefix."""
+    rng = np.random.default_rng(61)
+    B = 4
+    a = rng.integers(0, 151936, size=8 * B, dtype=np.int32)
+    ext = np.concatenate([a, rng.integers(0, 151936, size=3 * B, dtype=np.int32)])
+    tiny = a[:B - 1]
+    reqs = [a, a, ext, ext, tiny, a]
+    users = [1, 1, 1, 2, 3, 3]
+    turns = [0, 0, 1, 1, 0, 1]
+    parent, session = _link(L, B, reqs, users, turns)
+    assert parent.tolist() == [-1, -1, 1, -1, -1, 4]
+    assert session.tolist() == [0, 1, 1, 3, 4, 4]
+    parent, _ = _link(L, B, [a, ext], [1, 1], [0, 2])  # turn gap
+    assert parent.tolist() == [-1, -1]
+    # a chain of four turns: every request's session is the first one
+    ext2 = np.concatenate([ext, rng.integers(0, 151936, size=2 * B, dtype=np.int32)])
+    ext3 = np.concatenate([ext2, rng.integers(0, 151936, size=5, dtype=np.int32)])
+    parent, session = _link(L, B, [a, ext, ext2, ext3], [7] * 4, [0, 1, 2, 3])
+    assert parent.tolist() == [-1, 0, 1, 2] and session.tolist() == [0, 0, 0, 0]
+
+
 ALL_CHECKS = [
     check_published_vector,
     check_bijection,
@@ -656,4 +739,7 @@ ALL_CHECKS = [
     check_coloc_tpot_filter,
     check_coloc_lmetric_product,
     check_coloc_no_last_resort,
+    check_link_against_token_prefixes,
+    check_link_recovers_generated_sessions,
+    check_link_special_cases,
 ]

@@ -63,6 +63,12 @@ MUTANTS = {
     "coloc_prev_not_checked": ("meets_prev && cand[prev];", "meets_prev;"),
     "coloc_sum_not_product": ("(unsigned __int128)(uint64_t)est2[i] * (uint64_t)num_requests[i];",
                               "(unsigned __int128)((uint64_t)est2[i] + (uint64_t)num_requests[i]);"),
+    "link_earliest_parent": ("for (int32_t p = r - 1; p >= 0; --p) {", "for (int32_t p = 0; p < r; ++p) {"),
+    "link_turn_ignored": ("|| (int64_t)turns[p] != (int64_t)turns[r] - 1) continue;", ") continue;"),
+    "link_user_ignored": ("if (users[p] != users[r] || ", "if ("),
+    "link_longer_parent": ("if (np > nr) continue;", ";"),
+    "link_session_is_parent": ("session[r] = parent[r] < 0 ? r : session[parent[r]];",
+                               "session[r] = parent[r] < 0 ? r : parent[r];"),
     "coloc_product_64_bit": ("(unsigned __int128)(uint64_t)est2[i] * (uint64_t)num_requests[i];",
                              "(unsigned __int128)((uint64_t)est2[i] * (uint64_t)num_requests[i]);"),
 }
