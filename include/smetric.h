@@ -250,6 +250,22 @@ int smetric_route_batch_policy_coloc(smetric_index* idx, const int32_t* d_tokens
                                      int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
                                      int64_t hashes_cap, smetric_stream_t stream);
 
+/* Session reconstruction from block hashes (Appendix A): in a batch of
+ * requests in arrival order, request r follows the latest earlier request p
+ * of the same user (d_users) with d_turns[p] = d_turns[r] - 1 whose
+ * block-hash sequence is a prefix of r's (equal and empty sequences
+ * included); d_parent[r] = p, or -1. d_session[r] = the first request of
+ * r's chain of parents. Hashes are the index's (its block size and seed);
+ * same token and offset rules as smetric_route_batch. Uses the index's
+ * route scratch (no route may run on the index concurrently). Invalid
+ * offsets latch INVALID_ARG and write -1 to both outputs. Prefixes are
+ * compared by the hash of p's last block, which decides as a full comparison
+ * does up to a 64-bit collision of the chain hash. */
+int smetric_link_sessions(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                          const int64_t* d_offsets, int32_t n_requests, const int64_t* d_users,
+                          const int32_t* d_turns, int32_t* d_parent, int32_t* d_session,
+                          smetric_stream_t stream);
+
 /* Flags of smetric_index_commit_batch. */
 #define SMETRIC_COMMIT_GLOBAL 1 /* also add every block to the global tier */
 

@@ -45,7 +45,7 @@ EXPORTED = (
     "smetric_route_batch_host", "smetric_status", "smetric_strerror",
     "smetric_profile_enable", "smetric_profile_read", "smetric_profile_kernel_name",
     "smetric_launch_count", "smetric_block_hashes_noalloc", "smetric_route_batch_policy",
-    "smetric_index_commit_batch", "smetric_route_batch_policy_coloc",
+    "smetric_index_commit_batch", "smetric_route_batch_policy_coloc", "smetric_link_sessions",
 )
 
 
@@ -108,6 +108,7 @@ def lib():
             "smetric_route_batch_policy": (C.c_int, [P, P, I64, P, I32, P, P, P, smetric_policy, P, P,
                                                      P, P, P, P, I64, P]),
             "smetric_index_commit_batch": (C.c_int, [P, P, I32, P, P, P, I32, P, P]),
+            "smetric_link_sessions": (C.c_int, [P, P, I64, P, I32, P, P, P, P, P]),
             "smetric_route_batch_policy_coloc": (C.c_int, [P, P, I64, P, I32, P, P, P, P, P, smetric_policy,
                                                            P, P, P, P, P, P, I64, P]),
             "smetric_block_hashes": (C.c_int, [P, P, I64, P, I32, P, P, I64, P]),
@@ -242,6 +243,13 @@ def smetric_route_batch_policy_coloc(idx: int, d_tokens, n_tokens: int, d_offset
         _ptr(d_num_requests), _ptr(d_turn), _ptr(d_est_hit), _policy(policy), _ptr(d_instance),
         _ptr(d_local_hit), _ptr(d_global_hit), _ptr(d_stick), _ptr(d_session_key), _ptr(d_block_hashes),
         hashes_cap, _stream(stream)), "smetric_route_batch_policy_coloc")
+
+
+def smetric_link_sessions(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int, d_users, d_turns,
+                          d_parent, d_session, stream=None) -> None:
+    _check(lib().smetric_link_sessions(idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests, _ptr(d_users),
+                                       _ptr(d_turns), _ptr(d_parent), _ptr(d_session), _stream(stream)),
+           "smetric_link_sessions")
 
 
 def smetric_index_commit_batch(idx: int, d_offsets, n_requests: int, d_instance, d_local_hit,
@@ -433,6 +441,16 @@ class SMetricIndex:
                                          out["global_hit"], out["stick"], out["session_key"], hb,
                                          hb.numel() if hb is not None else 0, stream)
         return out
+
+    def link_sessions(self, tokens, offsets, users, turns, stream=None):
+        """Session reconstruction (Appendix A): returns (parent, session), int32 per request."""
+        import torch
+        n = offsets.numel() - 1
+        parent = torch.empty(n, dtype=torch.int32, device=offsets.device)
+        session = torch.empty(n, dtype=torch.int32, device=offsets.device)
+        smetric_link_sessions(self.handle, tokens, tokens.numel(), offsets, n, users, turns, parent, session,
+                              stream)
+        return parent, session
 
     def commit_batch(self, offsets, out, also_global=False, load=None, stream=None):
         """Add the routed batch's blocks (`out` from route_batch(..., want_hashes=True)

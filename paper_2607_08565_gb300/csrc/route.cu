@@ -1157,6 +1157,107 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
 }
 
 // ---------------------------------------------------------------------------
+// session links
+// ---------------------------------------------------------------------------
+
+// Fingerprint of (user, turn, number of blocks, last block hash) for the
+// session-link table; 0 marks an empty slot.
+__device__ __forceinline__ uint64_t link_key(int64_t user, int64_t turn, int64_t nb, uint64_t last) {
+  uint64_t x = mix64((uint64_t)user ^ kGamma);
+  x = mix64(x ^ (uint64_t)turn);
+  x = mix64(x ^ (uint64_t)nb);
+  x = mix64(x ^ last);
+  return x ? x : 1;
+}
+
+// Thread per request p: (key, p) into the table (a multi-map: every request
+// takes its own slot), and parent[p] = -1.
+__global__ void __launch_bounds__(256)
+    k_link_insert(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
+                  const uint64_t* __restrict__ H, const int64_t* __restrict__ users,
+                  const int32_t* __restrict__ turns, uint64_t* __restrict__ table, uint64_t gmask,
+                  int32_t* __restrict__ parent) {
+  const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= n || !*batch_ok) return;
+  parent[p] = -1;
+  const int64_t bo = block_off[p], nb = block_off[p + 1] - bo;
+  const uint64_t key = link_key(users[p], turns[p], nb, nb ? H[bo + nb - 1] : 0);
+  uint64_t s = key & gmask;
+  for (uint64_t t = 0; t <= gmask; ++t) {
+    unsigned long long* const slot = reinterpret_cast<unsigned long long*>(table + 2 * s);
+    if (atomicCAS(slot, 0ull, (unsigned long long)key) == 0ull) {
+      slot[1] = (unsigned long long)p;
+      return;
+    }
+    s = (s + 1) & gmask;
+  }
+}
+
+// Thread per (request r, prefix length k <= n_r): the latest earlier request
+// of r's user, of turn turn_r - 1, with exactly k blocks, the last equal to
+// r's block k - 1, raises parent[r] to it. Candidates from the table are
+// checked field by field.
+__global__ void __launch_bounds__(256)
+    k_link_find(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
+                const uint64_t* __restrict__ H, const int64_t* __restrict__ users,
+                const int32_t* __restrict__ turns, const uint64_t* __restrict__ table, uint64_t gmask,
+                int32_t* __restrict__ parent) {
+  if (!*batch_ok) return;
+  const int64_t total = block_off[n] + n;  // sum over r of n_r + 1
+  int32_t r = 0;
+  for (int64_t f = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; f < total;
+       f += (int64_t)gridDim.x * blockDim.x) {
+    int32_t lo = r, hi = n;  // largest r with block_off[r] + r <= f
+    while (hi - lo > 1) {
+      const int32_t mid = (lo + hi) >> 1;
+      if (__ldg(block_off + mid) + mid <= f) lo = mid; else hi = mid;
+    }
+    r = lo;
+    const int64_t bo = __ldg(block_off + r), k = f - (bo + r);
+    const int64_t user = users[r], turn = (int64_t)turns[r] - 1;
+    const uint64_t last = k ? __ldg(H + bo + k - 1) : 0;
+    const uint64_t key = link_key(user, turn, k, last);
+    int32_t best = -1;
+    uint64_t s = key & gmask;
+    for (uint64_t t = 0; t <= gmask; ++t) {
+      const uint64_t kk = __ldg(table + 2 * s);
+      if (kk == 0) break;
+      if (kk == key) {
+        const int32_t p = (int32_t)__ldg(table + 2 * s + 1);
+        const int64_t pbo = __ldg(block_off + p);
+        if (p < r && p > best && users[p] == user && (int64_t)turns[p] == turn &&
+            __ldg(block_off + p + 1) - pbo == k && (k == 0 || __ldg(H + pbo + k - 1) == last))
+          best = p;
+      }
+      s = (s + 1) & gmask;
+    }
+    if (best >= 0) atomicMax(parent + r, best);
+  }
+}
+
+// One CTA: session[r] = the head of r's chain of parents (pointer jumping;
+// parents are earlier requests, so every chain ends), then the link table
+// emptied for the next route.
+__global__ void __launch_bounds__(1024)
+    k_link_heads(int32_t n, const int32_t* __restrict__ batch_ok, int32_t* __restrict__ parent,
+                 int32_t* __restrict__ session, uint4* __restrict__ table, int64_t table_vecs) {
+  if (*batch_ok) {
+    for (int32_t r = threadIdx.x; r < n; r += blockDim.x) session[r] = parent[r] < 0 ? r : parent[r];
+    __syncthreads();
+    for (int64_t span = 1; span < n; span <<= 1) {
+      for (int32_t r = threadIdx.x; r < n; r += blockDim.x) {
+        const int32_t a = session[r];
+        session[r] = session[a];  // an ancestor either way: the heads are reached all the same
+      }
+      __syncthreads();
+    }
+  } else {  // invalid offsets: no links
+    for (int32_t r = threadIdx.x; r < n; r += blockDim.x) { parent[r] = -1; session[r] = -1; }
+  }
+  for (int64_t i = threadIdx.x; i < table_vecs; i += blockDim.x) table[i] = make_uint4(0, 0, 0, 0);
+}
+
+// ---------------------------------------------------------------------------
 // commit
 // ---------------------------------------------------------------------------
 
@@ -1604,6 +1705,35 @@ int smetric_index_commit_batch(smetric_index* idx, const int64_t* d_offsets, int
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   return launch_commit(idx, d_instance, d_block_hashes, n_requests, c.max_batch_tokens / c.block_size,
                        (flags & SMETRIC_COMMIT_GLOBAL) != 0, s);
+}
+
+int smetric_link_sessions(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                          const int64_t* d_offsets, int32_t n_requests, const int64_t* d_users,
+                          const int32_t* d_turns, int32_t* d_parent, int32_t* d_session,
+                          smetric_stream_t stream) {
+  int rc = check_device(idx);
+  if (rc) return rc;
+  if (n_requests < 0 || n_requests > idx->cfg.max_batch_requests) return SMETRIC_ERR_INVALID_ARG;
+  if (n_requests == 0) return SMETRIC_OK;
+  if (!d_users || !d_turns || !d_parent || !d_session) return SMETRIC_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // block hashes of the batch into the index's scratch
+  if ((rc = route_common<false>(idx, d_tokens, n_tokens, d_offsets, n_requests, nullptr, smetric_weights{0, 0, 0},
+                                nullptr, nullptr, nullptr, idx->sk_tmp, idx->hashes,
+                                n_tokens / idx->cfg.block_size, s)))
+    return rc;
+  const uint64_t gmask = group_slots_for(n_requests) - 1;
+  const unsigned g = (unsigned)((n_requests + 255) / 256);
+  k_link_insert<<<g, 256, 0, s>>>(idx->block_off, n_requests, idx->batch_ok, idx->hashes, d_users, d_turns,
+                                  idx->groups, gmask, d_parent);
+  const int64_t want = (n_tokens / idx->cfg.block_size + n_requests + 255) / 256;
+  const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
+  k_link_find<<<grid, 256, 0, s>>>(idx->block_off, n_requests, idx->batch_ok, idx->hashes, d_users, d_turns,
+                                   idx->groups, gmask, d_parent);
+  k_link_heads<<<1, 1024, 0, s>>>(n_requests, idx->batch_ok, d_parent, d_session,
+                                  reinterpret_cast<uint4*>(idx->groups), (int64_t)(gmask + 1));
+  idx->launches += 3;
+  return cuda_status(cudaGetLastError());
 }
 
 int smetric_block_hashes(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
