@@ -59,6 +59,8 @@ def parse():
     ap.add_argument("--commit", action="store_true",
                     help="time device-side index maintenance (route, then commit the batch's blocks "
                          "and drain the queues) over a config-2 replay (one GPU; its own JSON line)")
+    ap.add_argument("--link", action="store_true",
+                    help="time session reconstruction (Appendix A) over a config-3 trace (one GPU; its own line)")
     ap.add_argument("--coloc", action="store_true",
                     help="with --policy: the PD-colocation variant (Appendix B)")
     ap.add_argument("--policy", action="store_true",
@@ -738,6 +740,64 @@ def run_policy(args):
 
 
 # ---------------------------------------------------------------------------
+# session reconstruction over a config-3 trace
+# ---------------------------------------------------------------------------
+
+def run_link(args, scale=0.5):
+    import torch
+    import oracle
+    import paper_2607_08565_gb300 as pkg
+    from paper_2607_08565_gb300 import build_lib
+    from synth import agent_trace
+    from synth.traces import pack
+
+    build_lib.build()
+    torch.cuda.set_device(0)
+    tr = agent_trace("c3_long", scale=scale, seed=7)
+    p = tr.params
+    reqs, users, turns = [], [], []
+    for bt in tr.batches():
+        for r in range(bt.n_requests):
+            reqs.append(bt.tokens[bt.offsets[r]:bt.offsets[r + 1]])
+        users.extend(bt.sessions.tolist())
+        turns.extend(bt.turns.tolist())
+    tok, off = pack(reqs)
+    n = len(reqs)
+    ix = pkg.SMetricIndex(p.num_instances, p.block_size, p.session_blocks, capacity_slots=1 << 16,
+                          max_batch_requests=n, max_batch_tokens=len(tok), hash_seed=p.hash_seed)
+    d = [torch.from_numpy(np.ascontiguousarray(a)).cuda() for a in (tok, off, np.array(users, np.int64),
+                                                                    np.array(turns, np.int32))]
+    for _ in range(3):
+        parent, session = ix.link_sessions(*d)
+    torch.cuda.synchronize()
+    ix.check()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    steps = 20
+    e0.record()
+    for _ in range(steps):
+        ix.link_sessions(*d)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    m = min(n, 4096)  # the oracle compares every earlier request: the first two turn waves
+    t0 = time.perf_counter()
+    op, _ = oracle.link_sessions(p.block_size, p.hash_seed, tok[:off[m]], off[:m + 1], users[:m], turns[:m])
+    dt = time.perf_counter() - t0
+    if not np.array_equal(op, parent.cpu().numpy()[:m]):
+        raise RuntimeError("session links differ from the oracle")
+    line = {"metric": "requests linked into sessions per second (Appendix A)", "value": n / (ms / 1e3),
+            "unit": "requests/s", "n_gpus": 1, "steps": steps, "warmup": 3, "ms_per_step": ms,
+            "higher_is_better": True, "data": "synthetic",
+            "config": {"workload": f"c3_long agent trace at scale {scale}: {n} requests, {len(tok)} tokens, "
+                                   f"B = {p.block_size}, one call", "sessions": int(len(set(users))),
+                       "chains": int((parent.cpu().numpy() < 0).sum())},
+            "cpu_baseline": {"value": m / dt, "unit": "requests/s", "cores": 1, "kind": "oracle",
+                             "sample": f"first {m} requests ({dt:.1f} s, one thread)"}}
+    print(json.dumps(line), flush=True)
+    ix.close()
+
+
+# ---------------------------------------------------------------------------
 # device-side index maintenance over a config-2 replay
 # ---------------------------------------------------------------------------
 
@@ -912,6 +972,9 @@ def main():
         return
     if args.commit:
         run_commit(args)
+        return
+    if args.link:
+        run_link(args)
         return
     rank, world, local, dist = dist_setup(args)
     if args.impl == "reference":
