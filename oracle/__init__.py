@@ -68,6 +68,10 @@ def load_library(path: str):
         C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p, i64p, i64p, i32p, i64p,
         C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_int32,
         i32p, i32p, i32p, i32p, u64p]
+    L.oracle_route_batch_baseline.restype = C.c_int
+    L.oracle_route_batch_baseline.argtypes = [
+        C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, C.c_int32, i64p, i64p,
+        C.c_int64, C.c_int64, i32p, i32p, i32p, u64p]
     L.oracle_link_sessions.restype = C.c_int
     L.oracle_link_sessions.argtypes = [C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p, i32p, i32p, i32p]
     return L
@@ -235,3 +239,24 @@ class OracleIndex:
         inst, lh, gh, st = outs
         return dict(instance=inst[:n], local_hit=lh[:n], global_hit=gh[:n], stick=st[:n],
                     session_key=sk[:n])
+
+    def route_batch_baseline(self, block_size: int, session_blocks: int, seed: int, tokens, offsets,
+                             scorer: int, queued, batch, lam_num: int = 1, lam_den: int = 2):
+        """Baseline scorers of Section 5.1: scorer 1 = Bailian, 2 = LMetric.
+        Returns dict(instance, local_hit, global_hit, session_key)."""
+        t = np.ascontiguousarray(tokens, dtype=np.int32)
+        o = np.ascontiguousarray(offsets, dtype=np.int64)
+        n = len(o) - 1
+        q = np.ascontiguousarray(queued, dtype=np.int64)
+        b = np.ascontiguousarray(batch, dtype=np.int64)
+        if len(q) != self.N or len(b) != self.N:
+            raise ValueError("queued and batch have one entry per instance")
+        outs = [np.zeros(max(n, 1), np.int32) for _ in range(3)]
+        sk = np.zeros(max(n, 1), np.uint64)
+        rc = self._L.oracle_route_batch_baseline(
+            self._h, block_size, session_blocks, seed & 0xFFFFFFFFFFFFFFFF,
+            t if len(t) else np.zeros(1, np.int32), o, n, scorer, q, b, lam_num, lam_den, *outs, sk)
+        if rc != 0:
+            raise ValueError(f"oracle_route_batch_baseline: {rc}")
+        inst, lh, gh = outs
+        return dict(instance=inst[:n], local_hit=lh[:n], global_hit=gh[:n], session_key=sk[:n])

@@ -84,6 +84,15 @@
  *              runs (LMetric's multiplicative score), compared exactly in
  *              128 bits.
  *
+ * Baseline scorers of Section 5.1 (oracle_route_batch_baseline), argmin with
+ * ties to the lowest id over the same c_i:
+ *    Bailian: f_i = (1 - LAMBDA) * l_i / max_j l_j + LAMBDA * (1 - B*c_i / L_r)
+ *             (l_i instance i's batch size; the load term is 0 when every
+ *             l_j is 0 and the hit ratio is 0 for an empty prompt);
+ *             LAMBDA = LAM_NUM / LAM_DEN; compared exactly on f_i times
+ *             LAM_DEN * max_j l_j * L_r in 128 bits.
+ *    LMetric: f_i = (q_i + L_r - B*c_i) * l_i (q_i the queued prefill tokens).
+ *
  * Session reconstruction (Appendix A; oracle_link_sessions): request r
  * follows request p when p is earlier (p < r, requests in arrival order), of
  * the same user, of turn turn_r - 1, and p's block-hash sequence is a prefix
@@ -544,4 +553,72 @@ int oracle_link_sessions(int32_t B, uint64_t seed, const int32_t* tokens, const 
   free(h);
   free(first);
   return ORACLE_OK;
+}
+
+/* Baseline scorers (Section 5.1): scorer 1 = Bailian's weighted sum of the
+ * normalised batch size and miss ratio, 2 = LMetric's product. Limits:
+ * 0 <= l_i <= 2^20, 0 <= q_i <= 2^40, 0 <= LAM_NUM <= LAM_DEN <= 2^20,
+ * LAM_DEN >= 1, L_r < 2^31. */
+int oracle_route_batch_baseline(const oracle_index* x, int32_t B, int32_t S, uint64_t seed,
+                                const int32_t* tokens, const int64_t* offsets, int32_t n_requests,
+                                int32_t scorer, const int64_t* queued, const int64_t* batch, int64_t lam_num,
+                                int64_t lam_den, int32_t* instance, int32_t* local_hit, int32_t* global_hit,
+                                uint64_t* session_key) {
+  if (!x || B < 2 || (B % 2) != 0 || S < 1 || n_requests < 0 || (scorer != 1 && scorer != 2))
+    return ORACLE_ERR_INVALID_ARG;
+  const int32_t N = x->N;
+  if (lam_den < 1 || lam_den > (1LL << 20) || lam_num < 0 || lam_num > lam_den) return ORACLE_ERR_INVALID_ARG;
+  int64_t lmax = 0;
+  for (int32_t i = 0; i < N; ++i) {
+    if (batch[i] < 0 || batch[i] > (1LL << 20) || queued[i] < 0 || queued[i] > (1LL << 40))
+      return ORACLE_ERR_INVALID_ARG;
+    if (batch[i] > lmax) lmax = batch[i];
+  }
+  for (int32_t r = 0; r < n_requests; ++r)
+    if (offsets[r + 1] < offsets[r] || offsets[r] < 0 || offsets[r + 1] - offsets[r] >= (1LL << 31))
+      return ORACLE_ERR_INVALID_ARG;
+  int64_t* c = (int64_t*)malloc((size_t)N * sizeof(int64_t));
+  uint64_t* h = NULL;
+  int64_t cap = 0;
+  int rc = c ? ORACLE_OK : ORACLE_ERR_OOM;
+  for (int32_t r = 0; r < n_requests && rc == ORACLE_OK; ++r) {
+    const int64_t L = offsets[r + 1] - offsets[r];
+    const int64_t n = L / B;
+    if (n + 1 > cap) {
+      free(h);
+      cap = n + 1;
+      h = (uint64_t*)malloc((size_t)cap * sizeof(uint64_t));
+      if (!h) { rc = ORACLE_ERR_OOM; break; }
+    }
+    oracle_block_hashes(tokens + offsets[r], L, B, seed, h);
+    int64_t g;
+    oracle_prefix_hits(x, h, n, c, &g);
+    int32_t best = -1;
+    unsigned __int128 best_f = 0;
+    for (int32_t i = 0; i < N; ++i) {
+      unsigned __int128 f;
+      if (scorer == 2) {
+        f = (unsigned __int128)(uint64_t)(queued[i] + L - (int64_t)B * c[i]) * (uint64_t)batch[i];
+      } else {
+        /* f_i * LAM_DEN * lmax * L, with the load term dropped when lmax = 0
+         * and the miss ratio taken as 1 when L = 0 */
+        const uint64_t miss = (uint64_t)(L - (int64_t)B * c[i]);
+        const uint64_t Lm = (uint64_t)(lmax > 0 ? lmax : 1), Lr = (uint64_t)(L > 0 ? L : 1);
+        const unsigned __int128 load_term =
+            lmax > 0 ? (unsigned __int128)(uint64_t)((lam_den - lam_num) * batch[i]) * Lr : 0;
+        const unsigned __int128 miss_term =
+            (unsigned __int128)(uint64_t)lam_num * (L > 0 ? miss : 1) * Lm;
+        f = load_term + miss_term;
+      }
+      if (best < 0 || f < best_f) { best = i; best_f = f; }
+    }
+    const int64_t gb = c[best] > g ? c[best] : g;
+    instance[r] = best;
+    local_hit[r] = (int32_t)((int64_t)B * c[best]);
+    global_hit[r] = (int32_t)((int64_t)B * (gb - c[best]));
+    session_key[r] = n == 0 ? 0 : h[(n < S ? n : S) - 1];
+  }
+  free(h);
+  free(c);
+  return rc;
 }

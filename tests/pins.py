@@ -712,6 +712,74 @@ def check_link_special_cases(L):
     assert parent.tolist() == [-1, 0, 1, 2] and session.tolist() == [0, 0, 0, 0]
 
 
+# ---------------------------------------------------------------------------
+# baseline scorers (Section 5.1)
+# ---------------------------------------------------------------------------
+
+def _baseline(ix, B, reqs, scorer, queued, batch, lam=(1, 2)):
+    from synth.traces import pack
+    tokens, offsets = pack(reqs)
+    return ix.route_batch_baseline(B, 1, 0, tokens, offsets, scorer, np.asarray(queued, np.int64),
+                                   np.asarray(batch, np.int64), *lam)
+
+
+def _bailian_f(l, lmax, hit_tokens, Lp, lam):
+    """Section 5.1's weighted sum, exactly: (1 - lambda) * l / max l +
+    lambda * (1 - hit ratio)."""
+    lh = Fraction(l, lmax) if lmax else Fraction(0)
+    ch = Fraction(hit_tokens, Lp) if Lp else Fraction(0)
+    return (1 - lam) * lh + lam * (1 - ch)
+
+
+def check_baselines_against_their_definitions(L):
+    """Bailian's normalised weighted sum and LMetric's product, evaluated in
+    exact rationals from hits found by token comparison, against the
+    oracle's choice (ties to the lowest id)."""
+    rng = np.random.default_rng(70)
+    B = 2
+    for trial in range(60):
+        N = int(rng.integers(1, 7))
+        base = rng.integers(0, 3, size=10 * B, dtype=np.int32)
+        stored = {i: [_mutate(rng, base, int(rng.integers(0, 11 * B)))
+                      for _ in range(int(rng.integers(0, 3)))] for i in range(N)}
+        ix = oracle.OracleIndex(N, L)
+        for i, ps in stored.items():
+            for p_ in ps:
+                ix.insert(oracle.block_hashes(p_, B, 0, L), i)
+        req = _mutate(rng, base, int(rng.integers(0, 11 * B)))
+        c = [brute_hit(req, stored[i], B) for i in range(N)]
+        Lp = len(req)
+        batch = rng.integers(0, [1, 4, 50][trial % 3], size=N)
+        q = rng.integers(0, 40, size=N)
+        lam = (int(rng.integers(0, 7)), 6)
+        f = [_bailian_f(int(batch[i]), int(batch.max()), B * c[i], Lp, Fraction(*lam)) for i in range(N)]
+        out = _baseline(ix, B, [req], 1, q, batch, lam)
+        assert int(out["instance"][0]) == min(range(N), key=lambda i: (f[i], i)), (trial, f)
+        g = [(int(q[i]) + Lp - B * c[i]) * int(batch[i]) for i in range(N)]
+        out = _baseline(ix, B, [req], 2, q, batch)
+        assert int(out["instance"][0]) == min(range(N), key=lambda i: (g[i], i)), (trial, g)
+
+
+def check_baselines_special_cases(L):
+    """Bailian with lambda = 0 is join-the-shortest-batch; with lambda = 1 it
+    is the longest local hit; scaling every batch size leaves it unchanged.
+    LMetric sends work to an idle instance (no requests) first."""
+    rng = np.random.default_rng(71)
+    B = 4
+    t = rng.integers(0, 151936, size=60, dtype=np.int32)
+    ix = oracle.OracleIndex(4, L)
+    _held(L, ix, t, B, {2: 9, 3: 4})
+    batch = np.array([5, 3, 9, 3])
+    assert int(_baseline(ix, B, [t], 1, [0] * 4, batch, (0, 5))["instance"][0]) == 1
+    assert int(_baseline(ix, B, [t], 1, [0] * 4, batch, (5, 5))["instance"][0]) == 2
+    for lam in ((1, 3), (2, 3), (7, 10)):
+        a = _baseline(ix, B, [t], 1, [0] * 4, batch, lam)["instance"][0]
+        b = _baseline(ix, B, [t], 1, [0] * 4, batch * 1000, lam)["instance"][0]
+        assert a == b
+    out = _baseline(ix, B, [t], 2, [10 ** 9, 0, 0, 0], [0, 3, 1, 2])
+    assert int(out["instance"][0]) == 0
+
+
 ALL_CHECKS = [
     check_published_vector,
     check_bijection,
@@ -742,4 +810,6 @@ ALL_CHECKS = [
     check_link_against_token_prefixes,
     check_link_recovers_generated_sessions,
     check_link_special_cases,
+    check_baselines_against_their_definitions,
+    check_baselines_special_cases,
 ]

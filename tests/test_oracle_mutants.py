@@ -69,6 +69,17 @@ MUTANTS = {
     "link_longer_parent": ("if (np > nr) continue;", ";"),
     "link_session_is_parent": ("session[r] = parent[r] < 0 ? r : session[parent[r]];",
                                "session[r] = parent[r] < 0 ? r : parent[r];"),
+    "bailian_no_normalisation": ("(unsigned __int128)(uint64_t)((lam_den - lam_num) * batch[i]) * Lr : 0;",
+                                 "(unsigned __int128)(uint64_t)((lam_den - lam_num) * batch[i]) * Lr * Lm : 0;"),
+    "bailian_weights_swapped": ("(unsigned __int128)(uint64_t)((lam_den - lam_num) * batch[i]) * Lr : 0;",
+                                "(unsigned __int128)(uint64_t)(lam_num * batch[i]) * Lr : 0;"),
+    "bailian_hit_for_miss": ("(unsigned __int128)(uint64_t)lam_num * (L > 0 ? miss : 1) * Lm;",
+                             "(unsigned __int128)(uint64_t)lam_num * (L > 0 ? (uint64_t)L - miss : 1) * Lm;"),
+    "lmetric_sum": ("(unsigned __int128)(uint64_t)(queued[i] + L - (int64_t)B * c[i]) * (uint64_t)batch[i];",
+                    "(unsigned __int128)(uint64_t)(queued[i] + L - (int64_t)B * c[i]) + (uint64_t)batch[i];"),
+    "lmetric_drops_queue": ("(uint64_t)(queued[i] + L - (int64_t)B * c[i])", "(uint64_t)(L - (int64_t)B * c[i])"),
+    "baseline_tie_to_highest": ("if (best < 0 || f < best_f) { best = i; best_f = f; }",
+                                "if (best < 0 || f <= best_f) { best = i; best_f = f; }"),
     "coloc_product_64_bit": ("(unsigned __int128)(uint64_t)est2[i] * (uint64_t)num_requests[i];",
                              "(unsigned __int128)((uint64_t)est2[i] * (uint64_t)num_requests[i]);"),
 }
