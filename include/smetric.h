@@ -266,6 +266,28 @@ int smetric_link_sessions(smetric_index* idx, const int32_t* d_tokens, int64_t n
                           const int32_t* d_turns, int32_t* d_parent, int32_t* d_session,
                           smetric_stream_t stream);
 
+/* Baseline scorers of Section 5.1 as the routing decision (argmin over the
+ * same local hits c_i, ties to the lowest id). */
+#define SMETRIC_SCORER_BAILIAN 1 /* (1-lambda)*l_i/max_j l_j + lambda*(1 - B*c_i/L) */
+#define SMETRIC_SCORER_LMETRIC 2 /* (q_i + L - B*c_i) * l_i */
+
+/*   d_queued  int64 [N], each in [0, SMETRIC_MAX_LOAD]: queued prefill tokens
+ *             q_i (LMetric; unused by Bailian's score but still checked).
+ *   d_batch   int64 [N], each in [0, SMETRIC_POLICY_MAX_REQUESTS]: batch
+ *             sizes l_i. Bailian normalises them by their maximum (the load
+ *             term is 0 when every l_j is 0) and takes the hit ratio as 0 for
+ *             an empty prompt; lambda = lam_num / lam_den,
+ *             0 <= lam_num <= lam_den, 1 <= lam_den <= 2^20. Scores are
+ *             compared exactly (128-bit integers).
+ * Outputs as smetric_route_batch. Out-of-range parameters return
+ * INVALID_ARG; out-of-range queues or batch sizes latch OVERFLOW. */
+int smetric_route_batch_baseline(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                                 const int64_t* d_offsets, int32_t n_requests, int32_t scorer,
+                                 const int64_t* d_queued, const int64_t* d_batch, int64_t lam_num,
+                                 int64_t lam_den, int32_t* d_instance, int32_t* d_local_hit,
+                                 int32_t* d_global_hit, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                                 int64_t hashes_cap, smetric_stream_t stream);
+
 /* Flags of smetric_index_commit_batch. */
 #define SMETRIC_COMMIT_GLOBAL 1 /* also add every block to the global tier */
 

@@ -37,6 +37,8 @@ SMETRIC_POLICY_MAX_QUEUED = 1 << 59
 SMETRIC_COMMIT_GLOBAL = 1
 SMETRIC_POLICY_MAX_TPOT = 1 << 60
 SMETRIC_POLICY_MAX_REQUESTS = 1 << 20
+SMETRIC_SCORER_BAILIAN = 1
+SMETRIC_SCORER_LMETRIC = 2
 
 EXPORTED = (
     "smetric_index_create", "smetric_index_destroy", "smetric_index_clear",
@@ -46,6 +48,7 @@ EXPORTED = (
     "smetric_profile_enable", "smetric_profile_read", "smetric_profile_kernel_name",
     "smetric_launch_count", "smetric_block_hashes_noalloc", "smetric_route_batch_policy",
     "smetric_index_commit_batch", "smetric_route_batch_policy_coloc", "smetric_link_sessions",
+    "smetric_route_batch_baseline",
 )
 
 
@@ -109,6 +112,8 @@ def lib():
                                                      P, P, P, P, I64, P]),
             "smetric_index_commit_batch": (C.c_int, [P, P, I32, P, P, P, I32, P, P]),
             "smetric_link_sessions": (C.c_int, [P, P, I64, P, I32, P, P, P, P, P]),
+            "smetric_route_batch_baseline": (C.c_int, [P, P, I64, P, I32, I32, P, P, I64, I64, P, P, P, P, P,
+                                                       I64, P]),
             "smetric_route_batch_policy_coloc": (C.c_int, [P, P, I64, P, I32, P, P, P, P, P, smetric_policy,
                                                            P, P, P, P, P, P, I64, P]),
             "smetric_block_hashes": (C.c_int, [P, P, I64, P, I32, P, P, I64, P]),
@@ -243,6 +248,16 @@ def smetric_route_batch_policy_coloc(idx: int, d_tokens, n_tokens: int, d_offset
         _ptr(d_num_requests), _ptr(d_turn), _ptr(d_est_hit), _policy(policy), _ptr(d_instance),
         _ptr(d_local_hit), _ptr(d_global_hit), _ptr(d_stick), _ptr(d_session_key), _ptr(d_block_hashes),
         hashes_cap, _stream(stream)), "smetric_route_batch_policy_coloc")
+
+
+def smetric_route_batch_baseline(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int, scorer: int,
+                                 d_queued, d_batch, lam_num: int, lam_den: int, d_instance, d_local_hit,
+                                 d_global_hit, d_session_key, d_block_hashes=None, hashes_cap: int = 0,
+                                 stream=None) -> None:
+    _check(lib().smetric_route_batch_baseline(
+        idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests, scorer, _ptr(d_queued), _ptr(d_batch),
+        lam_num, lam_den, _ptr(d_instance), _ptr(d_local_hit), _ptr(d_global_hit), _ptr(d_session_key),
+        _ptr(d_block_hashes), hashes_cap, _stream(stream)), "smetric_route_batch_baseline")
 
 
 def smetric_link_sessions(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int, d_users, d_turns,
@@ -440,6 +455,21 @@ class SMetricIndex:
                                          num_requests, turn, est_hit, policy, out["instance"], out["local_hit"],
                                          out["global_hit"], out["stick"], out["session_key"], hb,
                                          hb.numel() if hb is not None else 0, stream)
+        return out
+
+    def route_batch_baseline(self, tokens, offsets, scorer, queued, batch, lam=(1, 2), stream=None):
+        """A baseline scorer of Section 5.1 (SMETRIC_SCORER_BAILIAN or _LMETRIC).
+        Returns dict(instance, local_hit, global_hit, session_key)."""
+        import torch
+        n = offsets.numel() - 1
+        dev = offsets.device
+        out = dict(instance=torch.empty(n, dtype=torch.int32, device=dev),
+                   local_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                   global_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                   session_key=torch.empty(n, dtype=torch.uint64, device=dev))
+        smetric_route_batch_baseline(self.handle, tokens, tokens.numel(), offsets, n, scorer, queued, batch,
+                                     lam[0], lam[1], out["instance"], out["local_hit"], out["global_hit"],
+                                     out["session_key"], None, 0, stream)
         return out
 
     def link_sessions(self, tokens, offsets, users, turns, stream=None):

@@ -824,7 +824,7 @@ __global__ void __launch_bounds__(256)
 
 // The session-centric policy (Figure 10) as the walk's decision; off for
 // the argmin cost of smetric_route_batch.
-enum Decide { kArgmin = 0, kSession = 1, kColoc = 2 };
+enum Decide { kArgmin = 0, kSession = 1, kColoc = 2, kBailian = 3, kLMetric = 4 };
 
 struct WalkPolicy {
   int on;    // a Decide value; 0 = the argmin cost
@@ -834,7 +834,8 @@ struct WalkPolicy {
   const int64_t* est_hit;
   int32_t* stick;
   const int64_t* tpot;  // colocation: prefill cost each instance's live decodes absorb
-  const int64_t* nreq;  // colocation: requests each instance runs
+  const int64_t* nreq;  // colocation: requests each instance runs; baselines: batch sizes
+  int64_t lam_num, lam_den;  // Bailian's weight
 };
 
 // One warp per request, lanes = 32 consecutive blocks. The masks are
@@ -884,7 +885,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
     for (int64_t r = (int64_t)blockIdx.x * kMatchWarps + warp; r < n; r += tw)
       if (lane == 0) {
         inst_out[r] = -1; lhit_out[r] = 0; ghit_out[r] = 0;
-        if (DECIDE != kArgmin) pol.stick[r] = 0;
+        if (DECIDE == kSession || DECIDE == kColoc) pol.stick[r] = 0;
       }
   // k_group's lists: leaders from the front of `order`, members from the back
   const int64_t count = !ok ? 0 : MEMBERS ? counts[1] : counts[0];
@@ -1036,8 +1037,14 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
     auto less128 = [](uint64_t h1, uint64_t l1, int32_t r1, uint64_t h2, uint64_t l2, int32_t r2) {
       return h1 < h2 || (h1 == h2 && (l1 < l2 || (l1 == l2 && r1 < r2)));
     };
-    const int32_t s0 = DECIDE != kArgmin ? (int32_t)(((int64_t)pol.rr_base + r) % N) : 0;
-    const int64_t budget2 = DECIDE != kArgmin ? 2 * (pol.d0 + pol.d1 * L) : 0;
+    int64_t lmax = 0;  // Bailian: the largest batch size
+    if (DECIDE == kBailian) {
+      for (int i = lane; i < N; i += 32) lmax = max(lmax, __ldg(pol.nreq + i));
+#pragma unroll
+      for (int dd = 16; dd > 0; dd >>= 1) lmax = max(lmax, __shfl_xor_sync(kFull, lmax, dd));
+    }
+    const int32_t s0 = DECIDE == kSession || DECIDE == kColoc ? (int32_t)(((int64_t)pol.rr_base + r) % N) : 0;
+    const int64_t budget2 = DECIDE == kSession || DECIDE == kColoc ? 2 * (pol.d0 + pol.d1 * L) : 0;
     int32_t* const out_c = summ + r * (N + 1);
 #pragma unroll
     for (int t = 0; t < CT; ++t) {
@@ -1060,6 +1067,18 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
         const int64_t gi = ci > g ? ci : g;
         const int64_t cost = w_load * load_s[i] + w_miss * (L - B * gi) + w_glob * B * (gi - ci);
         if (cost < best_cost) { best_cost = cost; best = i; best_c = ci; }
+      } else if (DECIDE == kLMetric) {
+        // (q_i + L - B c_i) * l_i, below 2^61
+        const int64_t f = (load_s[i] + L - B * ci) * __ldg(pol.nreq + i);
+        if (less128(0, (uint64_t)f, i, ahi, alo, arot)) { ahi = 0; alo = (uint64_t)f; arot = i; ac = ci; }
+      } else if (DECIDE == kBailian) {
+        // f_i * LAM_DEN * max l * L = (LAM_DEN - LAM_NUM) l_i L + LAM_NUM (L - B c_i) max l, in 128 bits
+        const uint64_t Lm = lmax > 0 ? (uint64_t)lmax : 1, Lr = L > 0 ? (uint64_t)L : 1;
+        const uint64_t a1 = lmax > 0 ? (uint64_t)((pol.lam_den - pol.lam_num) * __ldg(pol.nreq + i)) : 0;
+        const uint64_t a2 = (uint64_t)pol.lam_num * (L > 0 ? (uint64_t)(L - B * ci) : 1);
+        const uint64_t l1 = a1 * Lr, h1 = __umul64hi(a1, Lr), l2 = a2 * Lm, h2 = __umul64hi(a2, Lm);
+        const uint64_t lo = l1 + l2, hi = h1 + h2 + (lo < l1 ? 1 : 0);
+        if (less128(hi, lo, i, ahi, alo, arot)) { ahi = hi; alo = lo; arot = i; ac = ci; }
       } else {
         // Eq. 1 doubled: 2*c_lin*n + c_att*n*(2L - n), n = new tokens, plus 2*q_i
         const int64_t nn = L - B * ci;
@@ -1081,7 +1100,21 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
       }
     }
     if (!MEMBERS && lane == 0) out_c[N] = (int32_t)g;
-    if (DECIDE == kArgmin) {
+    if (DECIDE == kBailian || DECIDE == kLMetric) {
+#pragma unroll
+      for (int dd = 16; dd > 0; dd >>= 1) {
+        const uint64_t oh = __shfl_xor_sync(kFull, ahi, dd), ol = __shfl_xor_sync(kFull, alo, dd);
+        const int32_t oi = __shfl_xor_sync(kFull, arot, dd);
+        const int64_t oc2 = __shfl_xor_sync(kFull, ac, dd);
+        if (less128(oh, ol, oi, ahi, alo, arot)) { ahi = oh; alo = ol; arot = oi; ac = oc2; }
+      }
+      if (lane == 0) {
+        const int64_t gb = ac > g ? ac : g;
+        inst_out[r] = arot;
+        lhit_out[r] = (int32_t)(B * ac);
+        ghit_out[r] = (int32_t)(B * (gb - ac));
+      }
+    } else if (DECIDE == kArgmin) {
 #pragma unroll
       for (int dd = 16; dd > 0; dd >>= 1) {
         const int64_t oc = __shfl_xor_sync(kFull, best_cost, dd);
@@ -1508,9 +1541,11 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
   // leaders, then members (which read the leaders' run ends)
   using WalkKernel = decltype(&k_walk<W, false, kArgmin>);  // every instantiation has this signature
-  const WalkKernel kerns[2] = {
-      pol.on == kColoc ? k_walk<W, false, kColoc> : pol.on == kSession ? k_walk<W, false, kSession> : k_walk<W, false, kArgmin>,
-      pol.on == kColoc ? k_walk<W, true, kColoc> : pol.on == kSession ? k_walk<W, true, kSession> : k_walk<W, true, kArgmin>};
+  const WalkKernel leaders[5] = {k_walk<W, false, kArgmin>, k_walk<W, false, kSession>, k_walk<W, false, kColoc>,
+                                 k_walk<W, false, kBailian>, k_walk<W, false, kLMetric>};
+  const WalkKernel members[5] = {k_walk<W, true, kArgmin>, k_walk<W, true, kSession>, k_walk<W, true, kColoc>,
+                                 k_walk<W, true, kBailian>, k_walk<W, true, kLMetric>};
+  const WalkKernel kerns[2] = {leaders[pol.on], members[pol.on]};
   for (const WalkKernel kern : kerns) {
     if (smem > 48 * 1024 &&
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
@@ -1580,10 +1615,12 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
   if (!PROBE && !hashes) return SMETRIC_ERR_INVALID_ARG;
 
   profile_begin(idx, s);
+  // the policies' Eq. 1 arithmetic has its own limits on queues and lengths
+  const bool eq1 = pol && (pol->on == kSession || pol->on == kColoc);
   k_prep<<<1, 1024, 0, s>>>(d_offsets, n, n_tokens, c.block_size, d_load, PROBE ? c.num_instances : 0,
                             idx->block_off, idx->chunk_off, idx->batch_ok, idx->status,
-                            pol ? SMETRIC_POLICY_MAX_QUEUED : SMETRIC_MAX_LOAD,
-                            pol ? SMETRIC_POLICY_MAX_LEN : (int64_t)INT32_MAX, pol ? pol->est_hit : nullptr,
+                            eq1 ? SMETRIC_POLICY_MAX_QUEUED : SMETRIC_MAX_LOAD,
+                            eq1 ? SMETRIC_POLICY_MAX_LEN : (int64_t)INT32_MAX, pol ? pol->est_hit : nullptr,
                             pol ? pol->tpot : nullptr, SMETRIC_POLICY_MAX_TPOT,
                             pol ? pol->nreq : nullptr, SMETRIC_POLICY_MAX_REQUESTS);
   idx->launches++;
@@ -1654,6 +1691,25 @@ int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_t
   return route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance,
                             d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap,
                             reinterpret_cast<cudaStream_t>(stream));
+}
+
+int smetric_route_batch_baseline(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                                 const int64_t* d_offsets, int32_t n_requests, int32_t scorer,
+                                 const int64_t* d_queued, const int64_t* d_batch, int64_t lam_num,
+                                 int64_t lam_den, int32_t* d_instance, int32_t* d_local_hit,
+                                 int32_t* d_global_hit, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                                 int64_t hashes_cap, smetric_stream_t stream) {
+  if (!idx || !d_batch || (scorer != SMETRIC_SCORER_BAILIAN && scorer != SMETRIC_SCORER_LMETRIC) ||
+      lam_den < 1 || lam_den > (1LL << 20) || lam_num < 0 || lam_num > lam_den)
+    return SMETRIC_ERR_INVALID_ARG;
+  WalkPolicy pol = {};
+  pol.on = scorer == SMETRIC_SCORER_BAILIAN ? kBailian : kLMetric;
+  pol.nreq = d_batch;
+  pol.lam_num = lam_num;
+  pol.lam_den = lam_den;
+  return route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_queued, smetric_weights{0, 0, 0},
+                            d_instance, d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap,
+                            reinterpret_cast<cudaStream_t>(stream), &pol);
 }
 
 int smetric_route_batch_policy_coloc(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,

@@ -219,3 +219,50 @@ def test_coloc_rejects_out_of_range_inputs():
                                       good)
     assert ix.status() == pkg.SMETRIC_OK
     ix.close()
+
+
+# ---------------------------------------------------------------------------
+# baseline scorers (Section 5.1)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("N,B", [(1, 4), (3, 2), (8, 16), (64, 4), (256, 8)])
+def test_baselines_match_oracle_tiny_alphabet(N, B):
+    rng = np.random.default_rng(N * 313 + B)
+    stored, reqs = tiny_alphabet_case(rng, N, B, n_req=300, max_blocks=12)
+    ix = make_index(N, B, 2, cap=8192)
+    ox = oracle.OracleIndex(N)
+    populate_both(ix, ox, stored, B)
+    tok, off = pack(reqs)
+    for case in range(8):
+        scorer = pkg.SMETRIC_SCORER_BAILIAN if case % 2 == 0 else pkg.SMETRIC_SCORER_LMETRIC
+        queued = rng.integers(0, [1 << 40, 100, 1, 1 << 20][case // 2], size=N)
+        batch = rng.integers(0, [1 << 20, 8, 1, 300][case // 2], size=N)  # all zero in case 4-5
+        den = int(rng.integers(1, 1 << 20))
+        lam = (int(rng.integers(0, den + 1)), den)
+        out = ix.route_batch_baseline(T(tok), T(off), scorer, T(np.asarray(queued, np.int64)),
+                                      T(np.asarray(batch, np.int64)), lam)
+        ix.check()
+        g = {k: v.cpu().numpy() for k, v in out.items()}
+        o = ox.route_batch_baseline(B, 2, 0, tok, off, scorer, queued, batch, *lam)
+        assert_outputs_equal(g, o, fields=("instance", "local_hit", "global_hit", "session_key"),
+                             ctx=f"N={N} B={B} case={case}")
+    ix.close()
+
+
+def test_baselines_refusals():
+    rng = np.random.default_rng(80)
+    N, B = 4, 16
+    ix = make_index(N, B, 1)
+    tok = rng.integers(0, 151936, size=1000, dtype=np.int32)
+    off = np.array([0, 100, 400, 1000], np.int64)
+    q, b = T(np.zeros(N, np.int64)), T(np.ones(N, np.int64))
+    for scorer, lam in ((0, (1, 2)), (3, (1, 2)), (1, (3, 2)), (1, (0, 0)), (2, (1, (1 << 20) + 1))):
+        with pytest.raises(pkg.SmetricError):
+            ix.route_batch_baseline(T(tok), T(off), scorer, q, b, lam)
+    for queued, batch in ((np.array([0, (1 << 40) + 1, 0, 0]), np.ones(N)),
+                          (np.zeros(N), np.array([0, (1 << 20) + 1, 0, 0]))):
+        out = ix.route_batch_baseline(T(tok), T(off), pkg.SMETRIC_SCORER_LMETRIC, T(np.asarray(queued, np.int64)),
+                                      T(np.asarray(batch, np.int64)))
+        assert ix.status() == pkg.SMETRIC_ERR_OVERFLOW
+        assert np.all(out["instance"].cpu().numpy() == -1)
+    ix.close()
