@@ -72,6 +72,10 @@ def load_library(path: str):
     L.oracle_route_batch_baseline.argtypes = [
         C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, C.c_int32, i64p, i64p,
         C.c_int64, C.c_int64, i32p, i32p, i32p, u64p]
+    L.oracle_route_batch_sequential.restype = C.c_int
+    L.oracle_route_batch_sequential.argtypes = [
+        C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p,
+        C.c_int64, C.c_int64, C.c_int64, i32p, i32p, i32p, u64p, i64p]
     L.oracle_link_sessions.restype = C.c_int
     L.oracle_link_sessions.argtypes = [C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p, i32p, i32p, i32p]
     return L
@@ -260,3 +264,23 @@ class OracleIndex:
             raise ValueError(f"oracle_route_batch_baseline: {rc}")
         inst, lh, gh = outs
         return dict(instance=inst[:n], local_hit=lh[:n], global_hit=gh[:n], session_key=sk[:n])
+
+    def route_batch_sequential(self, block_size: int, session_blocks: int, seed: int, tokens, offsets, load,
+                               w_load: int, w_miss: int, w_glob: int):
+        """The argmin cost with loads updated request by request. Returns
+        dict(instance, local_hit, global_hit, session_key, load_after)."""
+        t = np.ascontiguousarray(tokens, dtype=np.int32)
+        o = np.ascontiguousarray(offsets, dtype=np.int64)
+        ld = np.ascontiguousarray(load, dtype=np.int64)
+        n = len(o) - 1
+        outs = [np.zeros(max(n, 1), np.int32) for _ in range(3)]
+        sk = np.zeros(max(n, 1), np.uint64)
+        after = np.zeros(self.N, np.int64)
+        rc = self._L.oracle_route_batch_sequential(
+            self._h, block_size, session_blocks, seed & 0xFFFFFFFFFFFFFFFF,
+            t if len(t) else np.zeros(1, np.int32), o, n, ld, w_load, w_miss, w_glob, *outs, sk, after)
+        if rc != 0:
+            raise ValueError(f"oracle_route_batch_sequential: {rc}")
+        inst, lh, gh = outs
+        return dict(instance=inst[:n], local_hit=lh[:n], global_hit=gh[:n], session_key=sk[:n],
+                    load_after=after)

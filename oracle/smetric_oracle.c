@@ -84,6 +84,13 @@
  *              runs (LMetric's multiplicative score), compared exactly in
  *              128 bits.
  *
+ * Sequential-update variant (oracle_route_batch_sequential; Figure 10 routes
+ * one request at a time, so each request sees the queues its predecessors
+ * in the batch joined): requests in order, each takes the argmin cost above
+ * with the current loads, then load_{i*} += L_r - B*c_{i*} (the tokens the
+ * chosen instance must prefill or fetch). Limits: max_i load_i plus the
+ * batch's tokens at most 2^42.
+ *
  * Baseline scorers of Section 5.1 (oracle_route_batch_baseline), argmin with
  * ties to the lowest id over the same c_i:
  *    Bailian: f_i = (1 - LAMBDA) * l_i / max_j l_j + LAMBDA * (1 - B*c_i / L_r)
@@ -620,5 +627,62 @@ int oracle_route_batch_baseline(const oracle_index* x, int32_t B, int32_t S, uin
   }
   free(h);
   free(c);
+  return rc;
+}
+
+/* The argmin cost with the loads updated request by request (one request at
+ * a time, as Figure 10 routes). load_after (may be NULL) receives the loads
+ * after the batch. */
+int oracle_route_batch_sequential(const oracle_index* x, int32_t B, int32_t S, uint64_t seed,
+                                  const int32_t* tokens, const int64_t* offsets, int32_t n_requests,
+                                  const int64_t* load, int64_t w_load, int64_t w_miss, int64_t w_glob,
+                                  int32_t* instance, int32_t* local_hit, int32_t* global_hit,
+                                  uint64_t* session_key, int64_t* load_after) {
+  if (!x || B < 2 || (B % 2) != 0 || S < 1 || n_requests < 0) return ORACLE_ERR_INVALID_ARG;
+  const int32_t N = x->N;
+  int64_t top = 0;
+  for (int32_t i = 0; i < N; ++i) {
+    if (load[i] < 0) return ORACLE_ERR_INVALID_ARG;
+    if (load[i] > top) top = load[i];
+  }
+  for (int32_t r = 0; r < n_requests; ++r)
+    if (offsets[r + 1] < offsets[r] || offsets[r] < 0) return ORACLE_ERR_INVALID_ARG;
+  if (n_requests > 0 && top + (offsets[n_requests] - offsets[0]) > (1LL << 42)) return ORACLE_ERR_INVALID_ARG;
+  int64_t* q = (int64_t*)malloc((size_t)N * sizeof(int64_t));
+  int64_t* c = (int64_t*)malloc((size_t)N * sizeof(int64_t));
+  uint64_t* h = NULL;
+  int64_t cap = 0;
+  int rc = q && c ? ORACLE_OK : ORACLE_ERR_OOM;
+  if (rc == ORACLE_OK) memcpy(q, load, (size_t)N * sizeof(int64_t));
+  for (int32_t r = 0; r < n_requests && rc == ORACLE_OK; ++r) {
+    const int64_t L = offsets[r + 1] - offsets[r];
+    const int64_t n = L / B;
+    if (n + 1 > cap) {
+      free(h);
+      cap = n + 1;
+      h = (uint64_t*)malloc((size_t)cap * sizeof(uint64_t));
+      if (!h) { rc = ORACLE_ERR_OOM; break; }
+    }
+    oracle_block_hashes(tokens + offsets[r], L, B, seed, h);
+    int64_t g;
+    oracle_prefix_hits(x, h, n, c, &g);
+    int32_t best = -1;
+    int64_t best_cost = 0;
+    for (int32_t i = 0; i < N; ++i) {
+      const int64_t gi = c[i] > g ? c[i] : g;
+      const int64_t cost = w_load * q[i] + w_miss * (L - (int64_t)B * gi) + w_glob * (int64_t)B * (gi - c[i]);
+      if (best < 0 || cost < best_cost) { best = i; best_cost = cost; }
+    }
+    q[best] += L - (int64_t)B * c[best];  /* the chosen queue grows before the next request */
+    const int64_t gb = c[best] > g ? c[best] : g;
+    instance[r] = best;
+    local_hit[r] = (int32_t)((int64_t)B * c[best]);
+    global_hit[r] = (int32_t)((int64_t)B * (gb - c[best]));
+    session_key[r] = n == 0 ? 0 : h[(n < S ? n : S) - 1];
+  }
+  if (rc == ORACLE_OK && load_after) memcpy(load_after, q, (size_t)N * sizeof(int64_t));
+  free(h);
+  free(c);
+  free(q);
   return rc;
 }

@@ -780,6 +780,63 @@ def check_baselines_special_cases(L):
     assert int(out["instance"][0]) == 0
 
 
+# ---------------------------------------------------------------------------
+# sequential-update variant (reading 7)
+# ---------------------------------------------------------------------------
+
+def _seq(ix, B, reqs, load, w, S=1):
+    from synth.traces import pack
+    tokens, offsets = pack(reqs)
+    return ix.route_batch_sequential(B, S, 0, tokens, offsets, np.asarray(load, np.int64), *w)
+
+
+def check_sequential_matches_snapshot_without_load(L):
+    """With w_load = 0 the loads never matter: the sequential decisions are
+    the snapshot ones, and the final loads are the starting loads plus each
+    request's work on its instance."""
+    rng = np.random.default_rng(80)
+    B = 2
+    for trial in range(30):
+        N = int(rng.integers(1, 7))
+        base = rng.integers(0, 3, size=10 * B, dtype=np.int32)
+        ix = oracle.OracleIndex(N, L)
+        for i in range(N):
+            for _ in range(int(rng.integers(0, 3))):
+                ix.insert(oracle.block_hashes(_mutate(rng, base, int(rng.integers(0, 11 * B))), B, 0, L), i)
+        reqs = [_mutate(rng, base, int(rng.integers(0, 11 * B))) for _ in range(12)]
+        load = rng.integers(0, 100, size=N)
+        a = _seq(ix, B, reqs, load, (0, 3, 1))
+        b = _route(ix, B, 1, reqs, load, w=(0, 3, 1))
+        for k in ("instance", "local_hit", "global_hit", "session_key"):
+            assert np.array_equal(a[k], b[k]), (trial, k)
+        work = np.zeros(N, np.int64)
+        for r, t in enumerate(reqs):
+            work[b["instance"][r]] += len(t) - int(b["local_hit"][r])
+        assert np.array_equal(a["load_after"], load + work)
+
+
+def check_sequential_join_shortest_queue(L):
+    """Empty index, equal loads, equal prompts: each request joins the
+    shortest queue and lengthens it, so request r goes to r mod N; with
+    unequal prompts the choice follows the running queues exactly."""
+    rng = np.random.default_rng(81)
+    for N in (1, 2, 3, 7):
+        ix = oracle.OracleIndex(N, L)
+        reqs = [rng.integers(0, 151936, size=40, dtype=np.int32) for _ in range(15)]
+        out = _seq(ix, 4, reqs, [0] * N, (1, 4, 2))
+        assert np.array_equal(out["instance"], np.arange(15) % N)
+        lens = rng.integers(1, 200, size=15)
+        reqs = [rng.integers(0, 151936, size=int(x), dtype=np.int32) for x in lens]
+        q = np.array(rng.integers(0, 300, size=N))
+        want = []
+        for x in lens:
+            i = int(np.argmin(q))  # w_load * q + w_miss * L: only q differs
+            want.append(i)
+            q[i] += x
+        out = _seq(ix, 4, reqs, q - np.bincount(want, weights=lens, minlength=N).astype(np.int64), (1, 4, 2))
+        assert out["instance"].tolist() == want
+
+
 ALL_CHECKS = [
     check_published_vector,
     check_bijection,
@@ -812,4 +869,6 @@ ALL_CHECKS = [
     check_link_special_cases,
     check_baselines_against_their_definitions,
     check_baselines_special_cases,
+    check_sequential_matches_snapshot_without_load,
+    check_sequential_join_shortest_queue,
 ]

@@ -80,6 +80,8 @@ MUTANTS = {
     "lmetric_drops_queue": ("(uint64_t)(queued[i] + L - (int64_t)B * c[i])", "(uint64_t)(L - (int64_t)B * c[i])"),
     "baseline_tie_to_highest": ("if (best < 0 || f < best_f) { best = i; best_f = f; }",
                                 "if (best < 0 || f <= best_f) { best = i; best_f = f; }"),
+    "sequential_no_update": ("q[best] += L - (int64_t)B * c[best];", ";"),
+    "sequential_update_global": ("q[best] += L - (int64_t)B * c[best];", "q[best] += L - (int64_t)B * g;"),
     "coloc_product_64_bit": ("(unsigned __int128)(uint64_t)est2[i] * (uint64_t)num_requests[i];",
                              "(unsigned __int128)((uint64_t)est2[i] * (uint64_t)num_requests[i]);"),
 }
