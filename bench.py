@@ -59,6 +59,8 @@ def parse():
     ap.add_argument("--commit", action="store_true",
                     help="time device-side index maintenance (route, then commit the batch's blocks "
                          "and drain the queues) over a config-2 replay (one GPU; its own JSON line)")
+    ap.add_argument("--sequential", action="store_true",
+                    help="time the sequential-update variant on the config-4 workload (one GPU; its own line)")
     ap.add_argument("--link", action="store_true",
                     help="time session reconstruction (Appendix A) over a config-3 trace (one GPU; its own line)")
     ap.add_argument("--coloc", action="store_true",
@@ -740,6 +742,55 @@ def run_policy(args):
 
 
 # ---------------------------------------------------------------------------
+# sequential-update variant on the config-4 workload
+# ---------------------------------------------------------------------------
+
+def run_sequential(args, steps=50):
+    import torch
+    import paper_2607_08565_gb300 as pkg
+    from paper_2607_08565_gb300 import build_lib
+
+    build_lib.build()
+    torch.cuda.set_device(0)
+    tr = c4_trace(args)
+    p = tr.params
+    host = [tr.batch(k) for k in range(2)]
+    nkeys = tr.n_prefix_blocks()
+    chunk = 4096
+    ix = pkg.SMetricIndex(p.num_instances, p.block_size, p.session_blocks, capacity_slots=int(nkeys / 0.7) + 1,
+                          max_batch_requests=max(tr.batch_size, chunk),
+                          max_batch_tokens=max(max(b.n_tokens for b in host), chunk * int(tr.prefix_len.max())),
+                          hash_seed=p.hash_seed)
+    populate_index(ix, tr, torch.device("cuda", 0), chunk)
+    dev = [[torch.from_numpy(a).cuda() for a in (b.tokens, b.offsets, b.load)] for b in host]
+    w = (p.w_load, p.w_miss, p.w_glob)
+    times = {}
+    for name, fn in (("snapshot", lambda d: ix.route_batch(*d, w)),
+                     ("sequential", lambda d: ix.route_batch_sequential(*d, w))):
+        for i in range(3):
+            fn(dev[i % 2])
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for i in range(steps):
+            out = fn(dev[i % 2])
+        e1.record()
+        torch.cuda.synchronize()
+        ix.check()
+        times[name] = e0.elapsed_time(e1) / steps
+    seq = ix.route_batch_sequential(*dev[0], w)
+    snap = ix.route_batch(*dev[0], w)
+    changed = float((seq["instance"] != snap["instance"]).float().mean().item())
+    line = {"metric": "routed requests/sec, loads updated request by request (sequential variant)",
+            "value": host[0].n_requests / (times["sequential"] / 1e3), "unit": "requests/s", "n_gpus": 1,
+            "steps": steps, "warmup": 3, "ms_per_step": times["sequential"], "snapshot_ms_per_step": times["snapshot"],
+            "higher_is_better": True, "data": "synthetic",
+            "config": {"workload": workload_name(args), "decisions_differing_from_snapshot": changed}}
+    print(json.dumps(line), flush=True)
+    ix.close()
+
+
+# ---------------------------------------------------------------------------
 # session reconstruction over a config-3 trace
 # ---------------------------------------------------------------------------
 
@@ -975,6 +1026,9 @@ def main():
         return
     if args.link:
         run_link(args)
+        return
+    if args.sequential:
+        run_sequential(args)
         return
     rank, world, local, dist = dist_setup(args)
     if args.impl == "reference":

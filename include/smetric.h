@@ -266,6 +266,21 @@ int smetric_link_sessions(smetric_index* idx, const int32_t* d_tokens, int64_t n
                           const int32_t* d_turns, int32_t* d_parent, int32_t* d_session,
                           smetric_stream_t stream);
 
+/* smetric_route_batch with the loads updated request by request (Figure 10
+ * routes one request at a time, so each request sees the queues the batch's
+ * earlier requests joined): requests in batch order, each takes the argmin
+ * cost with the current loads, then load_{i*} += L_r - B*c_{i*}. The hits
+ * are those of the index snapshot, as in smetric_route_batch. The decisions
+ * run on one warp, request after request. d_load_after (int64 [N], may be
+ * NULL) receives the loads after the batch; d_load is read, not written.
+ * The largest load plus the batch's tokens must be at most 2^42, else the
+ * call latches OVERFLOW and writes instance -1 and zero hits. */
+int smetric_route_batch_sequential(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                                   const int64_t* d_offsets, int32_t n_requests, const int64_t* d_load,
+                                   smetric_weights w, int32_t* d_instance, int32_t* d_local_hit,
+                                   int32_t* d_global_hit, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                                   int64_t hashes_cap, int64_t* d_load_after, smetric_stream_t stream);
+
 /* Baseline scorers of Section 5.1 as the routing decision (argmin over the
  * same local hits c_i, ties to the lowest id). */
 #define SMETRIC_SCORER_BAILIAN 1 /* (1-lambda)*l_i/max_j l_j + lambda*(1 - B*c_i/L) */

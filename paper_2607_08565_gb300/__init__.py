@@ -48,7 +48,7 @@ EXPORTED = (
     "smetric_profile_enable", "smetric_profile_read", "smetric_profile_kernel_name",
     "smetric_launch_count", "smetric_block_hashes_noalloc", "smetric_route_batch_policy",
     "smetric_index_commit_batch", "smetric_route_batch_policy_coloc", "smetric_link_sessions",
-    "smetric_route_batch_baseline",
+    "smetric_route_batch_baseline", "smetric_route_batch_sequential",
 )
 
 
@@ -112,6 +112,8 @@ def lib():
                                                      P, P, P, P, I64, P]),
             "smetric_index_commit_batch": (C.c_int, [P, P, I32, P, P, P, I32, P, P]),
             "smetric_link_sessions": (C.c_int, [P, P, I64, P, I32, P, P, P, P, P]),
+            "smetric_route_batch_sequential": (C.c_int, [P, P, I64, P, I32, P, smetric_weights, P, P, P, P, P,
+                                                         I64, P, P]),
             "smetric_route_batch_baseline": (C.c_int, [P, P, I64, P, I32, I32, P, P, I64, I64, P, P, P, P, P,
                                                        I64, P]),
             "smetric_route_batch_policy_coloc": (C.c_int, [P, P, I64, P, I32, P, P, P, P, P, smetric_policy,
@@ -258,6 +260,15 @@ def smetric_route_batch_baseline(idx: int, d_tokens, n_tokens: int, d_offsets, n
         idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests, scorer, _ptr(d_queued), _ptr(d_batch),
         lam_num, lam_den, _ptr(d_instance), _ptr(d_local_hit), _ptr(d_global_hit), _ptr(d_session_key),
         _ptr(d_block_hashes), hashes_cap, _stream(stream)), "smetric_route_batch_baseline")
+
+
+def smetric_route_batch_sequential(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int, d_load, w,
+                                   d_instance, d_local_hit, d_global_hit, d_session_key, d_block_hashes=None,
+                                   hashes_cap: int = 0, d_load_after=None, stream=None) -> None:
+    _check(lib().smetric_route_batch_sequential(
+        idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests, _ptr(d_load), _weights(w), _ptr(d_instance),
+        _ptr(d_local_hit), _ptr(d_global_hit), _ptr(d_session_key), _ptr(d_block_hashes), hashes_cap,
+        _ptr(d_load_after), _stream(stream)), "smetric_route_batch_sequential")
 
 
 def smetric_link_sessions(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int, d_users, d_turns,
@@ -470,6 +481,22 @@ class SMetricIndex:
         smetric_route_batch_baseline(self.handle, tokens, tokens.numel(), offsets, n, scorer, queued, batch,
                                      lam[0], lam[1], out["instance"], out["local_hit"], out["global_hit"],
                                      out["session_key"], None, 0, stream)
+        return out
+
+    def route_batch_sequential(self, tokens, offsets, load, weights=(1, 4, 2), stream=None):
+        """The argmin cost with loads updated request by request. Returns
+        dict(instance, local_hit, global_hit, session_key, load_after)."""
+        import torch
+        n = offsets.numel() - 1
+        dev = offsets.device
+        out = dict(instance=torch.empty(n, dtype=torch.int32, device=dev),
+                   local_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                   global_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                   session_key=torch.empty(n, dtype=torch.uint64, device=dev),
+                   load_after=torch.empty(self.N, dtype=torch.int64, device=dev))
+        smetric_route_batch_sequential(self.handle, tokens, tokens.numel(), offsets, n, load, weights,
+                                       out["instance"], out["local_hit"], out["global_hit"], out["session_key"],
+                                       None, 0, out["load_after"], stream)
         return out
 
     def link_sessions(self, tokens, offsets, users, turns, stream=None):

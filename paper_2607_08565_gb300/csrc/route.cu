@@ -1062,7 +1062,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
         for (int e = 0; e < ne; ++e)
           if (ev_mask[e * W + wi] & bi) { ci = ev_pos[e]; break; }
       }
-      if (!MEMBERS) out_c[i] = (int32_t)ci;
+      out_c[i] = (int32_t)ci;  // every request's run ends (members' for the sequential variant)
       if (DECIDE == kArgmin) {
         const int64_t gi = ci > g ? ci : g;
         const int64_t cost = w_load * load_s[i] + w_miss * (L - B * gi) + w_glob * B * (gi - ci);
@@ -1099,7 +1099,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
         }
       }
     }
-    if (!MEMBERS && lane == 0) out_c[N] = (int32_t)g;
+    if (lane == 0) out_c[N] = (int32_t)g;
     if (DECIDE == kBailian || DECIDE == kLMetric) {
 #pragma unroll
       for (int dd = 16; dd > 0; dd >>= 1) {
@@ -1187,6 +1187,79 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
          i += (int64_t)gridDim.x * blockDim.x)
       groups[i] = make_uint4(0, 0, 0, 0);
   }
+}
+
+// ---------------------------------------------------------------------------
+// sequential-update variant
+// ---------------------------------------------------------------------------
+
+// One warp, requests in batch order: the a4-a5 argmin over the run ends the
+// walk recorded (summ: c_i for every instance, then g) with the current
+// loads, then the chosen load grows by L_r - B*c_{i*}. The next request's
+// row is loaded while this one is decided.
+__global__ void __launch_bounds__(32)
+    k_seq(int N, int B, const int64_t* __restrict__ off, int32_t n, const int64_t* __restrict__ load,
+          int64_t w_load, int64_t w_miss, int64_t w_glob, const int32_t* __restrict__ summ,
+          const int32_t* __restrict__ batch_ok, int32_t* __restrict__ inst_out, int32_t* __restrict__ lhit_out,
+          int32_t* __restrict__ ghit_out, int64_t* __restrict__ load_after, int32_t* status) {
+  __shared__ int64_t q[SMETRIC_MAX_INSTANCES];
+  const int lane = threadIdx.x;
+  if (!*batch_ok) return;  // the route already wrote the invalid batch's outputs
+  int64_t top = 0;
+  for (int i = lane; i < N; i += 32) { q[i] = load[i]; top = max(top, q[i]); }
+#pragma unroll
+  for (int dd = 16; dd > 0; dd >>= 1) top = max(top, __shfl_xor_sync(kFull, top, dd));
+  if (top + (off[n] - off[0]) > (1LL << 42)) {
+    for (int32_t r = lane; r < n; r += 32) { inst_out[r] = -1; lhit_out[r] = 0; ghit_out[r] = 0; }
+    if (lane == 0) latch_error(status, SMETRIC_ERR_OVERFLOW);
+    return;
+  }
+  __syncwarp();
+  constexpr int MT = (SMETRIC_MAX_INSTANCES + 1 + 31) / 32;  // row entries per lane
+  int32_t cur[MT], nxt[MT];
+  auto load_row = [&](int32_t r, int32_t (&dst)[MT]) {
+#pragma unroll
+    for (int t = 0; t < MT; ++t) {
+      const int i = 32 * t + lane;
+      dst[t] = r < n && i <= N ? summ[(int64_t)r * (N + 1) + i] : 0;
+    }
+  };
+  load_row(0, cur);
+  for (int32_t r = 0; r < n; ++r) {
+    load_row(r + 1, nxt);
+    const int64_t L = off[r + 1] - off[r];
+    const int32_t g = __shfl_sync(kFull, cur[N >> 5], N & 31);
+    int64_t best_cost = INT64_MAX, best_c = 0;
+    int32_t best = N;
+#pragma unroll
+    for (int t = 0; t < MT; ++t) {
+      const int i = 32 * t + lane;
+      if (i < N) {
+        const int64_t ci = cur[t], gi = ci > g ? ci : g;
+        const int64_t cost = w_load * q[i] + w_miss * (L - B * gi) + w_glob * B * (gi - ci);
+        if (cost < best_cost) { best_cost = cost; best = i; best_c = ci; }
+      }
+    }
+#pragma unroll
+    for (int dd = 16; dd > 0; dd >>= 1) {
+      const int64_t oc = __shfl_xor_sync(kFull, best_cost, dd);
+      const int32_t oi = __shfl_xor_sync(kFull, best, dd);
+      const int64_t ocb = __shfl_xor_sync(kFull, best_c, dd);
+      if (oc < best_cost || (oc == best_cost && oi < best)) { best_cost = oc; best = oi; best_c = ocb; }
+    }
+    if (lane == 0) {
+      const int64_t gb = best_c > g ? best_c : g;
+      inst_out[r] = best;
+      lhit_out[r] = (int32_t)(B * best_c);
+      ghit_out[r] = (int32_t)(B * (gb - best_c));
+      q[best] += L - B * best_c;
+    }
+    __syncwarp();
+#pragma unroll
+    for (int t = 0; t < MT; ++t) cur[t] = nxt[t];
+  }
+  if (load_after)
+    for (int i = lane; i < N; i += 32) load_after[i] = q[i];
 }
 
 // ---------------------------------------------------------------------------
@@ -1691,6 +1764,22 @@ int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_t
   return route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance,
                             d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap,
                             reinterpret_cast<cudaStream_t>(stream));
+}
+
+int smetric_route_batch_sequential(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                                   const int64_t* d_offsets, int32_t n_requests, const int64_t* d_load,
+                                   smetric_weights w, int32_t* d_instance, int32_t* d_local_hit,
+                                   int32_t* d_global_hit, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                                   int64_t hashes_cap, int64_t* d_load_after, smetric_stream_t stream) {
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int rc = route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance, d_local_hit,
+                              d_global_hit, d_session_key, d_block_hashes, hashes_cap, s);
+  if (rc || n_requests == 0) return rc;
+  k_seq<<<1, 32, 0, s>>>(idx->cfg.num_instances, idx->cfg.block_size, d_offsets, n_requests, d_load, w.w_load,
+                         w.w_miss, w.w_glob, idx->summ, idx->batch_ok, d_instance, d_local_hit, d_global_hit,
+                         d_load_after, idx->status);
+  idx->launches++;
+  return cuda_status(cudaGetLastError());
 }
 
 int smetric_route_batch_baseline(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,

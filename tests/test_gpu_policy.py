@@ -266,3 +266,40 @@ def test_baselines_refusals():
         assert ix.status() == pkg.SMETRIC_ERR_OVERFLOW
         assert np.all(out["instance"].cpu().numpy() == -1)
     ix.close()
+
+
+# ---------------------------------------------------------------------------
+# sequential-update variant
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("N,B", [(1, 4), (3, 2), (8, 16), (64, 4), (256, 8)])
+def test_sequential_matches_oracle(N, B):
+    rng = np.random.default_rng(N * 71 + B)
+    stored, reqs = tiny_alphabet_case(rng, N, B, n_req=400, max_blocks=12)
+    ix = make_index(N, B, 2, cap=8192)
+    ox = oracle.OracleIndex(N)
+    populate_both(ix, ox, stored, B)
+    tok, off = pack(reqs)
+    for w in ((1, 4, 2), (1, 1, 0), (5, 1, 7), (0, 3, 1), (2 ** 20, 2 ** 20, 2 ** 20)):
+        load = rng.integers(0, [1 << 30, 50][w[0] > 1000], size=N)
+        out = ix.route_batch_sequential(T(tok), T(off), T(np.asarray(load, np.int64)), w)
+        ix.check()
+        g = {k: v.cpu().numpy() for k, v in out.items()}
+        o = ox.route_batch_sequential(B, 2, 0, tok, off, load, *w)
+        assert_outputs_equal(g, o, fields=("instance", "local_hit", "global_hit", "session_key"),
+                             ctx=f"N={N} B={B} w={w}")
+        assert np.array_equal(g["load_after"], o["load_after"])
+    ix.close()
+
+
+def test_sequential_overflow_guard():
+    N, B = 3, 4
+    ix = make_index(N, B, 1)
+    tok = np.zeros(64, np.int32)
+    off = np.array([0, 32, 64], np.int64)
+    out = ix.route_batch_sequential(T(tok), T(off), T(np.array([0, (1 << 42) - 63, 0], np.int64)))
+    assert ix.status() == pkg.SMETRIC_ERR_OVERFLOW
+    assert np.all(out["instance"].cpu().numpy() == -1)
+    out = ix.route_batch_sequential(T(tok), T(off), T(np.array([0, (1 << 40), 0], np.int64)))
+    assert ix.status() == pkg.SMETRIC_OK and out["instance"].cpu().numpy().tolist() == [0, 2]
+    ix.close()
