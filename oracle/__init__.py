@@ -76,6 +76,9 @@ def load_library(path: str):
     L.oracle_route_batch_sequential.argtypes = [
         C.c_void_p, C.c_int32, C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p,
         C.c_int64, C.c_int64, C.c_int64, i32p, i32p, i32p, u64p, i64p]
+    L.oracle_reuse_breakdown.restype = C.c_int
+    L.oracle_reuse_breakdown.argtypes = [C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i32p, i32p,
+                                         i32p, i32p, i32p, i32p]
     L.oracle_link_sessions.restype = C.c_int
     L.oracle_link_sessions.argtypes = [C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p, i32p, i32p, i32p]
     return L
@@ -118,6 +121,24 @@ def link_sessions(block_size: int, seed: int, tokens, offsets, users, turns, L=N
     if rc != 0:
         raise ValueError(f"oracle_link_sessions: {rc}")
     return parent[:n], session[:n]
+
+
+def reuse_breakdown(block_size: int, seed: int, tokens, offsets, sessions, sys_blocks, L=None):
+    """Reuse against an unbounded store of every earlier request's blocks:
+    dict(hit, sys, intra, inter), int32 blocks per request."""
+    t = np.ascontiguousarray(tokens, dtype=np.int32)
+    o = np.ascontiguousarray(offsets, dtype=np.int64)
+    n = len(o) - 1
+    ss = np.ascontiguousarray(sessions, dtype=np.int32)
+    sb = np.ascontiguousarray(sys_blocks, dtype=np.int32)
+    outs = [np.zeros(max(n, 1), np.int32) for _ in range(4)]
+    rc = (L or lib()).oracle_reuse_breakdown(block_size, seed & 0xFFFFFFFFFFFFFFFF,
+                                             t if len(t) else np.zeros(1, np.int32), o, n,
+                                             ss if n else np.zeros(1, np.int32), sb if n else np.zeros(1, np.int32),
+                                             *outs)
+    if rc != 0:
+        raise ValueError(f"oracle_reuse_breakdown: {rc}")
+    return dict(zip(("hit", "sys", "intra", "inter"), (x[:n] for x in outs)))
 
 
 class OracleIndex:

@@ -100,6 +100,14 @@
  *             LAM_DEN * max_j l_j * L_r in 128 bits.
  *    LMetric: f_i = (q_i + L_r - B*c_i) * l_i (q_i the queued prefill tokens).
  *
+ * Reuse breakdown (Section 3.1, Findings 1-3; oracle_reuse_breakdown): against
+ * an idealised KV$ store of unbounded capacity holding every block of every
+ * earlier request, request r's hit is its longest block prefix whose blocks
+ * the store holds (hash h_b occurs in some earlier request). Each hit block
+ * is attributed to the earliest request p holding it: to the system prompt
+ * when b < sys_r (the request's leading system-prompt blocks), else
+ * intra-session when session_p = session_r, else inter-session.
+ *
  * Session reconstruction (Appendix A; oracle_link_sessions): request r
  * follows request p when p is earlier (p < r, requests in arrival order), of
  * the same user, of turn turn_r - 1, and p's block-hash sequence is a prefix
@@ -685,4 +693,42 @@ int oracle_route_batch_sequential(const oracle_index* x, int32_t B, int32_t S, u
   free(c);
   free(q);
   return rc;
+}
+
+/* Reuse breakdown, by definition: for every hit candidate, every earlier
+ * request is searched for the block hash, earliest first. Outputs per
+ * request (int32): hit blocks and their split into system-prompt,
+ * intra-session and inter-session blocks. */
+int oracle_reuse_breakdown(int32_t B, uint64_t seed, const int32_t* tokens, const int64_t* offsets,
+                           int32_t n_requests, const int32_t* sessions, const int32_t* sys_blocks, int32_t* hit,
+                           int32_t* sys, int32_t* intra, int32_t* inter) {
+  if (B < 2 || (B % 2) != 0 || n_requests < 0) return ORACLE_ERR_INVALID_ARG;
+  for (int32_t r = 0; r < n_requests; ++r)
+    if (offsets[r + 1] < offsets[r] || offsets[r] < 0 || sys_blocks[r] < 0) return ORACLE_ERR_INVALID_ARG;
+  int64_t* first = (int64_t*)malloc((size_t)(n_requests + 1) * sizeof(int64_t));
+  if (!first) return ORACLE_ERR_OOM;
+  first[0] = 0;
+  for (int32_t r = 0; r < n_requests; ++r) first[r + 1] = first[r] + (offsets[r + 1] - offsets[r]) / B;
+  uint64_t* h = (uint64_t*)malloc((size_t)(first[n_requests] + 1) * sizeof(uint64_t));
+  if (!h) { free(first); return ORACLE_ERR_OOM; }
+  for (int32_t r = 0; r < n_requests; ++r)
+    oracle_block_hashes(tokens + offsets[r], offsets[r + 1] - offsets[r], B, seed, h + first[r]);
+  for (int32_t r = 0; r < n_requests; ++r) {
+    hit[r] = sys[r] = intra[r] = inter[r] = 0;
+    for (int64_t b = 0; b < first[r + 1] - first[r]; ++b) {
+      const uint64_t key = h[first[r] + b];
+      int32_t producer = -1;  /* the earliest earlier request holding the block */
+      for (int32_t p = 0; p < r && producer < 0; ++p)
+        for (int64_t k = first[p]; k < first[p + 1]; ++k)
+          if (h[k] == key) { producer = p; break; }
+      if (producer < 0) break;  /* the prefix ends at the first block the store lacks */
+      hit[r]++;
+      if (b < sys_blocks[r]) sys[r]++;
+      else if (sessions[producer] == sessions[r]) intra[r]++;
+      else inter[r]++;
+    }
+  }
+  free(h);
+  free(first);
+  return ORACLE_OK;
 }

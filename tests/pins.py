@@ -837,6 +837,70 @@ def check_sequential_join_shortest_queue(L):
         assert out["instance"].tolist() == want
 
 
+# ---------------------------------------------------------------------------
+# reuse breakdown (Section 3.1)
+# ---------------------------------------------------------------------------
+
+def check_reuse_against_token_prefixes(L):
+    """Brute force by token comparison: block b of r is reused when an
+    earlier request starts with r's first b+1 blocks; the prefix stops at the
+    first block that is not; each reused block goes to the system prompt when
+    b < sys_r, else to intra- or inter-session by the earliest such request's
+    session."""
+    from synth.traces import pack
+    rng = np.random.default_rng(90)
+    B = 2
+    for trial in range(25):
+        base = rng.integers(0, 3, size=12 * B, dtype=np.int32)
+        n = int(rng.integers(1, 30))
+        reqs = [_mutate(rng, base, int(rng.integers(0, 12 * B))) for _ in range(n)]
+        sessions = rng.integers(0, 4, size=n)
+        sys_b = rng.integers(0, 4, size=n)
+        tokens, offsets = pack(reqs)
+        out = oracle.reuse_breakdown(B, 0, tokens, offsets, sessions, sys_b, L)
+        for r in range(n):
+            want = dict(hit=0, sys=0, intra=0, inter=0)
+            for b in range(len(reqs[r]) // B):
+                pre = reqs[r][:(b + 1) * B]
+                prod = next((q for q in range(r) if len(reqs[q]) >= len(pre) and
+                             np.array_equal(reqs[q][:len(pre)], pre)), -1)
+                if prod < 0:
+                    break
+                want["hit"] += 1
+                key = "sys" if b < sys_b[r] else "intra" if sessions[prod] == sessions[r] else "inter"
+                want[key] += 1
+            for k in want:
+                assert int(out[k][r]) == want[k], (trial, r, k)
+
+
+def check_reuse_on_a_multi_turn_trace(L):
+    """Turn t of a session resends turn t-1 whole: with one session per user
+    and no truncation, every follow-up reuses at least its parent's blocks,
+    first turns reuse only the shared system prompt, and the parts add up."""
+    from synth import agent_trace
+    from synth.traces import pack
+    tr = agent_trace("c1_tiny", scale=0.25, seed=9)
+    B = tr.params.block_size
+    reqs, sess, turns = [], [], []
+    for bt in tr.batches():
+        for r in range(bt.n_requests):
+            reqs.append(bt.tokens[bt.offsets[r]:bt.offsets[r + 1]])
+        sess.extend(bt.sessions.tolist())
+        turns.extend(bt.turns.tolist())
+    tokens, offsets = pack(reqs)
+    sys_b = np.full(len(reqs), tr.system_prompt_len // B, np.int32)
+    out = oracle.reuse_breakdown(B, 0, tokens, offsets, sess, sys_b, L)
+    assert np.array_equal(out["hit"], out["sys"] + out["intra"] + out["inter"])
+    last = {}
+    for r, (s_, t_) in enumerate(zip(sess, turns)):
+        if t_ > 0:
+            assert out["hit"][r] >= len(reqs[last[s_]]) // B
+        else:
+            assert out["intra"][r] == 0
+        last[s_] = r
+    assert out["intra"].sum() > 0 and out["sys"].sum() > 0
+
+
 ALL_CHECKS = [
     check_published_vector,
     check_bijection,
@@ -871,4 +935,6 @@ ALL_CHECKS = [
     check_baselines_special_cases,
     check_sequential_matches_snapshot_without_load,
     check_sequential_join_shortest_queue,
+    check_reuse_against_token_prefixes,
+    check_reuse_on_a_multi_turn_trace,
 ]

@@ -82,6 +82,12 @@ MUTANTS = {
                                 "if (best < 0 || f <= best_f) { best = i; best_f = f; }"),
     "sequential_no_update": ("q[best] += L - (int64_t)B * c[best];", ";"),
     "sequential_update_global": ("q[best] += L - (int64_t)B * c[best];", "q[best] += L - (int64_t)B * g;"),
+    "reuse_latest_producer": ("for (int32_t p = 0; p < r && producer < 0; ++p)",
+                              "for (int32_t p = r - 1; p >= 0 && producer < 0; --p)"),
+    "reuse_system_off_by_one": ("if (b < sys_blocks[r]) sys[r]++;", "if (b <= sys_blocks[r]) sys[r]++;"),
+    "reuse_self_hit": ("for (int32_t p = 0; p < r && producer < 0; ++p)",
+                       "for (int32_t p = 0; p <= r && producer < 0; ++p)"),
+    "reuse_system_by_session": ("if (b < sys_blocks[r]) sys[r]++;", "if (b < sys_blocks[r] && sessions[producer] != sessions[r]) sys[r]++;"),
     "coloc_product_64_bit": ("(unsigned __int128)(uint64_t)est2[i] * (uint64_t)num_requests[i];",
                              "(unsigned __int128)((uint64_t)est2[i] * (uint64_t)num_requests[i]);"),
 }
