@@ -63,6 +63,9 @@ def parse():
                     help="time the sequential-update variant on the config-4 workload (one GPU; its own line)")
     ap.add_argument("--link", action="store_true",
                     help="time session reconstruction (Appendix A) over a config-3 trace (one GPU; its own line)")
+    ap.add_argument("--reuse", action="store_true",
+                    help="time the KV$ reuse breakdown (Section 3.1) over a whole config-2 window "
+                         "(one GPU; its own line)")
     ap.add_argument("--coloc", action="store_true",
                     help="with --policy: the PD-colocation variant (Appendix B)")
     ap.add_argument("--policy", action="store_true",
@@ -849,6 +852,78 @@ def run_link(args, scale=0.5):
 
 
 # ---------------------------------------------------------------------------
+# KV$ reuse breakdown over a whole config-2 window
+# ---------------------------------------------------------------------------
+
+def run_reuse(args, k_sessions=20):
+    import torch
+    import oracle
+    import paper_2607_08565_gb300 as pkg
+    from paper_2607_08565_gb300 import build_lib
+    from synth import agent_trace
+    from synth.traces import pack
+
+    build_lib.build()
+    torch.cuda.set_device(0)
+    tr = agent_trace("c2_medium", scale=1.0, seed=7)
+    p = tr.params
+    reqs, sess = [], []
+    for bt in tr.batches():
+        for r in range(bt.n_requests):
+            reqs.append(bt.tokens[bt.offsets[r]:bt.offsets[r + 1]])
+        sess.extend(bt.sessions.tolist())
+    tok, off = pack(reqs)
+    n = len(off) - 1
+    sys_b = np.full(n, tr.system_prompt_len // p.block_size, np.int32)
+    # the oracle's sample: every turn of the first sessions, a window of its own
+    keep = np.nonzero(np.asarray(sess) < k_sessions)[0]
+    s_tok, s_off = pack([reqs[i] for i in keep])
+    s_sess, s_sys = np.asarray(sess, np.int32)[keep], sys_b[keep]
+    del reqs
+    ix = pkg.SMetricIndex(p.num_instances, p.block_size, p.session_blocks, capacity_slots=1 << 16,
+                          max_batch_requests=n, max_batch_tokens=len(tok), hash_seed=p.hash_seed)
+    d = [torch.from_numpy(np.ascontiguousarray(a)).cuda() for a in (tok, off, np.asarray(sess, np.int32), sys_b)]
+    ws = torch.empty(pkg.smetric_reuse_workspace_bytes(len(tok) // p.block_size), dtype=torch.uint8, device="cuda")
+    for _ in range(3):
+        out = ix.reuse_breakdown(*d, workspace=ws)
+    torch.cuda.synchronize()
+    ix.check()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    steps = 10
+    e0.record()
+    for _ in range(steps):
+        ix.reuse_breakdown(*d, workspace=ws)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    g = {k: v.cpu().numpy() for k, v in out.items()}
+    if not np.array_equal(g["hit"], g["sys"] + g["intra"] + g["inter"]):
+        raise RuntimeError("reuse parts do not add up")
+    sg = ix.reuse_breakdown(*(torch.from_numpy(np.ascontiguousarray(a)).cuda()
+                              for a in (s_tok, s_off, s_sess, s_sys)))
+    ix.check()
+    t0 = time.perf_counter()
+    o = oracle.reuse_breakdown(p.block_size, p.hash_seed, s_tok, s_off, s_sess, s_sys)
+    dt = time.perf_counter() - t0
+    if any(not np.array_equal(o[k], sg[k].cpu().numpy()) for k in o):
+        raise RuntimeError("reuse breakdown differs from the oracle")
+    nb = int((np.diff(off) // p.block_size).sum())
+    line = {"metric": "requests analysed for KV$ reuse per second (Section 3.1)", "value": n / (ms / 1e3),
+            "unit": "requests/s", "n_gpus": 1, "steps": steps, "warmup": 3, "ms_per_step": ms,
+            "higher_is_better": True, "data": "synthetic",
+            "config": {"workload": f"c2_medium agent trace: {n} requests, {len(tok)} tokens, {nb} blocks, "
+                                   f"B = {p.block_size}, one call",
+                       "tokens_per_s": len(tok) / (ms / 1e3),
+                       "blocks": {k: int(g[k].sum()) for k in g}},
+            "cpu_baseline": {"value": len(keep) / dt, "unit": "requests/s", "cores": 1, "kind": "oracle",
+                             "sample": f"every turn of sessions 0-{k_sessions - 1} ({len(keep)} requests, "
+                                       f"{len(s_tok)} tokens) as a window of its own ({dt:.1f} s, one thread; "
+                                       f"the oracle's cost grows with the square of the window)"}}
+    print(json.dumps(line), flush=True)
+    ix.close()
+
+
+# ---------------------------------------------------------------------------
 # device-side index maintenance over a config-2 replay
 # ---------------------------------------------------------------------------
 
@@ -1029,6 +1104,9 @@ def main():
         return
     if args.sequential:
         run_sequential(args)
+        return
+    if args.reuse:
+        run_reuse(args)
         return
     rank, world, local, dist = dist_setup(args)
     if args.impl == "reference":

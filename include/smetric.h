@@ -250,6 +250,25 @@ int smetric_route_batch_policy_coloc(smetric_index* idx, const int32_t* d_tokens
                                      int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
                                      int64_t hashes_cap, smetric_stream_t stream);
 
+/* KV$ reuse breakdown of a trace window (Section 3.1, Findings 1-3):
+ * against an unbounded store of every earlier request's blocks (requests in
+ * arrival order), request r reuses its longest block prefix the store holds.
+ * Each reused block b counts as system prompt when b < d_sys_blocks[r], else
+ * as intra-session when the earliest request holding it has r's session
+ * (d_sessions, e.g. from smetric_link_sessions), else as inter-session.
+ * Outputs (int32 [n_requests], blocks): d_hit = d_sys + d_intra + d_inter.
+ * The caller provides a 16-byte aligned device workspace of at least
+ * smetric_reuse_workspace_bytes(n_tokens / block_size) bytes (nothing is
+ * allocated). Uses the index's hashing and route scratch. Invalid offsets
+ * latch INVALID_ARG and write -1 everywhere; a negative system span latches
+ * INVALID_ARG and counts as 0. */
+int64_t smetric_reuse_workspace_bytes(int64_t n_blocks);
+int smetric_reuse_breakdown(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                            const int64_t* d_offsets, int32_t n_requests, const int32_t* d_sessions,
+                            const int32_t* d_sys_blocks, void* d_workspace, int64_t workspace_bytes,
+                            int32_t* d_hit, int32_t* d_sys, int32_t* d_intra, int32_t* d_inter,
+                            smetric_stream_t stream);
+
 /* Session reconstruction from block hashes (Appendix A): in a batch of
  * requests in arrival order, request r follows the latest earlier request p
  * of the same user (d_users) with d_turns[p] = d_turns[r] - 1 whose

@@ -48,7 +48,8 @@ EXPORTED = (
     "smetric_profile_enable", "smetric_profile_read", "smetric_profile_kernel_name",
     "smetric_launch_count", "smetric_block_hashes_noalloc", "smetric_route_batch_policy",
     "smetric_index_commit_batch", "smetric_route_batch_policy_coloc", "smetric_link_sessions",
-    "smetric_route_batch_baseline", "smetric_route_batch_sequential",
+    "smetric_route_batch_baseline", "smetric_route_batch_sequential", "smetric_reuse_workspace_bytes",
+    "smetric_reuse_breakdown",
 )
 
 
@@ -112,6 +113,8 @@ def lib():
                                                      P, P, P, P, I64, P]),
             "smetric_index_commit_batch": (C.c_int, [P, P, I32, P, P, P, I32, P, P]),
             "smetric_link_sessions": (C.c_int, [P, P, I64, P, I32, P, P, P, P, P]),
+            "smetric_reuse_workspace_bytes": (I64, [I64]),
+            "smetric_reuse_breakdown": (C.c_int, [P, P, I64, P, I32, P, P, P, I64, P, P, P, P, P]),
             "smetric_route_batch_sequential": (C.c_int, [P, P, I64, P, I32, P, smetric_weights, P, P, P, P, P,
                                                          I64, P, P]),
             "smetric_route_batch_baseline": (C.c_int, [P, P, I64, P, I32, I32, P, P, I64, I64, P, P, P, P, P,
@@ -269,6 +272,19 @@ def smetric_route_batch_sequential(idx: int, d_tokens, n_tokens: int, d_offsets,
         idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests, _ptr(d_load), _weights(w), _ptr(d_instance),
         _ptr(d_local_hit), _ptr(d_global_hit), _ptr(d_session_key), _ptr(d_block_hashes), hashes_cap,
         _ptr(d_load_after), _stream(stream)), "smetric_route_batch_sequential")
+
+
+def smetric_reuse_workspace_bytes(n_blocks: int) -> int:
+    return int(lib().smetric_reuse_workspace_bytes(n_blocks))
+
+
+def smetric_reuse_breakdown(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int, d_sessions,
+                            d_sys_blocks, d_workspace, workspace_bytes: int, d_hit, d_sys, d_intra, d_inter,
+                            stream=None) -> None:
+    _check(lib().smetric_reuse_breakdown(idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests,
+                                         _ptr(d_sessions), _ptr(d_sys_blocks), _ptr(d_workspace), workspace_bytes,
+                                         _ptr(d_hit), _ptr(d_sys), _ptr(d_intra), _ptr(d_inter), _stream(stream)),
+           "smetric_reuse_breakdown")
 
 
 def smetric_link_sessions(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int, d_users, d_turns,
@@ -497,6 +513,20 @@ class SMetricIndex:
         smetric_route_batch_sequential(self.handle, tokens, tokens.numel(), offsets, n, load, weights,
                                        out["instance"], out["local_hit"], out["global_hit"], out["session_key"],
                                        None, 0, out["load_after"], stream)
+        return out
+
+    def reuse_breakdown(self, tokens, offsets, sessions, sys_blocks, workspace=None, stream=None):
+        """KV$ reuse against an unbounded store of the earlier requests:
+        dict(hit, sys, intra, inter), int32 blocks per request."""
+        import torch
+        n = offsets.numel() - 1
+        dev = offsets.device
+        need = smetric_reuse_workspace_bytes(tokens.numel() // self.B)
+        if workspace is None:
+            workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+        out = {k: torch.empty(n, dtype=torch.int32, device=dev) for k in ("hit", "sys", "intra", "inter")}
+        smetric_reuse_breakdown(self.handle, tokens, tokens.numel(), offsets, n, sessions, sys_blocks, workspace,
+                                workspace.numel(), out["hit"], out["sys"], out["intra"], out["inter"], stream)
         return out
 
     def link_sessions(self, tokens, offsets, users, turns, stream=None):

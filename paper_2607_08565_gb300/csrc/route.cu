@@ -1263,6 +1263,99 @@ __global__ void __launch_bounds__(32)
 }
 
 // ---------------------------------------------------------------------------
+// reuse breakdown
+// ---------------------------------------------------------------------------
+
+uint64_t reuse_slots_for(int64_t n_blocks) {
+  uint64_t g = 64;
+  while (g < 2 * (uint64_t)n_blocks) g <<= 1;
+  return g;
+}
+
+// Thread per block of the batch: its hash into the workspace table with the
+// earliest request holding it (pairs (hash, INT32_MAX - request), atomicMax).
+__global__ void __launch_bounds__(256)
+    k_reuse_insert(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
+                   const uint64_t* __restrict__ H, uint64_t* __restrict__ table, uint64_t mask) {
+  if (!*batch_ok) return;
+  const int64_t total = block_off[n];
+  int32_t r = 0;
+  for (int64_t f = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; f < total;
+       f += (int64_t)gridDim.x * blockDim.x) {
+    r = find_request(block_off, r, n, f);
+    const uint64_t key = H[f];
+    uint64_t s = key & mask;
+    for (uint64_t t = 0; t <= mask; ++t) {
+      unsigned long long* const slot = reinterpret_cast<unsigned long long*>(table + 2 * s);
+      const unsigned long long k = atomicCAS(slot, 0ull, (unsigned long long)key);
+      if (k == 0ull || k == key) {
+        atomicMax(slot + 1, (unsigned long long)(INT32_MAX - r));
+        break;
+      }
+      s = (s + 1) & mask;
+    }
+  }
+}
+
+// Warp per request, 32 blocks per round: block b is reused when its earliest
+// holder precedes the request; the run stops at the first block that is not.
+// Reused blocks split into system prompt (b < sys_r), intra-session (the
+// holder is of r's session) and inter-session.
+__global__ void __launch_bounds__(256)
+    k_reuse_walk(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
+                 const uint64_t* __restrict__ H, const uint64_t* __restrict__ table, uint64_t mask,
+                 const int32_t* __restrict__ sessions, const int32_t* __restrict__ sys_blocks,
+                 int32_t* __restrict__ hit, int32_t* __restrict__ sys, int32_t* __restrict__ intra,
+                 int32_t* __restrict__ inter, int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t tw = (int64_t)gridDim.x * (blockDim.x >> 5);
+  const bool ok = *batch_ok != 0;
+  for (int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n; r += tw) {
+    int32_t nh = 0, ns = 0, ni = 0, ne = 0;
+    if (ok) {
+      const int64_t bo = block_off[r], nb = block_off[r + 1] - bo;
+      int64_t sb = sys_blocks[r];
+      if (sb < 0) {
+        if (lane == 0) latch_error(status, SMETRIC_ERR_INVALID_ARG);
+        sb = 0;
+      }
+      const int32_t sr = sessions[r];
+      for (int64_t base = 0; base < nb; base += 32) {
+        const int64_t b = base + lane;
+        int32_t producer = INT32_MAX;
+        if (b < nb) {
+          const uint64_t key = H[bo + b];
+          uint64_t s = key & mask;
+          for (uint64_t t = 0; t <= mask; ++t) {
+            const uint64_t k = table[2 * s];
+            if (k == key) { producer = INT32_MAX - (int32_t)table[2 * s + 1]; break; }
+            if (k == 0) break;
+            s = (s + 1) & mask;
+          }
+        }
+        const bool reused = b < nb && producer < r;
+        const unsigned miss = __ballot_sync(kFull, !reused);
+        const unsigned run = miss ? (1u << (__ffs(miss) - 1)) - 1 : kFull;  // lanes before the first miss
+        const bool in = (run >> lane) & 1;
+        const bool is_sys = in && b < sb;
+        const bool is_intra = in && !is_sys && sessions[producer] == sr;
+        nh += __popc(run);
+        ns += __popc(__ballot_sync(kFull, is_sys));
+        ni += __popc(__ballot_sync(kFull, is_intra));
+        ne += __popc(__ballot_sync(kFull, in && !is_sys && !is_intra));
+        if (miss) break;
+      }
+    }
+    if (lane == 0) {
+      hit[r] = ok ? nh : -1;
+      sys[r] = ok ? ns : -1;
+      intra[r] = ok ? ni : -1;
+      inter[r] = ok ? ne : -1;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
 // session links
 // ---------------------------------------------------------------------------
 
@@ -1850,6 +1943,41 @@ int smetric_index_commit_batch(smetric_index* idx, const int64_t* d_offsets, int
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   return launch_commit(idx, d_instance, d_block_hashes, n_requests, c.max_batch_tokens / c.block_size,
                        (flags & SMETRIC_COMMIT_GLOBAL) != 0, s);
+}
+
+int64_t smetric_reuse_workspace_bytes(int64_t n_blocks) {
+  return n_blocks < 0 ? 0 : (int64_t)(2 * sizeof(uint64_t) * reuse_slots_for(n_blocks));
+}
+
+int smetric_reuse_breakdown(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                            const int64_t* d_offsets, int32_t n_requests, const int32_t* d_sessions,
+                            const int32_t* d_sys_blocks, void* d_workspace, int64_t workspace_bytes,
+                            int32_t* d_hit, int32_t* d_sys, int32_t* d_intra, int32_t* d_inter,
+                            smetric_stream_t stream) {
+  int rc = check_device(idx);
+  if (rc) return rc;
+  if (n_requests < 0 || n_requests > idx->cfg.max_batch_requests || n_tokens < 0) return SMETRIC_ERR_INVALID_ARG;
+  if (n_requests == 0) return SMETRIC_OK;
+  const int64_t n_blocks = n_tokens / idx->cfg.block_size;
+  if (!d_sessions || !d_sys_blocks || !d_hit || !d_sys || !d_intra || !d_inter || !d_workspace ||
+      workspace_bytes < smetric_reuse_workspace_bytes(n_blocks) || (reinterpret_cast<uintptr_t>(d_workspace) & 15))
+    return SMETRIC_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((rc = route_common<false>(idx, d_tokens, n_tokens, d_offsets, n_requests, nullptr, smetric_weights{0, 0, 0},
+                                nullptr, nullptr, nullptr, idx->sk_tmp, idx->hashes, n_blocks, s)))
+    return rc;
+  const uint64_t slots = reuse_slots_for(n_blocks);
+  uint64_t* table = static_cast<uint64_t*>(d_workspace);
+  if (cudaMemsetAsync(table, 0, 2 * sizeof(uint64_t) * slots, s) != cudaSuccess) return cuda_status(cudaErrorUnknown);
+  const int64_t want = (n_blocks + 255) / 256;
+  const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
+  k_reuse_insert<<<grid, 256, 0, s>>>(idx->block_off, n_requests, idx->batch_ok, idx->hashes, table, slots - 1);
+  const unsigned wgrid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(((int64_t)n_requests + 7) / 8,
+                                                                          (int64_t)idx->num_sms * 8));
+  k_reuse_walk<<<wgrid, 256, 0, s>>>(idx->block_off, n_requests, idx->batch_ok, idx->hashes, table, slots - 1,
+                                     d_sessions, d_sys_blocks, d_hit, d_sys, d_intra, d_inter, idx->status);
+  idx->launches += 2;
+  return cuda_status(cudaGetLastError());
 }
 
 int smetric_link_sessions(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
