@@ -1272,29 +1272,92 @@ uint64_t reuse_slots_for(int64_t n_blocks) {
   return g;
 }
 
-// Thread per block of the batch: its hash into the workspace table with the
-// earliest request holding it (pairs (hash, INT32_MAX - request), atomicMax).
+// The first table tried holds an eighth of the window's blocks at load 1/2
+// (67 MB for 16M blocks, so it stays in L2); windows whose distinct blocks
+// exceed that fall back on the device to the full table, sized for every
+// block distinct.
+uint64_t reuse_small_slots_for(int64_t n_blocks) { return reuse_slots_for((n_blocks + 7) / 8); }
+constexpr int kReuseSmallProbe = 64;  // longer probes in the first table also fall back
+
+// Workspace header after the table: [0] the fallback flag, [1] distinct keys
+// in the first table.
+struct ReuseHeader {
+  int32_t big;
+  uint32_t distinct;
+  int64_t pad;
+};
+
+// Warp per request, 32 blocks per round: each block's hash into the table
+// with the earliest request holding it and that request's session, packed as
+// (INT32_MAX - request) << 32 | session so that atomicMax keeps the earliest.
+// A slot that already names an earlier (or the same) request is left alone,
+// which spares most atomics: warps take requests in arrival order, so the
+// first holder of a shared block is usually in before its later ones. The
+// pre-checks are plain loads, so a block every request shares (a system
+// prompt) is read from L1; a stale copy only shows an empty key or a smaller
+// value, and both fall through to the atomics. The order of a request's
+// blocks does not matter, so each request starts at a round of its own and
+// wraps around, which spreads the requests in flight over the table.
+// BIG = false fills the first table and raises the fallback flag when it
+// runs full (more distinct keys than limit, or a probe longer than
+// kReuseSmallProbe); BIG = true runs only after that, on the cleared full
+// table.
+template <bool BIG>
 __global__ void __launch_bounds__(256)
     k_reuse_insert(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
-                   const uint64_t* __restrict__ H, uint64_t* __restrict__ table, uint64_t mask) {
+                   const uint64_t* __restrict__ H, const int32_t* __restrict__ sessions,
+                   uint64_t* __restrict__ table, uint64_t mask, ReuseHeader* hdr, uint32_t limit) {
   if (!*batch_ok) return;
-  const int64_t total = block_off[n];
-  int32_t r = 0;
-  for (int64_t f = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; f < total;
-       f += (int64_t)gridDim.x * blockDim.x) {
-    r = find_request(block_off, r, n, f);
-    const uint64_t key = H[f];
-    uint64_t s = key & mask;
-    for (uint64_t t = 0; t <= mask; ++t) {
-      unsigned long long* const slot = reinterpret_cast<unsigned long long*>(table + 2 * s);
-      const unsigned long long k = atomicCAS(slot, 0ull, (unsigned long long)key);
-      if (k == 0ull || k == key) {
-        atomicMax(slot + 1, (unsigned long long)(INT32_MAX - r));
-        break;
+  if (BIG && !__ldcg(&hdr->big)) return;
+  const int lane = threadIdx.x & 31;
+  const int64_t tw = (int64_t)gridDim.x * (blockDim.x >> 5);
+  for (int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n; r += tw) {
+    if (!BIG && __shfl_sync(kFull, lane == 0 ? __ldcg(&hdr->big) : 0, 0)) return;
+    const int64_t bo = block_off[r], nb = block_off[r + 1] - bo;
+    const unsigned long long val = ((unsigned long long)(INT32_MAX - r) << 32) | (uint32_t)sessions[r];
+    const int64_t rounds = (nb + 31) >> 5;
+    int64_t round = rounds ? r % rounds : 0;
+    uint32_t fresh_n = 0;
+    for (int64_t i = 0; i < rounds; ++i, round = round + 1 == rounds ? 0 : round + 1) {
+      const int64_t b = round * 32 + lane;
+      bool full = false;
+      if (b < nb) {
+        const uint64_t key = H[bo + b];
+        uint64_t s = key & mask;
+        const uint64_t probes = BIG ? mask + 1 : kReuseSmallProbe;
+        full = true;
+        for (uint64_t t = 0; t < probes; ++t) {
+          unsigned long long* const slot = reinterpret_cast<unsigned long long*>(table + 2 * s);
+          unsigned long long k = slot[0];
+          if (k == 0ull) {
+            k = atomicCAS(slot, 0ull, (unsigned long long)key);
+            fresh_n += k == 0ull;
+          }
+          if (k == 0ull || k == key) {
+            if (slot[1] < val) atomicMax(slot + 1, val);
+            full = false;
+            break;
+          }
+          s = (s + 1) & mask;
+        }
       }
-      s = (s + 1) & mask;
+      if (!BIG && __any_sync(kFull, full)) {
+        if (lane == 0) atomicExch(&hdr->big, 1);
+        return;
+      }
+    }
+    if (!BIG) {
+      for (int o = 16; o; o >>= 1) fresh_n += __shfl_xor_sync(kFull, fresh_n, o);
+      if (lane == 0 && fresh_n && atomicAdd(&hdr->distinct, fresh_n) + fresh_n > limit) atomicExch(&hdr->big, 1);
     }
   }
+}
+
+// Clears the full table once the first one has run full.
+__global__ void __launch_bounds__(256) k_reuse_clear(const ReuseHeader* hdr, uint4* table, int64_t n16) {
+  if (!*reinterpret_cast<const volatile int32_t*>(&hdr->big)) return;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n16; i += (int64_t)gridDim.x * blockDim.x)
+    table[i] = make_uint4(0, 0, 0, 0);
 }
 
 // Warp per request, 32 blocks per round: block b is reused when its earliest
@@ -1303,13 +1366,15 @@ __global__ void __launch_bounds__(256)
 // holder is of r's session) and inter-session.
 __global__ void __launch_bounds__(256)
     k_reuse_walk(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
-                 const uint64_t* __restrict__ H, const uint64_t* __restrict__ table, uint64_t mask,
-                 const int32_t* __restrict__ sessions, const int32_t* __restrict__ sys_blocks,
+                 const uint64_t* __restrict__ H, const uint64_t* __restrict__ table, uint64_t mask_small,
+                 uint64_t mask_big, const ReuseHeader* hdr, const int32_t* __restrict__ sessions,
+                 const int32_t* __restrict__ sys_blocks,
                  int32_t* __restrict__ hit, int32_t* __restrict__ sys, int32_t* __restrict__ intra,
                  int32_t* __restrict__ inter, int32_t* status) {
   const int lane = threadIdx.x & 31;
   const int64_t tw = (int64_t)gridDim.x * (blockDim.x >> 5);
   const bool ok = *batch_ok != 0;
+  const uint64_t mask = hdr->big ? mask_big : mask_small;
   for (int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n; r += tw) {
     int32_t nh = 0, ns = 0, ni = 0, ne = 0;
     if (ok) {
@@ -1322,13 +1387,18 @@ __global__ void __launch_bounds__(256)
       const int32_t sr = sessions[r];
       for (int64_t base = 0; base < nb; base += 32) {
         const int64_t b = base + lane;
-        int32_t producer = INT32_MAX;
+        int32_t producer = INT32_MAX, psess = 0;
         if (b < nb) {
           const uint64_t key = H[bo + b];
           uint64_t s = key & mask;
           for (uint64_t t = 0; t <= mask; ++t) {
             const uint64_t k = table[2 * s];
-            if (k == key) { producer = INT32_MAX - (int32_t)table[2 * s + 1]; break; }
+            if (k == key) {
+              const uint64_t v = table[2 * s + 1];
+              producer = INT32_MAX - (int32_t)(v >> 32);
+              psess = (int32_t)(uint32_t)v;
+              break;
+            }
             if (k == 0) break;
             s = (s + 1) & mask;
           }
@@ -1338,7 +1408,7 @@ __global__ void __launch_bounds__(256)
         const unsigned run = miss ? (1u << (__ffs(miss) - 1)) - 1 : kFull;  // lanes before the first miss
         const bool in = (run >> lane) & 1;
         const bool is_sys = in && b < sb;
-        const bool is_intra = in && !is_sys && sessions[producer] == sr;
+        const bool is_intra = in && !is_sys && psess == sr;
         nh += __popc(run);
         ns += __popc(__ballot_sync(kFull, is_sys));
         ni += __popc(__ballot_sync(kFull, is_intra));
@@ -1946,7 +2016,7 @@ int smetric_index_commit_batch(smetric_index* idx, const int64_t* d_offsets, int
 }
 
 int64_t smetric_reuse_workspace_bytes(int64_t n_blocks) {
-  return n_blocks < 0 ? 0 : (int64_t)(2 * sizeof(uint64_t) * reuse_slots_for(n_blocks));
+  return n_blocks < 0 ? 0 : (int64_t)(2 * sizeof(uint64_t) * reuse_slots_for(n_blocks) + sizeof(ReuseHeader));
 }
 
 int smetric_reuse_breakdown(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
@@ -1966,17 +2036,23 @@ int smetric_reuse_breakdown(smetric_index* idx, const int32_t* d_tokens, int64_t
   if ((rc = route_common<false>(idx, d_tokens, n_tokens, d_offsets, n_requests, nullptr, smetric_weights{0, 0, 0},
                                 nullptr, nullptr, nullptr, idx->sk_tmp, idx->hashes, n_blocks, s)))
     return rc;
-  const uint64_t slots = reuse_slots_for(n_blocks);
+  const uint64_t slots = reuse_slots_for(n_blocks), small = reuse_small_slots_for(n_blocks);
   uint64_t* table = static_cast<uint64_t*>(d_workspace);
-  if (cudaMemsetAsync(table, 0, 2 * sizeof(uint64_t) * slots, s) != cudaSuccess) return cuda_status(cudaErrorUnknown);
-  const int64_t want = (n_blocks + 255) / 256;
-  const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
-  k_reuse_insert<<<grid, 256, 0, s>>>(idx->block_off, n_requests, idx->batch_ok, idx->hashes, table, slots - 1);
+  ReuseHeader* hdr = reinterpret_cast<ReuseHeader*>(table + 2 * slots);
+  if (cudaMemsetAsync(table, 0, 2 * sizeof(uint64_t) * small, s) != cudaSuccess ||
+      cudaMemsetAsync(hdr, 0, sizeof(ReuseHeader), s) != cudaSuccess)
+    return cuda_status(cudaErrorUnknown);
   const unsigned wgrid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(((int64_t)n_requests + 7) / 8,
                                                                           (int64_t)idx->num_sms * 8));
-  k_reuse_walk<<<wgrid, 256, 0, s>>>(idx->block_off, n_requests, idx->batch_ok, idx->hashes, table, slots - 1,
-                                     d_sessions, d_sys_blocks, d_hit, d_sys, d_intra, d_inter, idx->status);
-  idx->launches += 2;
+  k_reuse_insert<false><<<wgrid, 256, 0, s>>>(idx->block_off, n_requests, idx->batch_ok, idx->hashes, d_sessions,
+                                              table, small - 1, hdr, (uint32_t)(small / 2));
+  k_reuse_clear<<<idx->num_sms * 8, 256, 0, s>>>(hdr, reinterpret_cast<uint4*>(table), (int64_t)slots);
+  k_reuse_insert<true><<<wgrid, 256, 0, s>>>(idx->block_off, n_requests, idx->batch_ok, idx->hashes, d_sessions,
+                                             table, slots - 1, hdr, 0);
+  k_reuse_walk<<<wgrid, 256, 0, s>>>(idx->block_off, n_requests, idx->batch_ok, idx->hashes, table, small - 1,
+                                     slots - 1, hdr, d_sessions, d_sys_blocks, d_hit, d_sys, d_intra, d_inter,
+                                     idx->status);
+  idx->launches += 4;
   return cuda_status(cudaGetLastError());
 }
 

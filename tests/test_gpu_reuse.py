@@ -152,6 +152,37 @@ def test_reuse_edge_cases():
     ix.close()
 
 
+def _first_table_limit(n_blocks):
+    """Distinct blocks the L2-sized first table takes before the kernels fall
+    back to the full table: half its slots, a power of two >= 2 ceil(n/8)."""
+    g = 64
+    while g < 2 * ((n_blocks + 7) // 8):
+        g <<= 1
+    return g // 2
+
+
+@pytest.mark.parametrize("distinct", [True, False])
+def test_reuse_first_table_and_fallback(distinct):
+    """All blocks distinct (the first table overflows, the full one takes
+    over) and few distinct (the first table holds them): both equal to the
+    oracle."""
+    rng = np.random.default_rng(17)
+    B, n = 4, 600
+    if distinct:
+        reqs = [rng.integers(0, 1 << 30, size=int(rng.integers(0, 60 * B)), dtype=np.int32) for _ in range(n)]
+    else:
+        pool = [rng.integers(0, 1 << 30, size=100 * B, dtype=np.int32) for _ in range(4)]
+        reqs = [pool[i % 4][:int(rng.integers(0, 100 * B))] for i in range(n)]
+    sessions = rng.integers(0, 3, size=n)
+    sys_b = rng.integers(0, 10, size=n)
+    g, o = _both(B, 1, reqs, sessions, sys_b)
+    _assert_equal(g, o, f"distinct={distinct}")
+    nb = np.array([len(r) // B for r in reqs])
+    fresh = int((nb - o["hit"]).sum())  # blocks no earlier request holds
+    limit = _first_table_limit(int(nb.sum()))
+    assert (fresh > limit) == distinct, (fresh, limit)
+
+
 def test_reuse_full_window_properties():
     """A whole c2_medium window (16,384 requests, 256M tokens) at once: the
     parts add up, first turns reuse no intra-session blocks, every
