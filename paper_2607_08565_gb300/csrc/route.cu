@@ -1284,8 +1284,20 @@ constexpr int kReuseSmallProbe = 64;  // longer probes in the first table also f
 struct ReuseHeader {
   int32_t big;
   uint32_t distinct;
-  int64_t pad;
+  uint32_t next[3];  // work counters of the two inserts and the walk
+  uint32_t pad[3];
 };
+
+// Warps take requests from a counter in arrival order, so that a warp done
+// with a short request takes the next one instead of idling behind a long one.
+__device__ __forceinline__ int64_t next_request(uint32_t* ctr, int lane) {
+  uint32_t r = 0;
+  if (lane == 0) r = atomicAdd(ctr, 1u);
+  return __shfl_sync(kFull, r, 0);
+}
+
+// Rounds of 32 blocks that a warp loads ahead before it uses them.
+constexpr int kReuseAhead = 4;
 
 // Warp per request, 32 blocks per round: each block's hash into the table
 // with the earliest request holding it and that request's session, packed as
@@ -1310,36 +1322,50 @@ __global__ void __launch_bounds__(256)
   if (!*batch_ok) return;
   if (BIG && !__ldcg(&hdr->big)) return;
   const int lane = threadIdx.x & 31;
-  const int64_t tw = (int64_t)gridDim.x * (blockDim.x >> 5);
-  for (int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n; r += tw) {
+  for (int64_t r = next_request(&hdr->next[BIG], lane); r < n; r = next_request(&hdr->next[BIG], lane)) {
     if (!BIG && __shfl_sync(kFull, lane == 0 ? __ldcg(&hdr->big) : 0, 0)) return;
     const int64_t bo = block_off[r], nb = block_off[r + 1] - bo;
     const unsigned long long val = ((unsigned long long)(INT32_MAX - r) << 32) | (uint32_t)sessions[r];
     const int64_t rounds = (nb + 31) >> 5;
-    int64_t round = rounds ? r % rounds : 0;
+    const int64_t start = rounds ? r % rounds : 0;
     uint32_t fresh_n = 0;
-    for (int64_t i = 0; i < rounds; ++i, round = round + 1 == rounds ? 0 : round + 1) {
-      const int64_t b = round * 32 + lane;
+    for (int64_t i = 0; i < rounds; i += kReuseAhead) {
+      int64_t b[kReuseAhead];
+      uint64_t key[kReuseAhead];
+      ulonglong2 sl[kReuseAhead];
+#pragma unroll
+      for (int u = 0; u < kReuseAhead; ++u) {
+        int64_t rd = start + i + u;
+        rd = rd >= rounds ? rd - rounds : rd;
+        b[u] = i + u < rounds ? rd * 32 + lane : nb;
+        key[u] = b[u] < nb ? H[bo + b[u]] : 0;
+      }
+#pragma unroll
+      for (int u = 0; u < kReuseAhead; ++u)
+        if (b[u] < nb) sl[u] = *reinterpret_cast<const ulonglong2*>(table + 2 * (key[u] & mask));
       bool full = false;
-      if (b < nb) {
-        const uint64_t key = H[bo + b];
-        uint64_t s = key & mask;
+#pragma unroll
+      for (int u = 0; u < kReuseAhead; ++u) {
+        // already held by this or an earlier request: nothing to do
+        if (b[u] >= nb || (sl[u].x == key[u] && sl[u].y >= val)) continue;
+        uint64_t s = key[u] & mask;
         const uint64_t probes = BIG ? mask + 1 : kReuseSmallProbe;
-        full = true;
+        bool placed = false;
         for (uint64_t t = 0; t < probes; ++t) {
           unsigned long long* const slot = reinterpret_cast<unsigned long long*>(table + 2 * s);
           unsigned long long k = slot[0];
           if (k == 0ull) {
-            k = atomicCAS(slot, 0ull, (unsigned long long)key);
+            k = atomicCAS(slot, 0ull, (unsigned long long)key[u]);
             fresh_n += k == 0ull;
           }
-          if (k == 0ull || k == key) {
+          if (k == 0ull || k == key[u]) {
             if (slot[1] < val) atomicMax(slot + 1, val);
-            full = false;
+            placed = true;
             break;
           }
           s = (s + 1) & mask;
         }
+        full |= !placed;
       }
       if (!BIG && __any_sync(kFull, full)) {
         if (lane == 0) atomicExch(&hdr->big, 1);
@@ -1367,15 +1393,14 @@ __global__ void __launch_bounds__(256) k_reuse_clear(const ReuseHeader* hdr, uin
 __global__ void __launch_bounds__(256)
     k_reuse_walk(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
                  const uint64_t* __restrict__ H, const uint64_t* __restrict__ table, uint64_t mask_small,
-                 uint64_t mask_big, const ReuseHeader* hdr, const int32_t* __restrict__ sessions,
+                 uint64_t mask_big, ReuseHeader* hdr, const int32_t* __restrict__ sessions,
                  const int32_t* __restrict__ sys_blocks,
                  int32_t* __restrict__ hit, int32_t* __restrict__ sys, int32_t* __restrict__ intra,
                  int32_t* __restrict__ inter, int32_t* status) {
   const int lane = threadIdx.x & 31;
-  const int64_t tw = (int64_t)gridDim.x * (blockDim.x >> 5);
   const bool ok = *batch_ok != 0;
   const uint64_t mask = hdr->big ? mask_big : mask_small;
-  for (int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n; r += tw) {
+  for (int64_t r = next_request(&hdr->next[2], lane); r < n; r = next_request(&hdr->next[2], lane)) {
     int32_t nh = 0, ns = 0, ni = 0, ne = 0;
     if (ok) {
       const int64_t bo = block_off[r], nb = block_off[r + 1] - bo;
@@ -1385,35 +1410,51 @@ __global__ void __launch_bounds__(256)
         sb = 0;
       }
       const int32_t sr = sessions[r];
-      for (int64_t base = 0; base < nb; base += 32) {
-        const int64_t b = base + lane;
-        int32_t producer = INT32_MAX, psess = 0;
-        if (b < nb) {
-          const uint64_t key = H[bo + b];
-          uint64_t s = key & mask;
-          for (uint64_t t = 0; t <= mask; ++t) {
-            const uint64_t k = table[2 * s];
-            if (k == key) {
-              const uint64_t v = table[2 * s + 1];
-              producer = INT32_MAX - (int32_t)(v >> 32);
-              psess = (int32_t)(uint32_t)v;
-              break;
+      bool stop = false;
+      for (int64_t base = 0; base < nb && !stop; base += 32 * kReuseAhead) {
+        uint64_t key[kReuseAhead];
+        ulonglong2 sl[kReuseAhead];
+#pragma unroll
+        for (int u = 0; u < kReuseAhead; ++u) {
+          const int64_t b = base + 32 * u + lane;
+          key[u] = b < nb ? H[bo + b] : 0;
+        }
+#pragma unroll
+        for (int u = 0; u < kReuseAhead; ++u)
+          if (base + 32 * u + lane < nb) sl[u] = *reinterpret_cast<const ulonglong2*>(table + 2 * (key[u] & mask));
+#pragma unroll
+        for (int u = 0; u < kReuseAhead; ++u) {
+          const int64_t b = base + 32 * u + lane;
+          int32_t producer = INT32_MAX, psess = 0;
+          if (b < nb) {
+            uint64_t s = key[u] & mask;
+            ulonglong2 e = sl[u];
+            for (uint64_t t = 0; t <= mask; ++t) {
+              if (e.x == key[u]) {
+                producer = INT32_MAX - (int32_t)(e.y >> 32);
+                psess = (int32_t)(uint32_t)e.y;
+                break;
+              }
+              if (e.x == 0) break;
+              s = (s + 1) & mask;
+              e = *reinterpret_cast<const ulonglong2*>(table + 2 * s);
             }
-            if (k == 0) break;
-            s = (s + 1) & mask;
+          }
+          const bool reused = b < nb && producer < r;
+          const unsigned miss = __ballot_sync(kFull, !reused);
+          const unsigned run = miss ? (1u << (__ffs(miss) - 1)) - 1 : kFull;  // lanes before the first miss
+          const bool in = (run >> lane) & 1;
+          const bool is_sys = in && b < sb;
+          const bool is_intra = in && !is_sys && psess == sr;
+          nh += __popc(run);
+          ns += __popc(__ballot_sync(kFull, is_sys));
+          ni += __popc(__ballot_sync(kFull, is_intra));
+          ne += __popc(__ballot_sync(kFull, in && !is_sys && !is_intra));
+          if (miss) {
+            stop = true;
+            break;
           }
         }
-        const bool reused = b < nb && producer < r;
-        const unsigned miss = __ballot_sync(kFull, !reused);
-        const unsigned run = miss ? (1u << (__ffs(miss) - 1)) - 1 : kFull;  // lanes before the first miss
-        const bool in = (run >> lane) & 1;
-        const bool is_sys = in && b < sb;
-        const bool is_intra = in && !is_sys && psess == sr;
-        nh += __popc(run);
-        ns += __popc(__ballot_sync(kFull, is_sys));
-        ni += __popc(__ballot_sync(kFull, is_intra));
-        ne += __popc(__ballot_sync(kFull, in && !is_sys && !is_intra));
-        if (miss) break;
       }
     }
     if (lane == 0) {
