@@ -66,6 +66,9 @@ def parse():
     ap.add_argument("--reuse", action="store_true",
                     help="time the KV$ reuse breakdown (Section 3.1) over a whole config-2 window "
                          "(one GPU; its own line)")
+    ap.add_argument("--imbalance", action="store_true",
+                    help="time the windowed load imbalance (Section 3.2) over a day of running intervals "
+                         "(one GPU; its own line)")
     ap.add_argument("--coloc", action="store_true",
                     help="with --policy: the PD-colocation variant (Appendix B)")
     ap.add_argument("--policy", action="store_true",
@@ -924,6 +927,62 @@ def run_reuse(args, k_sessions=20):
 
 
 # ---------------------------------------------------------------------------
+# windowed load imbalance over a day of running intervals
+# ---------------------------------------------------------------------------
+
+def run_imbalance(args, n_requests=3_456_000, num_instances=32, window=30_000, n_windows=2_880, sample=400_000):
+    import torch
+    import oracle
+    import paper_2607_08565_gb300 as pkg
+    from paper_2607_08565_gb300 import build_lib
+    from synth import running_intervals
+
+    build_lib.build()
+    torch.cuda.set_device(0)
+    inst, start, end = running_intervals(n_requests, num_instances, seed=4)
+    ix = pkg.SMetricIndex(num_instances, 16, 1, capacity_slots=1 << 10, max_batch_requests=1,
+                          max_batch_tokens=16)
+    d = [torch.from_numpy(np.ascontiguousarray(a)).cuda() for a in (inst, start, end)]
+    ws = torch.empty(pkg.smetric_imbalance_workspace_bytes(n_windows, num_instances) // 8, dtype=torch.int64,
+                     device="cuda")
+    for _ in range(3):
+        out = ix.window_imbalance(*d, window, n_windows, workspace=ws)
+    torch.cuda.synchronize()
+    ix.check()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    steps = 20
+    e0.record()
+    for _ in range(steps):
+        ix.window_imbalance(*d, window, n_windows, workspace=ws)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    g = {k: v.cpu().numpy() for k, v in out.items()}
+    # the oracle on the first requests, over the windows they reach, as a window set of its own
+    m = sample
+    nw_s = int(end[:m].max() // window) + 1
+    t0 = time.perf_counter()
+    o = oracle.window_imbalance(num_instances, window, nw_s, inst[:m], start[:m], end[:m])
+    dt = time.perf_counter() - t0
+    sg = ix.window_imbalance(*(x[:m] for x in d), window, nw_s)
+    ix.check()
+    if any(not np.array_equal(o[k], sg[k].cpu().numpy()) for k in o):
+        raise RuntimeError("window imbalance differs from the oracle")
+    busy = g["sum"] > 0
+    imb = num_instances * g["max"][busy] / g["sum"][busy]
+    line = {"metric": "requests folded into windowed load imbalance per second (Section 3.2)",
+            "value": n_requests / (ms / 1e3), "unit": "requests/s", "n_gpus": 1, "steps": steps, "warmup": 3,
+            "ms_per_step": ms, "higher_is_better": True, "data": "synthetic",
+            "config": {"workload": f"{n_requests} running intervals over a day, {num_instances} instances, "
+                                   f"{n_windows} windows of {window} ms, one call",
+                       "imbalance_p50": float(np.median(imb)), "imbalance_p95": float(np.percentile(imb, 95))},
+            "cpu_baseline": {"value": m / dt, "unit": "requests/s", "cores": 1, "kind": "oracle",
+                             "sample": f"first {m} requests over their {nw_s} windows ({dt:.1f} s, one thread)"}}
+    print(json.dumps(line), flush=True)
+    ix.close()
+
+
+# ---------------------------------------------------------------------------
 # device-side index maintenance over a config-2 replay
 # ---------------------------------------------------------------------------
 
@@ -1107,6 +1166,9 @@ def main():
         return
     if args.reuse:
         run_reuse(args)
+        return
+    if args.imbalance:
+        run_imbalance(args)
         return
     rank, world, local, dist = dist_setup(args)
     if args.impl == "reference":

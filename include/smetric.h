@@ -269,6 +269,34 @@ int smetric_reuse_breakdown(smetric_index* idx, const int32_t* d_tokens, int64_t
                             int32_t* d_hit, int32_t* d_sys, int32_t* d_intra, int32_t* d_inter,
                             smetric_stream_t stream);
 
+/* Windowed load imbalance (Section 3.2, Figure 3(c)): an instance's load in
+ * a time window is its average number of running requests there; the
+ * window's imbalance is the maximum load over the mean across the index's N
+ * instances. Request r runs on instance d_instance[r] over the integer time
+ * interval [d_start[r], d_end[r]) (ticks of the caller's choosing). Window
+ * w < n_windows is [w*window, (w+1)*window); running time after the last
+ * window is not counted. With S_i(w) the ticks instance i's requests run
+ * inside window w, the outputs (device, [n_windows]) are d_max[w] =
+ * max_i S_i(w) (int64), d_argmax[w] = the lowest instance attaining it
+ * (int32) and d_sum[w] = sum_i S_i(w) (int64); the imbalance is
+ * N * d_max[w] / d_sum[w] (no running request: all three are 0). The caller
+ * provides an 8-byte aligned device workspace of at least
+ * smetric_imbalance_workspace_bytes(n_windows, N) bytes. Limits: 1 <= window
+ * <= SMETRIC_IMBALANCE_MAX_WINDOW, n_windows * window <= 2^62, n_requests <=
+ * SMETRIC_IMBALANCE_MAX_REQUESTS, n_windows * N <= SMETRIC_IMBALANCE_MAX_CELLS
+ * (else INVALID_ARG before any launch). A request with an instance outside
+ * [0, N), a negative start or end < start latches INVALID_ARG and is left
+ * out; the others are counted. Does not touch the index's tables or route
+ * scratch. */
+#define SMETRIC_IMBALANCE_MAX_WINDOW (1LL << 36)
+#define SMETRIC_IMBALANCE_MAX_REQUESTS (1 << 26)
+#define SMETRIC_IMBALANCE_MAX_CELLS (1LL << 31)
+int64_t smetric_imbalance_workspace_bytes(int32_t n_windows, int32_t num_instances);
+int smetric_window_imbalance(smetric_index* idx, const int32_t* d_instance, const int64_t* d_start,
+                             const int64_t* d_end, int32_t n_requests, int64_t window, int32_t n_windows,
+                             void* d_workspace, int64_t workspace_bytes, int64_t* d_max, int32_t* d_argmax,
+                             int64_t* d_sum, smetric_stream_t stream);
+
 /* Session reconstruction from block hashes (Appendix A): in a batch of
  * requests in arrival order, request r follows the latest earlier request p
  * of the same user (d_users) with d_turns[p] = d_turns[r] - 1 whose

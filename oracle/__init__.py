@@ -79,6 +79,9 @@ def load_library(path: str):
     L.oracle_reuse_breakdown.restype = C.c_int
     L.oracle_reuse_breakdown.argtypes = [C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i32p, i32p,
                                          i32p, i32p, i32p, i32p]
+    L.oracle_window_imbalance.restype = C.c_int
+    L.oracle_window_imbalance.argtypes = [C.c_int32, C.c_int64, C.c_int32, i32p, i64p, i64p, C.c_int32, i64p, i32p,
+                                          i64p]
     L.oracle_link_sessions.restype = C.c_int
     L.oracle_link_sessions.argtypes = [C.c_int32, C.c_uint64, i32p, i64p, C.c_int32, i64p, i32p, i32p, i32p]
     return L
@@ -139,6 +142,24 @@ def reuse_breakdown(block_size: int, seed: int, tokens, offsets, sessions, sys_b
     if rc != 0:
         raise ValueError(f"oracle_reuse_breakdown: {rc}")
     return dict(zip(("hit", "sys", "intra", "inter"), (x[:n] for x in outs)))
+
+
+def window_imbalance(num_instances: int, window: int, n_windows: int, instance, start, end, L=None):
+    """Per window of `window` ticks: dict(max, argmax, sum) of the instances'
+    running-request ticks; the imbalance is num_instances * max / sum."""
+    inst = np.ascontiguousarray(instance, dtype=np.int32)
+    st = np.ascontiguousarray(start, dtype=np.int64)
+    en = np.ascontiguousarray(end, dtype=np.int64)
+    n = len(inst)
+    m = max(n_windows, 1)
+    mx, am, sm = np.zeros(m, np.int64), np.zeros(m, np.int32), np.zeros(m, np.int64)
+    rc = (L or lib()).oracle_window_imbalance(num_instances, window, n_windows,
+                                              inst if n else np.zeros(1, np.int32),
+                                              st if n else np.zeros(1, np.int64),
+                                              en if n else np.zeros(1, np.int64), n, mx, am, sm)
+    if rc != 0:
+        raise ValueError(f"oracle_window_imbalance: {rc}")
+    return dict(max=mx[:n_windows], argmax=am[:n_windows], sum=sm[:n_windows])
 
 
 class OracleIndex:

@@ -108,6 +108,16 @@
  * when b < sys_r (the request's leading system-prompt blocks), else
  * intra-session when session_p = session_r, else inter-session.
  *
+ * Windowed load imbalance (Section 3.2, Figure 3(c); oracle_window_imbalance):
+ * request r runs on instance inst_r over the integer time interval
+ * [start_r, end_r). Window w is [w*T, (w+1)*T). Instance i's load in window w
+ * is its average number of running requests there, S_i(w) / T with
+ *    S_i(w) = sum over r with inst_r = i of |[start_r, end_r) ∩ window w|
+ * (running-request time in ticks), and the window's imbalance is the maximum
+ * load over the mean across all N instances, N * max_i S_i(w) / sum_i S_i(w).
+ * Outputs per window: max_i S_i(w), its lowest maximising instance, and
+ * sum_i S_i(w) (exact integers; the ratio is formed by the caller).
+ *
  * Session reconstruction (Appendix A; oracle_link_sessions): request r
  * follows request p when p is earlier (p < r, requests in arrival order), of
  * the same user, of turn turn_r - 1, and p's block-hash sequence is a prefix
@@ -730,5 +740,38 @@ int oracle_reuse_breakdown(int32_t B, uint64_t seed, const int32_t* tokens, cons
   }
   free(h);
   free(first);
+  return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Windowed load imbalance                                                   */
+/* ------------------------------------------------------------------------ */
+
+int oracle_window_imbalance(int32_t N, int64_t T, int32_t n_windows, const int32_t* inst, const int64_t* start,
+                            const int64_t* end, int32_t n_requests, int64_t* out_max, int32_t* out_argmax,
+                            int64_t* out_sum) {
+  if (N < 1 || T < 1 || n_windows < 0 || n_requests < 0) return ORACLE_ERR_INVALID_ARG;
+  for (int32_t r = 0; r < n_requests; ++r)
+    if (inst[r] < 0 || inst[r] >= N || start[r] < 0 || end[r] < start[r]) return ORACLE_ERR_INVALID_ARG;
+  for (int32_t w = 0; w < n_windows; ++w) {
+    const int64_t lo = (int64_t)w * T, hi = lo + T;
+    out_max[w] = 0;
+    out_argmax[w] = 0;
+    out_sum[w] = 0;
+    for (int32_t i = 0; i < N; ++i) {
+      int64_t s = 0; /* running-request ticks of instance i in window w */
+      for (int32_t r = 0; r < n_requests; ++r) {
+        if (inst[r] != i) continue;
+        const int64_t a = start[r] > lo ? start[r] : lo;
+        const int64_t b = end[r] < hi ? end[r] : hi;
+        if (b > a) s += b - a;
+      }
+      out_sum[w] += s;
+      if (s > out_max[w]) {
+        out_max[w] = s;
+        out_argmax[w] = i;
+      }
+    }
+  }
   return ORACLE_OK;
 }

@@ -37,6 +37,9 @@ SMETRIC_POLICY_MAX_QUEUED = 1 << 59
 SMETRIC_COMMIT_GLOBAL = 1
 SMETRIC_POLICY_MAX_TPOT = 1 << 60
 SMETRIC_POLICY_MAX_REQUESTS = 1 << 20
+SMETRIC_IMBALANCE_MAX_WINDOW = 1 << 36
+SMETRIC_IMBALANCE_MAX_REQUESTS = 1 << 26
+SMETRIC_IMBALANCE_MAX_CELLS = 1 << 31
 SMETRIC_SCORER_BAILIAN = 1
 SMETRIC_SCORER_LMETRIC = 2
 
@@ -49,7 +52,7 @@ EXPORTED = (
     "smetric_launch_count", "smetric_block_hashes_noalloc", "smetric_route_batch_policy",
     "smetric_index_commit_batch", "smetric_route_batch_policy_coloc", "smetric_link_sessions",
     "smetric_route_batch_baseline", "smetric_route_batch_sequential", "smetric_reuse_workspace_bytes",
-    "smetric_reuse_breakdown",
+    "smetric_reuse_breakdown", "smetric_imbalance_workspace_bytes", "smetric_window_imbalance",
 )
 
 
@@ -114,6 +117,8 @@ def lib():
             "smetric_index_commit_batch": (C.c_int, [P, P, I32, P, P, P, I32, P, P]),
             "smetric_link_sessions": (C.c_int, [P, P, I64, P, I32, P, P, P, P, P]),
             "smetric_reuse_workspace_bytes": (I64, [I64]),
+            "smetric_imbalance_workspace_bytes": (I64, [I32, I32]),
+            "smetric_window_imbalance": (C.c_int, [P, P, P, P, I32, I64, I32, P, I64, P, P, P, P]),
             "smetric_reuse_breakdown": (C.c_int, [P, P, I64, P, I32, P, P, P, I64, P, P, P, P, P]),
             "smetric_route_batch_sequential": (C.c_int, [P, P, I64, P, I32, P, smetric_weights, P, P, P, P, P,
                                                          I64, P, P]),
@@ -285,6 +290,18 @@ def smetric_reuse_breakdown(idx: int, d_tokens, n_tokens: int, d_offsets, n_requ
                                          _ptr(d_sessions), _ptr(d_sys_blocks), _ptr(d_workspace), workspace_bytes,
                                          _ptr(d_hit), _ptr(d_sys), _ptr(d_intra), _ptr(d_inter), _stream(stream)),
            "smetric_reuse_breakdown")
+
+
+def smetric_imbalance_workspace_bytes(n_windows: int, num_instances: int) -> int:
+    return int(lib().smetric_imbalance_workspace_bytes(n_windows, num_instances))
+
+
+def smetric_window_imbalance(idx: int, d_instance, d_start, d_end, n_requests: int, window: int, n_windows: int,
+                             d_workspace, workspace_bytes: int, d_max, d_argmax, d_sum, stream=None) -> None:
+    _check(lib().smetric_window_imbalance(idx, _ptr(d_instance), _ptr(d_start), _ptr(d_end), n_requests, window,
+                                          n_windows, _ptr(d_workspace), workspace_bytes, _ptr(d_max),
+                                          _ptr(d_argmax), _ptr(d_sum), _stream(stream)),
+           "smetric_window_imbalance")
 
 
 def smetric_link_sessions(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int, d_users, d_turns,
@@ -527,6 +544,22 @@ class SMetricIndex:
         out = {k: torch.empty(n, dtype=torch.int32, device=dev) for k in ("hit", "sys", "intra", "inter")}
         smetric_reuse_breakdown(self.handle, tokens, tokens.numel(), offsets, n, sessions, sys_blocks, workspace,
                                 workspace.numel(), out["hit"], out["sys"], out["intra"], out["inter"], stream)
+        return out
+
+    def window_imbalance(self, instance, start, end, window: int, n_windows: int, workspace=None, stream=None):
+        """Per window: dict(max, argmax, sum) of the instances' running-request
+        ticks; the imbalance is N * max / sum."""
+        import torch
+        dev = start.device
+        if workspace is None:
+            workspace = torch.empty(max(1, smetric_imbalance_workspace_bytes(n_windows, self.N) // 8),
+                                    dtype=torch.int64, device=dev)
+        out = dict(max=torch.empty(n_windows, dtype=torch.int64, device=dev),
+                   argmax=torch.empty(n_windows, dtype=torch.int32, device=dev),
+                   sum=torch.empty(n_windows, dtype=torch.int64, device=dev))
+        smetric_window_imbalance(self.handle, instance, start, end, instance.numel(), window, n_windows, workspace,
+                                 workspace.numel() * workspace.element_size(), out["max"], out["argmax"],
+                                 out["sum"], stream)
         return out
 
     def link_sessions(self, tokens, offsets, users, turns, stream=None):

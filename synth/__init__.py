@@ -24,3 +24,4 @@ from .traces import (  # noqa: F401
     TRACE_CONFIGS,
 )
 from .replay import ReplayDriver  # noqa: F401
+from .intervals import running_intervals  # noqa: F401

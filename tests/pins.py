@@ -901,6 +901,76 @@ def check_reuse_on_a_multi_turn_trace(L):
     assert out["intra"].sum() > 0 and out["sys"].sum() > 0
 
 
+def _tick_loads(N, T, n_windows, inst, start, end):
+    """Running requests counted tick by tick: S_i(w) = sum over the ticks t of
+    window w of the requests on i with start <= t < end."""
+    S = np.zeros((n_windows, N), np.int64)
+    for w in range(n_windows):
+        for t in range(w * T, (w + 1) * T):
+            for i_, s_, e_ in zip(inst, start, end):
+                if s_ <= t < e_:
+                    S[w, i_] += 1
+    return S
+
+
+def check_imbalance_against_tick_counts(L):
+    """Brute force in discrete time: every tick of a window, count each
+    instance's running requests; the sums, their maximum (lowest instance on
+    ties) and their total per window."""
+    rng = np.random.default_rng(31)
+    for trial in range(150):
+        N = int(rng.integers(1, 6))
+        T = int(rng.integers(1, 8))
+        nw = int(rng.integers(0, 7))
+        n = int(rng.integers(0, 20))
+        inst = rng.integers(0, N, size=n)
+        start = rng.integers(0, 45, size=n)
+        end = start + rng.integers(0, 25, size=n)
+        out = oracle.window_imbalance(N, T, nw, inst, start, end, L)
+        S = _tick_loads(N, T, nw, inst, start, end)
+        assert np.array_equal(out["sum"], S.sum(axis=1)), trial
+        assert np.array_equal(out["max"], S.max(axis=1) if nw else S.sum(axis=1)), trial
+        assert np.array_equal(out["argmax"], S.argmax(axis=1) if nw else np.zeros(0)), trial
+
+
+def check_imbalance_special_cases(L):
+    """One instance: the maximum is the total (imbalance 1). Equal requests
+    dealt round-robin: every instance carries the same load (N max = sum).
+    Everything on one instance: that instance, and max = sum (imbalance N).
+    Conservation: the windows' totals add up to the requests' running time
+    inside the covered span; windows twice as long add pairs of totals."""
+    rng = np.random.default_rng(32)
+    n = 200
+    start = rng.integers(0, 5000, size=n)
+    end = start + rng.integers(0, 3000, size=n)
+    one = oracle.window_imbalance(1, 300, 20, np.zeros(n, np.int32), start, end, L)
+    assert np.array_equal(one["max"], one["sum"]) and (one["argmax"] == 0).all()
+    N = 8
+    rr = oracle.window_imbalance(N, 100, 30, np.arange(8 * 50) % N, np.repeat(np.arange(50) * 37, 8),
+                                 np.repeat(np.arange(50) * 37 + 450, 8), L)
+    assert np.array_equal(N * rr["max"], rr["sum"]) and rr["sum"].any()
+    assert (rr["argmax"][rr["sum"] > 0] == 0).all()
+    hot = oracle.window_imbalance(N, 300, 20, np.full(n, 5, np.int32), start, end, L)
+    busy = hot["sum"] > 0
+    assert np.array_equal(hot["max"], hot["sum"]) and (hot["argmax"][busy] == 5).all()
+    inst = rng.integers(0, N, size=n)
+    a = oracle.window_imbalance(N, 250, 32, inst, start, end, L)
+    covered = np.clip(end, 0, 250 * 32) - np.clip(start, 0, 250 * 32)
+    assert a["sum"].sum() == covered.sum()
+    b = oracle.window_imbalance(N, 500, 16, inst, start, end, L)
+    assert np.array_equal(b["sum"], a["sum"][0::2] + a["sum"][1::2])
+    assert (b["max"] <= a["max"][0::2] + a["max"][1::2]).all()
+    # an idle window reports zeros; invalid requests are refused
+    idle = oracle.window_imbalance(N, 10, 3, [1], [100], [200], L)
+    assert not idle["max"].any() and not idle["sum"].any() and not idle["argmax"].any()
+    for bad in (([N], [0], [1]), ([-1], [0], [1]), ([0], [-1], [1]), ([0], [5], [4])):
+        try:
+            oracle.window_imbalance(N, 10, 3, *bad, L)
+        except ValueError:
+            continue
+        raise AssertionError(bad)
+
+
 ALL_CHECKS = [
     check_published_vector,
     check_bijection,
@@ -937,4 +1007,6 @@ ALL_CHECKS = [
     check_sequential_join_shortest_queue,
     check_reuse_against_token_prefixes,
     check_reuse_on_a_multi_turn_trace,
+    check_imbalance_against_tick_counts,
+    check_imbalance_special_cases,
 ]

@@ -68,6 +68,30 @@ def test_create_rejects_bad_config_on_host(L, bad):
     assert rc == pkg.SMETRIC_ERR_INVALID_ARG and not h
 
 
+def test_binding_constants_match_the_header():
+    """Every #define SMETRIC_* value in the header equals the binding's."""
+    text = open(os.path.join(ROOT, "include", "smetric.h")).read()
+    seen = 0
+    for name, expr in re.findall(r"^#define (SMETRIC_\w+) ([^/\n]+)", text, re.M):
+        if name == "SMETRIC_H":
+            continue
+        value = eval(expr.replace("LL", "").strip(), {})
+        assert getattr(pkg, name) == value, name
+        seen += 1
+    assert seen >= 15
+
+
+def test_workspace_sizes(L):
+    # the reuse table: 16-byte slots for twice the blocks (a power of two, at least 64) and a 32-byte header
+    assert L.smetric_reuse_workspace_bytes(0) == 16 * 64 + 32
+    assert L.smetric_reuse_workspace_bytes(1000) == 16 * 2048 + 32
+    assert L.smetric_reuse_workspace_bytes(1024) == 16 * 2048 + 32
+    assert L.smetric_reuse_workspace_bytes(-1) == 0
+    # the imbalance grid: one int64 per (window, instance)
+    assert L.smetric_imbalance_workspace_bytes(30, 32) == 8 * 30 * 32
+    assert L.smetric_imbalance_workspace_bytes(-1, 32) == 0
+
+
 def test_null_handles_are_rejected(L):
     assert L.smetric_index_create(None, None) == pkg.SMETRIC_ERR_INVALID_ARG
     assert L.smetric_index_destroy(None) == pkg.SMETRIC_OK
@@ -78,6 +102,10 @@ def test_null_handles_are_rejected(L):
                                         pkg.smetric_policy(1, 1, 0, 0, 1, 2, 0, 0), None, None, None,
                                         None, None, None, 0, None) == pkg.SMETRIC_ERR_INVALID_ARG
     assert L.smetric_status(None, None) == pkg.SMETRIC_ERR_INVALID_ARG
+    assert L.smetric_reuse_breakdown(None, None, 0, None, 1, None, None, None, 0, None, None, None, None,
+                                     None) == pkg.SMETRIC_ERR_INVALID_ARG
+    assert L.smetric_window_imbalance(None, None, None, None, 0, 1, 1, None, 0, None, None, None,
+                                      None) == pkg.SMETRIC_ERR_INVALID_ARG
     assert L.smetric_index_mask_words(None) == 0
     assert L.smetric_launch_count(None) == 0
 

@@ -88,6 +88,12 @@ MUTANTS = {
     "reuse_self_hit": ("for (int32_t p = 0; p < r && producer < 0; ++p)",
                        "for (int32_t p = 0; p <= r && producer < 0; ++p)"),
     "reuse_system_by_session": ("if (b < sys_blocks[r]) sys[r]++;", "if (b < sys_blocks[r] && sessions[producer] != sessions[r]) sys[r]++;"),
+    "imbalance_window_end_inclusive": ("const int64_t b = end[r] < hi ? end[r] : hi;",
+                                       "const int64_t b = end[r] < hi + 1 ? end[r] : hi + 1;"),
+    "imbalance_counts_request_length": ("if (b > a) s += b - a;", "if (b > a) s += end[r] - start[r];"),
+    "imbalance_tie_to_highest": ("if (s > out_max[w]) {", "if (s >= out_max[w]) {"),
+    "imbalance_window_origin": ("const int64_t lo = (int64_t)w * T, hi = lo + T;",
+                                "const int64_t lo = (int64_t)w * T + 1, hi = lo + T;"),
     "coloc_product_64_bit": ("(unsigned __int128)(uint64_t)est2[i] * (uint64_t)num_requests[i];",
                              "(unsigned __int128)((uint64_t)est2[i] * (uint64_t)num_requests[i]);"),
 }
