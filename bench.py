@@ -231,7 +231,10 @@ def populate_index(ix, tr, device, chunk=4096):
 def algorithmic_bytes(lens, local_hit, global_hit, B, W):
     """Per-kernel bytes of one route call. k_digest: 4 B per hashed token (the
     method must read every token of every full block). k_probe: one index
-    entry (key + W mask words) per probed block, P_r = min(n_r, reach_r + 1).
+    entry (key + W mask words) per probed block, P_r = min(n_r, reach_r + 1),
+    with reach_r taken from the chosen instance's hits, g_{i*} = max(c_{i*}, g):
+    never above max(max_i c_i, g), and equal to it when the global tier holds
+    every local tier's blocks (config 4), so the count never overstates.
     k_chain: the digests it reads and hashes it writes (intermediates of this
     kernel split). k_walk: the masks it reads, offsets and outputs. k_prep:
     offsets and loads. path: the method's bytes per request,
