@@ -253,6 +253,29 @@ def algorithmic_bytes(lens, local_hit, global_hit, B, W):
     }
 
 
+def route_stats(lens_per_batch, outs_per_batch, num_instances):
+    """Serving-side view of the routed batches (the paper's reuse and
+    imbalance metrics, Sections 3.1-3.2, taken from the route's outputs):
+    the share of prompt tokens hit in the chosen instance's local tier and
+    fetched from the global tier, and the routed-token imbalance of each
+    batch, N * max_i (tokens routed to i) / (all tokens), averaged over the
+    batches."""
+    tok = loc = glob = 0
+    imb = []
+    for lens, o in zip(lens_per_batch, outs_per_batch):
+        lens = np.asarray(lens, np.int64)
+        tok += int(lens.sum())
+        loc += int(np.asarray(o["local_hit"], np.int64).sum())
+        glob += int(np.asarray(o["global_hit"], np.int64).sum())
+        per = np.bincount(np.asarray(o["instance"], np.int64), weights=lens, minlength=num_instances)
+        if per.sum() > 0:
+            imb.append(float(num_instances * per.max() / per.sum()))
+    return {"local_hit_ratio": loc / tok if tok else 0.0,
+            "global_hit_ratio": glob / tok if tok else 0.0,
+            "routed_token_imbalance": float(np.mean(imb)) if imb else None,
+            "batches": len(imb)}
+
+
 # ---------------------------------------------------------------------------
 # CPU oracle timing
 # ---------------------------------------------------------------------------
@@ -519,6 +542,7 @@ def run_ours(args, rank, world, local, dist):
             "roofline_path": {"achieved": path_gbs, "frac": path_gbs / peak,
                               "algorithmic_bytes_per_step": algo_mean["path"]},
             "kernels_ms_per_launch": {k: v[0] / max(v[1], 1) for k, v in prof.items()},
+            "route_stats": route_stats([b.lengths() for b in host], per_batch, N),
             "clocks": clk,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "steps": args.e2e_steps},

@@ -1,7 +1,8 @@
 """Host-side logic of bench.py, on the CPU: the algorithmic byte counts that
 the roofline fractions divide, the clock-record parsing that decides whether
-a measurement stands, and the keying of the committed ncu traffic to the
-kernel source it was taken on."""
+a measurement stands, the keying of the committed ncu traffic to the
+kernel source it was taken on, and the routed batches' hit and imbalance
+statistics."""
 
 import json
 import os
@@ -125,3 +126,40 @@ def test_peak_falls_back_only_without_a_measurement(tmp_path, monkeypatch):
     assert bench.peak_hbm() == (6800.0, "fallback")
     (tmp_path / "MEASURED_PEAKS.json").write_text(json.dumps({"hbm_gbs": 6798.6}))
     assert bench.peak_hbm() == (6798.6, "measured")
+
+
+def test_route_stats_hand_example():
+    lens = [np.array([100, 50, 30, 20], np.int64), np.array([10, 10], np.int64)]
+    outs = [dict(instance=np.array([0, 1, 0, 2], np.int32), local_hit=np.array([64, 0, 16, 0], np.int32),
+                 global_hit=np.array([32, 48, 0, 0], np.int32)),
+            dict(instance=np.array([1, 1], np.int32), local_hit=np.array([0, 0], np.int32),
+                 global_hit=np.array([0, 0], np.int32))]
+    s = bench.route_stats(lens, outs, 3)
+    assert s["local_hit_ratio"] == 80 / 220 and s["global_hit_ratio"] == 80 / 220
+    # batch 0: instance 0 gets 130 of 200 tokens; batch 1: one instance gets all 20
+    assert s["routed_token_imbalance"] == pytest.approx((3 * 130 / 200 + 3.0) / 2)
+    assert s["batches"] == 2
+    empty = bench.route_stats([np.zeros(0, np.int64)], [dict(instance=np.zeros(0, np.int32),
+                                                          local_hit=np.zeros(0, np.int32),
+                                                          global_hit=np.zeros(0, np.int32))], 4)
+    assert empty["local_hit_ratio"] == 0.0 and empty["routed_token_imbalance"] is None
+
+
+def test_route_stats_on_oracle_routed_burst_batches():
+    """The statistics of routed config-4-shaped batches (the oracle routes a
+    reduced burst trace) lie in their ranges: hits within the prompts and an
+    imbalance between 1 and N."""
+    import oracle
+    from synth import burst_trace
+    oracle.build()
+    tr = burst_trace(n_sessions=512, batch_size=64)
+    p = tr.params
+    host = [tr.batch(k) for k in range(2)]
+    ox = bench.oracle_index_for(tr, host)
+    outs = [ox.route_batch(p.block_size, p.session_blocks, p.hash_seed, b.tokens, b.offsets, b.load,
+                           p.w_load, p.w_miss, p.w_glob) for b in host]
+    ox.close()
+    s = bench.route_stats([b.lengths() for b in host], outs, p.num_instances)
+    assert 0.5 < s["local_hit_ratio"] + s["global_hit_ratio"] <= 1.0
+    assert 1.0 <= s["routed_token_imbalance"] <= p.num_instances
+    assert s["batches"] == 2
