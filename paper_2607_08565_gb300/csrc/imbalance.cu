@@ -17,6 +17,7 @@
 #include <algorithm>
 
 #include "smetric_impl.cuh"
+#include "call_range.cuh"
 
 using namespace smetric;
 
@@ -95,6 +96,7 @@ int smetric_window_imbalance(smetric_index* idx, const int32_t* d_instance, cons
                              const int64_t* d_end, int32_t n_requests, int64_t window, int32_t n_windows,
                              void* d_workspace, int64_t workspace_bytes, int64_t* d_max, int32_t* d_argmax,
                              int64_t* d_sum, smetric_stream_t stream) {
+  CallRange range("smetric_window_imbalance");
   int rc = check_device(idx);
   if (rc) return rc;
   const int32_t N = idx->cfg.num_instances;

@@ -19,6 +19,7 @@
 #include <new>
 
 #include "smetric_impl.cuh"
+#include "call_range.cuh"
 
 using namespace smetric;
 
@@ -272,6 +273,7 @@ void free_all(smetric_index* x) {
 extern "C" {
 
 int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
+  CallRange range("smetric_index_create");
   if (!out) return SMETRIC_ERR_INVALID_ARG;
   *out = nullptr;
   if (!cfg) return SMETRIC_ERR_INVALID_ARG;
@@ -347,6 +349,7 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
 }
 
 int smetric_index_destroy(smetric_index* idx) {
+  CallRange range("smetric_index_destroy");
   if (!idx) return SMETRIC_OK;
   int dev = -1;
   cudaGetDevice(&dev);
@@ -360,6 +363,7 @@ int smetric_index_destroy(smetric_index* idx) {
 }
 
 int smetric_index_clear(smetric_index* idx, smetric_stream_t stream) {
+  CallRange range("smetric_index_clear");
   int rc = check_device(idx);
   if (rc) return rc;
   const size_t slots = (size_t)idx->n_buckets * kBucket;
@@ -371,16 +375,19 @@ int smetric_index_clear(smetric_index* idx, smetric_stream_t stream) {
 
 int smetric_index_insert(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers,
                          int64_t n, smetric_stream_t stream) {
+  CallRange range("smetric_index_insert");
   return update(idx, d_keys, d_tiers, n, stream, kInsert);
 }
 
 int smetric_index_evict(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers,
                         int64_t n, smetric_stream_t stream) {
+  CallRange range("smetric_index_evict");
   return update(idx, d_keys, d_tiers, n, stream, kEvict);
 }
 
 int smetric_index_lookup(smetric_index* idx, const uint64_t* d_keys, int64_t n, uint64_t* d_masks,
                          smetric_stream_t stream) {
+  CallRange range("smetric_index_lookup");
   int rc = check_device(idx);
   if (rc) return rc;
   if (n < 0 || (n > 0 && (!d_keys || !d_masks))) return SMETRIC_ERR_INVALID_ARG;
@@ -395,6 +402,7 @@ int smetric_index_lookup(smetric_index* idx, const uint64_t* d_keys, int64_t n, 
 int32_t smetric_index_mask_words(const smetric_index* idx) { return idx ? idx->W : 0; }
 
 int smetric_status(smetric_index* idx, smetric_stream_t stream) {
+  CallRange range("smetric_status");
   int rc = check_device(idx);
   if (rc) return rc;
   if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)

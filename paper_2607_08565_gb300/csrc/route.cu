@@ -1958,6 +1958,8 @@ int route_policy(smetric_index* idx, int mode, const int32_t* d_tokens, int64_t 
 
 }  // namespace
 
+#include "call_range.cuh"
+
 extern "C" {
 
 int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
@@ -1965,6 +1967,7 @@ int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_t
                         smetric_weights w, int32_t* d_instance, int32_t* d_local_hit,
                         int32_t* d_global_hit, uint64_t* d_session_key, uint64_t* d_block_hashes,
                         int64_t hashes_cap, smetric_stream_t stream) {
+  CallRange range("smetric_route_batch");
   return route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance,
                             d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap,
                             reinterpret_cast<cudaStream_t>(stream));
@@ -1975,6 +1978,7 @@ int smetric_route_batch_sequential(smetric_index* idx, const int32_t* d_tokens, 
                                    smetric_weights w, int32_t* d_instance, int32_t* d_local_hit,
                                    int32_t* d_global_hit, uint64_t* d_session_key, uint64_t* d_block_hashes,
                                    int64_t hashes_cap, int64_t* d_load_after, smetric_stream_t stream) {
+  CallRange range("smetric_route_batch_sequential");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   int rc = route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance, d_local_hit,
                               d_global_hit, d_session_key, d_block_hashes, hashes_cap, s);
@@ -1992,6 +1996,7 @@ int smetric_route_batch_baseline(smetric_index* idx, const int32_t* d_tokens, in
                                  int64_t lam_den, int32_t* d_instance, int32_t* d_local_hit,
                                  int32_t* d_global_hit, uint64_t* d_session_key, uint64_t* d_block_hashes,
                                  int64_t hashes_cap, smetric_stream_t stream) {
+  CallRange range("smetric_route_batch_baseline");
   if (!idx || !d_batch || (scorer != SMETRIC_SCORER_BAILIAN && scorer != SMETRIC_SCORER_LMETRIC) ||
       lam_den < 1 || lam_den > (1LL << 20) || lam_num < 0 || lam_num > lam_den)
     return SMETRIC_ERR_INVALID_ARG;
@@ -2012,6 +2017,7 @@ int smetric_route_batch_policy_coloc(smetric_index* idx, const int32_t* d_tokens
                                      int32_t* d_instance, int32_t* d_local_hit, int32_t* d_global_hit,
                                      int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
                                      int64_t hashes_cap, smetric_stream_t stream) {
+  CallRange range("smetric_route_batch_policy_coloc");
   if (!idx || !d_tpot_budget || !d_num_requests) return SMETRIC_ERR_INVALID_ARG;
   return route_policy(idx, kColoc, d_tokens, n_tokens, d_offsets, n_requests, d_queued, d_tpot_budget,
                       d_num_requests, d_turn, d_est_hit, p, d_instance, d_local_hit, d_global_hit, d_stick,
@@ -2024,6 +2030,7 @@ int smetric_route_batch_policy(smetric_index* idx, const int32_t* d_tokens, int6
                                int32_t* d_instance, int32_t* d_local_hit, int32_t* d_global_hit,
                                int32_t* d_stick, uint64_t* d_session_key, uint64_t* d_block_hashes,
                                int64_t hashes_cap, smetric_stream_t stream) {
+  CallRange range("smetric_route_batch_policy");
   return route_policy(idx, kSession, d_tokens, n_tokens, d_offsets, n_requests, d_queued, nullptr, nullptr,
                       d_turn, d_est_hit, p, d_instance, d_local_hit, d_global_hit, d_stick, d_session_key,
                       d_block_hashes, hashes_cap, stream);
@@ -2034,6 +2041,7 @@ int smetric_index_commit_batch(smetric_index* idx, const int64_t* d_offsets, int
                                const int32_t* d_instance, const int32_t* d_local_hit,
                                const uint64_t* d_block_hashes, int32_t flags, int64_t* d_load,
                                smetric_stream_t stream) {
+  CallRange range("smetric_index_commit_batch");
   int rc = check_device(idx);
   if (rc) return rc;
   const smetric_index_config& c = idx->cfg;
@@ -2065,6 +2073,7 @@ int smetric_reuse_breakdown(smetric_index* idx, const int32_t* d_tokens, int64_t
                             const int32_t* d_sys_blocks, void* d_workspace, int64_t workspace_bytes,
                             int32_t* d_hit, int32_t* d_sys, int32_t* d_intra, int32_t* d_inter,
                             smetric_stream_t stream) {
+  CallRange range("smetric_reuse_breakdown");
   int rc = check_device(idx);
   if (rc) return rc;
   if (n_requests < 0 || n_requests > idx->cfg.max_batch_requests || n_tokens < 0) return SMETRIC_ERR_INVALID_ARG;
@@ -2101,6 +2110,7 @@ int smetric_link_sessions(smetric_index* idx, const int32_t* d_tokens, int64_t n
                           const int64_t* d_offsets, int32_t n_requests, const int64_t* d_users,
                           const int32_t* d_turns, int32_t* d_parent, int32_t* d_session,
                           smetric_stream_t stream) {
+  CallRange range("smetric_link_sessions");
   int rc = check_device(idx);
   if (rc) return rc;
   if (n_requests < 0 || n_requests > idx->cfg.max_batch_requests) return SMETRIC_ERR_INVALID_ARG;
@@ -2129,6 +2139,7 @@ int smetric_link_sessions(smetric_index* idx, const int32_t* d_tokens, int64_t n
 int smetric_block_hashes(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
                          const int64_t* d_offsets, int32_t n_requests, uint64_t* d_session_key,
                          uint64_t* d_block_hashes, int64_t hashes_cap, smetric_stream_t stream) {
+  CallRange range("smetric_block_hashes");
   smetric_weights w{0, 0, 0};
   return route_common<false>(idx, d_tokens, n_tokens, d_offsets, n_requests, nullptr, w, nullptr,
                              nullptr, nullptr, d_session_key, d_block_hashes, hashes_cap,
@@ -2139,6 +2150,7 @@ int smetric_route_batch_host(smetric_index* idx, const int32_t* h_tokens, int64_
                              const int64_t* h_offsets, int32_t n_requests, const int64_t* h_load,
                              smetric_weights w, int32_t* h_instance, int32_t* h_local_hit,
                              int32_t* h_global_hit, uint64_t* h_session_key, smetric_stream_t stream) {
+  CallRange range("smetric_route_batch_host");
   int rc = check_device(idx);
   if (rc) return rc;
   if (!(idx->cfg.flags & SMETRIC_FLAG_HOST_STAGING)) return SMETRIC_ERR_INVALID_ARG;
