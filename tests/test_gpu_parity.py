@@ -179,6 +179,19 @@ def test_index_full_reports_and_stays_consistent():
     assert int(ix.lookup(T(keys)).cpu().numpy().sum()) == 0
 
 
+def test_create_reports_oom_and_the_device_stays_usable():
+    """A table no device holds (2^40 slots of 16 bytes, 16 TiB) is refused
+    with SMETRIC_ERR_OOM and no index; the next index on the device works."""
+    with pytest.raises(pkg.SmetricError) as e:
+        make_index(4, 16, 1, cap=1 << 40)
+    assert e.value.code == pkg.SMETRIC_ERR_OOM
+    ix = make_index(4, 16, 1)
+    ix.insert(T(np.array([5], np.uint64)), T(np.array([2], np.int32)))
+    ix.check()
+    assert ix.lookup(T(np.array([5], np.uint64))).cpu().numpy()[0, 0] == 4
+    ix.close()
+
+
 # ---------------------------------------------------------------------------
 # (c)-(d): routing
 # ---------------------------------------------------------------------------
