@@ -123,3 +123,48 @@ def test_noalloc_hashes_refuse_on_host(L):
     assert f(None, 0, None, 0, 16, 1, 0, None, None, 0, None, None) == pkg.SMETRIC_OK
     assert pkg.smetric_strerror(pkg.SMETRIC_ERR_TOO_LARGE) == \
         "batch larger than the fixed no-allocation scratch"
+
+
+def test_header_is_plain_c_and_matches_the_binding_layout(tmp_path, L):
+    """include/smetric.h compiles as strict C99 with no CUDA header, links
+    against libsmetric.so, and its structs and enum agree byte for byte with
+    the ctypes binding; the refusals it makes from C need no GPU."""
+    import shutil
+    import subprocess
+    if shutil.which("gcc") is None:
+        pytest.skip("no C compiler")
+    exe = str(tmp_path / "c_abi_check")
+    libdir = os.path.dirname(build_lib.LIB)
+    subprocess.check_call(["gcc", "-std=c99", "-pedantic", "-Wall", "-Wextra", "-Werror",
+                           "-I", os.path.join(ROOT, "include"), os.path.join(ROOT, "tests", "c_abi_check.c"),
+                           "-o", exe, "-L", libdir, "-lsmetric", "-Wl,-rpath," + libdir])
+    out = subprocess.run([exe], capture_output=True, text=True, check=True).stdout.splitlines()
+    structs = {"smetric_index_config": pkg.smetric_index_config, "smetric_weights": pkg.smetric_weights,
+               "smetric_policy": pkg.smetric_policy}
+    fields = 0
+    for line in out:
+        kind, *rest = line.split(" ", 1)
+        rest = rest[0] if rest else ""
+        if kind == "sizeof":
+            name, size = rest.split()
+            assert C.sizeof(structs[name]) == int(size), name
+        elif kind == "offset":
+            qual, off, size = rest.split()
+            name, field = qual.split(".")
+            desc = getattr(structs[name], field)
+            assert (desc.offset, desc.size) == (int(off), int(size)), qual
+            fields += 1
+        elif kind == "enum":
+            name, value = rest.split()
+            assert getattr(pkg, name) == int(value), name
+        elif kind == "call":
+            what, *vals = rest.split()
+            want = {"create_odd_block": [pkg.SMETRIC_ERR_INVALID_ARG, 1],
+                    "route_null_index": [pkg.SMETRIC_ERR_INVALID_ARG],
+                    "destroy_null": [pkg.SMETRIC_OK]}[what]
+            assert [int(v) for v in vals] == want, what
+        elif kind == "strerror":
+            assert rest == pkg.smetric_strerror(pkg.SMETRIC_ERR_TABLE_FULL)
+    assert fields == 8 + 3 + 8
+    # every struct field of the binding was printed by the C side
+    assert fields == sum(len(s._fields_) for s in structs.values())
