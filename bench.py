@@ -66,6 +66,9 @@ def parse():
     ap.add_argument("--reuse", action="store_true",
                     help="time the KV$ reuse breakdown (Section 3.1) over a whole config-2 window "
                          "(one GPU; its own line)")
+    ap.add_argument("--pipeline", action="store_true",
+                    help="time smetric_route_batches (the config-4 batches routed four per call, "
+                         "alternating between two scratch sets) against one smetric_route_batch per batch")
     ap.add_argument("--imbalance", action="store_true",
                     help="time the windowed load imbalance (Section 3.2) over a day of running intervals "
                          "(one GPU; its own line)")
@@ -824,6 +827,86 @@ def run_sequential(args, steps=50):
 
 
 # ---------------------------------------------------------------------------
+# several batches per call, overlapped on two scratch sets
+# ---------------------------------------------------------------------------
+
+def run_pipelined(args, rounds=100):
+    """The config-4 batches routed four per smetric_route_batches call on an
+    index with a second scratch set, against the same batches routed one
+    smetric_route_batch call each; both timed with CUDA events over `rounds`
+    passes of the four batches, outputs compared bit for bit."""
+    import torch
+    import paper_2607_08565_gb300 as pkg
+    from paper_2607_08565_gb300 import build_lib
+
+    build_lib.build()
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    tr = c4_trace(args)
+    p = tr.params
+    host = [tr.batch(k) for k in range(N_DISTINCT_BATCHES)]
+    nkeys = tr.n_prefix_blocks()
+    chunk = 4096
+    ix = pkg.SMetricIndex(p.num_instances, p.block_size, p.session_blocks, capacity_slots=int(nkeys / 0.7) + 1,
+                          max_batch_requests=max(tr.batch_size, chunk),
+                          max_batch_tokens=max(max(b.n_tokens for b in host), chunk * int(tr.prefix_len.max())),
+                          hash_seed=p.hash_seed, pipeline=True)
+    populate_index(ix, tr, device, chunk)
+    batches = [tuple(torch.from_numpy(a).to(device) for a in (b.tokens, b.offsets, b.load)) for b in host]
+    w = (p.w_load, p.w_miss, p.w_glob)
+    one = [ix.route_batch(*b, w) for b in batches]
+    many = ix.route_batches(batches, w)
+    stream = torch.cuda.current_stream(device)
+
+    def per_batch():
+        for b, o in zip(batches, one):
+            pkg.smetric_route_batch(ix.handle, b[0], b[0].numel(), b[1], b[1].numel() - 1, b[2], w,
+                                    o["instance"], o["local_hit"], o["global_hit"], o["session_key"], None, 0,
+                                    stream)
+
+    def pipelined():
+        ix.route_batches(batches, w, out=many, stream=stream)
+
+    times = {}
+    for name, fn in (("per_batch", per_batch), ("pipelined", pipelined)):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(rounds):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ix.check()
+        times[name] = e0.elapsed_time(e1) / (rounds * len(batches))
+    for o1, o2 in zip(one, many):
+        for k in o1:
+            a, b = o1[k], o2[k]
+            if a.dtype == torch.uint64:  # compared as int64 words (uint64 has few CUDA kernels)
+                a, b = a.view(torch.int64), b.view(torch.int64)
+            if not torch.equal(a, b):
+                raise RuntimeError(f"smetric_route_batches differs from smetric_route_batch in {k}")
+    outs = [{k: v.cpu().numpy() for k, v in o.items()} for o in one]
+    algo = np.mean([algorithmic_bytes(b.lengths(), o["local_hit"], o["global_hit"], p.block_size, ix.W)["path"]
+                    for b, o in zip(host, outs)])
+    peak, peak_kind = peak_hbm()
+    reqs = np.mean([b.n_requests for b in host])
+    frac = {k: algo / (t / 1e3) / 1e9 / peak for k, t in times.items()}
+    line = {"metric": METRIC, "value": reqs / (times["pipelined"] / 1e3), "unit": UNIT, "n_gpus": 1,
+            "steps": rounds * len(batches), "warmup": 3 * len(batches), "ms_per_step": times["pipelined"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+            "per_batch_ms_per_step": times["per_batch"],
+            "roofline_path": {"frac_pipelined": frac["pipelined"], "frac_per_batch": frac["per_batch"],
+                              "algorithmic_bytes_per_step": float(algo), "peak": peak,
+                              "peak_kind": f"{peak_kind} copy"},
+            "config": {"workload": workload_name(args), "batches_per_call": len(batches),
+                       "outputs_equal_per_batch_route": True}}
+    print(json.dumps(line), flush=True)
+    ix.close()
+
+
+# ---------------------------------------------------------------------------
 # session reconstruction over a config-3 trace
 # ---------------------------------------------------------------------------
 
@@ -1196,6 +1279,9 @@ def main():
         return
     if args.imbalance:
         run_imbalance(args)
+        return
+    if args.pipeline:
+        run_pipelined(args)
         return
     rank, world, local, dist = dist_setup(args)
     if args.impl == "reference":

@@ -79,6 +79,7 @@ enum {
 
 /* smetric_index_config.flags */
 #define SMETRIC_FLAG_HOST_STAGING 1 /* allocate device staging buffers for smetric_route_batch_host */
+#define SMETRIC_FLAG_PIPELINE 2     /* allocate a second route scratch set for smetric_route_batches */
 
 typedef struct {
   int32_t num_instances;      /* N, 1..SMETRIC_MAX_INSTANCES (local tiers 0..N-1) */
@@ -441,6 +442,35 @@ int smetric_route_batch_host(smetric_index* idx, const int32_t* h_tokens, int64_
                              smetric_weights w, int32_t* h_instance, int32_t* h_local_hit,
                              int32_t* h_global_hit, uint64_t* h_session_key,
                              smetric_stream_t stream);
+
+/* Several batches routed in one call: batch j < n_batches is routed exactly
+ * as smetric_route_batch would route it with no block-hash output (tokens
+ * d_tokens[j] of n_tokens[j], offsets d_offsets[j], n_requests[j] requests,
+ * loads d_load[j], outputs d_instance[j], d_local_hit[j], d_global_hit[j],
+ * d_session_key[j]). Each d_ argument is a host array of n_batches device
+ * pointers; n_tokens and n_requests are host arrays of counts; the weights
+ * are shared. Every batch sees the index as of the call (routes do not
+ * change it) and its own loads, so the outputs equal those of n_batches
+ * smetric_route_batch calls in a row, and when the call returns every output
+ * is complete in `stream` order.
+ *
+ * With an index created with SMETRIC_FLAG_PIPELINE (and profiling off), the
+ * batches alternate between the index's two scratch sets and two streams,
+ * so that batch j+1's token read (the block digests, bound by HBM
+ * bandwidth) runs while batch j's tier lookups and walk (bound by random
+ * accesses and latency) finish: batch j+1 starts once batch j's hash chain
+ * is done. Without the flag the batches run one after another on `stream`.
+ * The outputs of different batches must not overlap (two batches may run at
+ * once); inputs may be shared. Nothing is allocated (the second set comes
+ * with the index). Host-detectable errors in any batch return before
+ * anything is enqueued; device-detected errors latch as for
+ * smetric_route_batch (a bad batch gets the invalid-batch outputs, the
+ * others are routed). */
+int smetric_route_batches(smetric_index* idx, int32_t n_batches, const int32_t* const* d_tokens,
+                          const int64_t* n_tokens, const int64_t* const* d_offsets, const int32_t* n_requests,
+                          const int64_t* const* d_load, smetric_weights w, int32_t* const* d_instance,
+                          int32_t* const* d_local_hit, int32_t* const* d_global_hit,
+                          uint64_t* const* d_session_key, smetric_stream_t stream);
 
 /* Wait for `stream`, then return and clear the first error the device latched
  * for this index since the last call (SMETRIC_OK if none). */

@@ -32,6 +32,7 @@ SMETRIC_MAX_WEIGHT = 1 << 20
 SMETRIC_MAX_LOAD = 1 << 40
 SMETRIC_MAX_PROBE = 65536
 SMETRIC_FLAG_HOST_STAGING = 1
+SMETRIC_FLAG_PIPELINE = 2
 SMETRIC_POLICY_MAX_LEN = 1 << 24
 SMETRIC_POLICY_MAX_QUEUED = 1 << 59
 SMETRIC_COMMIT_GLOBAL = 1
@@ -53,6 +54,7 @@ EXPORTED = (
     "smetric_index_commit_batch", "smetric_route_batch_policy_coloc", "smetric_link_sessions",
     "smetric_route_batch_baseline", "smetric_route_batch_sequential", "smetric_reuse_workspace_bytes",
     "smetric_reuse_breakdown", "smetric_imbalance_workspace_bytes", "smetric_window_imbalance",
+    "smetric_route_batches",
 )
 
 
@@ -112,6 +114,7 @@ def lib():
             "smetric_index_mask_words": (I32, [P]),
             "smetric_route_batch": (C.c_int, [P, P, I64, P, I32, P, smetric_weights, P, P, P, P, P,
                                               I64, P]),
+            "smetric_route_batches": (C.c_int, [P, I32, P, P, P, P, P, smetric_weights, P, P, P, P, P]),
             "smetric_route_batch_policy": (C.c_int, [P, P, I64, P, I32, P, P, P, smetric_policy, P, P,
                                                      P, P, P, P, I64, P]),
             "smetric_index_commit_batch": (C.c_int, [P, P, I32, P, P, P, I32, P, P]),
@@ -228,6 +231,21 @@ def smetric_route_batch(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests
                                      _ptr(d_load), _weights(w), _ptr(d_instance), _ptr(d_local_hit),
                                      _ptr(d_global_hit), _ptr(d_session_key), _ptr(d_block_hashes),
                                      hashes_cap, _stream(stream)), "smetric_route_batch")
+
+
+def smetric_route_batches(idx: int, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance,
+                          d_local_hit, d_global_hit, d_session_key, stream=None) -> None:
+    """Several batches in one call; every argument but idx, w and stream is a
+    sequence with one entry per batch (device arrays, or counts)."""
+    nb = len(n_requests)
+    if not all(len(x) == nb for x in (d_tokens, n_tokens, d_offsets, d_load, d_instance, d_local_hit,
+                                      d_global_hit, d_session_key)):
+        raise ValueError("every per-batch sequence needs one entry per batch")
+    ptrs = lambda xs: (C.c_void_p * max(nb, 1))(*[_ptr(x) for x in xs])
+    _check(lib().smetric_route_batches(idx, nb, ptrs(d_tokens), (C.c_int64 * max(nb, 1))(*n_tokens),
+                                       ptrs(d_offsets), (C.c_int32 * max(nb, 1))(*n_requests), ptrs(d_load),
+                                       _weights(w), ptrs(d_instance), ptrs(d_local_hit), ptrs(d_global_hit),
+                                       ptrs(d_session_key), _stream(stream)), "smetric_route_batches")
 
 
 def _policy(p) -> smetric_policy:
@@ -387,9 +405,10 @@ class SMetricIndex:
 
     def __init__(self, num_instances: int, block_size: int, session_blocks: int,
                  capacity_slots: int, max_batch_requests: int, max_batch_tokens: int,
-                 hash_seed: int = 0, host_staging: bool = False):
+                 hash_seed: int = 0, host_staging: bool = False, pipeline: bool = False):
         self.cfg = smetric_index_config(num_instances, block_size, session_blocks,
-                                        SMETRIC_FLAG_HOST_STAGING if host_staging else 0,
+                                        (SMETRIC_FLAG_HOST_STAGING if host_staging else 0)
+                                        | (SMETRIC_FLAG_PIPELINE if pipeline else 0),
                                         capacity_slots, hash_seed & 0xFFFFFFFFFFFFFFFF,
                                         max_batch_requests, max_batch_tokens)
         self.handle = smetric_index_create(self.cfg)
@@ -434,6 +453,26 @@ class SMetricIndex:
         import torch
         out = torch.empty((keys.numel(), self.W), dtype=torch.uint64, device=keys.device)
         smetric_index_lookup(self.handle, keys, keys.numel(), out, stream)
+        return out
+
+    def route_batches(self, batches, weights=(1, 4, 2), out=None, stream=None):
+        """Routes a list of (tokens, offsets, load) device batches in one call;
+        returns one dict(instance, local_hit, global_hit, session_key) per
+        batch (or fills `out`, a list of such dicts)."""
+        import torch
+        if out is None:
+            out = []
+            for tokens, offsets, _ in batches:
+                n, dev = offsets.numel() - 1, offsets.device
+                out.append(dict(instance=torch.empty(n, dtype=torch.int32, device=dev),
+                                local_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                                global_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                                session_key=torch.empty(n, dtype=torch.uint64, device=dev)))
+        smetric_route_batches(self.handle, [b[0] for b in batches], [b[0].numel() for b in batches],
+                              [b[1] for b in batches], [b[1].numel() - 1 for b in batches],
+                              [b[2] for b in batches], weights, [o["instance"] for o in out],
+                              [o["local_hit"] for o in out], [o["global_hit"] for o in out],
+                              [o["session_key"] for o in out], stream)
         return out
 
     def route_batch(self, tokens, offsets, load, weights=(1, 4, 2), want_hashes=False,

@@ -24,6 +24,13 @@
 using namespace smetric;
 
 namespace smetric {
+// The second route scratch set of SMETRIC_FLAG_PIPELINE (defined beside
+// smetric_route_batches, which uses it).
+int pipeline_attach(smetric_index* x);
+void pipeline_release(smetric_index* x);
+}  // namespace smetric
+
+namespace smetric {
 
 int cuda_status(cudaError_t e) {
   if (e == cudaSuccess) return SMETRIC_OK;
@@ -239,6 +246,7 @@ int launch_commit(smetric_index* idx, const int32_t* d_instance, const uint64_t*
 namespace {
 
 void free_all(smetric_index* x) {
+  pipeline_release(x);
   cudaFree(x->table);
   cudaFree(x->tags);
   cudaFree(x->status);
@@ -283,7 +291,7 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
   if (c.session_blocks < 1 || c.capacity_slots < 1) return SMETRIC_ERR_INVALID_ARG;
   if (c.max_batch_requests < 0 || c.max_batch_requests > INT32_MAX - 1) return SMETRIC_ERR_INVALID_ARG;
   if (c.max_batch_tokens < 0) return SMETRIC_ERR_INVALID_ARG;
-  if (c.flags & ~SMETRIC_FLAG_HOST_STAGING) return SMETRIC_ERR_INVALID_ARG;
+  if (c.flags & ~(SMETRIC_FLAG_HOST_STAGING | SMETRIC_FLAG_PIPELINE)) return SMETRIC_ERR_INVALID_ARG;
   const int W = (c.num_instances + 1 + 63) / 64;
   // slots (rounded up to whole buckets) * entry bytes must not overflow
   if (c.capacity_slots > (UINT64_MAX / 16) / (uint64_t)entry_words(W)) return SMETRIC_ERR_INVALID_ARG;
@@ -333,6 +341,7 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
          cudaMalloc(&x->st_out32, (3 * R + 1) * sizeof(int32_t)) == cudaSuccess &&
          cudaMalloc(&x->st_sk, (R + 1) * sizeof(uint64_t)) == cudaSuccess;
   }
+  if (ok && (c.flags & SMETRIC_FLAG_PIPELINE)) ok = pipeline_attach(x) == SMETRIC_OK;
   if (ok) ok = cudaMemset(x->table, 0, table_bytes) == cudaSuccess &&
                cudaMemset(x->tags, 0, slots) == cudaSuccess &&
                cudaMemset(x->status, 0, sizeof(int32_t)) == cudaSuccess &&

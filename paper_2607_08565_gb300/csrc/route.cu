@@ -1612,6 +1612,16 @@ __global__ void __launch_bounds__(1024)
 
 void profile_mark(smetric_index* idx, int k, cudaStream_t s);
 
+// How a batch shares the GPU with the batch before it (smetric_route_batches
+// on two scratch sets): an event recorded once its chain is enqueued, and
+// caps on the digest's and the probe's resident CTAs per SM so that both fit
+// on every SM at once (0 = no cap).
+struct Overlap {
+  cudaEvent_t after_chain;
+  int digest_ctas_per_sm;
+  int probe_ctas_per_sm;
+};
+
 // Launches a route kernel; with pdl the launch may begin while the previous
 // kernel on the stream is still running (the kernel waits in pdl_enter).
 template <typename... KArgs, typename... Args>
@@ -1677,7 +1687,7 @@ bool make_token_maps(TokenMaps& m, const int32_t* tokens, int64_t n_tokens, int 
 
 template <int HB>
 int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
-                  const int64_t* d_offsets, int32_t n, cudaStream_t s) {
+                  const int64_t* d_offsets, int32_t n, cudaStream_t s, int cap_per_sm) {
   const int B = idx->cfg.block_size;
   const uint64_t d_init = mix64(idx->cfg.hash_seed ^ (uint64_t)B);
   // request-aligned chunks (TMA kernel) number at most blocks / 32 + n
@@ -1701,7 +1711,8 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
         idx->digest_occ = occ < 1 ? 1 : occ;
       }
       const int64_t want = (max_chunks + warps - 1) / warps;
-      const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * idx->digest_occ));
+      const int occ = cap_per_sm > 0 ? std::min(cap_per_sm, idx->digest_occ) : idx->digest_occ;
+      const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * occ));
       idx->launches++;
       return launch_k(kern, dim3((unsigned)grid), dim3(warps * 32), smem, s, !idx->profiling, maps, d_tokens,
                       n_tokens, d_offsets, (const int64_t*)idx->block_off, (const int64_t*)idx->chunk_off, n, d_init,
@@ -1722,7 +1733,8 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
     idx->digest_occ = occ < 1 ? 1 : occ;
   }
   const int64_t want = (max_chunks + warps - 1) / warps;
-  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * idx->digest_occ));
+  const int occ = cap_per_sm > 0 ? std::min(cap_per_sm, idx->digest_occ) : idx->digest_occ;
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * occ));
   idx->launches++;
   if (HB > 0)
     return launch_k(kern, dim3((unsigned)grid), dim3(warps * 32), smem, s, !idx->profiling, d_tokens, n_tokens,
@@ -1734,12 +1746,12 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
 }
 
 int dispatch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
-                    const int64_t* d_offsets, int32_t n, cudaStream_t s) {
+                    const int64_t* d_offsets, int32_t n, cudaStream_t s, int cap_per_sm = 0) {
   switch (idx->cfg.block_size) {
-    case 16: return launch_digest<8>(idx, d_tokens, n_tokens, d_offsets, n, s);
-    case 32: return launch_digest<16>(idx, d_tokens, n_tokens, d_offsets, n, s);
-    case 64: return launch_digest<32>(idx, d_tokens, n_tokens, d_offsets, n, s);
-    default: return launch_digest<0>(idx, d_tokens, n_tokens, d_offsets, n, s);
+    case 16: return launch_digest<8>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm);
+    case 32: return launch_digest<16>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm);
+    case 64: return launch_digest<32>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm);
+    default: return launch_digest<0>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm);
   }
 }
 
@@ -1782,12 +1794,15 @@ int launch_group(smetric_index* idx, int32_t n, cudaStream_t s) {
 template <int W>
 int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
                  smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, uint64_t* hashes,
-                 uint64_t* sk, int64_t max_blocks, const WalkPolicy& pol, cudaStream_t s) {
+                 uint64_t* sk, int64_t max_blocks, const WalkPolicy& pol, cudaStream_t s,
+                 const Overlap* ov) {
+  const cudaEvent_t after_chain = ov ? ov->after_chain : nullptr;
   const int N = idx->cfg.num_instances;
   const uint64_t* H = hashes ? hashes : idx->hashes;
   int rc;
   if (idx->profiling) {  // one stream, so that each kernel's events bracket it alone
     if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, false, s))) return rc;
+    if (after_chain && cudaEventRecord(after_chain, s) != cudaSuccess) return cuda_status(cudaErrorUnknown);
     profile_mark(idx, kChain, s);
     if ((rc = launch_group(idx, n, s))) return rc;
     profile_mark(idx, kGroup, s);
@@ -1799,12 +1814,14 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
     if ((rc = launch_group(idx, n, idx->side))) return rc;
     if (cudaEventRecord(idx->join_ev, idx->side) != cudaSuccess) return cuda_status(cudaErrorUnknown);
     if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, false, s))) return rc;
+    if (after_chain && cudaEventRecord(after_chain, s) != cudaSuccess) return cuda_status(cudaErrorUnknown);
     if (cudaStreamWaitEvent(s, idx->join_ev, 0) != cudaSuccess) return cuda_status(cudaErrorUnknown);
   }
   {
     // probe: one thread per block, grid sized to the largest possible batch
     const int64_t want = (max_blocks + 255) / 256;
-    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
+    const int per_sm = ov && ov->probe_ctas_per_sm > 0 ? ov->probe_ctas_per_sm : 8;
+    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * per_sm));
     idx->launches++;
     // an ordinary launch: it follows the wait for the side stream
     if ((rc = launch_k(k_probe<W>, dim3((unsigned)grid), dim3(256), 0, s, false, idx->tags, idx->table,
@@ -1840,13 +1857,14 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
 
 int dispatch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
                    smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, uint64_t* hashes,
-                   uint64_t* sk, int64_t max_blocks, const WalkPolicy& pol, cudaStream_t s) {
+                   uint64_t* sk, int64_t max_blocks, const WalkPolicy& pol, cudaStream_t s,
+                   const Overlap* ov) {
   switch (idx->W) {
-    case 1: return launch_match<1>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s);
-    case 2: return launch_match<2>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s);
-    case 3: return launch_match<3>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s);
-    case 4: return launch_match<4>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s);
-    case 5: return launch_match<5>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s);
+    case 1: return launch_match<1>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s, ov);
+    case 2: return launch_match<2>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s, ov);
+    case 3: return launch_match<3>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s, ov);
+    case 4: return launch_match<4>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s, ov);
+    case 5: return launch_match<5>(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk, max_blocks, pol, s, ov);
     default: return SMETRIC_ERR_INVALID_ARG;
   }
 }
@@ -1878,7 +1896,7 @@ template <bool PROBE>
 int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, const int64_t* d_offsets,
                  int32_t n, const int64_t* d_load, smetric_weights w, int32_t* inst, int32_t* lhit,
                  int32_t* ghit, uint64_t* sk, uint64_t* hashes, int64_t hashes_cap, cudaStream_t s,
-                 const WalkPolicy* pol = nullptr) {
+                 const WalkPolicy* pol = nullptr, const Overlap* ov = nullptr) {
   int rc = check_device(idx);
   if (rc) return rc;
   const smetric_index_config& c = idx->cfg;
@@ -1904,13 +1922,14 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   profile_mark(idx, kPrep, s);
   if (n_tokens / c.block_size > 0) {
-    if ((rc = dispatch_digest(idx, d_tokens, n_tokens, d_offsets, n, s))) return rc;
+    if ((rc = dispatch_digest(idx, d_tokens, n_tokens, d_offsets, n, s, ov ? ov->digest_ctas_per_sm : 0)))
+      return rc;
   }
   profile_mark(idx, kDigest, s);
   if (PROBE) {
     const WalkPolicy off_pol = {};
     if ((rc = dispatch_match(idx, d_offsets, n, d_load, w, inst, lhit, ghit, hashes, sk,
-                             n_tokens / c.block_size, pol ? *pol : off_pol, s)))
+                             n_tokens / c.block_size, pol ? *pol : off_pol, s, ov)))
       return rc;
   } else {
     if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, !idx->profiling, s))) return rc;
@@ -1958,7 +1977,226 @@ int route_policy(smetric_index* idx, int mode, const int32_t* d_tokens, int64_t 
 
 }  // namespace
 
+#include <mutex>
+#include <new>
+#include <unordered_map>
+
 #include "call_range.cuh"
+
+// ---------------------------------------------------------------------------
+// batches overlapped on two scratch sets
+// ---------------------------------------------------------------------------
+
+namespace smetric {
+
+// The second route scratch set of an index created with SMETRIC_FLAG_PIPELINE:
+// the same buffers, with the same sizes, as the index's own set, and its own
+// side stream and events for the group stage.
+struct RouteScratchSet {
+  int64_t* block_off = nullptr;
+  int64_t* chunk_off = nullptr;
+  uint64_t* digest = nullptr;
+  uint64_t* hashes = nullptr;
+  uint64_t* masks = nullptr;
+  uint64_t* chunk_and = nullptr;
+  uint64_t* groups = nullptr;
+  int32_t* lead = nullptr;  // lead, then share at lead + max_batch_requests + 1
+  int32_t* summ = nullptr;
+  uint64_t* sk_tmp = nullptr;
+  int32_t* order = nullptr;
+  int32_t* batch_ok = nullptr;
+  cudaStream_t side = nullptr;
+  cudaEvent_t fork_ev = nullptr, join_ev = nullptr;
+};
+
+struct Pipeline {
+  RouteScratchSet alt;
+  cudaStream_t stream = nullptr;                   // runs the batches that use `alt`
+  cudaEvent_t chain_done[2] = {nullptr, nullptr};  // per set: its latest batch's chain has finished
+  cudaEvent_t start = nullptr, finish = nullptr;   // the caller's stream to `stream`, and back
+};
+
+static std::mutex& pipeline_mutex() {
+  static std::mutex m;
+  return m;
+}
+
+// Indexes created with SMETRIC_FLAG_PIPELINE and their second sets (kept
+// beside the index so that the index's layout stays as it is).
+static std::unordered_map<const smetric_index*, Pipeline*>& pipelines() {
+  static std::unordered_map<const smetric_index*, Pipeline*> table;
+  return table;
+}
+
+static Pipeline* pipeline_of(const smetric_index* idx) {
+  std::lock_guard<std::mutex> lock(pipeline_mutex());
+  auto it = pipelines().find(idx);
+  return it == pipelines().end() ? nullptr : it->second;
+}
+
+static void free_pipeline(Pipeline* p) {
+  RouteScratchSet& a = p->alt;
+  cudaFree(a.block_off);
+  cudaFree(a.chunk_off);
+  cudaFree(a.digest);
+  cudaFree(a.hashes);
+  cudaFree(a.masks);
+  cudaFree(a.chunk_and);
+  cudaFree(a.groups);
+  cudaFree(a.lead);
+  cudaFree(a.summ);
+  cudaFree(a.sk_tmp);
+  cudaFree(a.order);
+  cudaFree(a.batch_ok);
+  if (a.side) cudaStreamDestroy(a.side);
+  if (a.fork_ev) cudaEventDestroy(a.fork_ev);
+  if (a.join_ev) cudaEventDestroy(a.join_ev);
+  if (p->stream) cudaStreamDestroy(p->stream);
+  for (cudaEvent_t e : {p->chain_done[0], p->chain_done[1], p->start, p->finish})
+    if (e) cudaEventDestroy(e);
+  delete p;
+}
+
+// Exchanges the index's route scratch with set `a` (host pointers only: a
+// launch takes the pointers current when it is enqueued).
+static void swap_scratch(smetric_index* x, RouteScratchSet& a) {
+  std::swap(x->block_off, a.block_off);
+  std::swap(x->chunk_off, a.chunk_off);
+  std::swap(x->digest, a.digest);
+  std::swap(x->hashes, a.hashes);
+  std::swap(x->masks, a.masks);
+  std::swap(x->chunk_and, a.chunk_and);
+  std::swap(x->groups, a.groups);
+  std::swap(x->lead, a.lead);
+  x->share = x->lead + (x->cfg.max_batch_requests + 1);
+  std::swap(x->summ, a.summ);
+  std::swap(x->sk_tmp, a.sk_tmp);
+  std::swap(x->order, a.order);
+  std::swap(x->batch_ok, a.batch_ok);
+  std::swap(x->side, a.side);
+  std::swap(x->fork_ev, a.fork_ev);
+  std::swap(x->join_ev, a.join_ev);
+}
+
+// Allocates the second set of index x (called by smetric_index_create once
+// the index's own set exists). The sizes are those of the index's own set.
+int pipeline_attach(smetric_index* x) {
+  const smetric_index_config& c = x->cfg;
+  const size_t R = (size_t)c.max_batch_requests;
+  const size_t max_blocks = (size_t)(c.max_batch_tokens / c.block_size);
+  const size_t nb = max_blocks > 0 ? max_blocks : 1;
+  const size_t W = (size_t)x->W;
+  Pipeline* p = new (std::nothrow) Pipeline();
+  if (!p) return SMETRIC_ERR_OOM;
+  RouteScratchSet& a = p->alt;
+  bool ok = cudaMalloc(&a.block_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
+            cudaMalloc(&a.digest, nb * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&a.hashes, nb * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&a.masks, nb * W * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&a.chunk_and, (max_blocks / 32 + 1) * W * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&a.groups, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&a.lead, 2 * (R + 1) * sizeof(int32_t)) == cudaSuccess &&
+            cudaMalloc(&a.chunk_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
+            cudaMalloc(&a.order, (R + 2) * sizeof(int32_t)) == cudaSuccess &&
+            cudaMalloc(&a.sk_tmp, (R + 1) * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&a.summ, (R > 0 ? R : 1) * ((size_t)c.num_instances + 1) * sizeof(int32_t)) == cudaSuccess &&
+            cudaMalloc(&a.batch_ok, sizeof(int32_t)) == cudaSuccess &&
+            cudaMemset(a.groups, 0, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
+            cudaStreamCreateWithFlags(&a.side, cudaStreamNonBlocking) == cudaSuccess &&
+            cudaEventCreateWithFlags(&a.fork_ev, cudaEventDisableTiming) == cudaSuccess &&
+            cudaEventCreateWithFlags(&a.join_ev, cudaEventDisableTiming) == cudaSuccess &&
+            cudaStreamCreateWithFlags(&p->stream, cudaStreamNonBlocking) == cudaSuccess;
+  for (cudaEvent_t* e : {&p->chain_done[0], &p->chain_done[1], &p->start, &p->finish})
+    ok = ok && cudaEventCreateWithFlags(e, cudaEventDisableTiming) == cudaSuccess;
+  if (!ok) {
+    (void)cudaGetLastError();
+    free_pipeline(p);
+    return SMETRIC_ERR_OOM;
+  }
+  std::lock_guard<std::mutex> lock(pipeline_mutex());
+  pipelines()[x] = p;
+  return SMETRIC_OK;
+}
+
+// Frees the second set of index x, if it has one (the device is idle).
+void pipeline_release(smetric_index* x) {
+  Pipeline* p = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(pipeline_mutex());
+    auto it = pipelines().find(x);
+    if (it == pipelines().end()) return;
+    p = it->second;
+    pipelines().erase(it);
+  }
+  free_pipeline(p);
+}
+
+}  // namespace smetric
+
+namespace {
+
+// Resident CTAs per SM while two batches overlap: one digest CTA (24 warps,
+// 38 registers a thread) beside four probe CTAs (8 warps, 31 registers) fit
+// the SM's 64 warps and 64K registers together, so neither kernel's
+// persistent grid can shut the other out.
+constexpr int kOverlapDigestCtas = 1;
+constexpr int kOverlapProbeCtas = 4;
+
+// smetric_route_batches: the host checks of route_common for every batch
+// first, then the batches, alternating between the two sets when the index
+// has a second one. Batch j's first kernel waits for batch j - 1's chain, so
+// that batch j's digests (bound by HBM bandwidth) run while batch j - 1's
+// probe and walk (bound by random accesses and latency) finish, and batch
+// j's chain does not share the GPU with batch j - 1's digests.
+int route_batches(smetric_index* idx, int32_t nb, const int32_t* const* tok, const int64_t* ntok,
+                  const int64_t* const* off, const int32_t* nreq, const int64_t* const* load, smetric_weights w,
+                  int32_t* const* inst, int32_t* const* lhit, int32_t* const* ghit, uint64_t* const* sk,
+                  cudaStream_t s) {
+  int rc = check_device(idx);
+  if (rc) return rc;
+  if (nb < 0 || (nb > 0 && (!tok || !ntok || !off || !nreq || !load || !inst || !lhit || !ghit || !sk)))
+    return SMETRIC_ERR_INVALID_ARG;
+  const smetric_index_config& c = idx->cfg;
+  for (int32_t j = 0; j < nb; ++j) {
+    const int32_t n = nreq[j];
+    const int64_t nt = ntok[j];
+    if (n < 0 || n > c.max_batch_requests || nt < 0 || nt > c.max_batch_tokens) return SMETRIC_ERR_INVALID_ARG;
+    if (n == 0) continue;
+    if (!off[j] || !sk[j] || (nt > 0 && !tok[j])) return SMETRIC_ERR_INVALID_ARG;
+    if (tok[j] && (reinterpret_cast<uintptr_t>(tok[j]) & 15)) return SMETRIC_ERR_INVALID_ARG;
+    if (!load[j] || !inst[j] || !lhit[j] || !ghit[j] || !weights_ok(w)) return SMETRIC_ERR_INVALID_ARG;
+  }
+  Pipeline* p = pipeline_of(idx);
+  if (!p || idx->profiling || nb < 2) {
+    for (int32_t j = 0; j < nb; ++j)
+      if ((rc = route_common<true>(idx, tok[j], ntok[j], off[j], nreq[j], load[j], w, inst[j], lhit[j], ghit[j],
+                                   sk[j], nullptr, 0, s)))
+        return rc;
+    return SMETRIC_OK;
+  }
+  // the second stream starts from everything enqueued on the caller's stream
+  if (cudaEventRecord(p->start, s) != cudaSuccess || cudaStreamWaitEvent(p->stream, p->start, 0) != cudaSuccess)
+    return cuda_status(cudaErrorUnknown);
+  for (int32_t j = 0; j < nb && rc == SMETRIC_OK; ++j) {
+    const int set = j & 1;
+    cudaStream_t sj = set ? p->stream : s;
+    if (j > 0 && cudaStreamWaitEvent(sj, p->chain_done[set ^ 1], 0) != cudaSuccess) {
+      rc = cuda_status(cudaErrorUnknown);
+      break;
+    }
+    if (set) swap_scratch(idx, p->alt);
+    const Overlap ov = {p->chain_done[set], kOverlapDigestCtas, kOverlapProbeCtas};
+    rc = route_common<true>(idx, tok[j], ntok[j], off[j], nreq[j], load[j], w, inst[j], lhit[j], ghit[j], sk[j],
+                            nullptr, 0, sj, nullptr, &ov);
+    if (set) swap_scratch(idx, p->alt);
+  }
+  // the caller's stream continues after the second stream's batches
+  if (cudaEventRecord(p->finish, p->stream) != cudaSuccess || cudaStreamWaitEvent(s, p->finish, 0) != cudaSuccess)
+    return rc ? rc : cuda_status(cudaErrorUnknown);
+  return rc;
+}
+
+}  // namespace
 
 extern "C" {
 
@@ -1971,6 +2209,16 @@ int smetric_route_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_t
   return route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance,
                             d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap,
                             reinterpret_cast<cudaStream_t>(stream));
+}
+
+int smetric_route_batches(smetric_index* idx, int32_t n_batches, const int32_t* const* d_tokens,
+                          const int64_t* n_tokens, const int64_t* const* d_offsets, const int32_t* n_requests,
+                          const int64_t* const* d_load, smetric_weights w, int32_t* const* d_instance,
+                          int32_t* const* d_local_hit, int32_t* const* d_global_hit,
+                          uint64_t* const* d_session_key, smetric_stream_t stream) {
+  CallRange range("smetric_route_batches");
+  return route_batches(idx, n_batches, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance,
+                       d_local_hit, d_global_hit, d_session_key, reinterpret_cast<cudaStream_t>(stream));
 }
 
 int smetric_route_batch_sequential(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,

@@ -60,7 +60,7 @@ def _create(L, **kw):
 @pytest.mark.parametrize("bad", [
     dict(num_instances=0), dict(num_instances=257), dict(block_size=7), dict(block_size=0),
     dict(block_size=258), dict(session_blocks=0), dict(capacity_slots=0),
-    dict(max_batch_requests=-1), dict(max_batch_tokens=-5), dict(flags=8),
+    dict(max_batch_requests=-1), dict(max_batch_tokens=-5), dict(flags=8), dict(flags=4),
     dict(capacity_slots=(1 << 64) - 1),
 ])
 def test_create_rejects_bad_config_on_host(L, bad):
@@ -106,6 +106,9 @@ def test_null_handles_are_rejected(L):
                                      None) == pkg.SMETRIC_ERR_INVALID_ARG
     assert L.smetric_window_imbalance(None, None, None, None, 0, 1, 1, None, 0, None, None, None,
                                       None) == pkg.SMETRIC_ERR_INVALID_ARG
+    w = pkg.smetric_weights(1, 4, 2)
+    assert L.smetric_route_batches(None, 0, None, None, None, None, None, w, None, None, None, None,
+                                   None) == pkg.SMETRIC_ERR_INVALID_ARG
     assert L.smetric_index_mask_words(None) == 0
     assert L.smetric_launch_count(None) == 0
 
