@@ -2016,16 +2016,18 @@ struct Pipeline {
   cudaEvent_t start = nullptr, finish = nullptr;   // the caller's stream to `stream`, and back
 };
 
+// Both live until the process ends and are never destroyed, so that an index
+// destroyed late in process exit still finds them.
 static std::mutex& pipeline_mutex() {
-  static std::mutex m;
-  return m;
+  static std::mutex* m = new std::mutex;
+  return *m;
 }
 
 // Indexes created with SMETRIC_FLAG_PIPELINE and their second sets (kept
 // beside the index so that the index's layout stays as it is).
 static std::unordered_map<const smetric_index*, Pipeline*>& pipelines() {
-  static std::unordered_map<const smetric_index*, Pipeline*> table;
-  return table;
+  static auto* table = new std::unordered_map<const smetric_index*, Pipeline*>;
+  return *table;
 }
 
 static Pipeline* pipeline_of(const smetric_index* idx) {
