@@ -107,7 +107,8 @@ typedef struct {
  * tier masks, 2 * (max_batch_requests + 1) for per-request offsets, group
  * leaders and shared-block counts, and 2 * G for the group table, G the
  * smallest power of two >= max(64, 2 * max_batch_requests);
- * W = ceil((N+1)/64).
+ * W = ceil((N+1)/64). SMETRIC_FLAG_PIPELINE allocates a second route scratch
+ * of the same size (and two streams) for smetric_route_batches.
  * Returns SMETRIC_ERR_INVALID_ARG for an out-of-range field and
  * SMETRIC_ERR_OOM when a device allocation fails; *out is NULL then. */
 int smetric_index_create(const smetric_index_config* cfg, smetric_index** out);
