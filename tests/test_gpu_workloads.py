@@ -204,3 +204,44 @@ def test_config5_full_size_points_sampled(N, B, batch):
     assert_outputs_equal(sel, o, fields=("instance", "local_hit", "global_hit", "session_key"),
                          ctx=f"config 5 N={N} B={B} batch={batch}")
     ix.close()
+
+
+@pytest.mark.xfail(strict=False, reason="smetric_route_batches has not yet run on a GPU")
+@pytest.mark.parametrize("pipeline", [True, False])
+def test_route_batches_equal_one_route_per_batch(pipeline):
+    """Config-4-shaped batches (2,048 sessions, 512 requests a batch) routed
+    five per smetric_route_batches call, on an index with a second scratch
+    set (consecutive batches overlapped on two streams) and on one without:
+    every output of every batch equals that batch's own smetric_route_batch
+    call, including a batch with a decreasing offset (invalid-batch outputs
+    and the latched error) and an empty batch; repeated calls agree."""
+    tr = burst_trace(n_sessions=2048, batch_size=512)
+    p = tr.params
+    chunk = 512
+    host = [tr.batch(k) for k in range(3)]
+    max_tok = max(max(b.n_tokens for b in host), chunk * int(tr.prefix_len.max()))
+    ix = pkg.SMetricIndex(p.num_instances, p.block_size, p.session_blocks,
+                          capacity_slots=int(tr.n_prefix_blocks() / 0.7) + 1, max_batch_requests=chunk,
+                          max_batch_tokens=max_tok, hash_seed=p.hash_seed, pipeline=pipeline)
+    _populate_c4(ix, tr, chunk=chunk)
+    batches = [(T(b.tokens), T(b.offsets), T(b.load)) for b in host]
+    bad_off = host[2].offsets.copy()
+    bad_off[5] = bad_off[6] + 1
+    empty = (T(np.zeros(0, np.int32)), T(np.zeros(1, np.int64)), T(host[0].load))
+    batches = [batches[0], batches[1], (batches[2][0], T(bad_off), batches[2][2]), empty, batches[2]]
+    w = (p.w_load, p.w_miss, p.w_glob)
+    want, codes = [], []
+    for b in batches:
+        want.append({k: v.cpu().numpy() for k, v in ix.route_batch(*b, w).items()})
+        codes.append(ix.status())
+    assert codes == [pkg.SMETRIC_OK, pkg.SMETRIC_OK, pkg.SMETRIC_ERR_INVALID_ARG, pkg.SMETRIC_OK, pkg.SMETRIC_OK]
+    for rep in range(2):
+        got = ix.route_batches(batches, w)
+        assert ix.status() == pkg.SMETRIC_ERR_INVALID_ARG
+        assert len(got) == len(batches)
+        for j, (g, o) in enumerate(zip(got, want)):
+            g = {k: v.cpu().numpy() for k, v in g.items()}
+            assert_outputs_equal(g, o, fields=("instance", "local_hit", "global_hit", "session_key"),
+                                 ctx=f"pipeline={pipeline} call {rep} batch {j}")
+    assert np.all(want[2]["instance"] == -1) and np.all(want[4]["instance"] >= 0)
+    ix.close()
