@@ -317,6 +317,33 @@ def oracle_calibrate(tr, ox, bt, seconds, threads):
         m = min(bt.n_requests, max(m * 2, int(m * seconds / max(dt, 1e-3))))
 
 
+def cpu_baseline(tr, bt, batch_id, seconds, threads=None):
+    """The oracle timed on the host cores on batch `bt`: a bounded sample of
+    about `seconds` on every core (the whole batch repeated when it is
+    quicker), and a smaller sample on one thread."""
+    threads = threads or os.cpu_count() or 1
+    ox = oracle_index_for(tr, [bt])
+    m, dt = oracle_calibrate(tr, ox, bt, seconds, threads)
+    reps = 1
+    if m == bt.n_requests and dt < seconds / 2:
+        # the whole batch is quicker than the target: route it repeatedly
+        reps = max(2, int(seconds / max(dt, 1e-3)))
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            oracle_route(tr, ox, bt, m, threads)
+        dt = time.perf_counter() - t0
+    what = (f"{reps} passes over all {m} requests" if reps > 1 else
+            f"first {m} of the {bt.n_requests} requests")
+    m1, dt1 = oracle_calibrate(tr, ox, bt, seconds / 4, 1)
+    ox.close()
+    return {"value": reps * m / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"{what} of config-4 batch {batch_id} ({dt:.1f} s on {threads} threads), "
+                      f"oracle index holding that batch's sessions",
+            "tokens_per_s": reps * float(bt.offsets[m]) / dt,
+            "single_thread": {"value": m1 / dt1, "unit": UNIT, "cores": 1,
+                              "sample": f"first {m1} requests of the same batch ({dt1:.1f} s on one thread)"}}
+
+
 def run_reference(args, rank, world, dist):
     if rank != 0:
         return
@@ -510,23 +537,7 @@ def run_ours(args, rank, world, local, dist):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        threads = os.cpu_count() or 1
-        ox = oracle_index_for(tr, host[:1])
-        m, dt = oracle_calibrate(tr, ox, host[0], args.cpu_seconds, threads)
-        reps = 1
-        if m == host[0].n_requests and dt < args.cpu_seconds / 2:
-            # the whole batch is quicker than the target: route it repeatedly
-            reps = max(2, int(args.cpu_seconds / max(dt, 1e-3)))
-            t0 = time.perf_counter()
-            for _ in range(reps):
-                oracle_route(tr, ox, host[0], m, threads)
-            dt = time.perf_counter() - t0
-        what = (f"{reps} passes over all {m} requests" if reps > 1 else
-                f"first {m} of the {host[0].n_requests} requests")
-        cpu = {"value": reps * m / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
-               "sample": f"{what} of config-4 batch {ids[0]} ({dt:.1f} s on {threads} threads), "
-                         f"oracle index holding that batch's sessions",
-               "tokens_per_s": reps * float(host[0].offsets[m]) / dt}
+        cpu = cpu_baseline(tr, host[0], ids[0], args.cpu_seconds)
 
     if rank == 0:
         line = {

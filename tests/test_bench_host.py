@@ -163,3 +163,18 @@ def test_route_stats_on_oracle_routed_burst_batches():
     assert 0.5 < s["local_hit_ratio"] + s["global_hit_ratio"] <= 1.0
     assert 1.0 <= s["routed_token_imbalance"] <= p.num_instances
     assert s["batches"] == 2
+
+
+def test_cpu_baseline_reports_all_cores_and_one_thread():
+    """The oracle timing the bench line carries: a bounded sample on the
+    given cores and one on a single thread, each with its sample stated."""
+    import oracle
+    from synth import burst_trace
+    oracle.build()
+    tr = burst_trace(n_sessions=512, batch_size=64)
+    bt = tr.batch(0)
+    c = bench.cpu_baseline(tr, bt, 0, seconds=0.4, threads=2)
+    assert c["kind"] == "oracle" and c["cores"] == 2 and c["unit"] == bench.UNIT
+    assert c["value"] > 0 and c["tokens_per_s"] > 0 and "batch 0" in c["sample"]
+    one = c["single_thread"]
+    assert one["cores"] == 1 and one["value"] > 0 and "one thread" in one["sample"]
