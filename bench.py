@@ -122,7 +122,31 @@ class ClockSampler:
             self.proc = None
         self.t0 = time.time()
 
-    def stop(self):
+    def n_samples(self) -> int:
+        """Rows written so far."""
+        try:
+            with open(self.f.name) as g:
+                return sum(1 for r in g if r.strip())
+        except OSError:
+            return 0
+
+    def soak(self, step, min_samples=8, max_seconds=6.0):
+        """Runs `step(i)` (untimed, synchronising every 50 calls) until the
+        sampler holds at least `min_samples` rows or `max_seconds` pass, so
+        that a short timed region still gets a clock record of the same load
+        around it. Returns the number of steps run."""
+        import torch
+        if self.proc is None:
+            return 0
+        t0, i = time.time(), 0
+        while self.n_samples() < min_samples and time.time() - t0 < max_seconds:
+            for _ in range(50):
+                step(i)
+                i += 1
+            torch.cuda.synchronize()
+        return i
+
+    def stop(self, window="warm-up and timed steps"):
         if self.proc is not None:
             self.proc.terminate()
             try:
@@ -147,7 +171,7 @@ class ClockSampler:
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None,
                 "reasons": sorted(reasons), "samples": len(sm),
-                "window": "warm-up and timed steps"}
+                "window": window}
 
 
 def peak_hbm():
@@ -458,7 +482,9 @@ def run_ours(args, rank, world, local, dist):
     torch.cuda.synchronize()
     ms = ev0.elapsed_time(ev1)
     launches = pkg.smetric_launch_count(ix.handle) - launches0
-    clk = clocks.stop()
+    soaked = clocks.soak(step)
+    clk = clocks.stop("warm-up and timed steps" + (f", then {soaked} more of the same steps (untimed) so that "
+                                                   f"the sampler, every 100 ms, records the load" if soaked else ""))
     rc = ix.status()
     if rc != pkg.SMETRIC_OK:
         raise pkg.SmetricError(rc, "bench")
@@ -675,7 +701,9 @@ def run_policy(args):
     torch.cuda.synchronize()
     ms = ev0.elapsed_time(ev1)
     launches = pkg.smetric_launch_count(ix.handle) - launches0
-    clk = clocks.stop()
+    soaked = clocks.soak(step)
+    clk = clocks.stop("warm-up and timed steps" + (f", then {soaked} more of the same steps (untimed)"
+                                                   if soaked else ""))
     if ix.status() != pkg.SMETRIC_OK:
         raise RuntimeError("policy bench: device error")
     reqs = float(np.mean([b.n_requests for b in host]))

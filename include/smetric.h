@@ -408,7 +408,10 @@ int smetric_block_hashes(smetric_index* idx, const int32_t* d_tokens, int64_t n_
  * existing from module load). The first call on each device, with that
  * device current, looks up the array's device address once
  * (cudaGetSymbolAddress) and caches it; make that first call before any
- * stream capture on the device.
+ * stream capture on the device. The cached address belongs to the device's
+ * context as it was at that first call: after cudaDeviceReset (or anything
+ * else that destroys and recreates the primary context) it is stale, so do
+ * not call this function again in that process after such a reset.
  *
  * Limits: n_requests <= SMETRIC_NOALLOC_MAX_REQUESTS and
  * n_tokens / block_size <= SMETRIC_NOALLOC_MAX_BLOCKS; a larger batch returns

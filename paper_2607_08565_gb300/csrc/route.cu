@@ -2498,6 +2498,8 @@ std::atomic<uint64_t*> na_addr[kNaMaxDevices];
 
 // Device address of na_scratch on the current device, looked up once per
 // device (the first call on a device should not be under stream capture).
+// The cached address is not refreshed after a device reset (a reset
+// recreates the context and reloads the module).
 int na_scratch_for(int dev, uint64_t** out) {
   if (dev < 0 || dev >= kNaMaxDevices) return SMETRIC_ERR_INVALID_ARG;
   uint64_t* p = na_addr[dev].load(std::memory_order_acquire);

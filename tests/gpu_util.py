@@ -58,9 +58,14 @@ def assert_outputs_equal(g, o, fields=FIELDS + ("block_hashes",), ctx=""):
                               f"gpu {a[bad[:5]]} oracle {b[bad[:5]]}"
 
 
-def replay_both(trace, n_batches=None, cap=None, n_threads=8):
+def replay_both(trace, n_batches=None, cap=None, n_threads=8, shared_driver=False):
     """Replay an agent trace through the GPU and through the oracle, each
-    side driving its own index from its own outputs; compare every batch."""
+    side driving its own index from its own outputs; compare every batch.
+
+    With shared_driver, one replay driver serves both sides: every batch's
+    outputs are asserted equal before the driver consumes them, so the two
+    drivers would receive identical inputs and produce identical insert and
+    evict lists; sharing halves the host-side LRU work of the long replays."""
     p = trace.params
     batches = list(itertools.islice(trace.batches(), n_batches))
     total_blocks = sum(n_blocks(b.offsets, p.block_size) for b in batches)
@@ -71,7 +76,7 @@ def replay_both(trace, n_batches=None, cap=None, n_threads=8):
     ox = oracle.OracleIndex(p.num_instances)
     kw = dict(local_cap=trace.local_cap, global_policy=trace.global_policy, global_cap=trace.global_cap)
     dg = ReplayDriver(p.num_instances, p.block_size, **kw)
-    do = ReplayDriver(p.num_instances, p.block_size, **kw)
+    do = dg if shared_driver else ReplayDriver(p.num_instances, p.block_size, **kw)
     w = (p.w_load, p.w_miss, p.w_glob)
     stats = dict(batches=0, requests=0, local=0, glob=0, evicted=0)
     for k, bt in enumerate(batches):
@@ -85,7 +90,8 @@ def replay_both(trace, n_batches=None, cap=None, n_threads=8):
         if len(ek):
             ix.evict(T(ek), T(et))
         ix.check()
-        ik, it_, ek, et = do.after_batch(bt.offsets, o["instance"], o["local_hit"], o["block_hashes"])
+        if not shared_driver:
+            ik, it_, ek, et = do.after_batch(bt.offsets, o["instance"], o["local_hit"], o["block_hashes"])
         ox.insert(ik, it_)
         ox.evict(ek, et)
         assert np.array_equal(dg.load, do.load)

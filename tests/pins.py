@@ -148,6 +148,60 @@ def check_sentinel_remap(L):
             assert int(h2[1]) == _py_mix64(((want + GAMMA) & M64) ^ d1)
 
 
+def _fold(x, words):
+    for w in words:
+        x = _py_mix64(x ^ w)
+    return x
+
+
+def _words_to_tokens(words):
+    out = []
+    for w in words:
+        out += [w & 0xFFFFFFFF, w >> 32]
+    return np.array(out, dtype=np.uint32).view(np.int32)
+
+
+def multiword_tokens(targets, B, seed, rng):
+    """Tokens of len(targets) blocks of B tokens (B/2 >= 2 words each) whose
+    chain values h_0, h_1, ... before the remap are the given targets. Every
+    word of a block but the last is random; the last is solved for by
+    inverting mix64, the chain step and the digest's final fold step, so the
+    construction relies on the words being folded first to last from
+    mix64(seed ^ B)."""
+    hb = B // 2
+    h = _py_mix64((seed + GAMMA) & M64)
+    words = []
+    for target in targets:
+        d = py_mix64_inverse(target) ^ ((h + GAMMA) & M64)  # h_b = mix64((h + G) ^ d_b)
+        head = [int(x) for x in rng.integers(0, 1 << 63, size=hb - 1, dtype=np.uint64)]
+        x = _fold(_py_mix64(seed ^ B), head)  # fold of every word but the last
+        words += head + [py_mix64_inverse(d) ^ x]  # d_b = mix64(x ^ w_last)
+        h = target if target >= 2 else target | 2
+    return _words_to_tokens(words)
+
+
+def check_multiword_digest(L):
+    """Blocks of several words: the digest folds the block's words in order,
+    first to last, each into the running value. Tokens built backwards from
+    chosen chain values (the last word of each block solved for through the
+    inverse of mix64) must hash to exactly those values, for B = 4, 6, 16 and
+    two seeds, including a chain value of 0 (remapped to 2) inside the run."""
+    rng = np.random.default_rng(12)
+    for B in (4, 6, 16):
+        for seed in (0, (1 << 63) + 5):
+            targets = [int(x) | 2 for x in rng.integers(0, 1 << 63, size=3, dtype=np.uint64)]
+            targets.insert(1, 0)
+            t = multiword_tokens(targets, B, seed, rng)
+            h = oracle.block_hashes(t, B, seed, L)
+            want = [x if x >= 2 else x | 2 for x in targets]
+            assert [int(v) for v in h] == want, (B, seed)
+            # one word of the first block moved: every chain value changes
+            u = t.copy()
+            u[[0, 2]] = u[[2, 0]]
+            hu = oracle.block_hashes(u, B, seed, L)
+            assert all(int(a) != int(b) for a, b in zip(hu, h)), (B, seed)
+
+
 # ---------------------------------------------------------------------------
 # routing
 # ---------------------------------------------------------------------------
@@ -978,6 +1032,7 @@ ALL_CHECKS = [
     check_tail_and_empty,
     check_seed_and_block_size,
     check_sentinel_remap,
+    check_multiword_digest,
     check_session_key,
     check_brute_force_prefix,
     check_non_prefix_closed,

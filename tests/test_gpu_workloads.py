@@ -4,10 +4,13 @@ Configs 1-3 are multi-batch replays: after every batch each side inserts the
 routed blocks into its own index, evicts by LRU and drains its load, so the
 two replays stay identical only if every batch's outputs are bit-exact.
 Config 4 runs at full size in the launch configuration the benchmark times
-(65,536 sessions, 64 instances, B = 32, a batch of 8,192 requests): the
-oracle recomputes a sample of requests one by one, and invariants that hold
-at any size are checked on every request.
+(65,536 sessions, 64 instances, B = 32, batches of 8,192 requests): every
+request of the four batches the benchmark rotates is compared with the
+oracle, and invariants that hold at any size are checked on every request.
+Configs 2 and 3 are also replayed whole (the long cases carry the slow mark).
 """
+
+import os
 
 import numpy as np
 import pytest
@@ -48,6 +51,27 @@ def test_replay_config3_reduced_with_truncation_and_eviction():
     tr.local_cap = 400
     tr.global_cap = 3000
     st = replay_both(tr)
+    assert st["evicted"] > 0
+
+
+@pytest.mark.slow
+def test_replay_config2_full():
+    """Config 2 at full size: 1024 sessions x 16 turns, 64 batches of 256
+    requests, local tiers LRU-capped at 200k blocks, every block in the
+    global tier; both replays compared batch by batch."""
+    st = replay_both(agent_trace("c2_medium"), shared_driver=True)
+    assert st["batches"] == 64 and st["requests"] == 64 * 256
+    assert st["glob"] > 0 and st["local"] > 0
+
+
+@pytest.mark.slow
+def test_replay_config3_full():
+    """Config 3 at full size: 4096 sessions x 32 turns, 128 batches of 1024
+    requests with half the turns truncated, local tiers LRU-capped at 1M
+    blocks and the global tier at 16M; both replays compared batch by
+    batch."""
+    st = replay_both(agent_trace("c3_long"), shared_driver=True)
+    assert st["batches"] == 128 and st["requests"] == 128 * 1024
     assert st["evicted"] > 0
 
 
@@ -123,6 +147,42 @@ def test_config4_full_size_sampled():
         one = {f: g[f][r:r + 1] for f in ("instance", "local_hit", "global_hit", "session_key")}
         assert_outputs_equal(one, o, fields=("instance", "local_hit", "global_hit", "session_key"),
                              ctx=f"config 4 request {r}")
+    ix.close()
+
+
+@pytest.mark.slow
+def test_config4_bench_batches_every_request():
+    """The four config-4 batches the benchmark rotates (65,536 sessions,
+    64 instances, B = 32, 8,192 requests each), routed in the benchmark's
+    launch configuration on the fully populated index: every output of every
+    request, and every block hash, equals the oracle's. The oracle's index
+    holds the prefixes of every session the four batches use; requests hit
+    only their own session's blocks (the reach check below), so the rest of
+    the GPU index does not change any decision."""
+    tr = burst_trace()
+    p = tr.params
+    N, B = p.num_instances, p.block_size
+    nkeys = tr.n_prefix_blocks()
+    host = [tr.batch(k) for k in range(4)]
+    ix = make_index(N, B, p.session_blocks, cap=int(nkeys / 0.7) + 1,
+                    max_req=max(max(b.n_requests for b in host), 4096),
+                    max_tok=max(max(b.n_tokens for b in host), 4096 * int(tr.prefix_len.max())))
+    _populate_c4(ix, tr)
+    ox = oracle.OracleIndex(N)
+    sessions = np.unique(np.concatenate([b.sessions for b in host]))
+    for s in sessions.tolist():
+        h = oracle.block_hashes(tr.session_prefix(s), B, p.hash_seed)
+        for t in tr.session_tiers(s):
+            ox.insert(h, t)
+    w = (p.w_load, p.w_miss, p.w_glob)
+    for k, bt in enumerate(host):
+        g = gpu_route(ix, bt.tokens, bt.offsets, bt.load, w, want_hashes=True)
+        o = ox.route_batch(B, p.session_blocks, p.hash_seed, bt.tokens, bt.offsets, bt.load, *w,
+                           want_hashes=True, n_threads=os.cpu_count() or 1)
+        assert_outputs_equal(g, o, ctx=f"config 4 batch {k}")
+        reach = (o["local_hit"] + o["global_hit"]) // B
+        assert np.all(reach == tr.prefix_len[bt.sessions] // B)
+    ox.close()
     ix.close()
 
 
@@ -206,7 +266,6 @@ def test_config5_full_size_points_sampled(N, B, batch):
     ix.close()
 
 
-@pytest.mark.xfail(strict=False, reason="smetric_route_batches has not yet run on a GPU")
 @pytest.mark.parametrize("pipeline", [True, False])
 def test_route_batches_equal_one_route_per_batch(pipeline):
     """Config-4-shaped batches (2,048 sessions, 512 requests a batch) routed

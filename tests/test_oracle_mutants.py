@@ -27,6 +27,12 @@ MUTANTS = {
     "chain_xor_for_add": ("h = oracle_mix64((h + ORACLE_GAMMA) ^ d);",
                           "h = oracle_mix64((h ^ ORACLE_GAMMA) ^ d);"),
     "no_sentinel_remap": ("if (h < 2) h |= 2;", ""),
+    "digest_fold_reversed": ("for (int32_t k = 0; k < B / 2; ++k) d = oracle_mix64(",
+                             "for (int32_t k = B / 2 - 1; k >= 0; --k) d = oracle_mix64("),
+    "digest_skips_word0": ("for (int32_t k = 0; k < B / 2; ++k) d = oracle_mix64(",
+                           "for (int32_t k = 1; k < B / 2; ++k) d = oracle_mix64("),
+    "digest_last_word_only": ("d = oracle_mix64(d ^ oracle_word(tokens, b * B + 2 * k));",
+                              "d = oracle_mix64(oracle_mix64(seed ^ (uint64_t)B) ^ oracle_word(tokens, b * B + 2 * k));"),
     "word_index_off_by_one": ("oracle_word(tokens, b * B + 2 * k)",
                               "oracle_word(tokens, b * B + k)"),
     "session_key_index": ("session_key[r] = h[(n < S ? n : S) - 1];",

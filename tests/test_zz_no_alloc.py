@@ -1,8 +1,8 @@
 """smetric_block_hashes_noalloc: block hashes and session keys from the fixed
 scratch compiled into the library, with no index and no allocation. Its
 outputs must equal those of smetric_block_hashes (an index's scratch) on the
-same batches, call after call, and a batch beyond the fixed scratch must be
-refused before anything is enqueued.
+same batches, call after call, and those of the CPU oracle; a batch beyond
+the fixed scratch must be refused before anything is enqueued.
 
 The file name sorts last so that the test also runs after every other GPU
 test has used the library in the same process."""
@@ -11,6 +11,7 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 import paper_2607_08565_gb300 as pkg
 from synth.traces import pack
 
@@ -53,6 +54,16 @@ def _with_index(tok, off, B, S, seed):
     return U(hb), U(sk)
 
 
+def _oracle(tok, off, B, S, seed):
+    """Block hashes (request-major) and session keys from the CPU oracle."""
+    hs, keys = [], []
+    for r in range(len(off) - 1):
+        h = oracle.block_hashes(tok[off[r]:off[r + 1]], B, seed)
+        hs.append(h)
+        keys.append(int(h[min(len(h), S) - 1]) if len(h) else 0)
+    return np.concatenate(hs).astype(np.uint64), np.array(keys, dtype=np.uint64)
+
+
 def U(t):
     """A device tensor of 64-bit words as a host uint64 array."""
     return t.cpu().view(torch.int64).numpy().view(np.uint64)
@@ -79,6 +90,10 @@ def test_two_calls_in_a_row_equal_the_index_path(B, S, seed):
         m = _used_blocks(off, B)
         assert np.array_equal(U(hb)[:m], rhb[:m])
         assert np.array_equal(U(sk)[: len(off) - 1], rsk[: len(off) - 1])
+        # and the CPU oracle's own hashes and session keys, request by request
+        ohb, osk = _oracle(tok, off, B, S, seed)
+        assert np.array_equal(U(hb)[:m], ohb)
+        assert np.array_equal(U(sk)[: len(off) - 1], osk)
 
 
 def test_largest_accepted_batch_and_refusals():
@@ -96,6 +111,8 @@ def test_largest_accepted_batch_and_refusals():
     assert rc == pkg.SMETRIC_OK
     rhb, rsk = _with_index(tok, off, B, 2, 9)
     assert np.array_equal(U(hb), rhb[:nb_max]) and np.array_equal(U(sk), rsk[:n_max])
+    ohb, osk = _oracle(tok, off, B, 2, 9)
+    assert np.array_equal(U(hb), ohb) and np.array_equal(U(sk), osk)
     assert int(status.item()) == 0
 
     # one request or one block more: refused, outputs untouched
