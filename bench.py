@@ -263,18 +263,18 @@ def algorithmic_bytes(lens, local_hit, global_hit, B, W):
     with reach_r taken from the chosen instance's hits, g_{i*} = max(c_{i*}, g):
     never above max(max_i c_i, g), and equal to it when the global tier holds
     every local tier's blocks (config 4), so the count never overstates.
-    k_chain: the digests it reads and hashes it writes (intermediates of this
-    kernel split). k_walk: the masks it reads, offsets and outputs. k_prep:
-    offsets and loads. path: the method's bytes per request,
-    4 L_r + P_r (8 + 8W) + 8 + 20."""
+    k_chain_probe adds to those entries the digests the chain reads and the
+    hashes it writes (8 B each per block). k_walk: the masks it reads, offsets
+    and outputs. k_prep: offsets and loads. path: the method's bytes per
+    request, 4 L_r + P_r (8 + 8W) + 8 + 20."""
     nb = lens // B
     reach = (local_hit.astype(np.int64) + global_hit) // B
     probes = np.minimum(nb, reach + 1)
     n = len(lens)
     return {
         "k_digest": int(4 * B * nb.sum()),
-        "k_chain": int(16 * nb.sum() + 24 * n),
         "k_probe": int(probes.sum() * (8 + 8 * W)),
+        "k_chain_probe": int(16 * nb.sum() + 24 * n + probes.sum() * (8 + 8 * W)),
         "k_walk": int(8 * W * probes.sum() + 28 * n),
         "k_prep": int(16 * n),
         "path": int(4 * lens.sum() + probes.sum() * (8 + 8 * W) + 8 * (n + 1) + 20 * n),

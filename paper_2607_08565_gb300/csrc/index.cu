@@ -317,10 +317,12 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
             cudaMalloc(&x->tags, slots) == cudaSuccess &&
             cudaMalloc(&x->status, sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->block_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
-            cudaMalloc(&x->digest, (max_blocks > 0 ? max_blocks : 1) * sizeof(uint64_t)) == cudaSuccess &&
+            // two spare words: k_chain_probe copies a chunk's digests in whole 16-byte pieces
+            cudaMalloc(&x->digest, (max_blocks + 2) * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->hashes, (max_blocks > 0 ? max_blocks : 1) * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->masks, (max_blocks > 0 ? max_blocks : 1) * W * sizeof(uint64_t)) == cudaSuccess &&
-            cudaMalloc(&x->chunk_and, (max_blocks / 32 + 1) * W * sizeof(uint64_t)) == cudaSuccess &&
+            // one per request-aligned 32-block chunk: at most max_blocks / 32 + R
+            cudaMalloc(&x->chunk_and, (max_blocks / 32 + R + 1) * W * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->groups, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->lead, 2 * (R + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->chunk_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&

@@ -83,14 +83,18 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
                                               int32_t* status, int64_t max_load, int64_t max_len,
                                               const int64_t* __restrict__ est_hit,
                                               const int64_t* __restrict__ aux0 = nullptr, int64_t aux0_max = 0,
-                                              const int64_t* __restrict__ aux1 = nullptr, int64_t aux1_max = 0) {
+                                              const int64_t* __restrict__ aux1 = nullptr, int64_t aux1_max = 0,
+                                              int32_t* __restrict__ zero2 = nullptr) {
   constexpr int NS = 2;  // scans: full blocks, and 32-block chunks (when chunk_off is wanted)
   constexpr int R = kPrepRounds;
   __shared__ int64_t warp_tot[NS][32];
   __shared__ int64_t pass_tot[NS];
   __shared__ int bad_all;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
-  if (tid == 0) bad_all = 0;
+  if (tid == 0) {
+    bad_all = 0;
+    if (zero2) { zero2[0] = 0; zero2[1] = 0; }  // the group stage's leader and member counts
+  }
   __syncthreads();
   int bad = 0;  // bit 0: invalid offsets, bit 1: out-of-range length or load
   for (int i = tid; i < n_load; i += blockDim.x) {
@@ -188,6 +192,33 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
 // digest
 // ---------------------------------------------------------------------------
 
+// The group stage works from the digests, so that it runs beside the chain:
+// a request's first-block hash h_0 = chain step from h_init over d_0 is the
+// group key, and the shared-prefix length is the number of leading blocks
+// whose digests equal the leader's. Equal digests from equal previous hashes
+// give equal hashes, so the leader's masks serve those blocks exactly.
+__device__ __forceinline__ uint64_t first_hash(uint64_t h_init, uint64_t d0) {
+  uint64_t h = mix64((h_init + kGamma) ^ d0);
+  return h < 2 ? (h | 2) : h;
+}
+
+// Requests whose first block hashes are equal form a group; its leader is
+// the lowest request id. Table of (key, INT32_MAX - leader) word pairs,
+// key 0 = empty (block hashes are >= 2), linear probing, at most half full.
+__device__ __forceinline__ void group_insert(uint64_t* __restrict__ groups, uint64_t gmask, uint64_t key,
+                                             int32_t r) {
+  uint64_t s = key & gmask;
+  for (uint64_t t = 0; t <= gmask; ++t) {
+    unsigned long long* const slot = reinterpret_cast<unsigned long long*>(groups + 2 * s);
+    const unsigned long long k = atomicCAS(slot, 0ull, (unsigned long long)key);
+    if (k == 0ull || k == key) {
+      atomicMax(slot + 1, (unsigned long long)(INT32_MAX - r));
+      return;
+    }
+    s = (s + 1) & gmask;
+  }
+}
+
 // Largest r in [lo, n) with block_off[r] <= f, given block_off[lo] <= f < block_off[n].
 __device__ __forceinline__ int32_t find_request(const int64_t* __restrict__ block_off, int32_t lo,
                                                 int32_t n, int64_t f) {
@@ -250,7 +281,8 @@ template <int HB>
 __global__ void __launch_bounds__(kDigestWarps * 32)
     k_digest(const int32_t* __restrict__ tokens, int64_t n_tokens, const int64_t* __restrict__ off,
              const int64_t* __restrict__ block_off, int32_t n, uint64_t d_init,
-             const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ digest) {
+             const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ digest,
+             uint64_t* __restrict__ groups, uint64_t gmask, uint64_t h_init) {
   pdl_enter();
   constexpr int B = 2 * HB;
   constexpr int PB = HB > 0 ? HB / 2 : 1;  // 16-byte pieces per block (k_digest<0> is never launched)
@@ -275,16 +307,21 @@ __global__ void __launch_bounds__(kDigestWarps * 32)
     int64_t tok0;  // this lane's first token
     int64_t a0;    // byte offset of piece 0 (fast path)
     int nv;        // valid lanes (a prefix of the warp)
-    bool valid, fast;
+    int32_t req;   // this lane's request
+    bool valid, fast, head;  // head: the lane's block is its request's block 0
   };
   uint4 buf[NP];
   // locate chunk c and load its bytes into registers
   auto load = [&](int64_t c, Chunk& ch) {
     const int64_t f = c * kChunk + lane;
     ch.valid = f < total;
+    ch.head = false;
+    ch.req = r;
     if (ch.valid) {
       if (__ldg(block_off + r + 1) <= f) r = find_request(block_off, r + 1, n, f);
       ch.tok0 = __ldg(off + r) + (f - __ldg(block_off + r)) * B;
+      ch.head = f == __ldg(block_off + r);
+      ch.req = r;
     } else {
       ch.tok0 = 0;
     }
@@ -332,7 +369,9 @@ __global__ void __launch_bounds__(kDigestWarps * 32)
     if (cur.valid) {
       const int delta = (int)((cur.tok0 * 4) & 15);  // 0, 4, 8 or 12
       const uint64_t* row = reinterpret_cast<const uint64_t*>(st + lane * NP) + (delta >> 3);
-      digest[c * kChunk + lane] = digest_row<HB>(row, (delta & 4) != 0, HB, d_init);
+      const uint64_t d = digest_row<HB>(row, (delta & 4) != 0, HB, d_init);
+      digest[c * kChunk + lane] = d;
+      if (groups && cur.head) group_insert(groups, gmask, first_hash(h_init, d), cur.req);
     }
     __syncwarp();
     cur = nxt;
@@ -393,7 +432,8 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
     k_digest_tma(const __grid_constant__ TokenMaps maps, const int32_t* __restrict__ tokens,
                  int64_t n_tokens, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off,
                  const int64_t* __restrict__ chunk_off, int32_t n, uint64_t d_init, const int32_t* __restrict__ batch_ok,
-                 uint64_t* __restrict__ digest, int32_t* status) {
+                 uint64_t* __restrict__ digest, int32_t* status, uint64_t* __restrict__ groups, uint64_t gmask,
+                 uint64_t h_init) {
   pdl_enter();
   constexpr int B = 2 * HB;
   constexpr int NP = HB / 2 + 1;           // 16-byte pieces per row
@@ -428,8 +468,9 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
   int32_t r = find_request(chunk_off, 0, n, c_lo);  // warp-uniform
 
   // Start the copy of chunk c into stage s; returns this lane's first token
-  // and sets its digest index.
-  auto issue = [&](int64_t c, int s, bool& valid, int64_t& gidx) -> int64_t {
+  // and sets its digest index and its request (`head` when the lane has the
+  // request's block 0, whose digest also gives the request's group key).
+  auto issue = [&](int64_t c, int s, bool& valid, int64_t& gidx, int32_t& req, bool& head) -> int64_t {
     for (int i = 0; i < 4 && __ldg(chunk_off + r + 1) <= c; ++i) ++r;  // usually a step or two
     if (__ldg(chunk_off + r + 1) <= c) r = find_request(chunk_off, r + 1, n, c);
     const int64_t bo = __ldg(block_off + r), nbr = __ldg(block_off + r + 1) - bo;
@@ -437,6 +478,8 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
     valid = b < nbr;
     const int64_t tok0 = __ldg(off + r) + b * B;
     gidx = bo + b;
+    req = r;
+    head = b == 0;
     const int nv = (int)min((int64_t)kChunk, nbr - (b - lane));
     const int64_t a0 = (4 * __shfl_sync(kFull, tok0, 0)) & ~(int64_t)15;
     const int k = (int)((a0 % (4 * B)) >> 4);
@@ -466,31 +509,36 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
 
   uint32_t phase = 0;
   bool failed = false;
-  bool v[STAGES];
+  bool v[STAGES], hd[STAGES];
   int64_t t[STAGES], gi[STAGES];
+  int32_t rq[STAGES];
 #pragma unroll
   for (int s = 0; s < STAGES; ++s)
-    if (c_lo + s * warps < c_hi) t[s] = issue(c_lo + s * warps, s, v[s], gi[s]);
+    if (c_lo + s * warps < c_hi) t[s] = issue(c_lo + s * warps, s, v[s], gi[s], rq[s], hd[s]);
   int s = 0;
   for (int64_t c = c_lo; c < c_hi; c += warps) {
     if (!mbar_wait(mbar0 + 8u * (uint32_t)s, (phase >> s) & 1)) { failed = true; break; }
     phase ^= 1u << s;
-    bool vc = false;
+    bool vc = false, hc = false;
     int64_t tc = 0, gc = 0;
+    int32_t rc = 0;
 #pragma unroll
-    for (int q = 0; q < STAGES; ++q) if (q == s) { vc = v[q]; tc = t[q]; gc = gi[q]; }
+    for (int q = 0; q < STAGES; ++q) if (q == s) { vc = v[q]; tc = t[q]; gc = gi[q]; rc = rq[q]; hc = hd[q]; }
     if (vc) {
       const int delta = (int)((tc * 4) & 15);  // 0, 4, 8 or 12
       const uint64_t* row = reinterpret_cast<const uint64_t*>(stages + (size_t)s * STAGE + lane * ROW) + (delta >> 3);
-      digest[gc] = digest_row<HB>(row, (delta & 4) != 0, HB, d_init);
+      const uint64_t d = digest_row<HB>(row, (delta & 4) != 0, HB, d_init);
+      digest[gc] = d;
+      if (groups && hc) group_insert(groups, gmask, first_hash(h_init, d), rc);
     }
     __syncwarp();
     if (c + STAGES * warps < c_hi) {
-      bool vn;
+      bool vn, hn;
       int64_t gn = 0;
-      const int64_t tn = issue(c + STAGES * warps, s, vn, gn);
+      int32_t rn = 0;
+      const int64_t tn = issue(c + STAGES * warps, s, vn, gn, rn, hn);
 #pragma unroll
-      for (int q = 0; q < STAGES; ++q) if (q == s) { v[q] = vn; t[q] = tn; gi[q] = gn; }
+      for (int q = 0; q < STAGES; ++q) if (q == s) { v[q] = vn; t[q] = tn; gi[q] = gn; rq[q] = rn; hd[q] = hn; }
     }
     s = s + 1 == STAGES ? 0 : s + 1;
   }
@@ -507,7 +555,8 @@ __global__ void __launch_bounds__(kTmaWarps * 32)
 __global__ void __launch_bounds__(kDigestWarps * 32)
     k_digest_any(const int32_t* __restrict__ tokens, int64_t n_tokens, const int64_t* __restrict__ off,
                  const int64_t* __restrict__ block_off, int32_t n, int B, int nch, uint64_t d_init,
-                 const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ digest) {
+                 const int32_t* __restrict__ batch_ok, uint64_t* __restrict__ digest,
+                 uint64_t* __restrict__ groups, uint64_t gmask, uint64_t h_init) {
   pdl_enter();
   extern __shared__ uint4 dsm[];
   if (!*batch_ok) return;
@@ -531,8 +580,10 @@ __global__ void __launch_bounds__(kDigestWarps * 32)
     const int64_t a = (4 * tok0) & ~(int64_t)15;
     for (int i = 0; i < nch; ++i) row[i] = load_piece(tb, a + 16 * i, token_bytes - (a + 16 * i));
     const int delta = (int)((tok0 * 4) & 15);
-    digest[f] = digest_row<0>(reinterpret_cast<const uint64_t*>(row) + (delta >> 3), (delta & 4) != 0,
-                              B >> 1, d_init);
+    const uint64_t d = digest_row<0>(reinterpret_cast<const uint64_t*>(row) + (delta >> 3), (delta & 4) != 0,
+                                     B >> 1, d_init);
+    digest[f] = d;
+    if (groups && f == __ldg(block_off + r)) group_insert(groups, gmask, first_hash(h_init, d), r);
   }
 }
 
@@ -634,112 +685,6 @@ __global__ void __launch_bounds__(kChainThreads)
 // group
 // ---------------------------------------------------------------------------
 
-// The group stage works from the digests, so that it runs beside the chain:
-// a request's first-block hash h_0 = chain step from h_init over d_0 is the
-// group key, and the shared-prefix length is the number of leading blocks
-// whose digests equal the leader's. Equal digests from equal previous hashes
-// give equal hashes, so the leader's masks serve those blocks exactly.
-__device__ __forceinline__ uint64_t first_hash(uint64_t h_init, uint64_t d0) {
-  uint64_t h = mix64((h_init + kGamma) ^ d0);
-  return h < 2 ? (h | 2) : h;
-}
-
-// Requests whose first block hashes are equal form a group; its leader is
-// the lowest request id. Table of (key, INT32_MAX - leader) word pairs,
-// key 0 = empty (block hashes are >= 2), linear probing, at most half full.
-__device__ __forceinline__ void group_insert(uint64_t* __restrict__ groups, uint64_t gmask, uint64_t key,
-                                             int32_t r) {
-  uint64_t s = key & gmask;
-  for (uint64_t t = 0; t <= gmask; ++t) {
-    unsigned long long* const slot = reinterpret_cast<unsigned long long*>(groups + 2 * s);
-    const unsigned long long k = atomicCAS(slot, 0ull, (unsigned long long)key);
-    if (k == 0ull || k == key) {
-      atomicMax(slot + 1, (unsigned long long)(INT32_MAX - r));
-      return;
-    }
-    s = (s + 1) & gmask;
-  }
-}
-
-// One thread per request: its first-block hash into the group table.
-__global__ void __launch_bounds__(256)
-    k_group_insert(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
-                   const uint64_t* __restrict__ digest, uint64_t h_init, uint64_t* __restrict__ groups,
-                   uint64_t gmask, int32_t* __restrict__ counts) {
-  const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (r == 0) { counts[0] = 0; counts[1] = 0; }  // k_group's leader and member counts
-  if (r >= n || !*batch_ok) return;
-  const int64_t bo = block_off[r];
-  if (block_off[r + 1] > bo) group_insert(groups, gmask, first_hash(h_init, __ldg(digest + bo)), (int32_t)r);
-}
-
-// One warp per request: its leader (the group table's entry for its first
-// block hash) and share = the number of leading blocks whose digests equal
-// the leader's. Both sides look up the same finished table, so a request
-// that leads a group finds itself (share 0) and its masks cover all its
-// blocks; a member's mask for block b < share is the leader's, exact because
-// a block's tier masks are a function of its hash alone.
-__global__ void __launch_bounds__(256)
-    k_group(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
-            const uint64_t* __restrict__ groups, uint64_t gmask, const uint64_t* __restrict__ D,
-            uint64_t h_init, int32_t* __restrict__ lead, int32_t* __restrict__ share,
-            int32_t* __restrict__ order, int32_t* __restrict__ counts) {
-  if (!*batch_ok) return;
-  const int lane = threadIdx.x & 31;
-  const int64_t tw = (int64_t)gridDim.x * (blockDim.x >> 5);
-  for (int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < n; r += tw) {
-    const int64_t bo = block_off[r], nb = block_off[r + 1] - bo;
-    int32_t l = (int32_t)r;
-    int64_t sh = 0;
-    if (nb > 0) {
-      const uint64_t key = first_hash(h_init, __ldg(D + bo));
-      const uint64_t s0 = key & gmask;
-      for (uint64_t t = 0; t <= gmask; t += 32) {
-        const uint64_t sl = (s0 + t + lane) & gmask;
-        const uint64_t k = groups[2 * sl];
-        const unsigned hit = __ballot_sync(kFull, k == key), emp = __ballot_sync(kFull, k == 0);
-        const unsigned stop = hit | emp;
-        if (stop) {
-          const int first = __ffs(stop) - 1;
-          if (hit & (1u << first))
-            l = INT32_MAX - (int32_t)groups[2 * ((s0 + t + first) & gmask) + 1];
-          break;
-        }
-      }
-      if (l != (int32_t)r && l >= 0 && l < n) {
-        const int64_t lo = block_off[l], nl = block_off[l + 1] - lo;
-        const int64_t m = nb < nl ? nb : nl;
-        sh = m;
-        // kGroupAhead rounds of 32 blocks per iteration, all loads in flight
-        for (int64_t b = 0; b < m; b += 32 * kGroupAhead) {
-          bool ne[kGroupAhead];
-#pragma unroll
-          for (int u = 0; u < kGroupAhead; ++u) {
-            const int64_t bb = b + 32 * u + lane;
-            ne[u] = bb < m && __ldg(D + bo + bb) != __ldg(D + lo + bb);
-          }
-          int64_t first = -1;
-#pragma unroll
-          for (int u = 0; u < kGroupAhead; ++u) {
-            const unsigned x = __ballot_sync(kFull, ne[u]);
-            if (x && first < 0) first = 32 * u + __ffs(x) - 1;
-          }
-          if (first >= 0) { sh = b + first; break; }
-        }
-      } else {
-        l = (int32_t)r;
-      }
-    }
-    if (lane == 0) {
-      lead[r] = l;
-      share[r] = (int32_t)sh;
-      // leaders listed from the front, members from the back (any order)
-      if (l == (int32_t)r) order[atomicAdd(counts, 1)] = (int32_t)r;
-      else order[n - 1 - atomicAdd(counts + 1, 1)] = (int32_t)r;
-    }
-  }
-}
-
 // ---------------------------------------------------------------------------
 // match
 // ---------------------------------------------------------------------------
@@ -778,47 +723,330 @@ __device__ __forceinline__ void probe_one(const uint8_t* __restrict__ tags, cons
   }
 }
 
-// One thread per block of the batch: the tier masks of every block hash.
-// Each warp also stores the AND of its 32 blocks' masks (blocks 32k..32k+31
-// of the batch, a block the kernel skips counting as all ones): for a chunk
-// that lies wholly inside one request's probed blocks this is the set of
-// tiers holding every block of the chunk, which lets the walk cross such a
-// chunk in one step.
+// ---------------------------------------------------------------------------
+// chain, shared prefix and probe in one kernel
+// ---------------------------------------------------------------------------
+//
+// The chain is bound by the latency of its dependent mix64 steps and the
+// probe by random memory accesses, so one kernel runs both at once. One CTA
+// of 32 warps per SM; the SM deals a CTA's warps to its four schedulers in
+// turn (warp w to scheduler w mod 4). The chain warps (lane = request) are
+// warps 0 .. chain_warps - 1, one per scheduler, beside probe warps that
+// mostly wait on memory, so their dependent steps seldom wait for issue. The
+// other warps first find each request's group leader and shared prefix, then
+// probe the index for each 32-block chunk as soon as its chain has published
+// it.
+//
+// CTA c owns requests c, c + gridDim, c + 2 gridDim, ..., taken in groups of
+// up to 32 * chain_warps (one chain lane each). Chunk q of request r is its
+// blocks 32q .. 32q + 31; the chunk ANDs the walk reads are kept per such
+// request-aligned chunk, at index chunk_off[r] + q.
+constexpr int kCpWarps = 32;
+constexpr int kCpMaxChainWarps = 4;  // warps 0 .. 3, one per scheduler
+constexpr int kCpMaxGroup = 32 * kCpMaxChainWarps;
+constexpr int kCpRingDigests = 34;   // a chunk's 32 digests and one neighbour on each side
+constexpr int kCpRingBytes = 560;    // two such slots per chain lane, in 16-byte pieces
+constexpr int kCpProbes = 2;         // chunks a probe warp takes at once (probes in flight per lane)
+
+__device__ __forceinline__ int32_t ld_acquire_cta(const int32_t* p) {
+  int32_t v;
+  asm volatile("ld.acquire.cta.shared::cta.s32 %0, [%1];\n" : "=r"(v) : "r"(smem_u32(p)) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_cta(int32_t* p, int32_t v) {
+  asm volatile("st.release.cta.shared::cta.s32 [%0], %1;\n" ::"r"(smem_u32(p)), "r"(v) : "memory");
+}
+// A chain hash another warp of this CTA has published (ordered by ld_acquire_cta).
+__device__ __forceinline__ uint64_t ld_relaxed_cta(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.relaxed.cta.global.u64 %0, [%1];\n" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
+
+// One chain step: h_b from h_{b-1} and d_b, with the sentinel remap.
+__device__ __forceinline__ uint64_t chain_step(uint64_t hp, uint64_t db) {
+  uint64_t x = mix64_halves((hp + kGamma) ^ db);
+  if (x < 2) x |= 2;
+  return x;
+}
+
+// Bounded wait until a shared counter exceeds v; false on timeout.
+__device__ __forceinline__ bool wait_above(const int32_t* p, int32_t v) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    if (ld_acquire_cta(p) > v) return true;
+    __nanosleep(64);
+  }
+  return false;
+}
+
+// Tier masks of U keys at once: the home-bucket tags of all, then the first
+// tag match's entry of all, so that U pairs of dependent reads are in flight
+// together. A key whose first candidate is not it (another key with the same
+// tag, or a key stored past a full home bucket) takes the full probe_one.
+template <int W, int U>
+__device__ __forceinline__ void probe_many(const uint8_t* __restrict__ tags, const uint64_t* __restrict__ table,
+                                           uint64_t n_buckets, const bool (&act)[U], const uint64_t (&h)[U],
+                                           uint64_t (&M)[U][W]) {
+  constexpr int EW = entry_words(W);
+  constexpr int NV = (W + 2) / 2;
+  uint64_t bk[U];
+  uint4 tv[U];
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    bk[u] = act[u] ? home_bucket(h[u], n_buckets) : 0;
+    if (act[u]) tv[u] = __ldg(reinterpret_cast<const uint4*>(tags + bk[u] * kBucket));
+  }
+  ulonglong2 v[U][NV];
+  uint32_t cand[U];
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    cand[u] = act[u] ? tag_match(tv[u], key_tag(h[u])) : 0;
+    if (cand[u]) {
+      const ulonglong2* e = reinterpret_cast<const ulonglong2*>(table + (bk[u] * kBucket + __ffs(cand[u]) - 1) * EW);
+#pragma unroll
+      for (int q = 0; q < NV; ++q) v[u][q] = __ldg(e + q);
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+#pragma unroll
+    for (int w = 0; w < W; ++w) M[u][w] = 0;
+    if (!act[u]) continue;
+    if (cand[u] && v[u][0].x == h[u]) {
+#pragma unroll
+      for (int w = 0; w < W; ++w) M[u][w] = (w & 1) ? v[u][(w + 1) >> 1].x : v[u][(w + 1) >> 1].y;
+    } else if ((cand[u] & (cand[u] - 1)) || !tag_match(tv[u], 0)) {
+      probe_one<W>(tags, table, n_buckets, h[u], M[u]);  // more candidates, or later buckets
+    }
+    // else: no candidate left and the home bucket has an empty slot: absent
+  }
+}
+
 template <int W>
-__global__ void __launch_bounds__(256)
-    k_probe(const uint8_t* __restrict__ tags, const uint64_t* __restrict__ table, uint64_t n_buckets,
-            const int64_t* __restrict__ block_off, int32_t n, const uint64_t* __restrict__ H,
-            const int32_t* __restrict__ batch_ok, const int32_t* __restrict__ share,
-            uint64_t* __restrict__ masks, uint64_t* __restrict__ chunk_and) {
+__global__ void __launch_bounds__(kCpWarps * 32, 1)
+    k_chain_probe(const int64_t* __restrict__ block_off, const int64_t* __restrict__ chunk_off, int32_t n, int S,
+                  uint64_t h_init, const int32_t* __restrict__ batch_ok, const uint64_t* __restrict__ D,
+                  uint64_t* __restrict__ hashes, uint64_t* __restrict__ sk_out, const uint64_t* __restrict__ groups,
+                  uint64_t gmask, int32_t* __restrict__ lead, int32_t* __restrict__ share,
+                  int32_t* __restrict__ order, int32_t* __restrict__ counts, const uint8_t* __restrict__ tags,
+                  const uint64_t* __restrict__ table, uint64_t n_buckets, uint64_t* __restrict__ masks,
+                  uint64_t* __restrict__ chunk_and, int chain_warps, int32_t* status) {
   pdl_enter();
-  if (!*batch_ok) return;
-  const int64_t total = block_off[n];
-  const int lane = threadIdx.x & 31;
-  int32_t r = 0;
-  // warp-uniform loop over 32-aligned chunks (the stride is a multiple of 32)
-  for (int64_t f0 = blockIdx.x * (int64_t)blockDim.x + (threadIdx.x & ~31); f0 < total;
-       f0 += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t f = f0 + lane;
-    uint64_t M[W];
-    bool act = f < total;
-    if (act) {
-      r = find_request(block_off, r, n, f);
-      act = f - __ldg(block_off + r) >= __ldg(share + r);  // else the leader's mask serves
+  extern __shared__ __align__(128) unsigned char csm[];  // chain lanes' digest rings
+  __shared__ int32_t s_ready[kCpMaxGroup];  // chunks chained, per request of the group
+  __shared__ int32_t s_share[kCpMaxGroup];  // shared prefix per request (-1 until known)
+  __shared__ int32_t s_next0;               // work counter: share tasks
+  __shared__ unsigned long long s_next1;    // work counter: probe items
+  __shared__ int32_t s_maxch;               // most chunks of a request in the group
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // This CTA's requests are blockIdx.x + k * gridDim.x, k = 0, 1, ...: the
+  // batch's order (group leaders are the first requests of their sessions, so
+  // they crowd its front) is spread evenly over the CTAs.
+  const int32_t stride = (int32_t)gridDim.x;
+  const int32_t m = n > (int32_t)blockIdx.x ? (n - (int32_t)blockIdx.x + stride - 1) / stride : 0;
+  auto req_of = [&](int32_t k) { return (int32_t)blockIdx.x + k * stride; };
+  if (!*batch_ok) {
+    for (int32_t k = (int32_t)threadIdx.x; k < m; k += blockDim.x) sk_out[req_of(k)] = 0;
+    return;
+  }
+  // chain warps: warp k on scheduler k (one each); every other warp probes
+  const int cw = warp;
+  const bool chain = warp < chain_warps;
+  const bool prober = warp >= chain_warps;
+  const int G = 32 * chain_warps;
+
+  for (int32_t g0 = 0; g0 < m; g0 += G) {
+    const int mg = min(G, m - g0);
+    if ((int)threadIdx.x < mg) {
+      s_ready[threadIdx.x] = 0;
+      s_share[threadIdx.x] = -1;
     }
-    if (act) {
-      probe_one<W>(tags, table, n_buckets, __ldg(H + f), M);
-#pragma unroll
-      for (int w = 0; w < W; ++w) masks[f * W + w] = M[w];
-    } else {
-#pragma unroll
-      for (int w = 0; w < W; ++w) M[w] = ~0ull;
+    if (threadIdx.x == 0) {
+      s_next0 = 0;
+      s_next1 = 0;
+      s_maxch = 0;
     }
+    __syncthreads();
+    if ((int)threadIdx.x < mg)
+      atomicMax(&s_maxch, (int32_t)(chunk_off[req_of(g0 + threadIdx.x) + 1] - chunk_off[req_of(g0 + threadIdx.x)]));
+    __syncthreads();
+    const int32_t maxch = s_maxch;
+    if (chain) {
+      // lane = request j of the group: the chain over its digests, one chunk
+      // at a time from a two-slot ring in shared memory (slot q & 1 holds
+      // chunk q; chunk q + 1 is copied in while chunk q is chained)
+      const int j = 32 * cw + lane;
+      const bool act = j < mg;
+      const int32_t r = act ? req_of(g0 + j) : 0;
+      int64_t bo = 0, nb = 0;
+      if (act) {
+        bo = __ldg(block_off + r);
+        nb = __ldg(block_off + r + 1) - bo;
+      }
+      const int32_t nch = (int32_t)((nb + kChunk - 1) / kChunk);
+      int32_t wmax = nch;
 #pragma unroll
-    for (int w = 0; w < W; ++w) {
-      const uint64_t a = (uint64_t)__reduce_and_sync(kFull, (unsigned)M[w]) |
-                         ((uint64_t)__reduce_and_sync(kFull, (unsigned)(M[w] >> 32)) << 32);
-      if (lane == w) chunk_and[(f0 >> 5) * W + w] = a;
+      for (int dd = 16; dd > 0; dd >>= 1) wmax = max(wmax, __shfl_xor_sync(kFull, wmax, dd));
+      unsigned char* const ring = csm + (size_t)j * kCpRingBytes;
+      const uint32_t ring_s = smem_u32(ring);
+      // copies chunk q's digests [first, first + nv) in 16-byte pieces from the
+      // even index at or below first into slot q & 1
+      auto fetch = [&](int32_t q) {
+        const int64_t first = bo + (int64_t)kChunk * q;
+        const int64_t a = first & ~(int64_t)1;
+        const int nv = (int)min((int64_t)kChunk, nb - (int64_t)kChunk * q);
+        const int pieces = (int)((first + nv - a + 1) >> 1);
+        const uint32_t dst = ring_s + (uint32_t)((q & 1) * kCpRingDigests * 8);
+        for (int i = 0; i < pieces; ++i) cp_async16(dst + 16u * i, D + a + 2 * i);
+      };
+      if (act && nch > 0) fetch(0);
+      cp_async_commit();
+      uint64_t h = h_init;
+      for (int32_t q = 0; q < wmax; ++q) {
+        cp_async_wait_all();
+        if (q + 1 < nch) fetch(q + 1);
+        cp_async_commit();
+        if (q < nch) {
+          const int64_t b0 = (int64_t)kChunk * q;
+          const int nv = (int)min((int64_t)kChunk, nb - b0);
+          const uint64_t* dsm =
+              reinterpret_cast<const uint64_t*>(ring + (q & 1) * kCpRingDigests * 8) + ((bo + b0) & 1);
+          uint64_t* const ho = hashes + bo + b0;
+          for (int i = 0; i < nv; ++i) {
+            h = chain_step(h, dsm[i]);
+            ho[i] = h;
+          }
+          __threadfence_block();
+          st_release_cta(&s_ready[j], q + 1);  // the chunk's hashes are out
+        }
+      }
+      cp_async_wait_all();
+      if (act) sk_out[r] = nb > 0 ? hashes[bo + (nb < S ? nb : (int64_t)S) - 1] : 0;
+    } else if (prober) {
+      // Phase 1, a warp per request (taken from a counter): the group leader
+      // (lowest request id with the same first-block hash, from the table the
+      // digest kernel filled) and the number of leading blocks whose digests
+      // equal the leader's.
+      for (;;) {
+        int32_t j = 0;
+        if (lane == 0) j = atomicAdd(&s_next0, 1);
+        j = __shfl_sync(kFull, j, 0);
+        if (j >= mg) break;
+        const int32_t r = req_of(g0 + j);
+        const int64_t bo = __ldg(block_off + r), nb = __ldg(block_off + r + 1) - bo;
+        int32_t l = r;
+        int64_t sh = 0;
+        if (nb > 0) {
+          const uint64_t key = first_hash(h_init, __ldg(D + bo));
+          const uint64_t s0 = key & gmask;
+          for (uint64_t t = 0; t <= gmask; t += 32) {
+            const uint64_t sl = (s0 + t + lane) & gmask;
+            const uint64_t k = groups[2 * sl];
+            const unsigned hit = __ballot_sync(kFull, k == key), emp = __ballot_sync(kFull, k == 0);
+            const unsigned stop = hit | emp;
+            if (stop) {
+              const int first = __ffs(stop) - 1;
+              if (hit & (1u << first)) l = INT32_MAX - (int32_t)groups[2 * ((s0 + t + first) & gmask) + 1];
+              break;
+            }
+          }
+          if (l != r && l >= 0 && l < n) {
+            const int64_t lo = __ldg(block_off + l), nl = __ldg(block_off + l + 1) - lo;
+            const int64_t m = nb < nl ? nb : nl;
+            sh = m;
+            for (int64_t b = 0; b < m; b += 32 * kGroupAhead) {
+              bool ne[kGroupAhead];
+#pragma unroll
+              for (int u = 0; u < kGroupAhead; ++u) {
+                const int64_t bb = b + 32 * u + lane;
+                ne[u] = bb < m && __ldg(D + bo + bb) != __ldg(D + lo + bb);
+              }
+              int64_t first = -1;
+#pragma unroll
+              for (int u = 0; u < kGroupAhead; ++u) {
+                const unsigned x = __ballot_sync(kFull, ne[u]);
+                if (x && first < 0) first = 32 * u + __ffs(x) - 1;
+              }
+              if (first >= 0) {
+                sh = b + first;
+                break;
+              }
+            }
+          } else {
+            l = r;
+          }
+        }
+        if (lane == 0) {
+          lead[r] = l;
+          share[r] = (int32_t)sh;
+          // leaders listed from the front, members from the back (any order)
+          if (l == r) order[atomicAdd(counts, 1)] = r;
+          else order[n - 1 - atomicAdd(counts + 1, 1)] = r;
+          st_release_cta(&s_share[j], (int32_t)sh);
+        }
+      }
+      // Phase 2: items (q, j) in chunk-major order, kCpProbes at a time: the
+      // tier masks of chunk q's blocks of request j at or past its shared
+      // prefix, once its chain has published the chunk; and the chunk's AND
+      // (a block not probed counts as all ones).
+      const int64_t items = (int64_t)maxch * mg;
+      for (;;) {
+        int64_t t0 = 0;
+        if (lane == 0) t0 = (int64_t)atomicAdd(&s_next1, (unsigned long long)kCpProbes);
+        t0 = __shfl_sync(kFull, t0, 0);
+        if (t0 >= items) break;
+        bool act[kCpProbes];
+        uint64_t hv[kCpProbes];
+        int64_t f[kCpProbes], cidx[kCpProbes];
+#pragma unroll
+        for (int u = 0; u < kCpProbes; ++u) {
+          act[u] = false;
+          hv[u] = 0;
+          f[u] = 0;
+          cidx[u] = -1;
+          const int64_t t = t0 + u;
+          if (t >= items) continue;
+          const int32_t q = (int32_t)(t / mg), j = (int32_t)(t % mg);
+          const int32_t r = req_of(g0 + j);
+          const int64_t bo = __ldg(block_off + r), nb = __ldg(block_off + r + 1) - bo;
+          if ((int64_t)kChunk * q >= nb) continue;  // the request has no chunk q
+          bool ok = wait_above(&s_share[j], -1) && wait_above(&s_ready[j], q);
+          if (!ok) {
+            if (lane == 0) latch_error(status, SMETRIC_ERR_CUDA);
+            continue;
+          }
+          const int64_t sh = s_share[j];
+          const int64_t b = (int64_t)kChunk * q + lane;
+          act[u] = b < nb && b >= sh;
+          f[u] = bo + b;
+          cidx[u] = __ldg(chunk_off + r) + q;
+          if (act[u]) hv[u] = ld_relaxed_cta(hashes + bo + b);
+        }
+        uint64_t M[kCpProbes][W];
+        probe_many<W, kCpProbes>(tags, table, n_buckets, act, hv, M);
+#pragma unroll
+        for (int u = 0; u < kCpProbes; ++u) {
+          if (cidx[u] < 0) continue;  // warp-uniform
+          if (act[u]) {
+#pragma unroll
+            for (int w = 0; w < W; ++w) masks[f[u] * W + w] = M[u][w];
+          }
+#pragma unroll
+          for (int w = 0; w < W; ++w) {
+            const uint64_t x = act[u] ? M[u][w] : ~0ull;
+            const uint64_t a = (uint64_t)__reduce_and_sync(kFull, (unsigned)x) |
+                               ((uint64_t)__reduce_and_sync(kFull, (unsigned)(x >> 32)) << 32);
+            if (lane == w) chunk_and[cidx[u] * W + w] = a;
+          }
+        }
+      }
     }
+    __syncthreads();  // the group's shared state is rewritten by the next group
   }
 }
 
@@ -860,7 +1088,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
     k_walk(int N, int B, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n,
            const int64_t* __restrict__ load, int64_t w_load, int64_t w_miss, int64_t w_glob,
            const uint64_t* __restrict__ masks, const uint64_t* __restrict__ chunk_and,
-           const int32_t* __restrict__ batch_ok,
+           const int64_t* __restrict__ chunk_off, const int32_t* __restrict__ batch_ok,
            const int32_t* __restrict__ lead, const int32_t* __restrict__ share, int32_t* __restrict__ summ,
            const int32_t* __restrict__ order, const int32_t* __restrict__ counts,
            int32_t* __restrict__ inst_out, int32_t* __restrict__ lhit_out,
@@ -897,18 +1125,21 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
     const int64_t bo = block_off[r];
     const int64_t sh = MEMBERS ? share[r] : 0;
     const int32_t* const cl = summ + (int64_t)l * (N + 1);  // the leader's run ends
-    // the first step's loads (see below) go out with the leader's run ends
+    // the first step's loads (see below) go out with the leader's run ends;
+    // chunk ANDs are per request-aligned chunk: blocks 32q .. 32q + 31 of
+    // request r at index chunk_off[r] + q, so alignment is to b - bo
     int64_t f = bo + sh;
     const int64_t F1 = bo + nb;
-    const bool head_single = (f & 31) || F1 - f < 32;
+    const int64_t cbase = __ldg(chunk_off + r);
+    const bool head_single = ((f - bo) & 31) || F1 - f < 32;
     uint64_t pre[W];
 #pragma unroll
     for (int w = 0; w < W; ++w) {
       if (head_single) {
-        const int64_t len = min((int64_t)(32 - (f & 31)), F1 - f);
+        const int64_t len = min((int64_t)(32 - ((f - bo) & 31)), F1 - f);
         pre[w] = lane < len ? __ldg(masks + (f + lane) * W + w) : ~0ull;
       } else {
-        pre[w] = lane < ((F1 - f) >> 5) ? __ldg(chunk_and + ((f >> 5) + lane) * W + w) : 0;
+        pre[w] = lane < ((F1 - f) >> 5) ? __ldg(chunk_and + (cbase + ((f - bo) >> 5) + lane) * W + w) : 0;
       }
     }
     constexpr int CT = 2 * W;  // groups of 32 covering the N + 1 <= 64 W run ends
@@ -979,15 +1210,15 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
     bool dead = !galive;
 #pragma unroll
     for (int w = 0; w < W; ++w) dead &= A[w] == 0;
-    // From block sh: single blocks up to a 32-aligned batch position, then
+    // From block sh: single blocks up to a 32-aligned request position, then
     // 32 chunks per step from their AND summaries (lane = chunk); the first
     // chunk that ends an alive run is walked block by block, and the request's
     // last partial chunk too. The first step uses the loads issued above.
     bool first = true;
     while (!dead && f < F1) {
       uint64_t x[W];
-      if ((f & 31) || F1 - f < 32) {
-        const int len = (int)min((int64_t)(32 - (f & 31)), F1 - f);
+      if (((f - bo) & 31) || F1 - f < 32) {
+        const int len = (int)min((int64_t)(32 - ((f - bo) & 31)), F1 - f);
 #pragma unroll
         for (int w = 0; w < W; ++w)
           x[w] = first ? pre[w] : lane < len ? __ldg(masks + (f + lane) * W + w) : ~0ull;
@@ -999,7 +1230,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
       const int64_t nfull = (F1 - f) >> 5;
 #pragma unroll
       for (int w = 0; w < W; ++w)
-        x[w] = first ? pre[w] : lane < nfull ? __ldg(chunk_and + ((f >> 5) + lane) * W + w) : 0;
+        x[w] = first ? pre[w] : lane < nfull ? __ldg(chunk_and + (cbase + ((f - bo) >> 5) + lane) * W + w) : 0;
       first = false;
       bool stop = lane >= nfull;
 #pragma unroll
@@ -1685,11 +1916,23 @@ bool make_token_maps(TokenMaps& m, const int32_t* tokens, int64_t n_tokens, int 
   return true;
 }
 
+// Group-table slots a batch of n requests uses: a power of two >= 2n.
+uint64_t group_slots_for(int32_t n) {
+  uint64_t g = 64;
+  while (g < 2 * (uint64_t)n) g <<= 1;
+  return g;
+}
+
+// The digest kernel for the index's block size; with `group` it also puts
+// each request's first-block hash into the group table.
 template <int HB>
 int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
-                  const int64_t* d_offsets, int32_t n, cudaStream_t s, int cap_per_sm) {
+                  const int64_t* d_offsets, int32_t n, cudaStream_t s, int cap_per_sm, bool group) {
   const int B = idx->cfg.block_size;
   const uint64_t d_init = mix64(idx->cfg.hash_seed ^ (uint64_t)B);
+  const uint64_t h_init = mix64(idx->cfg.hash_seed + kGamma);
+  uint64_t* const groups = group ? idx->groups : nullptr;
+  const uint64_t gmask = group_slots_for(n) - 1;
   // request-aligned chunks (TMA kernel) number at most blocks / 32 + n
   const int64_t max_chunks = (n_tokens / B + kChunk - 1) / kChunk + (HB > 0 ? n : 0);
   // rows of 16*nch bytes: a block's 4B bytes start at most 12 bytes past a
@@ -1716,7 +1959,7 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
       idx->launches++;
       return launch_k(kern, dim3((unsigned)grid), dim3(warps * 32), smem, s, !idx->profiling, maps, d_tokens,
                       n_tokens, d_offsets, (const int64_t*)idx->block_off, (const int64_t*)idx->chunk_off, n, d_init,
-                      (const int32_t*)idx->batch_ok, idx->digest, idx->status);
+                      (const int32_t*)idx->batch_ok, idx->digest, idx->status, groups, gmask, h_init);
     }
   }
   const size_t per_warp = (size_t)kChunk * nch * 16;
@@ -1739,27 +1982,20 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
   if (HB > 0)
     return launch_k(kern, dim3((unsigned)grid), dim3(warps * 32), smem, s, !idx->profiling, d_tokens, n_tokens,
                     d_offsets, (const int64_t*)idx->block_off, n, d_init, (const int32_t*)idx->batch_ok,
-                    idx->digest);
+                    idx->digest, groups, gmask, h_init);
   return launch_k(k_digest_any, dim3((unsigned)grid), dim3(warps * 32), smem, s, !idx->profiling, d_tokens,
                   n_tokens, d_offsets, (const int64_t*)idx->block_off, n, B, nch, d_init,
-                  (const int32_t*)idx->batch_ok, idx->digest);
+                  (const int32_t*)idx->batch_ok, idx->digest, groups, gmask, h_init);
 }
 
 int dispatch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
-                    const int64_t* d_offsets, int32_t n, cudaStream_t s, int cap_per_sm = 0) {
+                    const int64_t* d_offsets, int32_t n, cudaStream_t s, int cap_per_sm, bool group) {
   switch (idx->cfg.block_size) {
-    case 16: return launch_digest<8>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm);
-    case 32: return launch_digest<16>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm);
-    case 64: return launch_digest<32>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm);
-    default: return launch_digest<0>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm);
+    case 16: return launch_digest<8>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm, group);
+    case 32: return launch_digest<16>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm, group);
+    case 64: return launch_digest<32>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm, group);
+    default: return launch_digest<0>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm, group);
   }
-}
-
-// Group-table slots a batch of n requests uses: a power of two >= 2n.
-uint64_t group_slots_for(int32_t n) {
-  uint64_t g = 64;
-  while (g < 2 * (uint64_t)n) g <<= 1;
-  return g;
 }
 
 int launch_chain(smetric_index* idx, const int64_t* d_offsets, int32_t n, uint64_t* hashes,
@@ -1772,25 +2008,6 @@ int launch_chain(smetric_index* idx, const int64_t* d_offsets, int32_t n, uint64
                   hashes ? hashes : idx->hashes, sk);
 }
 
-// The group stage (k_group_insert, then k_group) on stream s.
-int launch_group(smetric_index* idx, int32_t n, cudaStream_t s) {
-  const uint64_t h_init = mix64(idx->cfg.hash_seed + kGamma);
-  const uint64_t gmask = group_slots_for(n) - 1;
-  int32_t* const counts = idx->order + idx->cfg.max_batch_requests;
-  k_group_insert<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(idx->block_off, n, idx->batch_ok, idx->digest, h_init,
-                                                             idx->groups, gmask, counts);
-  idx->launches++;
-  int rc = cuda_status(cudaGetLastError());
-  if (rc) return rc;
-  const int64_t want = ((int64_t)n + 7) / 8;
-  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
-  k_group<<<(unsigned)grid, 256, 0, s>>>(idx->block_off, n, idx->batch_ok, idx->groups, gmask, idx->digest, h_init,
-                                         idx->lead, idx->share,
-                                         idx->order, counts);
-  idx->launches++;
-  return cuda_status(cudaGetLastError());
-}
-
 template <int W>
 int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const int64_t* d_load,
                  smetric_weights w, int32_t* inst, int32_t* lhit, int32_t* ghit, uint64_t* hashes,
@@ -1798,38 +2015,31 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
                  const Overlap* ov) {
   const cudaEvent_t after_chain = ov ? ov->after_chain : nullptr;
   const int N = idx->cfg.num_instances;
-  const uint64_t* H = hashes ? hashes : idx->hashes;
   int rc;
-  if (idx->profiling) {  // one stream, so that each kernel's events bracket it alone
-    if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, false, s))) return rc;
-    if (after_chain && cudaEventRecord(after_chain, s) != cudaSuccess) return cuda_status(cudaErrorUnknown);
-    profile_mark(idx, kChain, s);
-    if ((rc = launch_group(idx, n, s))) return rc;
-    profile_mark(idx, kGroup, s);
-  } else {
-    // the group stage needs only the digests: it runs on the side stream
-    // beside the latency-bound chain
-    if (cudaEventRecord(idx->fork_ev, s) != cudaSuccess || cudaStreamWaitEvent(idx->side, idx->fork_ev, 0) != cudaSuccess)
-      return cuda_status(cudaErrorUnknown);
-    if ((rc = launch_group(idx, n, idx->side))) return rc;
-    if (cudaEventRecord(idx->join_ev, idx->side) != cudaSuccess) return cuda_status(cudaErrorUnknown);
-    if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, false, s))) return rc;
-    if (after_chain && cudaEventRecord(after_chain, s) != cudaSuccess) return cuda_status(cudaErrorUnknown);
-    if (cudaStreamWaitEvent(s, idx->join_ev, 0) != cudaSuccess) return cuda_status(cudaErrorUnknown);
-  }
   {
-    // probe: one thread per block, grid sized to the largest possible batch
-    const int64_t want = (max_blocks + 255) / 256;
-    const int per_sm = ov && ov->probe_ctas_per_sm > 0 ? ov->probe_ctas_per_sm : 8;
-    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * per_sm));
+    // chain, group leaders and shared prefixes, and probe: one CTA per SM,
+    // a chain lane for each request a CTA owns (1 to 4 warps; more requests
+    // are taken in groups)
+    const int grid = idx->num_sms;
+    const int64_t per_cta = ((int64_t)n + grid - 1) / grid;
+    const int chain_warps = (int)std::max<int64_t>(1, std::min<int64_t>(kCpMaxChainWarps, (per_cta + 31) / 32));
+    const size_t smem = (size_t)chain_warps * 32 * kCpRingBytes;
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(k_chain_probe<W>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+      return cuda_status(cudaErrorInvalidValue);
     idx->launches++;
-    // an ordinary launch: it follows the wait for the side stream
-    if ((rc = launch_k(k_probe<W>, dim3((unsigned)grid), dim3(256), 0, s, false, idx->tags, idx->table,
-                       idx->n_buckets, idx->block_off, n, H, idx->batch_ok, idx->share, idx->masks,
-                       idx->chunk_and)))
+    if ((rc = launch_k(k_chain_probe<W>, dim3((unsigned)grid), dim3(kCpWarps * 32), smem, s, !idx->profiling,
+                       (const int64_t*)idx->block_off, (const int64_t*)idx->chunk_off, n, idx->cfg.session_blocks,
+                       mix64(idx->cfg.hash_seed + kGamma), (const int32_t*)idx->batch_ok,
+                       (const uint64_t*)idx->digest, hashes ? hashes : idx->hashes, sk, (const uint64_t*)idx->groups,
+                       group_slots_for(n) - 1, idx->lead, idx->share, idx->order,
+                       idx->order + idx->cfg.max_batch_requests, (const uint8_t*)idx->tags,
+                       (const uint64_t*)idx->table, idx->n_buckets, idx->masks, idx->chunk_and, chain_warps,
+                       idx->status)))
       return rc;
+    if (after_chain && cudaEventRecord(after_chain, s) != cudaSuccess) return cuda_status(cudaErrorUnknown);
   }
-  profile_mark(idx, kProbe, s);
+  profile_mark(idx, kChainProbe, s);
   const size_t smem = (size_t)N * sizeof(int64_t) + (size_t)kMatchWarps * N * (W + 1) * sizeof(uint64_t);
   const int64_t want = ((int64_t)n + kMatchWarps - 1) / kMatchWarps;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
@@ -1847,8 +2057,8 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
     idx->launches++;
     if ((rc = launch_k(kern, dim3((unsigned)grid), dim3(kMatchWarps * 32), smem, s, !idx->profiling, N,
                        idx->cfg.block_size, d_offsets, idx->block_off, n, d_load, w.w_load, w.w_miss, w.w_glob,
-                       idx->masks, idx->chunk_and, idx->batch_ok, idx->lead, idx->share, idx->summ, idx->order,
-                       idx->order + idx->cfg.max_batch_requests, inst, lhit, ghit,
+                       idx->masks, idx->chunk_and, (const int64_t*)idx->chunk_off, idx->batch_ok, idx->lead,
+                       idx->share, idx->summ, idx->order, idx->order + idx->cfg.max_batch_requests, inst, lhit, ghit,
                        reinterpret_cast<uint4*>(idx->groups), (int64_t)group_slots_for(n), pol)))
       return rc;
   }
@@ -1917,12 +2127,14 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
                             eq1 ? SMETRIC_POLICY_MAX_QUEUED : SMETRIC_MAX_LOAD,
                             eq1 ? SMETRIC_POLICY_MAX_LEN : (int64_t)INT32_MAX, pol ? pol->est_hit : nullptr,
                             pol ? pol->tpot : nullptr, SMETRIC_POLICY_MAX_TPOT,
-                            pol ? pol->nreq : nullptr, SMETRIC_POLICY_MAX_REQUESTS);
+                            pol ? pol->nreq : nullptr, SMETRIC_POLICY_MAX_REQUESTS,
+                            PROBE ? idx->order + c.max_batch_requests : nullptr);
   idx->launches++;
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   profile_mark(idx, kPrep, s);
+  // a route's digests also fill the group table (each request's first-block hash)
   if (n_tokens / c.block_size > 0) {
-    if ((rc = dispatch_digest(idx, d_tokens, n_tokens, d_offsets, n, s, ov ? ov->digest_ctas_per_sm : 0)))
+    if ((rc = dispatch_digest(idx, d_tokens, n_tokens, d_offsets, n, s, ov ? ov->digest_ctas_per_sm : 0, PROBE)))
       return rc;
   }
   profile_mark(idx, kDigest, s);
@@ -1933,9 +2145,7 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
       return rc;
   } else {
     if ((rc = launch_chain(idx, d_offsets, n, hashes, sk, !idx->profiling, s))) return rc;
-    profile_mark(idx, kChain, s);
-    profile_mark(idx, kGroup, s);
-    profile_mark(idx, kProbe, s);
+    profile_mark(idx, kChainProbe, s);
   }
   profile_mark(idx, kWalk, s);
   return SMETRIC_OK;
@@ -2092,10 +2302,10 @@ int pipeline_attach(smetric_index* x) {
   if (!p) return SMETRIC_ERR_OOM;
   RouteScratchSet& a = p->alt;
   bool ok = cudaMalloc(&a.block_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
-            cudaMalloc(&a.digest, nb * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&a.digest, (nb + 2) * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&a.hashes, nb * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&a.masks, nb * W * sizeof(uint64_t)) == cudaSuccess &&
-            cudaMalloc(&a.chunk_and, (max_blocks / 32 + 1) * W * sizeof(uint64_t)) == cudaSuccess &&
+            cudaMalloc(&a.chunk_and, (max_blocks / 32 + R + 1) * W * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&a.groups, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&a.lead, 2 * (R + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&a.chunk_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
@@ -2465,9 +2675,7 @@ const char* smetric_profile_kernel_name(int32_t k) {
   switch (k) {
     case kPrep: return "k_prep";
     case kDigest: return "k_digest";
-    case kChain: return "k_chain";
-    case kGroup: return "k_group";
-    case kProbe: return "k_probe";
+    case kChainProbe: return "k_chain_probe";
     case kWalk: return "k_walk";
     default: return "";
   }
@@ -2530,10 +2738,11 @@ int na_digest(const int32_t* d_tokens, int64_t n_tokens, const int64_t* d_offset
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)num_sms * std::max(occ, 1)));
   if (HB > 0)
     k_digest<(HB > 0 ? HB : 2)><<<(unsigned)grid, warps * 32, smem, s>>>(d_tokens, n_tokens, d_offsets,
-                                                                        block_off, n, d_init, ok, digest);
+                                                                        block_off, n, d_init, ok, digest,
+                                                                        nullptr, 0, 0);
   else
     k_digest_any<<<(unsigned)grid, warps * 32, smem, s>>>(d_tokens, n_tokens, d_offsets, block_off, n, B, nch,
-                                                          d_init, ok, digest);
+                                                          d_init, ok, digest, nullptr, 0, 0);
   return cuda_status(cudaGetLastError());
 }
 

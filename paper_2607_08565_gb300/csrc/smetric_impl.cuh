@@ -87,9 +87,9 @@ __device__ __forceinline__ void latch_error(int32_t* status, int32_t code) {
 __host__ __device__ constexpr int entry_words(int W) { return W == 1 ? 2 : (W <= 3 ? 4 : 8); }
 
 // Route kernels, in launch order; names returned by smetric_profile_kernel_name.
-enum RouteKernel {
-  kPrep = 0, kDigest = 1, kChain = 2, kGroup = 3, kProbe = 4, kWalk = 5, kNumRouteKernels = 6
-};
+// kChainProbe is k_chain_probe in a route (chain, group stage and probe in one
+// kernel) and k_chain in the calls that only hash.
+enum RouteKernel { kPrep = 0, kDigest = 1, kChainProbe = 2, kWalk = 3, kNumRouteKernels = 4 };
 
 struct ProfileSlot {
   cudaEvent_t ev[kNumRouteKernels + 1];
@@ -112,7 +112,7 @@ struct smetric_index {
   uint64_t* digest;    // max_batch_tokens / B: per-block digests d_b
   uint64_t* hashes;    // max_batch_tokens / B: per-block chain hashes h_b
   uint64_t* masks;     // W * max_batch_tokens / B: per-block tier masks
-  uint64_t* chunk_and; // W * ceil(max_batch_tokens / B / 32): AND of each 32-block chunk's masks
+  uint64_t* chunk_and; // W * (max_batch_tokens / B / 32 + R + 1): AND of each request-aligned 32-block chunk's masks
   uint64_t* groups;    // 2 * group_slots: (first-block hash, INT32_MAX - leader) pairs
   uint64_t group_slots;  // power of two >= 2 * max_batch_requests
   int32_t* lead;       // max_batch_requests: the request whose masks a request shares

@@ -44,8 +44,9 @@ def test_library_links_no_python_or_torch():
 def test_strerror_and_kernel_names(L):
     assert pkg.smetric_strerror(pkg.SMETRIC_ERR_TABLE_FULL) == "index table full"
     assert pkg.smetric_strerror(12345) == "unknown error"
-    assert [pkg.smetric_profile_kernel_name(k) for k in range(6)] == ["k_prep", "k_digest", "k_chain",
-                                                                      "k_group", "k_probe", "k_walk"]
+    assert [pkg.smetric_profile_kernel_name(k) for k in range(4)] == ["k_prep", "k_digest", "k_chain_probe",
+                                                                      "k_walk"]
+    assert pkg.smetric_profile_kernel_name(4) == ""
 
 
 def _create(L, **kw):

@@ -24,7 +24,7 @@ def test_algorithmic_bytes_hand_example():
     b = bench.algorithmic_bytes(lens, local, glob, 4, 1)
     assert b["k_digest"] == 4 * 4 * 6  # every token of the 6 full blocks
     assert b["k_probe"] == 5 * 16  # 2 + 0 + 3 probes, 16-byte entries
-    assert b["k_chain"] == 16 * 6 + 24 * 3
+    assert b["k_chain_probe"] == 16 * 6 + 24 * 3 + 5 * 16
     assert b["k_walk"] == 8 * 5 + 28 * 3
     assert b["k_prep"] == 16 * 3
     # 4 B per prompt token, an entry per probe, n + 1 offsets, 20 B of outputs per request
