@@ -779,7 +779,7 @@ __device__ __forceinline__ uint64_t chain_step(uint64_t hp, uint64_t db) {
 __device__ __forceinline__ bool wait_above(const int32_t* p, int32_t v) {
   for (uint32_t i = 0; i < kSpinLimit; ++i) {
     if (ld_acquire_cta(p) > v) return true;
-    __nanosleep(64);
+    __nanosleep(256);  // a long sleep keeps waiting warps off the chain warps' schedulers
   }
   return false;
 }
@@ -840,6 +840,8 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
   extern __shared__ __align__(128) unsigned char csm[];  // chain lanes' digest rings
   __shared__ int32_t s_ready[kCpMaxGroup];  // chunks chained, per request of the group
   __shared__ int32_t s_share[kCpMaxGroup];  // shared prefix per request (-1 until known)
+  __shared__ int32_t s_dead[kCpMaxGroup];   // first chunk whose AND is empty (INT32_MAX until one is)
+  __shared__ int32_t s_fin[kCpMaxGroup];    // chunks finished in order from the first unshared one
   __shared__ int32_t s_next0;               // work counter: share tasks
   __shared__ unsigned long long s_next1;    // work counter: probe items
   __shared__ int32_t s_maxch;               // most chunks of a request in the group
@@ -865,6 +867,8 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
     if ((int)threadIdx.x < mg) {
       s_ready[threadIdx.x] = 0;
       s_share[threadIdx.x] = -1;
+      s_dead[threadIdx.x] = INT32_MAX;
+      s_fin[threadIdx.x] = 0;
     }
     if (threadIdx.x == 0) {
       s_next0 = 0;
@@ -993,7 +997,16 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
       // Phase 2: items (q, j) in chunk-major order, kCpProbes at a time: the
       // tier masks of chunk q's blocks of request j at or past its shared
       // prefix, once its chain has published the chunk; and the chunk's AND
-      // (a block not probed counts as all ones).
+      // (a block not probed counts as all ones). Skipped with no wait: a chunk
+      // wholly inside the shared prefix (the walk starts past it). Skipped
+      // after waiting: any chunk after one whose AND is empty (that chunk
+      // lacks a block of every tier, so every run has ended there: the walk
+      // stops before reaching later chunks). When the probers' items in
+      // flight would span more than two rounds of the group (few requests per
+      // CTA), a request's chunk q starts only once its chunk q - 2 has
+      // finished (chunks then finish in order), so at most two of its chunks
+      // are probed ahead of knowing whether its runs are over.
+      const bool paced = (kCpWarps - chain_warps) * kCpProbes > 2 * mg;
       const int64_t items = (int64_t)maxch * mg;
       for (;;) {
         int64_t t0 = 0;
@@ -1003,24 +1016,39 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
         bool act[kCpProbes];
         uint64_t hv[kCpProbes];
         int64_t f[kCpProbes], cidx[kCpProbes];
+        int32_t qs[kCpProbes], js[kCpProbes], rel[kCpProbes];  // rel: chunk index counted from the first unshared one
 #pragma unroll
         for (int u = 0; u < kCpProbes; ++u) {
           act[u] = false;
           hv[u] = 0;
           f[u] = 0;
           cidx[u] = -1;
+          rel[u] = -1;
           const int64_t t = t0 + u;
           if (t >= items) continue;
           const int32_t q = (int32_t)(t / mg), j = (int32_t)(t % mg);
+          qs[u] = q;
+          js[u] = j;
           const int32_t r = req_of(g0 + j);
           const int64_t bo = __ldg(block_off + r), nb = __ldg(block_off + r + 1) - bo;
           if ((int64_t)kChunk * q >= nb) continue;  // the request has no chunk q
-          bool ok = wait_above(&s_share[j], -1) && wait_above(&s_ready[j], q);
-          if (!ok) {
+          if (!wait_above(&s_share[j], -1)) {
             if (lane == 0) latch_error(status, SMETRIC_ERR_CUDA);
             continue;
           }
           const int64_t sh = s_share[j];
+          if ((int64_t)kChunk * (q + 1) <= sh) continue;
+          rel[u] = paced ? q - (int32_t)(sh / kChunk) : -1;
+          if (paced && !wait_above(&s_fin[j], rel[u] - 2)) {  // chunk q - 2 has finished
+            if (lane == 0) latch_error(status, SMETRIC_ERR_CUDA);
+            rel[u] = -1;
+            continue;
+          }
+          if (ld_acquire_cta(&s_dead[j]) < q) continue;  // finished as skipped below
+          if (!wait_above(&s_ready[j], q)) {
+            if (lane == 0) latch_error(status, SMETRIC_ERR_CUDA);
+            continue;
+          }
           const int64_t b = (int64_t)kChunk * q + lane;
           act[u] = b < nb && b >= sh;
           f[u] = bo + b;
@@ -1036,13 +1064,26 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
 #pragma unroll
             for (int w = 0; w < W; ++w) masks[f[u] * W + w] = M[u][w];
           }
+          bool empty = true;
 #pragma unroll
           for (int w = 0; w < W; ++w) {
             const uint64_t x = act[u] ? M[u][w] : ~0ull;
             const uint64_t a = (uint64_t)__reduce_and_sync(kFull, (unsigned)x) |
                                ((uint64_t)__reduce_and_sync(kFull, (unsigned)(x >> 32)) << 32);
             if (lane == w) chunk_and[cidx[u] * W + w] = a;
+            empty &= a == 0;
           }
+          if (empty && lane == 0) atomicMin(&s_dead[js[u]], qs[u]);
+        }
+        // chunks finish in order: after the request's previous chunk
+#pragma unroll
+        for (int u = 0; u < kCpProbes; ++u) {
+          if (rel[u] < 0) continue;  // warp-uniform
+          if (lane == 0) {
+            if (!wait_above(&s_fin[js[u]], rel[u] - 1)) latch_error(status, SMETRIC_ERR_CUDA);
+            st_release_cta(&s_fin[js[u]], rel[u] + 1);
+          }
+          __syncwarp();
         }
       }
     }
