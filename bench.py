@@ -174,6 +174,24 @@ class ClockSampler:
                 "window": window}
 
 
+def h2d_link_gbs(pinned, device, reps=5):
+    """Host-to-device copy rate of one pinned buffer (GB/s): the ceiling of
+    the end-to-end number, which must move the batch's tokens every step."""
+    import torch
+    dst = torch.empty(pinned.numel(), dtype=pinned.dtype, device=device)
+    dst.copy_(pinned, non_blocking=True)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        dst.copy_(pinned, non_blocking=True)
+    e1.record()
+    torch.cuda.synchronize()
+    gbs = reps * pinned.numel() * pinned.element_size() / (e0.elapsed_time(e1) / 1e3) / 1e9
+    del dst
+    return gbs
+
+
 def peak_hbm():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -556,6 +574,7 @@ def run_ours(args, rank, world, local, dist):
     e2e_value = world * args.e2e_steps * e2e_reqs / e2e_s
     h2d = float(np.mean([4 * b["n_tokens"] + 8 * (b["n"] + 1) + 8 * N for b in pinned]))
     d2h = float(20 * e2e_reqs)
+    link = h2d_link_gbs(pinned[0]["tok"], device)
     # the host-buffer path must agree with the device path
     last = per_batch[(args.e2e_steps - 1) % len(pinned)]
     for k in hout:
@@ -587,7 +606,9 @@ def run_ours(args, rank, world, local, dist):
             "route_stats": route_stats([b.lengths() for b in host], per_batch, N),
             "clocks": clk,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h, "steps": args.e2e_steps},
+                    "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
+                    "h2d_link_gbs": link,
+                    "frac_of_link": (h2d * e2e_value / e2e_reqs / 1e9) / link if link else None},
             "gpu_launches": int(launches),
             "cpu_baseline": cpu,
         }

@@ -397,6 +397,57 @@ def test_route_host_buffers_match_device_path():
     assert_outputs_equal(h, o, fields=("instance", "local_hit", "global_hit", "session_key"))
 
 
+def test_route_host_buffers_large_batch():
+    """A larger host batch (600 requests, 9.6M tokens): outputs equal the
+    device path's, call after call, and for a sample the oracle's; offsets a
+    device check refuses give every request the invalid-batch outputs."""
+    rng = np.random.default_rng(29)
+    N, B = 16, 32
+    n = 600
+    lens = rng.integers(8000, 24000, size=n)
+    # requests share prefixes with a few stored prompts so that hits occur
+    base = [rng.integers(0, 151936, size=24000, dtype=np.int32) for _ in range(4)]
+    reqs = []
+    for L in lens.tolist():
+        b = base[int(rng.integers(0, 4))]
+        keep = int(rng.integers(0, L + 1))
+        reqs.append(np.concatenate([b[:keep], rng.integers(0, 151936, size=L - keep, dtype=np.int32)]))
+    tok, off = pack(reqs)
+    assert off[-1] >= 8 << 20
+    ix = make_index(N, B, 2, cap=1 << 16, host_staging=True, max_req=n, max_tok=len(tok))
+    ox = oracle.OracleIndex(N)
+    stored = {t: [base[t % 4][: 16000 + 512 * t]] for t in range(-1, N, 3)}
+    populate_both(ix, ox, stored, B)
+    load = rng.integers(0, 200000, size=N)
+    g = gpu_route(ix, tok, off, load, (1, 4, 2), want_hashes=False)
+
+    def host_route(offsets):
+        h = dict(instance=np.zeros(n, np.int32), local_hit=np.zeros(n, np.int32),
+                 global_hit=np.zeros(n, np.int32), session_key=np.zeros(n, np.uint64))
+        rc = pkg.smetric_route_batch_host(ix.handle, tok, len(tok), offsets, n, np.asarray(load, np.int64),
+                                          (1, 4, 2), h["instance"], h["local_hit"], h["global_hit"],
+                                          h["session_key"])
+        return rc, h
+
+    for rep in range(2):
+        rc, h = host_route(off)
+        assert rc == pkg.SMETRIC_OK
+        assert_outputs_equal(h, g, fields=("instance", "local_hit", "global_hit", "session_key"),
+                             ctx=f"host buffers, call {rep}")
+    sample = np.sort(rng.choice(n, size=40, replace=False))
+    st, so = pack([tok[off[r]:off[r + 1]] for r in sample])
+    o = ox.route_batch(B, 2, 0, st, so, load, 1, 4, 2)
+    assert_outputs_equal({k: v[sample] for k, v in h.items()}, o,
+                         fields=("instance", "local_hit", "global_hit", "session_key"))
+    assert np.any(h["local_hit"] > 0)
+    bad = off.copy()
+    bad[450] = bad[451] + 1  # decreasing, late in the batch
+    rc, hb = host_route(bad)
+    assert rc == pkg.SMETRIC_ERR_INVALID_ARG
+    assert np.all(hb["instance"] == -1) and not hb["session_key"].any()
+    ix.close()
+
+
 def test_profile_and_launch_count():
     rng = np.random.default_rng(24)
     ix = make_index(4, 16, 2)
