@@ -603,6 +603,14 @@ def run_ours(args, rank, world, local, dist):
                               "algorithmic_bytes_per_step": algo_mean["path"],
                               "frac_of_nominal": path_gbs / NOMINAL_HBM_GBS},
             "kernels_ms_per_launch": {k: v[0] / max(v[1], 1) for k, v in prof.items()},
+            # every kernel against the same copy peak: the digest streams the
+            # tokens (bound by its integer pipe at about this rate); the chain
+            # and probe kernel is bound by the chain's dependent steps and
+            # random entry reads, not by bandwidth
+            "kernels_roofline": {k: {"achieved_gbs": algo_mean[k] / (v[0] / max(v[1], 1) / 1e3) / 1e9,
+                                     "frac": algo_mean[k] / (v[0] / max(v[1], 1) / 1e3) / 1e9 / peak,
+                                     "traffic": ncu_traffic(k)}
+                                 for k, v in prof.items() if k in algo_mean and v[0] > 0},
             "route_stats": route_stats([b.lengths() for b in host], per_batch, N),
             "clocks": clk,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,

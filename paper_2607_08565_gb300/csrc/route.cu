@@ -842,6 +842,9 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
   __shared__ int32_t s_share[kCpMaxGroup];  // shared prefix per request (-1 until known)
   __shared__ int32_t s_dead[kCpMaxGroup];   // first chunk whose AND is empty (INT32_MAX until one is)
   __shared__ int32_t s_fin[kCpMaxGroup];    // chunks finished in order from the first unshared one
+  __shared__ int64_t s_bo[kCpMaxGroup];     // per request of the group: first block in the batch,
+  __shared__ int64_t s_cb[kCpMaxGroup];     // first request-aligned chunk,
+  __shared__ int32_t s_nb[kCpMaxGroup];     // and full blocks
   __shared__ int32_t s_next0;               // work counter: share tasks
   __shared__ unsigned long long s_next1;    // work counter: probe items
   __shared__ int32_t s_maxch;               // most chunks of a request in the group
@@ -869,6 +872,11 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
       s_share[threadIdx.x] = -1;
       s_dead[threadIdx.x] = INT32_MAX;
       s_fin[threadIdx.x] = 0;
+      const int32_t r = req_of(g0 + (int32_t)threadIdx.x);
+      const int64_t bo = block_off[r];
+      s_bo[threadIdx.x] = bo;
+      s_nb[threadIdx.x] = (int32_t)(block_off[r + 1] - bo);
+      s_cb[threadIdx.x] = chunk_off[r];
     }
     if (threadIdx.x == 0) {
       s_next0 = 0;
@@ -1013,6 +1021,9 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
         if (lane == 0) t0 = (int64_t)atomicAdd(&s_next1, (unsigned long long)kCpProbes);
         t0 = __shfl_sync(kFull, t0, 0);
         if (t0 >= items) break;
+        // item t is chunk t / mg of request t % mg; one division per grab
+        int32_t q0 = (int32_t)(t0 < INT32_MAX ? (uint32_t)t0 / (uint32_t)mg : t0 / mg);
+        int32_t j0 = (int32_t)(t0 - (int64_t)q0 * mg);
         bool act[kCpProbes];
         uint64_t hv[kCpProbes];
         int64_t f[kCpProbes], cidx[kCpProbes];
@@ -1025,12 +1036,15 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
           cidx[u] = -1;
           rel[u] = -1;
           const int64_t t = t0 + u;
+          const int32_t q = q0, j = j0;
+          if (++j0 == mg) {
+            j0 = 0;
+            ++q0;
+          }
           if (t >= items) continue;
-          const int32_t q = (int32_t)(t / mg), j = (int32_t)(t % mg);
           qs[u] = q;
           js[u] = j;
-          const int32_t r = req_of(g0 + j);
-          const int64_t bo = __ldg(block_off + r), nb = __ldg(block_off + r + 1) - bo;
+          const int64_t bo = s_bo[j], nb = s_nb[j];
           if ((int64_t)kChunk * q >= nb) continue;  // the request has no chunk q
           if (!wait_above(&s_share[j], -1)) {
             if (lane == 0) latch_error(status, SMETRIC_ERR_CUDA);
@@ -1052,7 +1066,7 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
           const int64_t b = (int64_t)kChunk * q + lane;
           act[u] = b < nb && b >= sh;
           f[u] = bo + b;
-          cidx[u] = __ldg(chunk_off + r) + q;
+          cidx[u] = s_cb[j] + q;
           if (act[u]) hv[u] = ld_relaxed_cta(hashes + bo + b);
         }
         uint64_t M[kCpProbes][W];
