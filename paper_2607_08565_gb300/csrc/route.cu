@@ -747,6 +747,7 @@ constexpr int kCpMaxGroup = 32 * kCpMaxChainWarps;
 constexpr int kCpRingDigests = 34;   // a chunk's 32 digests and one neighbour on each side
 constexpr int kCpRingBytes = 560;    // two such slots per chain lane, in 16-byte pieces
 constexpr int kCpProbes = 2;         // chunks a probe warp takes at once (probes in flight per lane)
+constexpr int kCpDealMax = 512;      // requests a CTA can own when leaders are dealt out
 
 __device__ __forceinline__ int32_t ld_acquire_cta(const int32_t* p) {
   int32_t v;
@@ -827,6 +828,32 @@ __device__ __forceinline__ void probe_many(const uint8_t* __restrict__ tags, con
   }
 }
 
+// One thread per request: 1 if the request leads its group (the group
+// table's lowest request with its first-block hash), else 0.
+__global__ void __launch_bounds__(256)
+    k_lead(const int64_t* __restrict__ block_off, int32_t n, const int32_t* __restrict__ batch_ok,
+           const uint64_t* __restrict__ D, uint64_t h_init, const uint64_t* __restrict__ groups, uint64_t gmask,
+           uint8_t* __restrict__ lead_flag) {
+  pdl_enter();
+  const int32_t r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= n || !*batch_ok) return;
+  const int64_t bo = block_off[r];
+  uint8_t f = 0;
+  if (block_off[r + 1] > bo) {
+    const uint64_t key = first_hash(h_init, __ldg(D + bo));
+    uint64_t sl = key & gmask;
+    for (uint64_t t = 0; t <= gmask; ++t, sl = (sl + 1) & gmask) {
+      const ulonglong2 pr = *reinterpret_cast<const ulonglong2*>(groups + 2 * sl);
+      if (pr.x == key) {
+        f = INT32_MAX - (int32_t)pr.y == r;
+        break;
+      }
+      if (pr.x == 0) break;
+    }
+  }
+  lead_flag[r] = f;
+}
+
 template <int W>
 __global__ void __launch_bounds__(kCpWarps * 32, 1)
     k_chain_probe(const int64_t* __restrict__ block_off, const int64_t* __restrict__ chunk_off, int32_t n, int S,
@@ -835,7 +862,8 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
                   uint64_t gmask, int32_t* __restrict__ lead, int32_t* __restrict__ share,
                   int32_t* __restrict__ order, int32_t* __restrict__ counts, const uint8_t* __restrict__ tags,
                   const uint64_t* __restrict__ table, uint64_t n_buckets, uint64_t* __restrict__ masks,
-                  uint64_t* __restrict__ chunk_and, int chain_warps, int32_t* status) {
+                  uint64_t* __restrict__ chunk_and, const uint8_t* __restrict__ lead_flag, int chain_warps,
+                  int32_t* status) {
   pdl_enter();
   extern __shared__ __align__(128) unsigned char csm[];  // chain lanes' digest rings
   __shared__ int32_t s_ready[kCpMaxGroup];  // chunks chained, per request of the group
@@ -849,12 +877,52 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
   __shared__ unsigned long long s_next1;    // work counter: probe items
   __shared__ int32_t s_maxch;               // most chunks of a request in the group
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // This CTA's requests are blockIdx.x + k * gridDim.x, k = 0, 1, ...: the
-  // batch's order (group leaders are the first requests of their sessions, so
-  // they crowd its front) is spread evenly over the CTAs.
+  // The CTAs' requests. A group leader (the lowest request with its first
+  // block, which probes its whole prefix) costs a member (which probes only
+  // past its shared prefix) many times over, so leaders are dealt round robin
+  // over the CTAs in request order, then the members after them: every CTA
+  // gets its share of each. k_lead has marked the leaders. Past 32 requests
+  // a thread, or kCpDealMax a CTA, requests are taken as blockIdx.x +
+  // k * gridDim.x instead.
+  __shared__ int32_t s_mine[kCpDealMax];
+  __shared__ int32_t s_nmine;
+  __shared__ int32_t s_wsum[kCpWarps];
   const int32_t stride = (int32_t)gridDim.x;
-  const int32_t m = n > (int32_t)blockIdx.x ? (n - (int32_t)blockIdx.x + stride - 1) / stride : 0;
-  auto req_of = [&](int32_t k) { return (int32_t)blockIdx.x + k * stride; };
+  const int32_t per_t = (n + (int32_t)blockDim.x - 1) / (int32_t)blockDim.x;
+  const bool dealt = *batch_ok && per_t <= 32 && (n + stride - 1) / stride <= kCpDealMax;
+  if (dealt) {
+    if (threadIdx.x == 0) s_nmine = 0;
+    const int32_t a = min(n, (int32_t)threadIdx.x * per_t), e = min(n, a + per_t);
+    uint32_t lead_bits = 0;  // bit i: request a + i leads its group (from k_lead)
+    for (int32_t r = a; r < e; ++r) lead_bits |= (uint32_t)__ldg(lead_flag + r) << (r - a);
+    // exclusive scan of the leader counts over the threads, in request order
+    const int32_t cnt = __popc(lead_bits);
+    int32_t incl = cnt;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const int32_t y = __shfl_up_sync(kFull, incl, d);
+      if (lane >= d) incl += y;
+    }
+    if (lane == 31) s_wsum[warp] = incl;
+    __syncthreads();
+    int32_t before = 0, total = 0;
+    for (int w2 = 0; w2 < kCpWarps; ++w2) {
+      const int32_t v = s_wsum[w2];
+      if (w2 < warp) before += v;
+      total += v;
+    }
+    int32_t lrank = before + incl - cnt;  // leaders before request a
+    for (int32_t r = a; r < e; ++r) {
+      const bool isl = (lead_bits >> (r - a)) & 1u;
+      // leaders by leader rank; members by member rank, continuing the deal
+      const int32_t cta = isl ? lrank % stride : (total + (r - lrank)) % stride;
+      if (isl) ++lrank;
+      if (cta == (int32_t)blockIdx.x) s_mine[atomicAdd(&s_nmine, 1)] = r;
+    }
+    __syncthreads();
+  }
+  const int32_t m = dealt ? s_nmine : n > (int32_t)blockIdx.x ? (n - (int32_t)blockIdx.x + stride - 1) / stride : 0;
+  auto req_of = [&](int32_t k) { return dealt ? s_mine[k] : (int32_t)blockIdx.x + k * stride; };
   if (!*batch_ok) {
     for (int32_t k = (int32_t)threadIdx.x; k < m; k += blockDim.x) sk_out[req_of(k)] = 0;
     return;
@@ -2079,6 +2147,14 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
     const int64_t per_cta = ((int64_t)n + grid - 1) / grid;
     const int chain_warps = (int)std::max<int64_t>(1, std::min<int64_t>(kCpMaxChainWarps, (per_cta + 31) / 32));
     const size_t smem = (size_t)chain_warps * 32 * kCpRingBytes;
+    // leader flags, one byte a request, in the scratch words k_link_sessions uses for its keys
+    uint8_t* const flags = reinterpret_cast<uint8_t*>(idx->sk_tmp);
+    idx->launches++;
+    if ((rc = launch_k(k_lead, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, !idx->profiling,
+                       (const int64_t*)idx->block_off, n, (const int32_t*)idx->batch_ok, (const uint64_t*)idx->digest,
+                       mix64(idx->cfg.hash_seed + kGamma), (const uint64_t*)idx->groups, group_slots_for(n) - 1,
+                       flags)))
+      return rc;
     if (smem > 48 * 1024 &&
         cudaFuncSetAttribute(k_chain_probe<W>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
       return cuda_status(cudaErrorInvalidValue);
@@ -2089,8 +2165,8 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
                        (const uint64_t*)idx->digest, hashes ? hashes : idx->hashes, sk, (const uint64_t*)idx->groups,
                        group_slots_for(n) - 1, idx->lead, idx->share, idx->order,
                        idx->order + idx->cfg.max_batch_requests, (const uint8_t*)idx->tags,
-                       (const uint64_t*)idx->table, idx->n_buckets, idx->masks, idx->chunk_and, chain_warps,
-                       idx->status)))
+                       (const uint64_t*)idx->table, idx->n_buckets, idx->masks, idx->chunk_and,
+                       (const uint8_t*)flags, chain_warps, idx->status)))
       return rc;
     if (after_chain && cudaEventRecord(after_chain, s) != cudaSuccess) return cuda_status(cudaErrorUnknown);
   }

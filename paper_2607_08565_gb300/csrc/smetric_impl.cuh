@@ -87,8 +87,9 @@ __device__ __forceinline__ void latch_error(int32_t* status, int32_t code) {
 __host__ __device__ constexpr int entry_words(int W) { return W == 1 ? 2 : (W <= 3 ? 4 : 8); }
 
 // Route kernels, in launch order; names returned by smetric_profile_kernel_name.
-// kChainProbe is k_chain_probe in a route (chain, group stage and probe in one
-// kernel) and k_chain in the calls that only hash.
+// kChainProbe is k_lead and k_chain_probe in a route (leader flags, then
+// chain, group stage and probe in one kernel) and k_chain in the calls that
+// only hash.
 enum RouteKernel { kPrep = 0, kDigest = 1, kChainProbe = 2, kWalk = 3, kNumRouteKernels = 4 };
 
 struct ProfileSlot {
@@ -118,7 +119,7 @@ struct smetric_index {
   int32_t* lead;       // max_batch_requests: the request whose masks a request shares
   int32_t* share;      // max_batch_requests: leading blocks taken from the leader
   int32_t* summ;       // max_batch_requests * (num_instances + 1): a leader's run ends c_i, then g
-  uint64_t* sk_tmp;     // max_batch_requests: session keys nobody reads (session links)
+  uint64_t* sk_tmp;     // max_batch_requests: session keys nobody reads (session links); a route's leader flags
   int32_t* order;      // max_batch_requests + 2: leaders from the front, members from the back, then both counts
   int64_t* chunk_off;  // max_batch_requests + 1: first 32-block chunk of each request
   cudaStream_t side;   // runs the group stage beside the chain
