@@ -1265,8 +1265,9 @@ def sweep_index(N, B, table_gb, max_req, max_tok, device):
     return tr, ix, slots * (entry + 1), tr.n_prefix_blocks() + max(n_fill, 0)
 
 
-def sweep_point(tr, ix, batch, device):
-    """Route one config-5 batch repeatedly; per-kernel device time."""
+def sweep_point(tr, ix, batch, device, gpu_id=None):
+    """Route one config-5 batch repeatedly; per-kernel device time, the whole
+    path's roofline fraction, and the clocks sampled around the timed steps."""
     import torch
     import paper_2607_08565_gb300 as pkg
     p = tr.params
@@ -1275,6 +1276,13 @@ def sweep_point(tr, ix, batch, device):
     off = torch.from_numpy(bt.offsets).to(device)
     load = torch.from_numpy(bt.load).to(device)
     w = (p.w_load, p.w_miss, p.w_glob)
+    out = ix.route_batch(tok, off, load, w, want_hashes=False)
+    ix.check()
+    algo = algorithmic_bytes(bt.lengths(), out["local_hit"].cpu().numpy(), out["global_hit"].cpu().numpy(),
+                             p.block_size, ix.W)
+    clocks = ClockSampler(gpu_id) if gpu_id is not None else None
+    if clocks:
+        clocks.start()
     for _ in range(3):
         ix.route_batch(tok, off, load, w, want_hashes=False)
     ix.check()
@@ -1287,6 +1295,13 @@ def sweep_point(tr, ix, batch, device):
     e1.record(stream)
     torch.cuda.synchronize()
     us = e0.elapsed_time(e1) * 1e3 / steps
+    clk = None
+    if clocks:
+        soaked = clocks.soak(lambda i: ix.route_batch(tok, off, load, w, want_hashes=False), min_samples=4)
+        clk = clocks.stop("warm-up and timed steps" + (f", then {soaked} more of the same steps (untimed)"
+                                                       if soaked else ""))
+    peak, peak_kind = peak_hbm()
+    path_frac = algo["path"] / (us / 1e6) / 1e9 / peak
     pkg.smetric_profile_enable(ix.handle, True)
     for _ in range(steps):
         ix.route_batch(tok, off, load, w, want_hashes=False)
@@ -1295,7 +1310,10 @@ def sweep_point(tr, ix, batch, device):
     ix.check()
     return {"batch": batch, "tokens": int(bt.n_tokens), "us_per_batch": us,
             "requests_per_s": batch / us * 1e6, "tokens_per_s": bt.n_tokens / us * 1e6,
-            "kernels_us": {k: v[0] * 1e3 / max(v[1], 1) for k, v in prof.items()}, "steps": steps}
+            "kernels_us": {k: v[0] * 1e3 / max(v[1], 1) for k, v in prof.items()}, "steps": steps,
+            "roofline_path": {"frac": path_frac, "algorithmic_bytes": algo["path"], "peak": peak,
+                              "peak_kind": f"{peak_kind} copy"},
+            "clocks": clk}
 
 
 def run_sweep(args):
@@ -1317,8 +1335,12 @@ def run_sweep(args):
         max_tok = int(tr0.session_len.max()) * max_req
         tr, ix, table_bytes, keys = sweep_index(N, B, args.table_gb, max_req, max_tok, device)
         build_s = time.perf_counter() - t0
+        try:
+            gpu_id = "GPU-" + str(torch.cuda.get_device_properties(0).uuid)
+        except Exception:
+            gpu_id = "0"
         for b in batches:
-            pt = sweep_point(tr, ix, b, device)
+            pt = sweep_point(tr, ix, b, device, gpu_id)
             pt.update({"sweep": "config-5", "num_instances": N, "block_size": B,
                        "table_bytes": table_bytes, "index_keys": int(keys), "build_s": build_s})
             print(json.dumps(pt), flush=True)

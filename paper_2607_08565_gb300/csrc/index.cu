@@ -261,9 +261,6 @@ void free_all(smetric_index* x) {
   cudaFree(x->groups);
   cudaFree(x->lead);
   cudaFree(x->chunk_off);
-  if (x->side) cudaStreamDestroy(x->side);
-  if (x->fork_ev) cudaEventDestroy(x->fork_ev);
-  if (x->join_ev) cudaEventDestroy(x->join_ev);
   cudaFree(x->batch_ok);
   cudaFree(x->st_tokens);
   cudaFree(x->st_offsets);
@@ -331,10 +328,6 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
             cudaMalloc(&x->summ, (R > 0 ? R : 1) * ((size_t)c.num_instances + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->batch_ok, sizeof(int32_t)) == cudaSuccess;
   if (ok) x->share = x->lead + (R + 1);
-  if (ok)
-    ok = cudaStreamCreateWithFlags(&x->side, cudaStreamNonBlocking) == cudaSuccess &&
-         cudaEventCreateWithFlags(&x->fork_ev, cudaEventDisableTiming) == cudaSuccess &&
-         cudaEventCreateWithFlags(&x->join_ev, cudaEventDisableTiming) == cudaSuccess;
   if (ok && (c.flags & SMETRIC_FLAG_HOST_STAGING)) {
     const size_t T = (size_t)(c.max_batch_tokens > 0 ? c.max_batch_tokens : 1);
     ok = cudaMalloc(&x->st_tokens, T * sizeof(int32_t)) == cudaSuccess &&

@@ -2,32 +2,33 @@
 // match, integer cost and argmin (Figure 6 and Figure 10 of the paper, with
 // every request of the batch routed against one snapshot of index and load).
 //
-// Kernels per batch, in stream order (the group stage on a side stream):
+// Kernels per batch, in stream order:
 //   k_prep        one CTA: validates offsets and loads; scans the per-request
 //                 full-block counts into block_off and the 32-block chunk
-//                 counts into chunk_off.
+//                 counts into chunk_off; zeroes the leader and member counts.
 //   k_digest_tma  HBM-bound block digests d_b: chunk q of request r is its
 //                 blocks 32q..32q+31, one 2D TMA tile of 32 overlapping rows
 //                 (each block's bytes rounded out to 16-byte boundaries); a
 //                 CTA takes a contiguous range of chunks, its warps
 //                 interleaved over it; lane j folds block j's B/2 words.
-//                 (k_digest and k_digest_any cover block sizes the tensor
-//                 maps do not.)
-//   k_group_insert, k_group   (side stream, beside k_chain) each request's
-//                 first-block hash into a group table, then its leader and
-//                 the number of leading blocks whose digests equal the
-//                 leader's.
-//   k_chain       one thread per request: the serial chain h_b over its
-//                 digests and the session key.
-//   k_probe       one thread per block not shared with the leader: the tier
-//                 masks of h_b from the index (16 tags of the home bucket,
-//                 then the matching entry), and per warp the AND of its 32
-//                 blocks' masks.
+//                 The lane holding a request's first block also inserts the
+//                 request's group key (its first-block hash) into the group
+//                 table. (k_digest and k_digest_any cover block sizes the
+//                 tensor maps do not.)
+//   k_lead        one thread per request: whether it leads its group (the
+//                 group's lowest request index).
+//   k_chain_probe one CTA per SM. Chain warps (one lane per request the CTA
+//                 owns) run the serial chain h_b over the digests and write
+//                 the session key; beside them, probe warps find each
+//                 member's shared prefix with its leader and probe every
+//                 block not shared: the tier masks of h_b from the index (16
+//                 tags of the home bucket, then the matching entry), and the
+//                 AND of each 32-block chunk's masks.
 //   k_walk        leaders, then members: one warp per request walks the runs
 //                 of the local tiers and the global tier, 32 chunks per step
 //                 from the chunk ANDs and block by block where a run ends;
 //                 then lanes = instances for the cost and a shuffle argmin
-//                 with ties to the lowest id.
+//                 with ties to the lowest id (or one of the policy scores).
 
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -192,7 +193,7 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
 // digest
 // ---------------------------------------------------------------------------
 
-// The group stage works from the digests, so that it runs beside the chain:
+// The group stage works from the digests, so that it needs no finished chain:
 // a request's first-block hash h_0 = chain step from h_init over d_0 is the
 // group key, and the shared-prefix length is the number of leading blocks
 // whose digests equal the leader's. Equal digests from equal previous hashes
@@ -1967,13 +1968,12 @@ __global__ void __launch_bounds__(1024)
 void profile_mark(smetric_index* idx, int k, cudaStream_t s);
 
 // How a batch shares the GPU with the batch before it (smetric_route_batches
-// on two scratch sets): an event recorded once its chain is enqueued, and
-// caps on the digest's and the probe's resident CTAs per SM so that both fit
-// on every SM at once (0 = no cap).
+// on two scratch sets): an event recorded once its chain and probe are
+// enqueued, and a cap on the digest's resident CTAs per SM (0 = no cap) so
+// that its digests leave room on every SM for the other batch's walk.
 struct Overlap {
   cudaEvent_t after_chain;
   int digest_ctas_per_sm;
-  int probe_ctas_per_sm;
 };
 
 // Launches a route kernel; with pdl the launch may begin while the previous
@@ -2331,8 +2331,7 @@ int route_policy(smetric_index* idx, int mode, const int32_t* d_tokens, int64_t 
 namespace smetric {
 
 // The second route scratch set of an index created with SMETRIC_FLAG_PIPELINE:
-// the same buffers, with the same sizes, as the index's own set, and its own
-// side stream and events for the group stage.
+// the same buffers, with the same sizes, as the index's own set.
 struct RouteScratchSet {
   int64_t* block_off = nullptr;
   int64_t* chunk_off = nullptr;
@@ -2346,8 +2345,6 @@ struct RouteScratchSet {
   uint64_t* sk_tmp = nullptr;
   int32_t* order = nullptr;
   int32_t* batch_ok = nullptr;
-  cudaStream_t side = nullptr;
-  cudaEvent_t fork_ev = nullptr, join_ev = nullptr;
 };
 
 struct Pipeline {
@@ -2391,9 +2388,6 @@ static void free_pipeline(Pipeline* p) {
   cudaFree(a.sk_tmp);
   cudaFree(a.order);
   cudaFree(a.batch_ok);
-  if (a.side) cudaStreamDestroy(a.side);
-  if (a.fork_ev) cudaEventDestroy(a.fork_ev);
-  if (a.join_ev) cudaEventDestroy(a.join_ev);
   if (p->stream) cudaStreamDestroy(p->stream);
   for (cudaEvent_t e : {p->chain_done[0], p->chain_done[1], p->start, p->finish})
     if (e) cudaEventDestroy(e);
@@ -2416,9 +2410,6 @@ static void swap_scratch(smetric_index* x, RouteScratchSet& a) {
   std::swap(x->sk_tmp, a.sk_tmp);
   std::swap(x->order, a.order);
   std::swap(x->batch_ok, a.batch_ok);
-  std::swap(x->side, a.side);
-  std::swap(x->fork_ev, a.fork_ev);
-  std::swap(x->join_ev, a.join_ev);
 }
 
 // Allocates the second set of index x (called by smetric_index_create once
@@ -2445,9 +2436,6 @@ int pipeline_attach(smetric_index* x) {
             cudaMalloc(&a.summ, (R > 0 ? R : 1) * ((size_t)c.num_instances + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&a.batch_ok, sizeof(int32_t)) == cudaSuccess &&
             cudaMemset(a.groups, 0, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
-            cudaStreamCreateWithFlags(&a.side, cudaStreamNonBlocking) == cudaSuccess &&
-            cudaEventCreateWithFlags(&a.fork_ev, cudaEventDisableTiming) == cudaSuccess &&
-            cudaEventCreateWithFlags(&a.join_ev, cudaEventDisableTiming) == cudaSuccess &&
             cudaStreamCreateWithFlags(&p->stream, cudaStreamNonBlocking) == cudaSuccess;
   for (cudaEvent_t* e : {&p->chain_done[0], &p->chain_done[1], &p->start, &p->finish})
     ok = ok && cudaEventCreateWithFlags(e, cudaEventDisableTiming) == cudaSuccess;
@@ -2478,12 +2466,10 @@ void pipeline_release(smetric_index* x) {
 
 namespace {
 
-// Resident CTAs per SM while two batches overlap: one digest CTA (24 warps,
-// 38 registers a thread) beside four probe CTAs (8 warps, 31 registers) fit
-// the SM's 64 warps and 64K registers together, so neither kernel's
-// persistent grid can shut the other out.
+// Resident digest CTAs per SM while two batches overlap: one digest CTA (24
+// warps) leaves 40 of the SM's 64 warps to the other batch's walk, so the
+// persistent digest grid cannot shut it out.
 constexpr int kOverlapDigestCtas = 1;
-constexpr int kOverlapProbeCtas = 4;
 
 // smetric_route_batches: the host checks of route_common for every batch
 // first, then the batches, alternating between the two sets when the index
@@ -2528,7 +2514,7 @@ int route_batches(smetric_index* idx, int32_t nb, const int32_t* const* tok, con
       break;
     }
     if (set) swap_scratch(idx, p->alt);
-    const Overlap ov = {p->chain_done[set], kOverlapDigestCtas, kOverlapProbeCtas};
+    const Overlap ov = {p->chain_done[set], kOverlapDigestCtas};
     rc = route_common<true>(idx, tok[j], ntok[j], off[j], nreq[j], load[j], w, inst[j], lhit[j], ghit[j], sk[j],
                             nullptr, 0, sj, nullptr, &ov);
     if (set) swap_scratch(idx, p->alt);

@@ -122,8 +122,6 @@ struct smetric_index {
   uint64_t* sk_tmp;     // max_batch_requests: session keys nobody reads (session links); a route's leader flags
   int32_t* order;      // max_batch_requests + 2: leaders from the front, members from the back, then both counts
   int64_t* chunk_off;  // max_batch_requests + 1: first 32-block chunk of each request
-  cudaStream_t side;   // runs the group stage beside the chain
-  cudaEvent_t fork_ev, join_ev;
   int32_t* batch_ok;   // device flag written by the prep kernel
   // staging for smetric_route_batch_host
   int32_t* st_tokens;
