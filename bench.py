@@ -1166,61 +1166,67 @@ def run_imbalance(args, n_requests=3_456_000, num_instances=32, window=30_000, n
 # device-side index maintenance over a config-2 replay
 # ---------------------------------------------------------------------------
 
-def run_commit(args, n_batches=24):
+def run_commit(args):
+    """Route then commit on the device, batch after batch, with the capped
+    tiers' evictions done by the device LRU inside the timed commit: one line
+    per agent trace (c2_medium: local tiers capped, global tier uncapped;
+    c3_long: both capped)."""
     import itertools
     import torch
     import paper_2607_08565_gb300 as pkg
     from paper_2607_08565_gb300 import build_lib
-    from synth import ReplayDriver, agent_trace
+    from synth import agent_trace
 
     build_lib.build()
     torch.cuda.set_device(0)
-    tr = agent_trace("c2_medium")
-    p = tr.params
-    batches = list(itertools.islice(tr.batches(), n_batches))
-    blocks = [int((b.lengths() // p.block_size).sum()) for b in batches]
-    ix = pkg.SMetricIndex(p.num_instances, p.block_size, p.session_blocks,
-                          capacity_slots=max(1024, int(sum(blocks) * 2 / 0.5)),
-                          max_batch_requests=max(b.n_requests for b in batches),
-                          max_batch_tokens=max(b.n_tokens for b in batches), hash_seed=p.hash_seed)
-    driver = ReplayDriver(p.num_instances, p.block_size, local_cap=tr.local_cap,
-                          global_policy=tr.global_policy, global_cap=tr.global_cap)
-    load = torch.zeros(p.num_instances, dtype=torch.int64, device="cuda")
-    w = (p.w_load, p.w_miss, p.w_glob)
-    stream = torch.cuda.current_stream()
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-    route_ms, commit_ms, done = 0.0, 0.0, 0
-    for k, bt in enumerate(batches):
-        tok = torch.from_numpy(bt.tokens).cuda()
-        off = torch.from_numpy(bt.offsets).cuda()
-        torch.cuda.synchronize()
-        ev[0].record(stream)
-        out = ix.route_batch(tok, off, load, w, want_hashes=True)
-        ev[1].record(stream)
-        ix.commit_batch(off, out, also_global=tr.global_policy != "none", load=load)
-        ev[2].record(stream)
-        torch.cuda.synchronize()
-        ix.check()
-        if k >= 2:  # the first batches warm up
-            route_ms += ev[0].elapsed_time(ev[1])
-            commit_ms += ev[1].elapsed_time(ev[2])
-            done += blocks[k]
-        # the capped local tiers evict on the host's orders, outside the timed region
-        g = {key: v.cpu().numpy() for key, v in out.items()}
-        _, _, ek, et = driver.after_batch(bt.offsets, g["instance"], g["local_hit"],
-                                          g["block_hashes"][:blocks[k]])
-        if len(ek):
-            ix.evict(torch.from_numpy(ek).cuda(), torch.from_numpy(et).cuda())
-    timed = len(batches) - 2
-    line = {"metric": "device-side commit of routed batches (blocks into the chosen local tier and the "
-                      "global tier, queue drain)", "value": done / (commit_ms / 1e3), "unit": "blocks/s",
-            "n_gpus": 1, "steps": timed, "warmup": 2, "ms_per_step": commit_ms / timed,
-            "route_ms_per_step": route_ms / timed, "higher_is_better": True, "data": "synthetic",
-            "config": {"workload": "c2_medium agent trace (16 instances, B = 16, 256 requests per batch)",
-                       "blocks_per_batch": float(np.mean(blocks[2:])), "tiers_per_block": 2,
-                       "evictions": "host LRU driver, outside the timed region"}}
-    print(json.dumps(line), flush=True)
-    ix.close()
+    for name, n_batches in (("c2_medium", 24), ("c3_long", 12)):
+        tr = agent_trace(name)
+        p = tr.params
+        batches = list(itertools.islice(tr.batches(), n_batches))
+        blocks = [int((b.lengths() // p.block_size).sum()) for b in batches]
+        local_cap = tr.local_cap or 0
+        global_cap = tr.global_cap if (tr.global_policy == "lru" and tr.global_cap) else 0
+        live = sum(blocks) if tr.global_policy == "all" or not local_cap else \
+            min(sum(blocks), p.num_instances * local_cap + global_cap)
+        ix = pkg.SMetricIndex(p.num_instances, p.block_size, p.session_blocks,
+                              capacity_slots=max(1024, int(live / 0.6)),
+                              max_batch_requests=max(b.n_requests for b in batches),
+                              max_batch_tokens=max(b.n_tokens for b in batches), hash_seed=p.hash_seed)
+        ix.set_lru(local_cap, global_cap)
+        load = torch.zeros(p.num_instances, dtype=torch.int64, device="cuda")
+        w = (p.w_load, p.w_miss, p.w_glob)
+        stream = torch.cuda.current_stream()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        route_ms, commit_ms, done = 0.0, 0.0, 0
+        for k, bt in enumerate(batches):
+            tok = torch.from_numpy(bt.tokens).cuda()
+            off = torch.from_numpy(bt.offsets).cuda()
+            torch.cuda.synchronize()
+            ev[0].record(stream)
+            out = ix.route_batch(tok, off, load, w, want_hashes=True)
+            ev[1].record(stream)
+            ix.commit_batch(off, out, also_global=tr.global_policy != "none", load=load)
+            ev[2].record(stream)
+            torch.cuda.synchronize()
+            ix.check()
+            if k >= 2:  # the first batches warm up
+                route_ms += ev[0].elapsed_time(ev[1])
+                commit_ms += ev[1].elapsed_time(ev[2])
+                done += blocks[k]
+        sizes = ix.lru_sizes().cpu().numpy()
+        timed = len(batches) - 2
+        line = {"metric": "device-side commit of routed batches (blocks into the chosen local tier and the "
+                          "global tier, queue drain, LRU evictions of capped tiers)",
+                "value": done / (commit_ms / 1e3), "unit": "blocks/s", "n_gpus": 1, "steps": timed,
+                "warmup": 2, "ms_per_step": commit_ms / timed, "route_ms_per_step": route_ms / timed,
+                "higher_is_better": True, "data": "synthetic",
+                "config": {"workload": f"{name} agent trace ({p.num_instances} instances, B = {p.block_size}, "
+                                       f"{batches[0].n_requests} requests per batch, first {n_batches} batches)",
+                           "blocks_per_batch": float(np.mean(blocks[2:])), "local_cap": local_cap,
+                           "global_cap": global_cap, "lru_blocks_at_end": int(sizes.sum()),
+                           "evictions": "device LRU, inside the timed commit"}}
+        print(json.dumps(line), flush=True)
+        ix.close()
 
 
 # ---------------------------------------------------------------------------
@@ -1242,7 +1248,7 @@ def sweep_index(N, B, table_gb, max_req, max_tok, device):
     tr = burst_trace("c5_sweep", num_instances=N, block_size=B, batch_size=max_req)
     W = (N + 1 + 63) // 64
     entry = 16 if W == 1 else (32 if W <= 3 else 64)
-    slots = int(table_gb * 1e9 / (entry + 1))
+    slots = int(table_gb * 1e9 / (entry + 16 / 15))  # entry + a 16-byte tag group per 15 slots
     chunk = 4096
     max_tok = max(max_tok, chunk * int(tr.prefix_len.max()))
     ix = pkg.SMetricIndex(N, B, tr.params.session_blocks, capacity_slots=slots,
@@ -1262,7 +1268,8 @@ def sweep_index(N, B, table_gb, max_req, max_tok, device):
         tiers = torch.randint(-1, N, (m,), device=device, generator=g, dtype=torch.int32)
         ix.insert(keys, tiers)
     ix.check()
-    return tr, ix, slots * (entry + 1), tr.n_prefix_blocks() + max(n_fill, 0)
+    nb = -(-slots // 15)
+    return tr, ix, nb * 15 * entry + nb * 16, tr.n_prefix_blocks() + max(n_fill, 0)
 
 
 def sweep_point(tr, ix, batch, device, gpu_id=None):

@@ -73,8 +73,9 @@ enum {
 #define SMETRIC_MAX_INSTANCES 256
 #define SMETRIC_MAX_WEIGHT (1LL << 20)
 #define SMETRIC_MAX_LOAD (1LL << 40)
-/* An insert that probes this many slots without finding its key or a free
- * slot reports SMETRIC_ERR_TABLE_FULL; lookups stop after as many probes. */
+/* An insert that visits SMETRIC_MAX_PROBE / 16 buckets (of 15 slots) without
+ * finding its key or a free slot reports SMETRIC_ERR_TABLE_FULL; lookups
+ * visit as many buckets at most. */
 #define SMETRIC_MAX_PROBE 65536
 
 /* smetric_index_config.flags */
@@ -86,7 +87,7 @@ typedef struct {
   int32_t block_size;         /* B, even, 2..256 tokens */
   int32_t session_blocks;     /* S >= 1: blocks that form the session key */
   int32_t flags;              /* SMETRIC_FLAG_* */
-  uint64_t capacity_slots;    /* index slots, >= 1; size for a load factor <= 0.7 */
+  uint64_t capacity_slots;    /* index slots, >= 1; size for a load factor <= 0.7 of the live keys */
   uint64_t hash_seed;         /* seed of the chain hash */
   int64_t max_batch_requests; /* largest n_requests a route call accepts */
   int64_t max_batch_tokens;   /* largest n_tokens a route call accepts */
@@ -100,9 +101,11 @@ typedef struct {
 } smetric_weights;
 
 /* Create an empty index and its route scratch on the current device.
- * The table holds capacity_slots (rounded up to a multiple of 16) entries of
+ * The table holds capacity_slots (rounded up to a multiple of 15) entries of
  * 16, 32 or 64 bytes (key plus ceil((N+1)/64) tier-mask words, padded to a
- * power of two) and one tag byte per slot. The route scratch holds, in 64-bit
+ * power of two) and a 16-byte tag group per 15 slots (a tag byte per slot
+ * and the bucket's overflow count). A key occupies a slot while some tier
+ * holds it: evictions give slots back. The route scratch holds, in 64-bit
  * words, (2 + W) * (max_batch_tokens/B) for per-block digests, hashes and
  * tier masks, 2 * (max_batch_requests + 1) for per-request offsets, group
  * leaders and shared-block counts, and 2 * G for the group table, G the
@@ -126,12 +129,16 @@ int smetric_index_clear(smetric_index* idx, smetric_stream_t stream);
  * (0..N-1 = local tier of that instance, -1 = global tier). Keys are block
  * hashes (>= 2). Set semantics: idempotent and order-independent within a
  * call. Errors latched: a key < 2 or tier out of range (INVALID_ARG, that
- * pair skipped), no free slot (TABLE_FULL). */
+ * pair skipped), no free slot (TABLE_FULL). A tier the device LRU caps
+ * (smetric_index_set_lru) is INVALID_ARG here: its keys enter through
+ * smetric_index_commit_batch only. */
 int smetric_index_insert(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers,
                          int64_t n, smetric_stream_t stream);
 
 /* Remove key d_keys[j] from tier d_tiers[j]; absent pairs are ignored. A key
- * that leaves its last tier keeps its slot and matches no tier. */
+ * that leaves its last tier gives its slot back for later inserts. A tier the
+ * device LRU caps is INVALID_ARG here (latched, pair skipped): it evicts on
+ * its own. */
 int smetric_index_evict(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers,
                         int64_t n, smetric_stream_t stream);
 
@@ -368,8 +375,10 @@ int smetric_route_batch_baseline(smetric_index* idx, const int32_t* d_tokens, in
  *                  smetric_route_batch writes them).
  *   d_load         int64 [N], read and written; NULL skips the drain.
  * Stream-ordered after the route; set semantics as smetric_index_insert
- * (inserting a key a tier holds is a no-op). Capped tiers are the caller's
- * to evict (smetric_index_evict): the index keeps no recency. Errors
+ * (inserting a key a tier holds is a no-op). Tiers capped by
+ * smetric_index_set_lru then evict their least recently used blocks down to
+ * the cap; other capped tiers are the caller's to evict
+ * (smetric_index_evict). Errors
  * latched: invalid offsets, an instance outside [-1, N) or a local hit
  * outside [0, L_r] (INVALID_ARG: nothing is committed and the loads are left
  * as they were), no free slot (TABLE_FULL). d_local_hit may be NULL when
@@ -378,6 +387,41 @@ int smetric_index_commit_batch(smetric_index* idx, const int64_t* d_offsets, int
                                const int32_t* d_instance, const int32_t* d_local_hit,
                                const uint64_t* d_block_hashes, int32_t flags, int64_t* d_load,
                                smetric_stream_t stream);
+
+/* One replay step on the device: smetric_route_batch, then
+ * smetric_index_commit_batch of its outputs, on one stream with no host
+ * round trip in between. d_load (int64 [N]) is read by the route and then
+ * drained in place by the commit. d_block_hashes is required (the commit
+ * reads it); flags as smetric_index_commit_batch. Arguments and errors as
+ * the two calls; an invalid batch routes every request to -1 and commits
+ * nothing. */
+int smetric_route_commit_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                               const int64_t* d_offsets, int32_t n_requests, int64_t* d_load,
+                               smetric_weights w, int32_t* d_instance, int32_t* d_local_hit,
+                               int32_t* d_global_hit, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                               int64_t hashes_cap, int32_t flags, smetric_stream_t stream);
+
+/* Device-side LRU for capped tiers (Section 2: an instance's local KV$ and
+ * the global store are bounded and keep their most recently used blocks).
+ * local_cap > 0 caps every local tier at that many blocks, global_cap > 0
+ * the global tier; 0 leaves a tier uncapped, and (0, 0) turns the LRU off.
+ * After each smetric_index_commit_batch, a capped tier holds its cap most
+ * recent blocks: a block touched by request r of a commit at block position
+ * b has recency (commit, r, -b) (later commits, later requests and, within a
+ * request, leading blocks are more recent), and the least recent leave
+ * first. Call it while the capped tiers are empty (after create or
+ * smetric_index_clear): keys already in them are not tracked. Synchronises
+ * the device; any earlier recency state is dropped. Device memory: 16 B per
+ * capped block (two record buffers), plus 16 B x 2 x max_blocks of touch
+ * lists, 16 B x 8 x max_blocks of per-batch sets and a byte per record and
+ * touch (max_blocks = max_batch_tokens / B).
+ * Errors: a negative cap or one above 2^40 (INVALID_ARG), an allocation
+ * failure (OOM: the LRU is off then). */
+int smetric_index_set_lru(smetric_index* idx, int64_t local_cap, int64_t global_cap);
+
+/* d_sizes[t] (int64 [N+1], device) = blocks the LRU tracks in tier t (local
+ * tiers 0..N-1, the global tier at N); 0 for uncapped tiers. Stream-ordered. */
+int smetric_index_lru_sizes(smetric_index* idx, int64_t* d_sizes, smetric_stream_t stream);
 
 /* Step (a)-(b) alone: block hashes and session keys of a batch, without
  * index lookups (Appendix A: a request's block-hash sequence starts with its

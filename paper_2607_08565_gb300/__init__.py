@@ -54,7 +54,7 @@ EXPORTED = (
     "smetric_index_commit_batch", "smetric_route_batch_policy_coloc", "smetric_link_sessions",
     "smetric_route_batch_baseline", "smetric_route_batch_sequential", "smetric_reuse_workspace_bytes",
     "smetric_reuse_breakdown", "smetric_imbalance_workspace_bytes", "smetric_window_imbalance",
-    "smetric_route_batches",
+    "smetric_route_batches", "smetric_index_set_lru", "smetric_index_lru_sizes", "smetric_route_commit_batch",
 )
 
 
@@ -118,6 +118,10 @@ def lib():
             "smetric_route_batch_policy": (C.c_int, [P, P, I64, P, I32, P, P, P, smetric_policy, P, P,
                                                      P, P, P, P, I64, P]),
             "smetric_index_commit_batch": (C.c_int, [P, P, I32, P, P, P, I32, P, P]),
+            "smetric_index_set_lru": (C.c_int, [P, I64, I64]),
+            "smetric_route_commit_batch": (C.c_int, [P, P, I64, P, I32, P, smetric_weights, P, P, P, P, P, I64,
+                                                     I32, P]),
+            "smetric_index_lru_sizes": (C.c_int, [P, P, P]),
             "smetric_link_sessions": (C.c_int, [P, P, I64, P, I32, P, P, P, P, P]),
             "smetric_reuse_workspace_bytes": (I64, [I64]),
             "smetric_imbalance_workspace_bytes": (I64, [I32, I32]),
@@ -233,6 +237,15 @@ def smetric_route_batch(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests
                                      hashes_cap, _stream(stream)), "smetric_route_batch")
 
 
+def smetric_route_commit_batch(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int, d_load, w,
+                               d_instance, d_local_hit, d_global_hit, d_session_key, d_block_hashes,
+                               hashes_cap: int, flags: int = 0, stream=None) -> None:
+    _check(lib().smetric_route_commit_batch(idx, _ptr(d_tokens), n_tokens, _ptr(d_offsets), n_requests,
+                                            _ptr(d_load), _weights(w), _ptr(d_instance), _ptr(d_local_hit),
+                                            _ptr(d_global_hit), _ptr(d_session_key), _ptr(d_block_hashes),
+                                            hashes_cap, flags, _stream(stream)), "smetric_route_commit_batch")
+
+
 def smetric_route_batches(idx: int, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance,
                           d_local_hit, d_global_hit, d_session_key, stream=None) -> None:
     """Several batches in one call; every argument but idx, w and stream is a
@@ -334,6 +347,14 @@ def smetric_index_commit_batch(idx: int, d_offsets, n_requests: int, d_instance,
     _check(lib().smetric_index_commit_batch(idx, _ptr(d_offsets), n_requests, _ptr(d_instance),
                                             _ptr(d_local_hit), _ptr(d_block_hashes), flags, _ptr(d_load),
                                             _stream(stream)), "smetric_index_commit_batch")
+
+
+def smetric_index_set_lru(idx: int, local_cap: int, global_cap: int) -> None:
+    _check(lib().smetric_index_set_lru(idx, local_cap, global_cap), "smetric_index_set_lru")
+
+
+def smetric_index_lru_sizes(idx: int, d_sizes, stream=None) -> None:
+    _check(lib().smetric_index_lru_sizes(idx, _ptr(d_sizes), _stream(stream)), "smetric_index_lru_sizes")
 
 
 def smetric_block_hashes(idx: int, d_tokens, n_tokens: int, d_offsets, n_requests: int,
@@ -495,6 +516,24 @@ class SMetricIndex:
                             out["session_key"], hb, hb.numel() if hb is not None else 0, stream)
         return out
 
+    def route_commit_batch(self, tokens, offsets, load, weights=(1, 4, 2), also_global=False, stream=None):
+        """route_batch then commit_batch on the device in one call; `load` is
+        read by the route and drained in place. Returns route_batch's dict
+        with block_hashes."""
+        import torch
+        n = offsets.numel() - 1
+        dev = offsets.device
+        out = dict(instance=torch.empty(n, dtype=torch.int32, device=dev),
+                   local_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                   global_hit=torch.empty(n, dtype=torch.int32, device=dev),
+                   session_key=torch.empty(n, dtype=torch.uint64, device=dev),
+                   block_hashes=torch.empty(max(tokens.numel() // self.B, 1), dtype=torch.uint64, device=dev))
+        hb = out["block_hashes"]
+        smetric_route_commit_batch(self.handle, tokens, tokens.numel(), offsets, n, load, weights, out["instance"],
+                                   out["local_hit"], out["global_hit"], out["session_key"], hb, hb.numel(),
+                                   SMETRIC_COMMIT_GLOBAL if also_global else 0, stream)
+        return out
+
     def route_batch_policy(self, tokens, offsets, queued, turn, est_hit, policy, want_hashes=False,
                            out=None, stream=None):
         """The session-centric policy (Figure 10). `policy` is a dict with c_lin,
@@ -618,6 +657,19 @@ class SMetricIndex:
         smetric_index_commit_batch(self.handle, offsets, offsets.numel() - 1, out["instance"],
                                    out["local_hit"], out["block_hashes"],
                                    SMETRIC_COMMIT_GLOBAL if also_global else 0, load, stream)
+
+    def set_lru(self, local_cap=0, global_cap=0):
+        """Caps the local tiers at `local_cap` blocks each and the global tier
+        at `global_cap` (0: uncapped); commit_batch then evicts each capped
+        tier's least recently used blocks on the device."""
+        smetric_index_set_lru(self.handle, int(local_cap), int(global_cap))
+
+    def lru_sizes(self, stream=None):
+        """Blocks the device LRU tracks per tier (int64 [N+1], global last)."""
+        import torch
+        out = torch.empty(self.N + 1, dtype=torch.int64, device="cuda")
+        smetric_index_lru_sizes(self.handle, out, stream)
+        return out
 
     def block_hashes(self, tokens, offsets, stream=None):
         """Returns (block_hashes, session_key) as device tensors."""

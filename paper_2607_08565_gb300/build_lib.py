@@ -16,7 +16,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libsmetric.so")
-SOURCES = ["index.cu", "route.cu", "imbalance.cu"]
+SOURCES = ["index.cu", "route.cu", "imbalance.cu", "lru.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

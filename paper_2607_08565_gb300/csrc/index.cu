@@ -5,12 +5,12 @@
 // block hash, which tiers hold the block. One table serves all tiers: an
 // entry is the 64-bit block hash followed by W = ceil((N+1)/64) mask words,
 // bit i < N = local tier of instance i, bit N = global tier. Slots are grouped
-// in buckets of kBucket; a one-byte tag per slot (0 = empty, else 0x80 | low
-// 7 key bits) lives in a separate tag array so that a lookup reads one
-// 16-byte tag group and then only the entry whose tag matches. Inserts take
-// the first empty slot in bucket order from the key's home bucket. Keys are
-// never removed: an evicted key keeps its slot with a cleared tier bit, so
-// lookups never meet tombstones and concurrent inserts cannot duplicate a key.
+// in buckets of kSlots; a one-byte tag per slot (0 = empty, else 0x80 | low
+// 7 key bits) and the bucket's overflow count live in a separate 16-byte tag
+// group, so that a lookup reads one tag group and then only the entry whose
+// tag matches. A key that leaves its last tier gives its slot back (the
+// primitives and their concurrency contract are in table.cuh), so a table
+// sized for the live keys serves any number of inserted and evicted ones.
 
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -19,6 +19,7 @@
 #include <new>
 
 #include "smetric_impl.cuh"
+#include "table.cuh"
 #include "call_range.cuh"
 
 using namespace smetric;
@@ -51,87 +52,10 @@ namespace {
 
 enum Op { kInsert = 0, kEvict = 1 };
 
-__device__ __forceinline__ uint64_t max_buckets(uint64_t n_buckets) {
-  const uint64_t m = SMETRIC_MAX_PROBE / kBucket;
-  return n_buckets < m ? n_buckets : m;
-}
-
-__device__ __forceinline__ uint4 load_tags_volatile(const uint8_t* p) {
-  const volatile uint32_t* q = reinterpret_cast<const volatile uint32_t*>(p);
-  return make_uint4(q[0], q[1], q[2], q[3]);
-}
-
-// Slot of `key`, or -1 when absent (at most SMETRIC_MAX_PROBE slots probed).
-// Used by kernels that do not run concurrently with inserts.
-__device__ __forceinline__ int64_t find_slot(const uint8_t* __restrict__ tags,
-                                             const uint64_t* __restrict__ table, int ew,
-                                             uint64_t n_buckets, uint64_t key) {
-  const uint32_t tg = key_tag(key);
-  uint64_t b = home_bucket(key, n_buckets);
-  const uint64_t mb = max_buckets(n_buckets);
-  for (uint64_t t = 0; t < mb; ++t) {
-    const uint4 tv = *reinterpret_cast<const uint4*>(tags + b * kBucket);
-    uint32_t cand = tag_match(tv, tg);
-    while (cand) {
-      const int sl = __ffs(cand) - 1;
-      cand &= cand - 1;
-      const uint64_t slot = b * kBucket + sl;
-      if (table[slot * ew] == key) return (int64_t)slot;
-    }
-    if (tag_match(tv, 0)) return -1;  // the bucket still has an empty slot
-    if (++b == n_buckets) b = 0;
-  }
-  return -1;
-}
-
-// Insert: set tier bit (word, m) of `key`, claiming the first empty slot in
-// bucket order if the key is new. A slot is claimed by a CAS on its key word
-// and published by setting its tag after a fence; a concurrent inserter of the
-// same key that meets the claimed-but-untagged slot sees its key in the failed
-// CAS and uses that slot. Returns false when no slot was found.
-__device__ bool insert_key(uint8_t* tags, uint64_t* table, int ew, uint64_t n_buckets,
-                           uint64_t key, int word, unsigned long long m) {
-  const uint32_t tg = key_tag(key);
-  uint64_t b = home_bucket(key, n_buckets);
-  const uint64_t mb = max_buckets(n_buckets);
-  for (uint64_t t = 0; t < mb; ++t) {
-    const uint4 tv = load_tags_volatile(tags + b * kBucket);
-    uint32_t cand = tag_match(tv, tg);
-    while (cand) {
-      const int sl = __ffs(cand) - 1;
-      cand &= cand - 1;
-      unsigned long long* e = reinterpret_cast<unsigned long long*>(table + (b * kBucket + sl) * ew);
-      if (*reinterpret_cast<volatile unsigned long long*>(e) == key) {
-        atomicOr(e + 1 + word, m);
-        return true;
-      }
-    }
-    uint32_t empty = tag_match(tv, 0);
-    while (empty) {
-      const int sl = __ffs(empty) - 1;
-      empty &= empty - 1;
-      unsigned long long* e = reinterpret_cast<unsigned long long*>(table + (b * kBucket + sl) * ew);
-      const unsigned long long old = atomicCAS(e, (unsigned long long)kEmpty, (unsigned long long)key);
-      if (old == kEmpty) {
-        __threadfence();
-        atomicOr(reinterpret_cast<unsigned int*>(tags + b * kBucket) + (sl >> 2), tg << (8 * (sl & 3)));
-        atomicOr(e + 1 + word, m);
-        return true;
-      }
-      if (old == key) {
-        atomicOr(e + 1 + word, m);
-        return true;
-      }
-    }
-    if (++b == n_buckets) b = 0;
-  }
-  return false;
-}
-
 // One thread per (key, tier) pair, grid-stride.
 template <int OP>
 __global__ void k_update(uint8_t* __restrict__ tags, uint64_t* __restrict__ table, uint64_t n_buckets,
-                         int ew, int N, const uint64_t* __restrict__ keys,
+                         int ew, int W, int N, bool lru_local, bool lru_global, const uint64_t* __restrict__ keys,
                          const int32_t* __restrict__ tiers, int64_t n, int32_t* status) {
   for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < n;
        j += (int64_t)gridDim.x * blockDim.x) {
@@ -142,14 +66,16 @@ __global__ void k_update(uint8_t* __restrict__ tags, uint64_t* __restrict__ tabl
       continue;
     }
     const int bit = tier < 0 ? N : tier;
+    if ((bit < N && lru_local) || (bit == N && lru_global)) {  // the device LRU owns capped tiers
+      latch_error(status, SMETRIC_ERR_INVALID_ARG);
+      continue;
+    }
     const unsigned long long m = 1ull << (bit & 63);
     if (OP == kInsert) {
       if (!insert_key(tags, table, ew, n_buckets, key, bit >> 6, m))
         latch_error(status, SMETRIC_ERR_TABLE_FULL);
     } else {
-      const int64_t slot = find_slot(tags, table, ew, n_buckets, key);
-      if (slot >= 0)
-        atomicAnd(reinterpret_cast<unsigned long long*>(table + slot * ew) + 1 + (bit >> 6), ~m);
+      remove_tier(tags, table, ew, W, n_buckets, key, bit >> 6, m);
     }
   }
 }
@@ -160,7 +86,7 @@ __global__ void k_lookup(const uint8_t* __restrict__ tags, const uint64_t* __res
   for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < n;
        j += (int64_t)gridDim.x * blockDim.x) {
     const uint64_t key = keys[j];
-    const int64_t slot = key >= 2 ? find_slot(tags, table, ew, n_buckets, key) : -1;
+    const int64_t slot = key >= 2 ? find_slot<false>(tags, table, ew, n_buckets, key) : -1;
     for (int w = 0; w < W; ++w) out[j * W + w] = slot >= 0 ? table[slot * ew + 1 + w] : 0;
   }
 }
@@ -214,14 +140,13 @@ int update(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers, i
   const int threads = 256;
   int grid = grid_for(idx, n, threads);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const bool ll = idx->lru && idx->lru->local_cap > 0, lg = idx->lru && idx->lru->global_cap > 0;
   if (op == kInsert)
-    k_update<kInsert><<<grid, threads, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->EW,
-                                               idx->cfg.num_instances, d_keys, d_tiers, n,
-                                               idx->status);
+    k_update<kInsert><<<grid, threads, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->EW, idx->W,
+                                               idx->cfg.num_instances, ll, lg, d_keys, d_tiers, n, idx->status);
   else
-    k_update<kEvict><<<grid, threads, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->EW,
-                                              idx->cfg.num_instances, d_keys, d_tiers, n,
-                                              idx->status);
+    k_update<kEvict><<<grid, threads, 0, s>>>(idx->tags, idx->table, idx->n_buckets, idx->EW, idx->W,
+                                              idx->cfg.num_instances, ll, lg, d_keys, d_tiers, n, idx->status);
   idx->launches++;
   return cuda_status(cudaGetLastError());
 }
@@ -247,6 +172,7 @@ namespace {
 
 void free_all(smetric_index* x) {
   pipeline_release(x);
+  lru_free(x);
   cudaFree(x->table);
   cudaFree(x->tags);
   cudaFree(x->status);
@@ -298,20 +224,21 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
   x->cfg = c;
   x->W = W;
   x->EW = entry_words(W);
-  x->n_buckets = (c.capacity_slots + kBucket - 1) / kBucket;
+  x->n_buckets = (c.capacity_slots + kSlots - 1) / kSlots;
   if (cudaGetDevice(&x->device) != cudaSuccess ||
       cudaDeviceGetAttribute(&x->num_sms, cudaDevAttrMultiProcessorCount, x->device) != cudaSuccess) {
     delete x;
     return cuda_status(cudaErrorInvalidDevice);
   }
-  const size_t slots = (size_t)x->n_buckets * kBucket;
+  const size_t slots = (size_t)x->n_buckets * kSlots;
   const size_t table_bytes = slots * x->EW * sizeof(uint64_t);
+  const size_t tag_bytes = (size_t)x->n_buckets * kBucket;
   const size_t max_blocks = (size_t)(c.max_batch_tokens / c.block_size);
   const size_t R = (size_t)c.max_batch_requests;
   x->group_slots = 64;
   while (x->group_slots < 2 * (uint64_t)R) x->group_slots <<= 1;
   bool ok = cudaMalloc(&x->table, table_bytes) == cudaSuccess &&
-            cudaMalloc(&x->tags, slots) == cudaSuccess &&
+            cudaMalloc(&x->tags, tag_bytes) == cudaSuccess &&
             cudaMalloc(&x->status, sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->block_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
             // two spare words: k_chain_probe copies a chunk's digests in whole 16-byte pieces
@@ -338,7 +265,7 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
   }
   if (ok && (c.flags & SMETRIC_FLAG_PIPELINE)) ok = pipeline_attach(x) == SMETRIC_OK;
   if (ok) ok = cudaMemset(x->table, 0, table_bytes) == cudaSuccess &&
-               cudaMemset(x->tags, 0, slots) == cudaSuccess &&
+               cudaMemset(x->tags, 0, tag_bytes) == cudaSuccess &&
                cudaMemset(x->status, 0, sizeof(int32_t)) == cudaSuccess &&
                cudaMemset(x->groups, 0, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
                cudaDeviceSynchronize() == cudaSuccess;
@@ -370,11 +297,12 @@ int smetric_index_clear(smetric_index* idx, smetric_stream_t stream) {
   CallRange range("smetric_index_clear");
   int rc = check_device(idx);
   if (rc) return rc;
-  const size_t slots = (size_t)idx->n_buckets * kBucket;
+  const size_t slots = (size_t)idx->n_buckets * kSlots;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (cudaMemsetAsync(idx->table, 0, slots * idx->EW * sizeof(uint64_t), s) != cudaSuccess)
+  if (cudaMemsetAsync(idx->table, 0, slots * idx->EW * sizeof(uint64_t), s) != cudaSuccess ||
+      cudaMemsetAsync(idx->tags, 0, (size_t)idx->n_buckets * kBucket, s) != cudaSuccess)
     return cuda_status(cudaErrorUnknown);
-  return cuda_status(cudaMemsetAsync(idx->tags, 0, slots, s));
+  return lru_reset(idx, s);
 }
 
 int smetric_index_insert(smetric_index* idx, const uint64_t* d_keys, const int32_t* d_tiers,

@@ -691,8 +691,8 @@ __global__ void __launch_bounds__(kChainThreads)
 // ---------------------------------------------------------------------------
 
 // Tier masks of key h (zeros when absent) from the read-only table: the home
-// bucket's 16 tags, then the entry of each tag match, then later buckets while
-// every slot of the bucket so far was full.
+// bucket's 15 tags, then the entry of each tag match, then later buckets while
+// the bucket just read has keys stored past it (its overflow count).
 template <int W>
 __device__ __forceinline__ void probe_one(const uint8_t* __restrict__ tags, const uint64_t* __restrict__ table,
                                           uint64_t n_buckets, uint64_t h, uint64_t (&M)[W]) {
@@ -702,14 +702,14 @@ __device__ __forceinline__ void probe_one(const uint8_t* __restrict__ tags, cons
   for (int w = 0; w < W; ++w) M[w] = 0;
   const uint32_t tg = key_tag(h);
   uint64_t b = home_bucket(h, n_buckets);
-  const uint64_t mb = n_buckets < SMETRIC_MAX_PROBE / kBucket ? n_buckets : SMETRIC_MAX_PROBE / kBucket;
+  const uint64_t mb = max_buckets(n_buckets);
   for (uint64_t t = 0; t < mb; ++t) {
     const uint4 tv = __ldg(reinterpret_cast<const uint4*>(tags + b * kBucket));
-    uint32_t cand = tag_match(tv, tg);
+    uint32_t cand = slot_match(tv, tg);
     while (cand) {
       const int sl = __ffs(cand) - 1;
       cand &= cand - 1;
-      const ulonglong2* e = reinterpret_cast<const ulonglong2*>(table + (b * kBucket + sl) * EW);
+      const ulonglong2* e = reinterpret_cast<const ulonglong2*>(table + (b * kSlots + sl) * EW);
       ulonglong2 v[NV];
 #pragma unroll
       for (int q = 0; q < NV; ++q) v[q] = __ldg(e + q);
@@ -719,7 +719,7 @@ __device__ __forceinline__ void probe_one(const uint8_t* __restrict__ tags, cons
         return;
       }
     }
-    if (tag_match(tv, 0)) return;
+    if (overflow_count(tv) == 0) return;
     if (++b == n_buckets) b = 0;
   }
 }
@@ -789,7 +789,7 @@ __device__ __forceinline__ bool wait_above(const int32_t* p, int32_t v) {
 // Tier masks of U keys at once: the home-bucket tags of all, then the first
 // tag match's entry of all, so that U pairs of dependent reads are in flight
 // together. A key whose first candidate is not it (another key with the same
-// tag, or a key stored past a full home bucket) takes the full probe_one.
+// tag, or a key stored past its home bucket) takes the full probe_one.
 template <int W, int U>
 __device__ __forceinline__ void probe_many(const uint8_t* __restrict__ tags, const uint64_t* __restrict__ table,
                                            uint64_t n_buckets, const bool (&act)[U], const uint64_t (&h)[U],
@@ -807,9 +807,9 @@ __device__ __forceinline__ void probe_many(const uint8_t* __restrict__ tags, con
   uint32_t cand[U];
 #pragma unroll
   for (int u = 0; u < U; ++u) {
-    cand[u] = act[u] ? tag_match(tv[u], key_tag(h[u])) : 0;
+    cand[u] = act[u] ? slot_match(tv[u], key_tag(h[u])) : 0;
     if (cand[u]) {
-      const ulonglong2* e = reinterpret_cast<const ulonglong2*>(table + (bk[u] * kBucket + __ffs(cand[u]) - 1) * EW);
+      const ulonglong2* e = reinterpret_cast<const ulonglong2*>(table + (bk[u] * kSlots + __ffs(cand[u]) - 1) * EW);
 #pragma unroll
       for (int q = 0; q < NV; ++q) v[u][q] = __ldg(e + q);
     }
@@ -822,10 +822,10 @@ __device__ __forceinline__ void probe_many(const uint8_t* __restrict__ tags, con
     if (cand[u] && v[u][0].x == h[u]) {
 #pragma unroll
       for (int w = 0; w < W; ++w) M[u][w] = (w & 1) ? v[u][(w + 1) >> 1].x : v[u][(w + 1) >> 1].y;
-    } else if ((cand[u] & (cand[u] - 1)) || !tag_match(tv[u], 0)) {
+    } else if ((cand[u] & (cand[u] - 1)) || overflow_count(tv[u])) {
       probe_one<W>(tags, table, n_buckets, h[u], M[u]);  // more candidates, or later buckets
     }
-    // else: no candidate left and the home bucket has an empty slot: absent
+    // else: no candidate left and no key stored past the home bucket: absent
   }
 }
 
@@ -1967,13 +1967,11 @@ __global__ void __launch_bounds__(1024)
 
 void profile_mark(smetric_index* idx, int k, cudaStream_t s);
 
-// How a batch shares the GPU with the batch before it (smetric_route_batches
+// How a batch shares the GPU with the batch after it (smetric_route_batches
 // on two scratch sets): an event recorded once its chain and probe are
-// enqueued, and a cap on the digest's resident CTAs per SM (0 = no cap) so
-// that its digests leave room on every SM for the other batch's walk.
+// enqueued, which the next batch's first kernel waits for.
 struct Overlap {
   cudaEvent_t after_chain;
-  int digest_ctas_per_sm;
 };
 
 // Launches a route kernel; with pdl the launch may begin while the previous
@@ -2050,7 +2048,7 @@ uint64_t group_slots_for(int32_t n) {
 // each request's first-block hash into the group table.
 template <int HB>
 int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
-                  const int64_t* d_offsets, int32_t n, cudaStream_t s, int cap_per_sm, bool group) {
+                  const int64_t* d_offsets, int32_t n, cudaStream_t s, bool group) {
   const int B = idx->cfg.block_size;
   const uint64_t d_init = mix64(idx->cfg.hash_seed ^ (uint64_t)B);
   const uint64_t h_init = mix64(idx->cfg.hash_seed + kGamma);
@@ -2077,8 +2075,7 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
         idx->digest_occ = occ < 1 ? 1 : occ;
       }
       const int64_t want = (max_chunks + warps - 1) / warps;
-      const int occ = cap_per_sm > 0 ? std::min(cap_per_sm, idx->digest_occ) : idx->digest_occ;
-      const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * occ));
+      const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * idx->digest_occ));
       idx->launches++;
       return launch_k(kern, dim3((unsigned)grid), dim3(warps * 32), smem, s, !idx->profiling, maps, d_tokens,
                       n_tokens, d_offsets, (const int64_t*)idx->block_off, (const int64_t*)idx->chunk_off, n, d_init,
@@ -2099,8 +2096,7 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
     idx->digest_occ = occ < 1 ? 1 : occ;
   }
   const int64_t want = (max_chunks + warps - 1) / warps;
-  const int occ = cap_per_sm > 0 ? std::min(cap_per_sm, idx->digest_occ) : idx->digest_occ;
-  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * occ));
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * idx->digest_occ));
   idx->launches++;
   if (HB > 0)
     return launch_k(kern, dim3((unsigned)grid), dim3(warps * 32), smem, s, !idx->profiling, d_tokens, n_tokens,
@@ -2112,12 +2108,12 @@ int launch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
 }
 
 int dispatch_digest(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
-                    const int64_t* d_offsets, int32_t n, cudaStream_t s, int cap_per_sm, bool group) {
+                    const int64_t* d_offsets, int32_t n, cudaStream_t s, bool group) {
   switch (idx->cfg.block_size) {
-    case 16: return launch_digest<8>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm, group);
-    case 32: return launch_digest<16>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm, group);
-    case 64: return launch_digest<32>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm, group);
-    default: return launch_digest<0>(idx, d_tokens, n_tokens, d_offsets, n, s, cap_per_sm, group);
+    case 16: return launch_digest<8>(idx, d_tokens, n_tokens, d_offsets, n, s, group);
+    case 32: return launch_digest<16>(idx, d_tokens, n_tokens, d_offsets, n, s, group);
+    case 64: return launch_digest<32>(idx, d_tokens, n_tokens, d_offsets, n, s, group);
+    default: return launch_digest<0>(idx, d_tokens, n_tokens, d_offsets, n, s, group);
   }
 }
 
@@ -2265,7 +2261,7 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
   profile_mark(idx, kPrep, s);
   // a route's digests also fill the group table (each request's first-block hash)
   if (n_tokens / c.block_size > 0) {
-    if ((rc = dispatch_digest(idx, d_tokens, n_tokens, d_offsets, n, s, ov ? ov->digest_ctas_per_sm : 0, PROBE)))
+    if ((rc = dispatch_digest(idx, d_tokens, n_tokens, d_offsets, n, s, PROBE)))
       return rc;
   }
   profile_mark(idx, kDigest, s);
@@ -2466,17 +2462,12 @@ void pipeline_release(smetric_index* x) {
 
 namespace {
 
-// Resident digest CTAs per SM while two batches overlap: one digest CTA (24
-// warps) leaves 40 of the SM's 64 warps to the other batch's walk, so the
-// persistent digest grid cannot shut it out.
-constexpr int kOverlapDigestCtas = 1;
-
 // smetric_route_batches: the host checks of route_common for every batch
 // first, then the batches, alternating between the two sets when the index
-// has a second one. Batch j's first kernel waits for batch j - 1's chain, so
-// that batch j's digests (bound by HBM bandwidth) run while batch j - 1's
-// probe and walk (bound by random accesses and latency) finish, and batch
-// j's chain does not share the GPU with batch j - 1's digests.
+// has a second one. Batch j's first kernel waits for batch j - 1's chain and
+// probe kernel, so that batch j's prep and digests (bound by the integer
+// pipe) run beside batch j - 1's walk (bound by latency), and batch j - 1's
+// chain does not share the GPU with batch j's digests.
 int route_batches(smetric_index* idx, int32_t nb, const int32_t* const* tok, const int64_t* ntok,
                   const int64_t* const* off, const int32_t* nreq, const int64_t* const* load, smetric_weights w,
                   int32_t* const* inst, int32_t* const* lhit, int32_t* const* ghit, uint64_t* const* sk,
@@ -2514,7 +2505,7 @@ int route_batches(smetric_index* idx, int32_t nb, const int32_t* const* tok, con
       break;
     }
     if (set) swap_scratch(idx, p->alt);
-    const Overlap ov = {p->chain_done[set], kOverlapDigestCtas};
+    const Overlap ov = {p->chain_done[set]};
     rc = route_common<true>(idx, tok[j], ntok[j], off[j], nreq[j], load[j], w, inst[j], lhit[j], ghit[j], sk[j],
                             nullptr, 0, sj, nullptr, &ov);
     if (set) swap_scratch(idx, p->alt);
@@ -2523,6 +2514,36 @@ int route_batches(smetric_index* idx, int32_t nb, const int32_t* const* tok, con
   if (cudaEventRecord(p->finish, p->stream) != cudaSuccess || cudaStreamWaitEvent(s, p->finish, 0) != cudaSuccess)
     return rc ? rc : cuda_status(cudaErrorUnknown);
   return rc;
+}
+
+// smetric_index_commit_batch's steps; with prep the batch's block offsets
+// and validity are computed here, else a route call just left them.
+int commit_common(smetric_index* idx, const int64_t* d_offsets, int32_t n_requests, const int32_t* d_instance,
+                  const int32_t* d_local_hit, const uint64_t* d_block_hashes, int32_t flags, int64_t* d_load,
+                  cudaStream_t s, bool prep) {
+  int rc = check_device(idx);
+  if (rc) return rc;
+  const smetric_index_config& c = idx->cfg;
+  if (n_requests < 0 || n_requests > c.max_batch_requests || (flags & ~SMETRIC_COMMIT_GLOBAL))
+    return SMETRIC_ERR_INVALID_ARG;
+  if (n_requests == 0) return SMETRIC_OK;
+  if (!d_offsets || !d_instance || !d_block_hashes || (d_load && !d_local_hit)) return SMETRIC_ERR_INVALID_ARG;
+  if (prep) {
+    // block offsets of the batch (and the offsets' checks) into the index's scratch
+    k_prep<<<1, 1024, 0, s>>>(d_offsets, n_requests, c.max_batch_tokens, c.block_size, nullptr, 0, idx->block_off,
+                              nullptr, idx->batch_ok, idx->status, SMETRIC_MAX_LOAD, (int64_t)INT32_MAX, nullptr);
+    idx->launches++;
+    if ((rc = cuda_status(cudaGetLastError()))) return rc;
+  }
+  // the checks (and the drain) first: a bad output commits nothing
+  k_drain<<<1, 1024, 0, s>>>(d_offsets, n_requests, c.num_instances, d_instance, d_local_hit, idx->batch_ok,
+                             d_load, idx->status);
+  idx->launches++;
+  if ((rc = cuda_status(cudaGetLastError()))) return rc;
+  if ((rc = launch_commit(idx, d_instance, d_block_hashes, n_requests, c.max_batch_tokens / c.block_size,
+                          (flags & SMETRIC_COMMIT_GLOBAL) != 0, s)))
+    return rc;
+  return lru_commit(idx, d_instance, d_block_hashes, n_requests, (flags & SMETRIC_COMMIT_GLOBAL) != 0, s);
 }
 
 }  // namespace
@@ -2619,26 +2640,24 @@ int smetric_index_commit_batch(smetric_index* idx, const int64_t* d_offsets, int
                                const uint64_t* d_block_hashes, int32_t flags, int64_t* d_load,
                                smetric_stream_t stream) {
   CallRange range("smetric_index_commit_batch");
-  int rc = check_device(idx);
-  if (rc) return rc;
-  const smetric_index_config& c = idx->cfg;
-  if (n_requests < 0 || n_requests > c.max_batch_requests || (flags & ~SMETRIC_COMMIT_GLOBAL))
-    return SMETRIC_ERR_INVALID_ARG;
-  if (n_requests == 0) return SMETRIC_OK;
-  if (!d_offsets || !d_instance || !d_block_hashes || (d_load && !d_local_hit)) return SMETRIC_ERR_INVALID_ARG;
+  return commit_common(idx, d_offsets, n_requests, d_instance, d_local_hit, d_block_hashes, flags, d_load,
+                       reinterpret_cast<cudaStream_t>(stream), true);
+}
+
+int smetric_route_commit_batch(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens,
+                               const int64_t* d_offsets, int32_t n_requests, int64_t* d_load,
+                               smetric_weights w, int32_t* d_instance, int32_t* d_local_hit,
+                               int32_t* d_global_hit, uint64_t* d_session_key, uint64_t* d_block_hashes,
+                               int64_t hashes_cap, int32_t flags, smetric_stream_t stream) {
+  CallRange range("smetric_route_commit_batch");
+  if ((flags & ~SMETRIC_COMMIT_GLOBAL) || !d_block_hashes) return SMETRIC_ERR_INVALID_ARG;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  // block offsets of the batch (and the offsets' checks) into the index's scratch
-  k_prep<<<1, 1024, 0, s>>>(d_offsets, n_requests, c.max_batch_tokens, c.block_size, nullptr, 0, idx->block_off,
-                            nullptr, idx->batch_ok, idx->status, SMETRIC_MAX_LOAD, (int64_t)INT32_MAX, nullptr);
-  idx->launches++;
-  if ((rc = cuda_status(cudaGetLastError()))) return rc;
-  // the checks (and the drain) first: a bad output commits nothing
-  k_drain<<<1, 1024, 0, s>>>(d_offsets, n_requests, c.num_instances, d_instance, d_local_hit, idx->batch_ok,
-                             d_load, idx->status);
-  idx->launches++;
-  if ((rc = cuda_status(cudaGetLastError()))) return rc;
-  return launch_commit(idx, d_instance, d_block_hashes, n_requests, c.max_batch_tokens / c.block_size,
-                       (flags & SMETRIC_COMMIT_GLOBAL) != 0, s);
+  const int rc = route_common<true>(idx, d_tokens, n_tokens, d_offsets, n_requests, d_load, w, d_instance,
+                                    d_local_hit, d_global_hit, d_session_key, d_block_hashes, hashes_cap, s);
+  if (rc) return rc;
+  // the route's prep left this batch's block offsets and validity in the scratch
+  return commit_common(idx, d_offsets, n_requests, d_instance, d_local_hit, d_block_hashes, flags, d_load, s,
+                       false);
 }
 
 int64_t smetric_reuse_workspace_bytes(int64_t n_blocks) {

@@ -21,14 +21,24 @@ __host__ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
   return z ^ (z >> 31);
 }
 
-// The table is an array of buckets of kBucket slots. Each slot has a one-byte
-// tag (0: empty; otherwise 0x80 | low 7 key bits) in a separate tag array and
-// an entry (key + tier-mask words) in the entry array. A key's home bucket is
-// the high 64 bits of key * n_buckets (Lemire's range reduction); inserts
-// take the first empty slot in bucket order from the home bucket (linear
-// probing over buckets). At load factor 0.7, 98.6% of keys sit in their home
-// bucket, so a lookup is one tag read plus one entry read.
-constexpr int kBucket = 16;
+// The table is an array of buckets of kSlots = 15 slots. A bucket's 16-byte
+// tag group (in a tag array of its own) holds a one-byte tag per slot (0:
+// empty; otherwise 0x80 | low 7 key bits) and, in byte 15, the bucket's
+// overflow count: how many keys stored past this bucket probed through it
+// (saturating at 255, which then stays). Entries (key + tier-mask words) are
+// in the entry array, slot sl of bucket b at b * kSlots + sl. A key's home
+// bucket is the high 64 bits of key * n_buckets (Lemire's range reduction);
+// an insert takes the first empty slot in bucket order from the home bucket
+// (linear probing over buckets) and counts itself in the overflow byte of
+// every bucket it passed; a lookup stops at the first bucket without the key
+// whose overflow count is 0. A key that leaves its last tier gives its slot
+// back (tag and key zeroed, the passed buckets' counts decremented), so the
+// table holds live keys only and no tombstones. At load factor 0.7 about 98%
+// of keys sit in their home bucket: a lookup is one tag read plus one entry
+// read.
+constexpr int kBucket = 16;  // bytes of a bucket's tag group
+constexpr int kSlots = 15;   // slots of a bucket
+constexpr uint32_t kSlotBits = (1u << kSlots) - 1;
 
 // mix64 on 32-bit halves, for the serial chain where only latency counts:
 // the high word of each product is one three-input sum of the low-by-low
@@ -76,6 +86,19 @@ __device__ __forceinline__ uint32_t tag_match(uint4 t, uint32_t tag) {
   return m;
 }
 
+// Bit s of the result is set where slot s's tag equals `tag` (byte 15, the
+// overflow count, left out).
+__device__ __forceinline__ uint32_t slot_match(uint4 t, uint32_t tag) { return tag_match(t, tag) & kSlotBits; }
+
+// A bucket's overflow count (byte 15 of its tag group).
+__device__ __forceinline__ uint32_t overflow_count(uint4 t) { return t.w >> 24; }
+
+// Buckets a lookup or an insert visits at most.
+__host__ __device__ __forceinline__ uint64_t max_buckets(uint64_t n_buckets) {
+  const uint64_t m = SMETRIC_MAX_PROBE / kBucket;
+  return n_buckets < m ? n_buckets : m;
+}
+
 // First error wins; later ones are dropped until the host reads and clears.
 __device__ __forceinline__ void latch_error(int32_t* status, int32_t code) {
   atomicCAS(reinterpret_cast<int*>(status), 0, code);
@@ -98,15 +121,39 @@ struct ProfileSlot {
 
 }  // namespace smetric
 
+namespace smetric {
+
+// Device-side LRU of the capped tiers (smetric_index_set_lru; kernels in
+// lru.cu). Each capped tier keeps its keys in recency order, least recent
+// first, in a region of one of two record buffers; a commit rewrites every
+// region from one buffer into the other.
+struct LruState {
+  int64_t local_cap = 0, global_cap = 0;  // blocks; 0 = uncapped
+  int n_tiers = 0;                        // N + 1
+  uint64_t* ring[2] = {nullptr, nullptr}; // records (keys), tier t's at its region offset
+  int cur = 0;                            // the buffer holding the current records
+  int64_t* plan = nullptr;                // kLruPlanFields rows of n_tiers + 1 int64 (lru.cu)
+  int64_t* req_off = nullptr;             // 2 * max_batch_requests: a request's first touch in its tiers
+  uint64_t* touches = nullptr;            // 2 * max_blocks: the batch's touches, tier after tier
+  uint64_t* set = nullptr;                // set_entries (key, last touch + 1) pairs
+  int64_t set_entries = 0;
+  uint8_t* keep = nullptr;                // max_tiles * kLruTile flags
+  int64_t* tile_cnt = nullptr;            // max_tiles + 1, then their exclusive scan
+  int64_t* tile_off = nullptr;
+  int64_t max_tiles = 0;
+};
+
+}  // namespace smetric
+
 struct smetric_index {
   smetric_index_config cfg;
   int device;
   int num_sms;
   int W;   // tier-mask words per key
   int EW;  // entry stride in 64-bit words
-  uint64_t n_buckets;  // ceil(capacity_slots / kBucket)
-  uint64_t* table;     // n_buckets * kBucket entries of EW words
-  uint8_t* tags;       // n_buckets * kBucket tag bytes
+  uint64_t n_buckets;  // ceil(capacity_slots / kSlots)
+  uint64_t* table;     // n_buckets * kSlots entries of EW words
+  uint8_t* tags;       // n_buckets tag groups of kBucket bytes
   int32_t* status;  // device: first latched error
   // route scratch
   int64_t* block_off;  // max_batch_requests + 1: first block of each request
@@ -130,6 +177,7 @@ struct smetric_index {
   int32_t* st_out32;    // 3 * max_batch_requests
   uint64_t* st_sk;      // max_batch_requests
   int digest_occ;  // resident digest CTAs per SM (0 until the first route)
+  smetric::LruState* lru;  // capped tiers' recency (NULL: no tier capped)
   // observability
   int64_t launches;
   bool profiling;
@@ -146,4 +194,12 @@ int cuda_status(cudaError_t e);
 // (and the global tier); block_off must hold the batch's block offsets.
 int launch_commit(smetric_index* idx, const int32_t* d_instance, const uint64_t* d_hashes, int32_t n,
                   int64_t max_blocks, bool global, cudaStream_t s);
+// After a commit's inserts: the capped tiers' recency lists take the batch's
+// touches and evict what exceeds each cap (no-op without an LRU).
+int lru_commit(smetric_index* idx, const int32_t* d_instance, const uint64_t* d_hashes, int32_t n, bool global,
+               cudaStream_t s);
+// Empties every recency list (after the table is cleared).
+int lru_reset(smetric_index* idx, cudaStream_t s);
+// Frees the LRU state.
+void lru_free(smetric_index* idx);
 }  // namespace smetric

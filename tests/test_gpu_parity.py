@@ -167,16 +167,21 @@ def test_index_rejects_bad_keys_and_tiers():
 
 
 def test_index_full_reports_and_stays_consistent():
-    ix = make_index(2, 16, 1, cap=100)  # rounded up to 7 buckets of 16 slots
+    ix = make_index(2, 16, 1, cap=100)  # rounded up to 7 buckets of 15 slots
     keys = np.arange(1000, 1300, dtype=np.uint64) * np.uint64(0x9E3779B97F4A7C15)
     keys = np.maximum(keys, 2)
     ix.insert(T(keys), T(np.zeros(len(keys), np.int32)))
     assert ix.status() == pkg.SMETRIC_ERR_TABLE_FULL
     m = ix.lookup(T(keys)).cpu().numpy()[:, 0]
-    assert int((m & 1).sum()) == 112  # exactly the slots that exist
+    assert int((m & 1).sum()) == 105  # exactly the slots that exist
     ix.evict(T(keys), T(np.zeros(len(keys), np.int32)))
     assert ix.status() == pkg.SMETRIC_OK
     assert int(ix.lookup(T(keys)).cpu().numpy().sum()) == 0
+    # every slot was given back: the table takes as many keys again
+    ix.insert(T(keys[::-1].copy()), T(np.ones(len(keys), np.int32)))
+    assert ix.status() == pkg.SMETRIC_ERR_TABLE_FULL
+    m = ix.lookup(T(keys)).cpu().numpy()[:, 0]
+    assert int(((m >> 1) & 1).sum()) == 105 and int((m & 1).sum()) == 0
 
 
 def test_create_reports_oom_and_the_device_stays_usable():
