@@ -221,13 +221,11 @@ def test_config5_corner_points_sampled(N, B):
     ix.close()
 
 
-@pytest.mark.parametrize("N,B,batch", [(256, 16, 8192), (8, 64, 8192), (64, 32, 32768)])
-def test_config5_full_size_points_sampled(N, B, batch):
-    """Config-5 sweep points at the full session count, in the benchmark's
-    launch configuration: the most instances with the smallest blocks, the
-    fewest with the largest, and the largest batch. Random filler keys with
-    random tiers pad the table to load factor 0.7 of its capacity; the
-    oracle recomputes a sample of requests one by one and invariants are
+def _config5_full_size(N, B, batch, n_sample):
+    """A config-5 sweep point at the full session count, in the benchmark's
+    launch configuration. Random filler keys with random tiers pad the
+    table to load factor 0.7 of its capacity; the oracle recomputes
+    `n_sample` requests (every request when None) and invariants are
     checked on every request."""
     tr = burst_trace("c5_sweep", num_instances=N, block_size=B, batch_size=batch)
     p = tr.params
@@ -241,12 +239,13 @@ def test_config5_full_size_points_sampled(N, B, batch):
     ix.insert(T(fk.view(np.int64)), T(ft))
     ix.check()
     w = (p.w_load, p.w_miss, p.w_glob)
-    g = gpu_route(ix, bt.tokens, bt.offsets, bt.load, w, want_hashes=False)
+    g = gpu_route(ix, bt.tokens, bt.offsets, bt.load, w, want_hashes=n_sample is None)
     lens = bt.lengths()
     assert np.all((g["instance"] >= 0) & (g["instance"] < N))
     assert np.all(g["local_hit"] + g["global_hit"] <= (lens // B) * B)
     rng = np.random.default_rng(N + B)
-    sample = np.sort(rng.choice(bt.n_requests, size=48, replace=False))
+    sample = np.arange(bt.n_requests) if n_sample is None else \
+        np.sort(rng.choice(bt.n_requests, size=n_sample, replace=False))
     ox = oracle.OracleIndex(N)
     sample_hashes = []
     for s in np.unique(bt.sessions[sample]).tolist():
@@ -255,15 +254,39 @@ def test_config5_full_size_points_sampled(N, B, batch):
         for t in tr.session_tiers(s):
             ox.insert(h, t)
     from synth.traces import pack
-    st, so = pack([bt.tokens[bt.offsets[r]:bt.offsets[r + 1]] for r in sample])
-    o = ox.route_batch(B, p.session_blocks, p.hash_seed, st, so, bt.load, *w, want_hashes=True)
+    if n_sample is None:
+        st, so = bt.tokens, bt.offsets
+    else:
+        st, so = pack([bt.tokens[bt.offsets[r]:bt.offsets[r + 1]] for r in sample])
+    o = ox.route_batch(B, p.session_blocks, p.hash_seed, st, so, bt.load, *w, want_hashes=True,
+                       n_threads=os.cpu_count() or 1)
     # the oracle leaves out the filler keys (tens of millions): exact as long
     # as none of them equals a block hash of the sample, which is checked
     assert not np.isin(np.concatenate(sample_hashes + [o["block_hashes"]]), fk).any()
-    sel = {f: g[f][sample] for f in ("instance", "local_hit", "global_hit", "session_key")}
-    assert_outputs_equal(sel, o, fields=("instance", "local_hit", "global_hit", "session_key"),
-                         ctx=f"config 5 N={N} B={B} batch={batch}")
+    fields = ("instance", "local_hit", "global_hit", "session_key")
+    if n_sample is None:
+        assert_outputs_equal(g, o, ctx=f"config 5 N={N} B={B} batch={batch}")
+    else:
+        sel = {f: g[f][sample] for f in fields}
+        assert_outputs_equal(sel, o, fields=fields, ctx=f"config 5 N={N} B={B} batch={batch}")
+    ox.close()
     ix.close()
+
+
+@pytest.mark.parametrize("N,B,batch", [(256, 16, 8192), (8, 64, 8192), (64, 32, 32768)])
+def test_config5_full_size_points_sampled(N, B, batch):
+    """Config-5 sweep points at the full session count: the most instances
+    with the smallest blocks, the fewest with the largest, and the largest
+    batch; 256 requests of each recomputed by the oracle."""
+    _config5_full_size(N, B, batch, 256)
+
+
+@pytest.mark.slow
+def test_config5_largest_point_every_request():
+    """The sweep's largest batch (32,768 requests, N = 64, B = 32) on the
+    filler-padded table: every output of every request, and every block
+    hash, equals the oracle's."""
+    _config5_full_size(64, 32, 32768, None)
 
 
 @pytest.mark.parametrize("pipeline", [True, False])
