@@ -162,6 +162,62 @@ def window_imbalance(num_instances: int, window: int, n_windows: int, instance, 
     return dict(max=mx[:n_windows], argmax=am[:n_windows], sum=sm[:n_windows])
 
 
+class OracleLRU:
+    """Contents of capped KV$ tiers under least-recently-used eviction
+    (Section 2: each instance's local KV$ and the global store are bounded).
+
+    Plain and slow, written from the recency rule itself: every commit k
+    touches, for each committed request r (in order) and each of its full
+    blocks b, the block's key in the request's local tier (and in the global
+    tier when asked) with stamp (k, r, -b), so that later commits, later
+    requests and, within a request, leading blocks are more recent. A key's
+    stamp in a tier is its largest; after the commit each capped tier keeps
+    its `cap` keys of largest stamp. Tier -1 is the global tier."""
+
+    def __init__(self, num_instances: int, local_cap: int = 0, global_cap: int = 0):
+        self.N = num_instances
+        self.caps = {t: local_cap for t in range(num_instances)}
+        self.caps[-1] = global_cap
+        self.stamp = {t: {} for t in range(-1, num_instances)}  # tier -> key -> stamp
+        self.k = 0
+
+    def commit(self, n_blocks, instance, hashes, also_global: bool):
+        """n_blocks[r] full blocks of request r (its hashes in order, request
+        after request); instance[r] < 0 commits nothing for r. Returns the
+        evicted (keys, tiers)."""
+        hashes = [int(x) for x in np.asarray(hashes, dtype=np.uint64)]
+        pos = 0
+        for r, (nb, i) in enumerate(zip(np.asarray(n_blocks).tolist(), np.asarray(instance).tolist())):
+            keys = hashes[pos:pos + nb]
+            pos += nb
+            if i < 0:
+                continue
+            for t in ([i, -1] if also_global else [i]):
+                if self.caps[t] <= 0:
+                    continue
+                tier = self.stamp[t]
+                for b, key in enumerate(keys):
+                    st = (self.k, r, -b)
+                    if key not in tier or tier[key] < st:
+                        tier[key] = st
+        self.k += 1
+        ev_k, ev_t = [], []
+        for t, tier in self.stamp.items():
+            over = len(tier) - self.caps[t]
+            if self.caps[t] > 0 and over > 0:
+                for key, _ in sorted(tier.items(), key=lambda kv: kv[1])[:over]:
+                    del tier[key]
+                    ev_k.append(key)
+                    ev_t.append(t)
+        return np.array(ev_k, dtype=np.uint64), np.array(ev_t, dtype=np.int32)
+
+    def holds(self, key: int, tier: int) -> bool:
+        return int(key) in self.stamp[tier]
+
+    def size(self, tier: int) -> int:
+        return len(self.stamp[tier]) if self.caps[tier] > 0 else 0
+
+
 class OracleIndex:
     """Two-tier KV$ index: local tier per instance plus one global tier (-1)."""
 

@@ -411,6 +411,65 @@ def check_batch_invariants(L):
     assert len(keys_by_session) == tr.n_sessions
 
 
+def check_lru_recency(L):
+    """The LRU oracle against recency worked out by hand, the rule's special
+    cases (one slot keeps the most recent touch: the last committed
+    request's first block; a cap above every key evicts nothing), and a
+    second formulation of the rule (move-to-back ordered dicts, deepest
+    block first within a request)."""
+    from collections import OrderedDict
+    # hand example: N = 2, local cap 3, global cap 0
+    lru = oracle.OracleLRU(2, local_cap=3)
+    ek, et = lru.commit([4], [1], [11, 12, 13, 14], also_global=False)
+    # stamps (0,0,0) (0,0,-1) (0,0,-2) (0,0,-3): the deepest block (14) leaves
+    assert ek.tolist() == [14] and et.tolist() == [1]
+    assert [lru.holds(k, 1) for k in (11, 12, 13, 14)] == [True, True, True, False]
+    ek, et = lru.commit([1, 2], [1, 0], [21, 31, 32], also_global=False)
+    # tier 1 now: 21 (1,0,0), 11 (0,0,0), 12 (0,0,-1), 13 (0,0,-2): 13 leaves
+    assert ek.tolist() == [13] and lru.size(1) == 3 and lru.size(0) == 2
+    ek, et = lru.commit([2, 1], [1, 1], [12, 41, 11], also_global=False)
+    # request 1 touches 11 at (2,1,0), request 0 touches 12 at (2,0,0) and 41
+    # at (2,0,-1): tier 1 holds 11, 12, 41, 21 by recency; 21 leaves
+    assert ek.tolist() == [21] and all(lru.holds(k, 1) for k in (11, 12, 41))
+    # one slot: the last committed request's first block
+    one = oracle.OracleLRU(3, local_cap=1, global_cap=1)
+    one.commit([3, 2, 2], [2, 0, 2], [1, 2, 3, 4, 5, 6, 7], also_global=True)
+    assert one.holds(6, 2) and one.size(2) == 1 and one.holds(4, 0) and one.holds(6, -1)
+    # a cap above every key: nothing leaves
+    big = oracle.OracleLRU(2, local_cap=100, global_cap=100)
+    ek, _ = big.commit([3, 3], [0, 1], [1, 2, 3, 1, 2, 3], also_global=True)
+    assert len(ek) == 0 and big.size(-1) == 3
+    # the second formulation, on random commits with repeated keys
+    rng = np.random.default_rng(15)
+    N, cap, gcap = 3, 7, 11
+    a = oracle.OracleLRU(N, local_cap=cap, global_cap=gcap)
+    od = {t: OrderedDict() for t in range(-1, N)}
+    for step in range(40):
+        n = int(rng.integers(1, 6))
+        nb = rng.integers(0, 6, size=n)
+        inst = rng.integers(-1, N, size=n)
+        h = rng.integers(2, 40, size=int(nb.sum())).astype(np.uint64)
+        ek, et = a.commit(nb, inst, h, also_global=True)
+        pos = 0
+        for r in range(n):
+            keys = h[pos:pos + nb[r]].tolist()
+            pos += int(nb[r])
+            if inst[r] < 0:
+                continue
+            for t in (int(inst[r]), -1):
+                for key in reversed(keys):  # deepest first: the least recent of the request
+                    od[t].pop(key, None)
+                    od[t][key] = None
+        want = []
+        for t, d in od.items():
+            c = gcap if t < 0 else cap
+            while len(d) > c:
+                want.append((d.popitem(last=False)[0], t))
+        assert sorted(zip(ek.tolist(), et.tolist())) == sorted(want), step
+        for t in range(-1, N):
+            assert set(a.stamp[t]) == set(od[t]), (step, t)
+
+
 def check_index_set_semantics(L):
     """Insert/evict behave as set operations per tier (against Python sets)."""
     rng = np.random.default_rng(14)
@@ -1043,6 +1102,7 @@ ALL_CHECKS = [
     check_hand_costs,
     check_batch_invariants,
     check_index_set_semantics,
+    check_lru_recency,
     check_policy_eq1_boundary,
     check_policy_first_turn_is_cost_argmin,
     check_policy_sticks_to_longest_local_hit,

@@ -297,13 +297,15 @@ def _tiny_batch(rng, n_req, B, alphabet=2, max_blocks=6):
 def test_lru_tiny_batches_every_key(N, local_cap, global_cap):
     """Tiny-alphabet batches (blocks shared within and across requests, keys
     touched several times in one batch): after every commit, every key ever
-    seen has exactly the host LRU's tiers, and the sizes match."""
+    seen has exactly the tiers of the LRU oracle (and of the host replay
+    driver's LRU), and the sizes match."""
     B = 4
     rng = np.random.default_rng(N * 100 + local_cap)
     ix = make_index(N, B, 1, cap=2048, max_req=64, max_tok=1 << 12)
     ix.set_lru(local_cap, global_cap)
     do = ReplayDriver(N, B, local_cap=local_cap or None, global_policy="lru" if global_cap else "all",
                       global_cap=global_cap or None)
+    ol = oracle.OracleLRU(N, local_cap=local_cap, global_cap=global_cap)
     seen = set()
     seen_local = [set() for _ in range(N)]
     for step in range(25):
@@ -318,6 +320,7 @@ def test_lru_tiny_batches_every_key(N, local_cap, global_cap):
         ix.commit_batch(T(off), out, also_global=True)
         ix.check()
         do.after_batch(off, inst, lh, hb_h)
+        ol.commit(np.diff(off) // B, inst, hb_h, also_global=True)
         seen.update(hb_h.tolist())
         nbr = np.diff(off) // B
         for r, i in enumerate(inst.tolist()):
@@ -325,14 +328,16 @@ def test_lru_tiny_batches_every_key(N, local_cap, global_cap):
             seen_local[i].update(hb_h[a:a + int(nbr[r])].tolist())
         model = {}
         for i in range(N):  # an uncapped tier holds every key committed to it
-            for key in (do.local_lru[i] if local_cap else seen_local[i]):
+            for key in (ol.stamp[i] if local_cap else seen_local[i]):
                 model.setdefault(key, set()).add(i)
-        for key in (do.global_lru if global_cap else seen):
+        for key in (ol.stamp[-1] if global_cap else seen):
             model.setdefault(key, set()).add(-1)
+        for i in range(N):  # the two host formulations agree
+            assert set(ol.stamp[i]) == (set(do.local_lru[i]) if local_cap else set())
+        assert set(ol.stamp[-1]) == (set(do.global_lru) if global_cap else set())
         _check_model(ix, model, N, extra_keys=seen)
         sizes = ix.lru_sizes().cpu().numpy().tolist()
-        assert sizes == [len(d) if local_cap else 0 for d in do.local_lru] + \
-            [len(do.global_lru) if global_cap else 0]
+        assert sizes == [ol.size(i) for i in range(N)] + [ol.size(-1)]
     ix.close()
 
 
