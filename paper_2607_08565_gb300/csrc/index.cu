@@ -182,7 +182,6 @@ void free_all(smetric_index* x) {
   cudaFree(x->masks);
   cudaFree(x->summ);
   cudaFree(x->chunk_and);
-  cudaFree(x->order);
   cudaFree(x->sk_tmp);
   cudaFree(x->groups);
   cudaFree(x->lead);
@@ -250,7 +249,6 @@ int smetric_index_create(const smetric_index_config* cfg, smetric_index** out) {
             cudaMalloc(&x->groups, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->lead, 2 * (R + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->chunk_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
-            cudaMalloc(&x->order, (R + 2) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->sk_tmp, (R + 1) * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&x->summ, (R > 0 ? R : 1) * ((size_t)c.num_instances + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&x->batch_ok, sizeof(int32_t)) == cudaSuccess;

@@ -5,7 +5,7 @@
 // Kernels per batch, in stream order:
 //   k_prep        one CTA: validates offsets and loads; scans the per-request
 //                 full-block counts into block_off and the 32-block chunk
-//                 counts into chunk_off; zeroes the leader and member counts.
+//                 counts into chunk_off.
 //   k_digest_tma  HBM-bound block digests d_b: chunk q of request r is its
 //                 blocks 32q..32q+31, one 2D TMA tile of 32 overlapping rows
 //                 (each block's bytes rounded out to 16-byte boundaries); a
@@ -24,11 +24,12 @@
 //                 block not shared: the tier masks of h_b from the index (16
 //                 tags of the home bucket, then the matching entry), and the
 //                 AND of each 32-block chunk's masks.
-//   k_walk        leaders, then members: one warp per request walks the runs
-//                 of the local tiers and the global tier, 32 chunks per step
-//                 from the chunk ANDs and block by block where a run ends;
-//                 then lanes = instances for the cost and a shuffle argmin
-//                 with ties to the lowest id (or one of the policy scores).
+//   k_walk        one warp per request walks the runs of the local tiers and
+//                 the global tier (a member over its leader's probes up to
+//                 its shared prefix), 32 chunks per step from the chunk ANDs
+//                 and block by block where a run ends; then lanes =
+//                 instances for the cost and a shuffle argmin with ties to
+//                 the lowest id (or one of the policy scores).
 
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -84,18 +85,14 @@ __global__ void __launch_bounds__(1024) k_prep(const int64_t* __restrict__ off, 
                                               int32_t* status, int64_t max_load, int64_t max_len,
                                               const int64_t* __restrict__ est_hit,
                                               const int64_t* __restrict__ aux0 = nullptr, int64_t aux0_max = 0,
-                                              const int64_t* __restrict__ aux1 = nullptr, int64_t aux1_max = 0,
-                                              int32_t* __restrict__ zero2 = nullptr) {
+                                              const int64_t* __restrict__ aux1 = nullptr, int64_t aux1_max = 0) {
   constexpr int NS = 2;  // scans: full blocks, and 32-block chunks (when chunk_off is wanted)
   constexpr int R = kPrepRounds;
   __shared__ int64_t warp_tot[NS][32];
   __shared__ int64_t pass_tot[NS];
   __shared__ int bad_all;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
-  if (tid == 0) {
-    bad_all = 0;
-    if (zero2) { zero2[0] = 0; zero2[1] = 0; }  // the group stage's leader and member counts
-  }
+  if (tid == 0) bad_all = 0;
   __syncthreads();
   int bad = 0;  // bit 0: invalid offsets, bit 1: out-of-range length or load
   for (int i = tid; i < n_load; i += blockDim.x) {
@@ -861,7 +858,7 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
                   uint64_t h_init, const int32_t* __restrict__ batch_ok, const uint64_t* __restrict__ D,
                   uint64_t* __restrict__ hashes, uint64_t* __restrict__ sk_out, const uint64_t* __restrict__ groups,
                   uint64_t gmask, int32_t* __restrict__ lead, int32_t* __restrict__ share,
-                  int32_t* __restrict__ order, int32_t* __restrict__ counts, const uint8_t* __restrict__ tags,
+                  const uint8_t* __restrict__ tags,
                   const uint64_t* __restrict__ table, uint64_t n_buckets, uint64_t* __restrict__ masks,
                   uint64_t* __restrict__ chunk_and, const uint8_t* __restrict__ lead_flag, int chain_warps,
                   int32_t* status) {
@@ -1065,9 +1062,6 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
         if (lane == 0) {
           lead[r] = l;
           share[r] = (int32_t)sh;
-          // leaders listed from the front, members from the back (any order)
-          if (l == r) order[atomicAdd(counts, 1)] = r;
-          else order[n - 1 - atomicAdd(counts + 1, 1)] = r;
           st_release_cta(&s_share[j], (int32_t)sh);
         }
       }
@@ -1200,21 +1194,19 @@ struct WalkPolicy {
 // if i held every block), the cost, and a shuffle argmin with ties to the
 // lowest id.
 //
-// Two passes. The first walks the group leaders over their own masks and
-// records each leader's run ends (c_i for every instance, then g) in `summ`.
-// The second walks the members: a member's blocks before `share` are the
-// leader's, so a run that ended there ended at the same block, and a run
-// alive through share - 1 continues over the member's own masks from block
-// `share` on. Members therefore start at `share` instead of re-reading the
-// leader's masks from block 0.
-template <int W, bool MEMBERS, int DECIDE>
-__global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (leaders) or 5 (members) CTAs per SM
+// One pass over every request. A member's blocks before `share` are its
+// leader's, whose masks and chunk ANDs the probe wrote (the member's own were
+// not probed there): its walk reads them from the leader up to block
+// `share` (a 32-block chunk that straddles `share` block by block), then its
+// own. Every request's run ends (c_i for every instance, then g) go to
+// `summ` for the sequential variant.
+template <int W, int DECIDE>
+__global__ void __launch_bounds__(kMatchWarps * 32, 5)
     k_walk(int N, int B, const int64_t* __restrict__ off, const int64_t* __restrict__ block_off, int32_t n,
            const int64_t* __restrict__ load, int64_t w_load, int64_t w_miss, int64_t w_glob,
            const uint64_t* __restrict__ masks, const uint64_t* __restrict__ chunk_and,
            const int64_t* __restrict__ chunk_off, const int32_t* __restrict__ batch_ok,
            const int32_t* __restrict__ lead, const int32_t* __restrict__ share, int32_t* __restrict__ summ,
-           const int32_t* __restrict__ order, const int32_t* __restrict__ counts,
            int32_t* __restrict__ inst_out, int32_t* __restrict__ lhit_out,
            int32_t* __restrict__ ghit_out, uint4* __restrict__ groups, int64_t group_vecs,
            const WalkPolicy pol) {
@@ -1233,63 +1225,53 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
   const int64_t tw = (int64_t)gridDim.x * kMatchWarps;
   const unsigned lt = (1u << lane) - 1;
 
-  if (!ok && !MEMBERS)
+  if (!ok)
     for (int64_t r = (int64_t)blockIdx.x * kMatchWarps + warp; r < n; r += tw)
       if (lane == 0) {
         inst_out[r] = -1; lhit_out[r] = 0; ghit_out[r] = 0;
         if (DECIDE == kSession || DECIDE == kColoc) pol.stick[r] = 0;
       }
-  // k_group's lists: leaders from the front of `order`, members from the back
-  const int64_t count = !ok ? 0 : MEMBERS ? counts[1] : counts[0];
-  for (int64_t k = (int64_t)blockIdx.x * kMatchWarps + warp; k < count; k += tw) {
-    const int64_t r = MEMBERS ? order[n - 1 - k] : order[k];
-    const int32_t l = lead[r];
+  for (int64_t r = (int64_t)blockIdx.x * kMatchWarps + warp; ok && r < n; r += tw) {
     const int64_t L = off[r + 1] - off[r];
     const int64_t nb = L / B;
     const int64_t bo = block_off[r];
-    const int64_t sh = MEMBERS ? share[r] : 0;
-    const int32_t* const cl = summ + (int64_t)l * (N + 1);  // the leader's run ends
-    // the first step's loads (see below) go out with the leader's run ends;
+    const int64_t sh = share[r];  // 0 for a leader
+    const int32_t l = sh > 0 ? lead[r] : (int32_t)r;
     // chunk ANDs are per request-aligned chunk: blocks 32q .. 32q + 31 of
-    // request r at index chunk_off[r] + q, so alignment is to b - bo
-    int64_t f = bo + sh;
-    const int64_t F1 = bo + nb;
+    // request r at index chunk_off[r] + q; block p < sh of the request is
+    // block p of its leader
     const int64_t cbase = __ldg(chunk_off + r);
-    const bool head_single = ((f - bo) & 31) || F1 - f < 32;
+    const int64_t lbo = sh > 0 ? __ldg(block_off + l) : bo;
+    const int64_t lcb = sh > 0 ? __ldg(chunk_off + l) : cbase;
+    auto mask_at = [&](int64_t p, int w) -> uint64_t {  // block p of the request
+      return __ldg(masks + ((p < sh ? lbo : bo) + p) * W + w);
+    };
+    auto and_at = [&](int64_t q, int w) -> uint64_t {  // its chunk q; 0 where the chunk straddles sh
+      if (32 * (q + 1) <= sh) return __ldg(chunk_and + (lcb + q) * W + w);
+      if (32 * q < sh) return 0ull;  // walked block by block
+      return __ldg(chunk_and + (cbase + q) * W + w);
+    };
+    int64_t f = bo;
+    const int64_t F1 = bo + nb;
+    const bool head_single = F1 - f < 32;
     uint64_t pre[W];
 #pragma unroll
     for (int w = 0; w < W; ++w) {
       if (head_single) {
-        const int64_t len = min((int64_t)(32 - ((f - bo) & 31)), F1 - f);
-        pre[w] = lane < len ? __ldg(masks + (f + lane) * W + w) : ~0ull;
+        const int64_t len = F1 - f;
+        pre[w] = lane < len ? mask_at(lane, w) : ~0ull;
       } else {
-        pre[w] = lane < ((F1 - f) >> 5) ? __ldg(chunk_and + (cbase + ((f - bo) >> 5) + lane) * W + w) : 0;
+        pre[w] = lane < (nb >> 5) ? and_at(lane, w) : 0;
       }
     }
-    constexpr int CT = 2 * W;  // groups of 32 covering the N + 1 <= 64 W run ends
-    int32_t cv[CT];            // cv[t] = the leader's run end of tier 32 t + lane (g at tier N)
+    constexpr int CT = 2 * W;  // groups of 32 covering the N + 1 <= 64 W tiers
     uint64_t A[W];  // local tiers holding every block so far (warp-uniform)
     bool galive = true;
     int64_t g = 0;
-    if (!MEMBERS) {
 #pragma unroll
-      for (int w = 0; w < W; ++w) {
-        const int lo = w * 64;
-        A[w] = N >= lo + 64 ? ~0ull : (N > lo ? (1ull << (N - lo)) - 1 : 0ull);
-      }
-    } else {
-#pragma unroll
-      for (int t = 0; t < CT; ++t) cv[t] = 32 * t + lane <= N ? __ldg(cl + 32 * t + lane) : 0;
-      int32_t gl = 0;
-#pragma unroll
-      for (int t = 0; t < CT; ++t) {
-        const unsigned alive = __ballot_sync(kFull, 32 * t + lane < N && cv[t] >= sh);
-        if ((t & 1) == 0) A[t >> 1] = alive;
-        else A[t >> 1] |= (uint64_t)alive << 32;
-        if (t == (N >> 5)) gl = __shfl_sync(kFull, cv[t], N & 31);
-      }
-      galive = gl >= sh;
-      g = galive ? sh : gl;
+    for (int w = 0; w < W; ++w) {
+      const int lo = w * 64;
+      A[w] = N >= lo + 64 ? ~0ull : (N > lo ? (1ull << (N - lo)) - 1 : 0ull);
     }
     int ne = 0;
     // `len` consecutive blocks from request block `base`, lane j < len holding
@@ -1345,7 +1327,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
         const int len = (int)min((int64_t)(32 - ((f - bo) & 31)), F1 - f);
 #pragma unroll
         for (int w = 0; w < W; ++w)
-          x[w] = first ? pre[w] : lane < len ? __ldg(masks + (f + lane) * W + w) : ~0ull;
+          x[w] = first ? pre[w] : lane < len ? mask_at(f - bo + lane, w) : ~0ull;
         first = false;
         dead = span(f - bo, len, x);
         f += len;
@@ -1353,8 +1335,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
       }
       const int64_t nfull = (F1 - f) >> 5;
 #pragma unroll
-      for (int w = 0; w < W; ++w)
-        x[w] = first ? pre[w] : lane < nfull ? __ldg(chunk_and + (cbase + ((f - bo) >> 5) + lane) * W + w) : 0;
+      for (int w = 0; w < W; ++w) x[w] = first ? pre[w] : lane < nfull ? and_at(((f - bo) >> 5) + lane, w) : 0;
       first = false;
       bool stop = lane >= nfull;
 #pragma unroll
@@ -1368,7 +1349,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
       if (galive) g = f - bo;
       if (j < nfull && j < 32) {
 #pragma unroll
-        for (int w = 0; w < W; ++w) x[w] = __ldg(masks + (f + lane) * W + w);
+        for (int w = 0; w < W; ++w) x[w] = mask_at(f - bo + lane, w);
         dead = span(f - bo, 32, x);
         f += 32;
       }
@@ -1411,9 +1392,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
 #pragma unroll
       for (int w = 0; w < W; ++w) if (w == wi) aw = A[w];
       int64_t ci = nb;
-      if (MEMBERS && cv[t] < sh) {
-        ci = cv[t];  // ended on the shared blocks, as in the leader
-      } else if (!(aw & bi)) {
+      if (!(aw & bi)) {
         for (int e = 0; e < ne; ++e)
           if (ev_mask[e * W + wi] & bi) { ci = ev_pos[e]; break; }
       }
@@ -1535,13 +1514,11 @@ __global__ void __launch_bounds__(kMatchWarps * 32, MEMBERS ? 5 : 4)  // 4 (lead
     }
     __syncwarp();
   }
-  if (MEMBERS) {
-    // k_group has read the group table: empty it for the next route (it is
-    // zero from index creation before the first)
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < group_vecs;
-         i += (int64_t)gridDim.x * blockDim.x)
-      groups[i] = make_uint4(0, 0, 0, 0);
-  }
+  // the group stage has read the group table: empty it for the next route
+  // (it is zero from index creation before the first)
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < group_vecs;
+       i += (int64_t)gridDim.x * blockDim.x)
+    groups[i] = make_uint4(0, 0, 0, 0);
 }
 
 // ---------------------------------------------------------------------------
@@ -2159,8 +2136,7 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
                        (const int64_t*)idx->block_off, (const int64_t*)idx->chunk_off, n, idx->cfg.session_blocks,
                        mix64(idx->cfg.hash_seed + kGamma), (const int32_t*)idx->batch_ok,
                        (const uint64_t*)idx->digest, hashes ? hashes : idx->hashes, sk, (const uint64_t*)idx->groups,
-                       group_slots_for(n) - 1, idx->lead, idx->share, idx->order,
-                       idx->order + idx->cfg.max_batch_requests, (const uint8_t*)idx->tags,
+                       group_slots_for(n) - 1, idx->lead, idx->share, (const uint8_t*)idx->tags,
                        (const uint64_t*)idx->table, idx->n_buckets, idx->masks, idx->chunk_and,
                        (const uint8_t*)flags, chain_warps, idx->status)))
       return rc;
@@ -2170,25 +2146,21 @@ int launch_match(smetric_index* idx, const int64_t* d_offsets, int32_t n, const 
   const size_t smem = (size_t)N * sizeof(int64_t) + (size_t)kMatchWarps * N * (W + 1) * sizeof(uint64_t);
   const int64_t want = ((int64_t)n + kMatchWarps - 1) / kMatchWarps;
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)idx->num_sms * 8));
-  // leaders, then members (which read the leaders' run ends)
-  using WalkKernel = decltype(&k_walk<W, false, kArgmin>);  // every instantiation has this signature
-  const WalkKernel leaders[5] = {k_walk<W, false, kArgmin>, k_walk<W, false, kSession>, k_walk<W, false, kColoc>,
-                                 k_walk<W, false, kBailian>, k_walk<W, false, kLMetric>};
-  const WalkKernel members[5] = {k_walk<W, true, kArgmin>, k_walk<W, true, kSession>, k_walk<W, true, kColoc>,
-                                 k_walk<W, true, kBailian>, k_walk<W, true, kLMetric>};
-  const WalkKernel kerns[2] = {leaders[pol.on], members[pol.on]};
-  for (const WalkKernel kern : kerns) {
-    if (smem > 48 * 1024 &&
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
-      return cuda_status(cudaErrorInvalidValue);
-    idx->launches++;
-    if ((rc = launch_k(kern, dim3((unsigned)grid), dim3(kMatchWarps * 32), smem, s, !idx->profiling, N,
-                       idx->cfg.block_size, d_offsets, idx->block_off, n, d_load, w.w_load, w.w_miss, w.w_glob,
-                       idx->masks, idx->chunk_and, (const int64_t*)idx->chunk_off, idx->batch_ok, idx->lead,
-                       idx->share, idx->summ, idx->order, idx->order + idx->cfg.max_batch_requests, inst, lhit, ghit,
-                       reinterpret_cast<uint4*>(idx->groups), (int64_t)group_slots_for(n), pol)))
-      return rc;
-  }
+  // every request in one pass (members read their leaders' probes)
+  using WalkKernel = decltype(&k_walk<W, kArgmin>);  // every instantiation has this signature
+  const WalkKernel kerns[5] = {k_walk<W, kArgmin>, k_walk<W, kSession>, k_walk<W, kColoc>, k_walk<W, kBailian>,
+                               k_walk<W, kLMetric>};
+  const WalkKernel kern = kerns[pol.on];
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+    return cuda_status(cudaErrorInvalidValue);
+  idx->launches++;
+  if ((rc = launch_k(kern, dim3((unsigned)grid), dim3(kMatchWarps * 32), smem, s, !idx->profiling, N,
+                     idx->cfg.block_size, d_offsets, idx->block_off, n, d_load, w.w_load, w.w_miss, w.w_glob,
+                     idx->masks, idx->chunk_and, (const int64_t*)idx->chunk_off, idx->batch_ok, idx->lead,
+                     idx->share, idx->summ, inst, lhit, ghit, reinterpret_cast<uint4*>(idx->groups),
+                     (int64_t)group_slots_for(n), pol)))
+    return rc;
   return SMETRIC_OK;
 }
 
@@ -2254,8 +2226,7 @@ int route_common(smetric_index* idx, const int32_t* d_tokens, int64_t n_tokens, 
                             eq1 ? SMETRIC_POLICY_MAX_QUEUED : SMETRIC_MAX_LOAD,
                             eq1 ? SMETRIC_POLICY_MAX_LEN : (int64_t)INT32_MAX, pol ? pol->est_hit : nullptr,
                             pol ? pol->tpot : nullptr, SMETRIC_POLICY_MAX_TPOT,
-                            pol ? pol->nreq : nullptr, SMETRIC_POLICY_MAX_REQUESTS,
-                            PROBE ? idx->order + c.max_batch_requests : nullptr);
+                            pol ? pol->nreq : nullptr, SMETRIC_POLICY_MAX_REQUESTS);
   idx->launches++;
   if ((rc = cuda_status(cudaGetLastError()))) return rc;
   profile_mark(idx, kPrep, s);
@@ -2339,7 +2310,6 @@ struct RouteScratchSet {
   int32_t* lead = nullptr;  // lead, then share at lead + max_batch_requests + 1
   int32_t* summ = nullptr;
   uint64_t* sk_tmp = nullptr;
-  int32_t* order = nullptr;
   int32_t* batch_ok = nullptr;
 };
 
@@ -2382,7 +2352,6 @@ static void free_pipeline(Pipeline* p) {
   cudaFree(a.lead);
   cudaFree(a.summ);
   cudaFree(a.sk_tmp);
-  cudaFree(a.order);
   cudaFree(a.batch_ok);
   if (p->stream) cudaStreamDestroy(p->stream);
   for (cudaEvent_t e : {p->chain_done[0], p->chain_done[1], p->start, p->finish})
@@ -2404,7 +2373,6 @@ static void swap_scratch(smetric_index* x, RouteScratchSet& a) {
   x->share = x->lead + (x->cfg.max_batch_requests + 1);
   std::swap(x->summ, a.summ);
   std::swap(x->sk_tmp, a.sk_tmp);
-  std::swap(x->order, a.order);
   std::swap(x->batch_ok, a.batch_ok);
 }
 
@@ -2427,7 +2395,6 @@ int pipeline_attach(smetric_index* x) {
             cudaMalloc(&a.groups, 2 * x->group_slots * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&a.lead, 2 * (R + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&a.chunk_off, (R + 1) * sizeof(int64_t)) == cudaSuccess &&
-            cudaMalloc(&a.order, (R + 2) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&a.sk_tmp, (R + 1) * sizeof(uint64_t)) == cudaSuccess &&
             cudaMalloc(&a.summ, (R > 0 ? R : 1) * ((size_t)c.num_instances + 1) * sizeof(int32_t)) == cudaSuccess &&
             cudaMalloc(&a.batch_ok, sizeof(int32_t)) == cudaSuccess &&

@@ -167,7 +167,6 @@ struct smetric_index {
   int32_t* share;      // max_batch_requests: leading blocks taken from the leader
   int32_t* summ;       // max_batch_requests * (num_instances + 1): a leader's run ends c_i, then g
   uint64_t* sk_tmp;     // max_batch_requests: session keys nobody reads (session links); a route's leader flags
-  int32_t* order;      // max_batch_requests + 2: leaders from the front, members from the back, then both counts
   int64_t* chunk_off;  // max_batch_requests + 1: first 32-block chunk of each request
   int32_t* batch_ok;   // device flag written by the prep kernel
   // staging for smetric_route_batch_host

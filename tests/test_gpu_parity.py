@@ -352,7 +352,7 @@ def test_batch_of_3100_requests_parity_and_late_errors():
     load = rng.integers(0, 50, size=N)
     before = pkg.smetric_launch_count(ix.handle)
     g = gpu_route(ix, tok, off, load, (1, 4, 2))
-    assert pkg.smetric_launch_count(ix.handle) - before == 6  # prep, digest, leaders, chain and probe, two walks
+    assert pkg.smetric_launch_count(ix.handle) - before == 5  # prep, digest, leaders, chain and probe, walk
     o = ox.route_batch(B, S, 0, tok, off, load, 1, 4, 2, want_hashes=True)
     assert_outputs_equal(g, o, ctx="3100 requests")
     for r in (0, 1500, 2600, 3099):  # ranges of the first, a middle and the last CTA
@@ -465,6 +465,6 @@ def test_profile_and_launch_count():
     prof = pkg.smetric_profile_read(ix.handle)
     assert set(prof) == {"k_prep", "k_digest", "k_chain_probe", "k_walk"}
     assert all(v[1] == 3 and v[0] > 0 for v in prof.values())
-    # 6 kernels per route: prep, digest, leaders, chain with group stage and probe, two walks
-    assert pkg.smetric_launch_count(ix.handle) - before == 18
+    # 5 kernels per route: prep, digest, leaders, chain with group stage and probe, walk
+    assert pkg.smetric_launch_count(ix.handle) - before == 15
     pkg.smetric_profile_enable(ix.handle, False)
