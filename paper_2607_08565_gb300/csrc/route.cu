@@ -1069,7 +1069,7 @@ __global__ void __launch_bounds__(kCpWarps * 32, 1)
       // tier masks of chunk q's blocks of request j at or past its shared
       // prefix, once its chain has published the chunk; and the chunk's AND
       // (a block not probed counts as all ones). Skipped with no wait: a chunk
-      // wholly inside the shared prefix (the walk starts past it). Skipped
+      // wholly inside the shared prefix (the walk reads the leader's). Skipped
       // after waiting: any chunk after one whose AND is empty (that chunk
       // lacks a block of every tier, so every run has ended there: the walk
       // stops before reaching later chunks). When the probers' items in
@@ -1396,7 +1396,7 @@ __global__ void __launch_bounds__(kMatchWarps * 32, 5)
         for (int e = 0; e < ne; ++e)
           if (ev_mask[e * W + wi] & bi) { ci = ev_pos[e]; break; }
       }
-      out_c[i] = (int32_t)ci;  // every request's run ends (members' for the sequential variant)
+      out_c[i] = (int32_t)ci;  // every request's run ends (for the sequential variant)
       if (DECIDE == kArgmin) {
         const int64_t gi = ci > g ? ci : g;
         const int64_t cost = w_load * load_s[i] + w_miss * (L - B * gi) + w_glob * B * (gi - ci);
