@@ -151,3 +151,55 @@ def test_mutant_is_caught(name, tmp_path):
     line = [x for x in p.stdout.splitlines() if x.startswith("FAILED_CHECKS")][-1]
     failed = line.split(" ", 1)[1].strip() if " " in line else ""
     assert failed, f"mutant {name} passed every pin"
+
+
+# The LRU oracle (plain Python): each mutant restates the recency rule with
+# one plausible slip and must fail pins.check_lru_recency.
+def _lru_mutant(stamp_of=None, keep_first_touch=False, evict_largest=False):
+    class Mutant(oracle.OracleLRU):
+        def commit(self, n_blocks, instance, hashes, also_global):
+            import numpy as np
+            hashes = [int(x) for x in np.asarray(hashes, dtype=np.uint64)]
+            pos = 0
+            for r, (nb, i) in enumerate(zip(np.asarray(n_blocks).tolist(), np.asarray(instance).tolist())):
+                keys = hashes[pos:pos + nb]
+                pos += nb
+                if i < 0:
+                    continue
+                for t in ([i, -1] if also_global else [i]):
+                    if self.caps[t] <= 0:
+                        continue
+                    tier = self.stamp[t]
+                    for b, key in enumerate(keys):
+                        st = stamp_of(self.k, r, b) if stamp_of else (self.k, r, -b)
+                        if key not in tier or (not keep_first_touch and tier[key] < st):
+                            tier[key] = st
+            self.k += 1
+            ev_k, ev_t = [], []
+            for t, tier in self.stamp.items():
+                over = len(tier) - self.caps[t]
+                if self.caps[t] > 0 and over > 0:
+                    order = sorted(tier.items(), key=lambda kv: kv[1], reverse=evict_largest)
+                    for key, _ in order[:over]:
+                        del tier[key]
+                        ev_k.append(key)
+                        ev_t.append(t)
+            return np.array(ev_k, dtype=np.uint64), np.array(ev_t, dtype=np.int32)
+    return Mutant
+
+
+LRU_MUTANTS = {
+    "deepest_block_most_recent": _lru_mutant(stamp_of=lambda k, r, b: (k, r, b)),
+    "earlier_request_more_recent": _lru_mutant(stamp_of=lambda k, r, b: (k, -r, -b)),
+    "batch_order_ignored": _lru_mutant(stamp_of=lambda k, r, b: (r, -b)),
+    "first_touch_kept": _lru_mutant(keep_first_touch=True),
+    "most_recent_evicted": _lru_mutant(evict_largest=True),
+}
+
+
+@pytest.mark.parametrize("name", sorted(LRU_MUTANTS))
+def test_lru_mutant_is_caught(name, monkeypatch):
+    from pins import check_lru_recency
+    monkeypatch.setattr(oracle, "OracleLRU", LRU_MUTANTS[name])
+    with pytest.raises(AssertionError):
+        check_lru_recency(None)
